@@ -46,7 +46,8 @@ __all__ = [
     "ln_series", "cos2pi_series", "make_inputs_x", "teacher_params",
     "teacher_labels", "init_params", "layer_offsets", "num_params",
     "make_schedule", "commit_bench_order", "commit_bench_acc",
-    "commit_bench_theta", "DEFAULT_SEED",
+    "commit_bench_theta", "normal_f32", "DEFAULT_SEED",
+    "SyntheticDataset", "workload_dataset", "workload_schedule",
 ]
 
 _M64 = (1 << 64) - 1
@@ -332,18 +333,57 @@ def commit_bench_order(seed: int, n: int, pulls_per_commit: int):
     return np.array(p, dtype=np.int32), pulls
 
 
+# float32 variant of the normal variate, used by the standalone commit
+# workload (hundreds of millions of draws per accumulator, generated on the
+# GPU): the same Box-Muller with float32 series, every operation a correctly
+# rounded float32 +, -, *, / or sqrt.
+_LN_TERMS_F32 = 6      # s^11/11 < 3e-10
+_COS_TERMS_F32 = 12    # pi^24/24! < 5e-13
+_F32 = np.float32
+
+
+def normal_f32(key: int, idx) -> np.ndarray:
+    """N(0,1) variate number i in float32 arithmetic (draws 2i and 2i+1)."""
+    idx = np.asarray(idx, dtype=_U64)
+    d1 = draw(key, idx * _U64(2))
+    d2 = draw(key, idx * _U64(2) + _U64(1))
+    u1 = ((d1 >> _U64(40)).astype(np.float64) * (2.0 ** -24)).astype(_F32)
+    u2 = ((d2 >> _U64(40)).astype(np.float64) * (2.0 ** -24)).astype(_F32)
+    x = _F32(1.0) - u1                                   # exact, in (0, 1]
+    f, e = np.frexp(x)
+    small = f < _F32(_SQRT_HALF)
+    f = np.where(small, f * _F32(2.0), f).astype(_F32)
+    e = np.where(small, e - 1, e).astype(_F32)
+    s = (f - _F32(1.0)) / (f + _F32(1.0))
+    s2 = s * s
+    p = np.full_like(s, _F32(1.0) / _F32(2 * (_LN_TERMS_F32 - 1) + 1))
+    for k in range(_LN_TERMS_F32 - 2, -1, -1):
+        p = p * s2 + _F32(1.0) / _F32(2 * k + 1)
+    ln = e * _F32(_LN2) + (_F32(2.0) * s) * p
+    r = np.sqrt(_F32(-2.0) * ln)
+    c = [_F32(1.0)]
+    for k in range(1, _COS_TERMS_F32):
+        c.append(_F32(-c[-1] / _F32((2 * k - 1) * (2 * k))))
+    th = u2 * _F32(_TWO_PI) - _F32(_PI)
+    th2 = th * th
+    q = np.full_like(th, c[-1])
+    for k in range(_COS_TERMS_F32 - 2, -1, -1):
+        q = q * th2 + c[k]
+    return (r * (-q)).astype(_F32)
+
+
 def commit_bench_acc(seed: int, P: int, k: int, idx=None) -> np.ndarray:
-    """Accumulator k, a_k ~ N(0, 1e-2): fp32(0.1 z), z = normal number k*P + i."""
+    """Accumulator k, a_k ~ N(0, 1e-2): fp32(0.1) * z, z = float32 normal number k*P + i."""
     key = stream_key(seed, STREAM_COMMIT_ACC)
     i = np.arange(P, dtype=_U64) if idx is None else np.asarray(idx, dtype=_U64)
-    return (normal_f64(key, _U64(k) * _U64(P) + i) * 0.1).astype(np.float32)
+    return normal_f32(key, _U64(k) * _U64(P) + i) * _F32(0.1)
 
 
 def commit_bench_theta(seed: int, P: int, idx=None) -> np.ndarray:
-    """Initial central variable of the commit workload, N(0,1) in float32."""
+    """Initial central variable of the commit workload: float32 normal number i."""
     key = stream_key(seed, STREAM_COMMIT_THETA)
     i = np.arange(P, dtype=_U64) if idx is None else np.asarray(idx, dtype=_U64)
-    return normal_f64(key, i).astype(np.float32)
+    return normal_f32(key, i)
 
 
 class SyntheticDataset:

@@ -1,0 +1,208 @@
+/*
+ * agn.h - C ABI of the GB300 implementation of the hot path of Accumulated
+ * Gradient Normalization (Hermans, Spanakis & Moeckel, ACML 2017).
+ *
+ * What the library computes (all of it in CUDA kernels on one GPU):
+ *   n workers, each a resident replica theta_k of the parameters, pull the
+ *   central variable theta~, take lambda local minibatch-SGD steps on their own
+ *   data shard while accumulating the gradients (Algorithm 1), and commit the
+ *   accumulated update normalised by lambda,
+ *       Delta theta^k = -(eta / lambda) * sum_i (1/m) sum_j grad L(theta_i; x_ij, y_ij)   (Eq. 1)
+ *   which the parameter server adds to theta~ in FIFO order (Eq. 2).  The
+ *   asynchrony is an explicit, seeded schedule: commit c belongs to worker w_c
+ *   and was computed from theta~ after v_c = c - tau_c commits (Fig. 1).
+ *
+ * Conventions for every entry point:
+ *   - Return 0 (AGN_OK) on success, a negative AGN_E_* code on failure; the
+ *     message of the last failure on a handle is agn_last_error(handle), and
+ *     that of a handle-less call is agn_last_error(NULL) (per thread).
+ *   - Host buffers are owned by the caller and given with a capacity in
+ *     elements; a short buffer gives AGN_E_INVALID and writes nothing.
+ *   - Device buffers passed in are owned by the caller and must stay valid
+ *     until the work queued on the given stream completes.
+ *   - A handle must not be used by two threads at once.
+ *   - Flat parameter order (the paper fixes none): for l = 1..L, W_l row-major
+ *     [d_l][d_{l-1}], then b_l [d_l].  P = sum_l (d_l d_{l-1} + d_l).
+ *   - The loss is softmax cross-entropy over the last layer's d_L outputs; the
+ *     hidden layers use ReLU.
+ */
+#ifndef AGN_H
+#define AGN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AGN_OK 0
+#define AGN_E_INVALID (-1)     /* bad sizes, pointers or options            */
+#define AGN_E_SCHEDULE (-2)    /* infeasible (worker, staleness) pair       */
+#define AGN_E_OOM (-3)         /* device or host allocation failed          */
+#define AGN_E_CUDA (-4)        /* a CUDA call failed (message has details)   */
+#define AGN_E_TIMEOUT (-5)     /* a bounded device wait gave up              */
+#define AGN_E_NONFINITE (-6)   /* a loss or a commit was not finite; the run
+                                  still completed and theta~ is readable     */
+#define AGN_E_UNSUPPORTED (-7) /* valid request this build cannot serve      */
+
+#define AGN_PREC_FP32 0        /* fp32 parameters, activations and GEMMs    */
+#define AGN_PREC_BF16 1        /* bf16 GEMM operands, fp32 accumulation, fp32
+                                  master replicas and accumulators            */
+
+#define AGN_DIST_UNIFORM 0     /* x ~ U[0,1)^d0 */
+#define AGN_DIST_NORMAL 1      /* x ~ N(0,1)^d0 */
+
+#define AGN_GEMM_AUTO 0        /* tensor cores where the build has them     */
+#define AGN_GEMM_SIMT 1        /* CUDA-core GEMM kernels                     */
+#define AGN_GEMM_TCGEN05 2     /* tcgen05/TMEM GEMM kernels (bf16 mode)      */
+
+typedef struct agn_handle agn_handle;
+
+/* Options of agn_create.  Fill with agn_default_options, then override. */
+typedef struct agn_options {
+  int32_t precision;            /* AGN_PREC_*, default fp32                    */
+  int32_t batch;                /* m, samples per minibatch per worker (32)    */
+  int64_t n_samples;            /* N, dataset rows, split into n equal shards of
+                                   S = N / n rows (the last N mod n unused)    */
+  int32_t input_dist;           /* AGN_DIST_*, default uniform                 */
+  const int32_t* teacher_dims;  /* labelling network dims (d_0 .. 10); NULL =
+                                   {d_0, 64, d_L}                             */
+  int32_t n_teacher_dims;
+  int32_t normalize;            /* 1 = AGN (divide by lambda, Eq. 1); 0 = the
+                                   un-normalised ablation (Fig. 3)            */
+  int32_t gemm;                 /* AGN_GEMM_*                                  */
+  int32_t tau_lo, tau_hi;       /* staleness range of the built-in schedule    */
+  void* stream;                 /* cudaStream_t for all work; NULL = a stream
+                                   the handle creates and owns                 */
+  /* Optional caller inputs (host, copied at create); NULL = generate from the
+     seed.  x: [n_samples][d_0] fp32 row-major, y: [n_samples] int32 in
+     [0, d_L), theta0: [P] fp32 flat order. */
+  const float* x_init;
+  const int32_t* y_init;
+  const float* theta_init;
+} agn_options;
+
+void agn_default_options(agn_options* opt);
+
+/*
+ * Create a handle: allocate theta~ [P], replicas theta_k [n][P] and
+ * accumulators a_k [n][P] (fp32; plus bf16 working copies [n][P] in bf16
+ * mode), the dataset and activation workspaces on the current device;
+ * generate (or copy) the dataset, teacher labels and theta~^0 (Glorot-uniform
+ * weights, zero biases); every replica pulls version 0.
+ *   dims     : d_0 .. d_L (n_dims = L + 1 >= 2), all > 0; d_L = classes.
+ *   n_workers: n >= 1;  lambda: local steps per commit >= 1 (Algorithm 1);
+ *   eta      : learning rate > 0 (constant: Section 4 uses no decay);
+ *   seed     : seeds every generated input;  opt: NULL = defaults.
+ * Errors: AGN_E_INVALID, AGN_E_OOM, AGN_E_CUDA, AGN_E_UNSUPPORTED.
+ */
+int agn_create(const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t lambda,
+               double eta, uint64_t seed, const agn_options* opt, agn_handle** out);
+
+/*
+ * Run the next n_commits commits (Algorithm 1 workers, Eq. 2 server).
+ * worker[i], staleness[i] (host, length n_schedule >= n_commits) describe
+ * commits V .. V+n_schedule-1, V = commits applied so far: commit c belongs
+ * to worker[c-V] and reads theta~ after c - staleness[c-V] commits.  Entries
+ * past n_commits are look-ahead: they tell the handle which version each
+ * worker must pull during this call.  Feasible iff prev(w) < v_c <= c with
+ * prev(w) the worker's previous commit (-1 before its first); a commit whose
+ * version was passed in an earlier call must match the pull made then.
+ * worker == NULL and staleness == NULL: use the built-in seeded round-robin
+ * schedule (agn_make_schedule with the handle's tau_lo/tau_hi and seed).
+ * Cumulative: repeated calls continue the commit index and the step counters.
+ * Queues the work on the handle's stream and waits for it.
+ * Errors: AGN_E_INVALID, AGN_E_SCHEDULE (nothing run), AGN_E_CUDA,
+ * AGN_E_NONFINITE (run completed; results readable).
+ */
+int agn_run(agn_handle* h, int32_t n_commits, const int32_t* worker,
+            const int32_t* staleness, int32_t n_schedule);
+
+/* theta~ after the commits run so far, fp32, flat order, into host out[P]. */
+int agn_central(agn_handle* h, float* out, int64_t cap);
+
+/* Replica theta_k (fp32 master), flat order, into host out[P]. */
+int agn_replica(agn_handle* h, int32_t k, float* out, int64_t cap);
+
+/* Per commit so far: the mean of its lambda minibatch losses (host out[C]). */
+int agn_loss(agn_handle* h, float* out, int64_t cap);
+
+/* Per commit so far: ||Delta_c||_2 (host out[C]). */
+int agn_delta_norm(agn_handle* h, float* out, int64_t cap);
+
+int64_t agn_num_params(const agn_handle* h);   /* P, or -1 for NULL */
+int64_t agn_num_commits(const agn_handle* h);  /* commits applied so far */
+
+/*
+ * Statistics of the last agn_run: [0] waves, [1] kernel launches, [2] GPU
+ * milliseconds (CUDA events around the queued work), [3] worker-steps.
+ */
+int agn_last_run_stats(const agn_handle* h, double* out, int64_t cap);
+
+/*
+ * Pure host helper: the inputs agn_create generates for these arguments,
+ * restricted to dataset rows [row0, row0 + n_rows): x [n_rows][d_0] fp32,
+ * y [n_rows] int32 (teacher labels), theta0 [P] fp32 flat (any may be NULL).
+ * teacher_dims NULL = {d_0, 64, d_L}.  Needs no GPU.
+ */
+int agn_generate_inputs(const int32_t* dims, int32_t n_dims, int32_t input_dist,
+                        const int32_t* teacher_dims, int32_t n_teacher_dims, uint64_t seed,
+                        int64_t row0, int64_t n_rows, float* x, int32_t* y, float* theta0);
+
+/* Copy the generated inputs (host, caller-owned, any may be NULL):
+   x [n_samples][d_0] fp32, y [n_samples] int32, theta0 [P] fp32 flat. */
+int agn_export_inputs(agn_handle* h, float* x, int32_t* y, float* theta0);
+
+const char* agn_last_error(const agn_handle* h);
+void agn_destroy(agn_handle* h);
+
+/*
+ * Seeded round-robin schedule (pure host helper): commit c belongs to worker
+ * c mod n, staleness tau_c = tau_lo + ((d_c >> 40)(tau_hi - tau_lo + 1)) >> 24
+ * with d_c the c-th draw of the schedule stream, clamped to c - prev(w_c) - 1.
+ * Outputs are host arrays of n_commits int32.
+ */
+int agn_make_schedule(int32_t n, int32_t n_commits, int32_t tau_lo, int32_t tau_hi,
+                      uint64_t seed, int32_t* worker_out, int32_t* tau_out);
+
+/*
+ * Standalone commit + pull (the parameter-server step, Eq. 1-2 and the
+ * Commit/Pull of Algorithm 1) on caller device buffers.  For c = 0 .. C-1 in
+ * order: k = commit_worker[c];
+ *     Delta = fp32(acc[k] * s), s = fp32(-eta/lambda) (fp32(-eta) when
+ *     normalize == 0), computed in double; theta_c = fp32(theta_c + Delta)
+ *     (no fused multiply-add, so results are bit-reproducible);
+ *     acc[k] = 0;  replica[p] = theta_c for every p in
+ *     pull_workers[pull_offsets[c] .. pull_offsets[c+1]).
+ *   theta_c   : device fp32 [P];  acc, replicas: device fp32 [n][ld],
+ *               ld >= P, ld % 4 == 0, all three 16-byte aligned.
+ *   replicas_bf16: optional device bf16 [n][ld] that receives bf16(theta_c)
+ *               (round to nearest even) at each pull; NULL = none.
+ *   commit_worker [C], pull_offsets [C+1], pull_workers: host int32.
+ *   delta_norm: optional device fp32 [C] receiving ||Delta_c||_2 (the
+ *               per-block partial sums are reduced in a fixed order).
+ *   stream    : cudaStream_t or NULL (legacy default stream).
+ * Queues the work and returns without waiting.  Scratch memory (the schedule
+ * and the norm partials) comes from the stream-ordered allocator.
+ * Errors: AGN_E_INVALID, AGN_E_OOM, AGN_E_CUDA.
+ */
+int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_bf16,
+                    int64_t P, int64_t ld, int32_t n, int32_t C,
+                    const int32_t* commit_worker, const int32_t* pull_offsets,
+                    const int32_t* pull_workers, double eta, int32_t lambda,
+                    int32_t normalize, float* delta_norm, void* stream);
+
+/*
+ * Fill the inputs of the standalone commit workload on the device with the
+ * seeded generator: theta_c[i] = fp32(N(0,1) number i of the commit-theta
+ * stream); acc[k][i] = fp32(0.1 * N(0,1) number k*P + i of the commit-acc
+ * stream) for k < n; replicas [n][ld] (optional) = theta_c.  Asynchronous.
+ */
+int agn_fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P,
+                           int64_t ld, int32_t n, uint64_t seed, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AGN_H */

@@ -1,0 +1,106 @@
+"""ctypes view of the AGN C ABI (include/agn.h): library loading and signatures.
+
+The library is built in-tree (`_build/libagn_gb300.so`, see build.py).  There
+is no fallback: if it is missing, loading raises.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libagn_gb300.so")
+
+AGN_OK = 0
+AGN_E_INVALID = -1
+AGN_E_SCHEDULE = -2
+AGN_E_OOM = -3
+AGN_E_CUDA = -4
+AGN_E_TIMEOUT = -5
+AGN_E_NONFINITE = -6
+AGN_E_UNSUPPORTED = -7
+
+AGN_PREC_FP32 = 0
+AGN_PREC_BF16 = 1
+AGN_DIST_UNIFORM = 0
+AGN_DIST_NORMAL = 1
+AGN_GEMM_AUTO = 0
+AGN_GEMM_SIMT = 1
+AGN_GEMM_TCGEN05 = 2
+
+ERROR_NAMES = {
+    AGN_E_INVALID: "AGN_E_INVALID", AGN_E_SCHEDULE: "AGN_E_SCHEDULE", AGN_E_OOM: "AGN_E_OOM",
+    AGN_E_CUDA: "AGN_E_CUDA", AGN_E_TIMEOUT: "AGN_E_TIMEOUT",
+    AGN_E_NONFINITE: "AGN_E_NONFINITE", AGN_E_UNSUPPORTED: "AGN_E_UNSUPPORTED",
+}
+
+
+class agn_options(C.Structure):
+    _fields_ = [
+        ("precision", C.c_int32),
+        ("batch", C.c_int32),
+        ("n_samples", C.c_int64),
+        ("input_dist", C.c_int32),
+        ("teacher_dims", C.POINTER(C.c_int32)),
+        ("n_teacher_dims", C.c_int32),
+        ("normalize", C.c_int32),
+        ("gemm", C.c_int32),
+        ("tau_lo", C.c_int32),
+        ("tau_hi", C.c_int32),
+        ("stream", C.c_void_p),
+        ("x_init", C.POINTER(C.c_float)),
+        ("y_init", C.POINTER(C.c_int32)),
+        ("theta_init", C.POINTER(C.c_float)),
+    ]
+
+
+_I32P = C.POINTER(C.c_int32)
+_F32P = C.POINTER(C.c_float)
+_F64P = C.POINTER(C.c_double)
+
+# name -> (restype, argtypes); every symbol the header declares.
+SIGNATURES = {
+    "agn_default_options": (None, [C.POINTER(agn_options)]),
+    "agn_create": (C.c_int, [_I32P, C.c_int32, C.c_int32, C.c_int32, C.c_double, C.c_uint64,
+                             C.POINTER(agn_options), C.POINTER(C.c_void_p)]),
+    "agn_run": (C.c_int, [C.c_void_p, C.c_int32, _I32P, _I32P, C.c_int32]),
+    "agn_central": (C.c_int, [C.c_void_p, _F32P, C.c_int64]),
+    "agn_replica": (C.c_int, [C.c_void_p, C.c_int32, _F32P, C.c_int64]),
+    "agn_loss": (C.c_int, [C.c_void_p, _F32P, C.c_int64]),
+    "agn_delta_norm": (C.c_int, [C.c_void_p, _F32P, C.c_int64]),
+    "agn_num_params": (C.c_int64, [C.c_void_p]),
+    "agn_num_commits": (C.c_int64, [C.c_void_p]),
+    "agn_last_run_stats": (C.c_int, [C.c_void_p, _F64P, C.c_int64]),
+    "agn_generate_inputs": (C.c_int, [_I32P, C.c_int32, C.c_int32, _I32P, C.c_int32, C.c_uint64,
+                                      C.c_int64, C.c_int64, _F32P, _I32P, _F32P]),
+    "agn_export_inputs": (C.c_int, [C.c_void_p, _F32P, _I32P, _F32P]),
+    "agn_last_error": (C.c_char_p, [C.c_void_p]),
+    "agn_destroy": (None, [C.c_void_p]),
+    "agn_make_schedule": (C.c_int, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_uint64,
+                                    _I32P, _I32P]),
+    "agn_commit_pull": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64,
+                                  C.c_int64, C.c_int32, C.c_int32, _I32P, _I32P, _I32P,
+                                  C.c_double, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]),
+    "agn_fill_commit_inputs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64,
+                                         C.c_int64, C.c_int32, C.c_uint64, C.c_void_p]),
+}
+
+_LIB = None
+
+
+def load():
+    """Load the library (once) and declare every signature; raise if missing."""
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"AGN CUDA library not found at {LIB_PATH}; build it first "
+                "(python -c 'import __graft_entry__ as g; g.build()')")
+        lib = C.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = lib
+    return _LIB

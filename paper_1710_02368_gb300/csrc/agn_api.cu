@@ -1,0 +1,877 @@
+// C ABI of the AGN library: handle life cycle, the host scheduler that turns
+// a (worker, staleness) schedule into waves of batched local steps and runs of
+// fused commits, and the standalone commit+pull entry point.
+//
+// Scheduling (Fig. 1's FIFO parameter server, Algorithm 1's workers): commit c
+// of worker w_c is computed from theta~ after v_c = c - tau_c commits, and is
+// a pure function of that version and the worker's data cursor.  So the host
+// groups the commits whose version is already available into a wave, runs
+// their lambda local steps as one batched launch sequence, then applies every
+// computed commit in FIFO order (one fused commit+pull launch per run of at
+// most kMaxCommitsPerLaunch commits); each pull happens right after the commit
+// that creates the version it reads.  This gives the same theta~ as applying
+// the commits one at a time in schedule order.
+#include <cmath>
+#include <cstdint>
+#include <new>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "host_inputs.h"
+#include "mlp.cuh"
+
+using agn::bf16;
+using agn::CommitPlan;
+using agn::Status;
+using agn::ceil_div;
+using agn::round_up;
+
+namespace {
+
+thread_local std::string g_error;   // message of the last handle-less failure
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+struct Wave {
+  int offset = 0;                 // first slot in the run's plan arrays
+  int slots = 0;
+  std::vector<CommitPlan> commits;
+};
+
+}  // namespace
+
+struct agn_handle {
+  // problem
+  std::vector<int> dims;
+  int L = 0, n = 0, lam = 0;
+  double eta = 0.0;
+  uint64_t seed = 0;
+  int prec = AGN_PREC_FP32, m = 32, dist = AGN_DIST_UNIFORM, normalize = 1, gemm = 0;
+  int tau_lo = 0, tau_hi = 0;
+  int64_t N = 0, S = 0;
+  std::vector<int> tdims;
+  int64_t P = 0, P_pad = 0;
+  std::vector<int64_t> woff, boff, woff_flat, boff_flat;   // per layer (index l-1)
+  int maxd = 0;
+  // CUDA
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+  std::vector<void*> allocs;
+  // device state
+  float* theta_c = nullptr;   // [P_pad]
+  float* rep = nullptr;       // [n][P_pad] fp32 master replicas
+  float* acc = nullptr;       // [n][P_pad] accumulators (sum of raw gradients)
+  bf16* rep_b = nullptr;      // [n][P_pad] bf16 working copies (bf16 mode)
+  void* X = nullptr;          // [N][d0] T
+  int* y = nullptr;           // [N]
+  void* Xb = nullptr;         // [n][m][d0] T
+  int* yb = nullptr;          // [n][m]
+  std::vector<void*> H;       // H[l] [n][m][d_l] T, l = 1..L-1 (H[0] = Xb)
+  float* Z = nullptr;         // [n][m][d_L]
+  void* dz[2] = {nullptr, nullptr};   // [n][m][maxd] T
+  int* flag = nullptr;
+  double* partials = nullptr;
+  int grid = 0;
+  float* loss = nullptr;      // [cap_commits]
+  float* dnorm = nullptr;     // [cap_commits]
+  int64_t cap_commits = 0;
+  float* loss_parts = nullptr;
+  int64_t cap_parts = 0;
+  int* plan_worker = nullptr;
+  int* plan_commit = nullptr;
+  long long* plan_t0 = nullptr;
+  int64_t cap_plan = 0;
+  int* pull_list = nullptr;   // [n]
+  // host state
+  std::vector<float> hX, htheta0;
+  std::vector<int32_t> hy;
+  int64_t V = 0;                                  // commits applied
+  std::vector<int64_t> prev, pulled_v, steps;     // per worker
+  std::string err;
+  double stats[4] = {0, 0, 0, 0};
+};
+
+namespace {
+
+int fail(agn_handle* h, const Status& s) {
+  if (h) h->err = s.msg; else g_error = s.msg;
+  return s.code;
+}
+int fail(agn_handle* h, int code, const std::string& msg) { return fail(h, Status::Err(code, msg)); }
+
+Status dalloc(agn_handle* h, void** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return Status::Err(AGN_E_OOM, "cudaMalloc of " + std::to_string(bytes) + " bytes failed: " +
+                                      cudaGetErrorString(e));
+  }
+  h->allocs.push_back(*p);
+  return Status::Ok();
+}
+
+void dfree(agn_handle* h, void* p) {
+  if (!p) return;
+  for (auto& a : h->allocs)
+    if (a == p) a = nullptr;
+  cudaFree(p);
+}
+
+template <typename Tp>
+Status dalloc_t(agn_handle* h, Tp** p, size_t count) {
+  void* v = nullptr;
+  AGN_TRY(dalloc(h, &v, count * sizeof(Tp)));
+  *p = static_cast<Tp*>(v);
+  return Status::Ok();
+}
+
+// Grow a device array (keeps the first `keep` elements).
+template <typename Tp>
+Status grow(agn_handle* h, Tp** p, int64_t* cap, int64_t need, int64_t keep) {
+  if (need <= *cap) return Status::Ok();
+  int64_t nc = std::max<int64_t>(need, *cap * 2);
+  Tp* np = nullptr;
+  AGN_TRY(dalloc_t(h, &np, (size_t)nc));
+  if (*p && keep > 0)
+    AGN_TRY_CUDA(cudaMemcpyAsync(np, *p, (size_t)keep * sizeof(Tp), cudaMemcpyDeviceToDevice,
+                                 h->stream));
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  dfree(h, *p);
+  *p = np;
+  *cap = nc;
+  return Status::Ok();
+}
+
+size_t elem_size(const agn_handle* h) { return h->prec == AGN_PREC_BF16 ? 2 : 4; }
+
+// ---------------------------------------------------------------------------
+// One wave: lambda local steps of every slot (Algorithm 1's inner loop)
+// ---------------------------------------------------------------------------
+
+template <typename T>
+Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
+  const int s = wv.slots;
+  const int* sw = h->plan_worker + wv.offset;
+  const int* sc = h->plan_commit + wv.offset;
+  const long long* st0 = h->plan_t0 + wv.offset;
+  const int m = h->m, L = h->L;
+  const T* W = h->prec == AGN_PREC_BF16 ? reinterpret_cast<const T*>(h->rep_b)
+                                         : reinterpret_cast<const T*>(h->rep);
+  const float eta = (float)h->eta;
+  for (int i = 0; i < h->lam; ++i) {
+    AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb), h->yb,
+                                 h->dims[0], m, h->S, sw, st0, i, s, h->stream));
+    ++*launches;
+    // forward, l = 1..L
+    for (int l = 1; l <= L; ++l) {
+      agn::GemmArgs g{};
+      const int fi = h->dims[l - 1], fo = h->dims[l];
+      g.M = m; g.N = fo; g.K = fi;
+      g.a = l == 1 ? h->Xb : h->H[l - 1]; g.lda = fi; g.a_bstride = (int64_t)m * fi;
+      g.b = W + h->woff[l - 1]; g.ldb = fi; g.b_bstride = h->P_pad; g.b_by_worker = 1;
+      g.slot_worker = sw;
+      g.out = l == L ? static_cast<void*>(h->Z) : h->H[l];
+      g.ldo = fo; g.out_bstride = (int64_t)m * fo;
+      g.relu = l < L;
+      g.theta = h->rep; g.ld_param = h->P_pad; g.boff = h->boff[l - 1];
+      AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
+      ++*launches;
+    }
+    AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dz[0]), m, h->dims[L],
+                                 h->loss_parts, sc, h->lam, i, h->flag, s, h->stream));
+    ++*launches;
+    // backward, l = L..1: dX (reads W_l before its update), then dW + update
+    int cur = 0;
+    for (int l = L; l >= 1; --l) {
+      const int fi = h->dims[l - 1], fo = h->dims[l];
+      const void* Hprev = l == 1 ? h->Xb : h->H[l - 1];
+      if (l > 1) {
+        agn::GemmArgs g{};
+        g.M = m; g.N = fi; g.K = fo;
+        g.a = h->dz[cur]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
+        g.b = W + h->woff[l - 1]; g.ldb = fi; g.b_bstride = h->P_pad; g.b_by_worker = 1;
+        g.slot_worker = sw;
+        g.out = h->dz[1 - cur]; g.ldo = fi; g.out_bstride = (int64_t)m * fi;
+        g.mask = Hprev; g.mask_bstride = (int64_t)m * fi;
+        g.theta = h->rep; g.ld_param = h->P_pad;
+        AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
+        ++*launches;
+      }
+      agn::GemmArgs g{};
+      g.M = fo; g.N = fi; g.K = m;
+      g.a = h->dz[cur]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
+      g.b = Hprev; g.ldb = fi; g.b_bstride = (int64_t)m * fi;
+      g.slot_worker = sw;
+      g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
+      g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
+      AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+      ++*launches;
+      cur = 1 - cur;
+    }
+  }
+  return Status::Ok();
+}
+
+// ---------------------------------------------------------------------------
+// Planning
+// ---------------------------------------------------------------------------
+
+struct RunPlan {
+  std::vector<int> start_pulls;
+  std::vector<Wave> waves;
+  std::vector<int> slot_worker, slot_commit;
+  std::vector<long long> slot_t0;
+  std::vector<int64_t> prev, pulled_v, steps;
+};
+
+Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32_t* tau, int ns,
+                  RunPlan* out) {
+  const int n = h->n;
+  const int64_t V0 = h->V;
+  std::vector<int64_t> prev = h->prev;
+  std::vector<int64_t> v(ns);
+  for (int i = 0; i < ns; ++i) {
+    const int64_t c = V0 + i;
+    const int w = worker[i];
+    if (w < 0 || w >= n)
+      return Status::Err(AGN_E_SCHEDULE, "commit " + std::to_string(c) + ": worker " +
+                                             std::to_string(w) + " out of range");
+    if (tau[i] < 0)
+      return Status::Err(AGN_E_SCHEDULE, "commit " + std::to_string(c) + ": negative staleness");
+    v[i] = c - tau[i];
+    if (v[i] <= prev[w])
+      return Status::Err(AGN_E_SCHEDULE,
+                         "commit " + std::to_string(c) + ": worker " + std::to_string(w) +
+                             " cannot read version " + std::to_string(v[i]) +
+                             " (its previous commit is " + std::to_string(prev[w]) + ")");
+    prev[w] = c;
+  }
+  // per-worker commits of this run and first look-ahead commit
+  std::vector<std::vector<int>> q(n);
+  std::vector<int> look(n, -1);
+  for (int i = 0; i < ns; ++i) {
+    const int w = worker[i];
+    if (i < k) q[w].push_back(i);
+    else if (look[w] < 0) look[w] = i;
+  }
+  std::vector<std::vector<int>> pulls_at(k + 1);   // pulls at version V0 + j
+  std::vector<int64_t> pulled = h->pulled_v;
+  for (int w = 0; w < n; ++w) {
+    std::vector<int> lst = q[w];
+    if (look[w] >= 0) lst.push_back(look[w]);
+    for (size_t e = 0; e < lst.size(); ++e) {
+      const int i = lst[e];
+      const int64_t vc = v[i];
+      if (e == 0) {
+        if (vc < V0) {
+          if (pulled[w] != vc)
+            return Status::Err(AGN_E_SCHEDULE,
+                               "commit " + std::to_string(V0 + i) + ": worker " +
+                                   std::to_string(w) + " reads version " + std::to_string(vc) +
+                                   ", which has passed without a pull (give the earlier call a "
+                                   "longer look-ahead)");
+          continue;
+        }
+        if (vc == V0) {
+          if (pulled[w] != V0) pulls_at[0].push_back(w);
+          pulled[w] = V0;
+          continue;
+        }
+      }
+      if (vc <= V0 + k) {
+        pulls_at[vc - V0].push_back(w);
+        pulled[w] = vc;
+      }
+    }
+    if (!q[w].empty()) {
+      // after its last commit of the run, the replica holds the pulled
+      // look-ahead version if there is one, else nothing usable
+      const int i_look = look[w];
+      pulled[w] = (i_look >= 0 && v[i_look] <= V0 + k) ? v[i_look] : -1;
+    }
+  }
+  out->start_pulls = pulls_at[0];
+  // waves
+  std::vector<int64_t> steps = h->steps;
+  std::vector<char> computed(k, 0);
+  std::vector<size_t> ptr(n, 0);
+  int64_t Vc = V0;
+  while (Vc < V0 + k) {
+    Wave wv;
+    wv.offset = (int)out->slot_worker.size();
+    for (int w = 0; w < n; ++w) {
+      if (ptr[w] < q[w].size()) {
+        const int i = q[w][ptr[w]];
+        if (v[i] <= Vc) {
+          out->slot_worker.push_back(w);
+          out->slot_commit.push_back(i);
+          out->slot_t0.push_back(steps[w]);
+          steps[w] += h->lam;
+          ++ptr[w];
+          computed[i] = 1;
+        }
+      }
+    }
+    wv.slots = (int)out->slot_worker.size() - wv.offset;
+    if (wv.slots == 0) return Status::Err(AGN_E_SCHEDULE, "internal: empty wave");
+    int j = (int)(Vc - V0);
+    const int j0 = j;
+    while (j < k && computed[j]) ++j;
+    CommitPlan cp{};
+    for (int i = j0; i < j; ++i) {
+      const int np = (int)pulls_at[i + 1].size();
+      if (cp.n_commits == agn::kMaxCommitsPerLaunch ||
+          cp.pull_begin[cp.n_commits] + np > agn::kMaxPullsPerLaunch) {
+        wv.commits.push_back(cp);
+        cp = CommitPlan{};
+      }
+      const int c = cp.n_commits;
+      cp.worker[c] = worker[i];
+      cp.norm_slot[c] = (int)(V0 + i);
+      int pb = cp.pull_begin[c];
+      for (int p : pulls_at[i + 1]) cp.pull_worker[pb++] = p;
+      cp.pull_begin[c + 1] = pb;
+      cp.n_commits = c + 1;
+    }
+    if (cp.n_commits > 0) wv.commits.push_back(cp);
+    out->waves.push_back(std::move(wv));
+    Vc = V0 + j;
+  }
+  out->prev = std::move(prev);
+  // prev must only advance over the commits actually run
+  for (int w = 0; w < n; ++w) out->prev[w] = h->prev[w];
+  for (int i = 0; i < k; ++i) out->prev[worker[i]] = V0 + i;
+  out->pulled_v = std::move(pulled);
+  out->steps = std::move(steps);
+  return Status::Ok();
+}
+
+Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, int ns) {
+  RunPlan plan;
+  AGN_TRY(build_plan(h, k, worker, tau, ns, &plan));
+  const int64_t V0 = h->V;
+  const int64_t total_slots = (int64_t)plan.slot_worker.size();
+  if (V0 + k > h->cap_commits) {   // loss and dnorm share one capacity
+    int64_t c1 = h->cap_commits, c2 = h->cap_commits;
+    AGN_TRY(grow(h, &h->loss, &c1, V0 + k, V0));
+    AGN_TRY(grow(h, &h->dnorm, &c2, V0 + k, V0));
+    h->cap_commits = c1;
+  }
+  AGN_TRY(grow(h, &h->loss_parts, &h->cap_parts, (int64_t)k * h->lam, 0));
+  if (total_slots > h->cap_plan) {  // the three plan arrays share one capacity
+    int64_t c1 = h->cap_plan, c2 = h->cap_plan, c3 = h->cap_plan;
+    AGN_TRY(grow(h, &h->plan_worker, &c1, total_slots, 0));
+    AGN_TRY(grow(h, &h->plan_commit, &c2, total_slots, 0));
+    AGN_TRY(grow(h, &h->plan_t0, &c3, total_slots, 0));
+    h->cap_plan = c1;
+  }
+  if (total_slots > 0) {
+    AGN_TRY_CUDA(cudaMemcpyAsync(h->plan_worker, plan.slot_worker.data(), total_slots * sizeof(int),
+                                 cudaMemcpyHostToDevice, h->stream));
+    AGN_TRY_CUDA(cudaMemcpyAsync(h->plan_commit, plan.slot_commit.data(), total_slots * sizeof(int),
+                                 cudaMemcpyHostToDevice, h->stream));
+    AGN_TRY_CUDA(cudaMemcpyAsync(h->plan_t0, plan.slot_t0.data(), total_slots * sizeof(long long),
+                                 cudaMemcpyHostToDevice, h->stream));
+  }
+  int64_t launches = 0;
+  AGN_TRY_CUDA(cudaEventRecord(h->ev0, h->stream));
+  if (!plan.start_pulls.empty()) {
+    AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, plan.start_pulls.data(),
+                                 plan.start_pulls.size() * sizeof(int), cudaMemcpyHostToDevice,
+                                 h->stream));
+    AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
+                               (int)plan.start_pulls.size(), h->stream));
+    ++launches;
+  }
+  const float scale = (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
+  for (const Wave& wv : plan.waves) {
+    if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
+    else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
+    for (const CommitPlan& cp : wv.commits) {
+      AGN_TRY(agn::launch_commit_pull(cp, h->theta_c, h->acc, h->rep, h->rep_b, h->P_pad,
+                                      h->P_pad, scale, true, h->partials, h->grid, h->dnorm,
+                                      h->flag, h->stream));
+      launches += 2;
+    }
+  }
+  AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, k, h->loss + V0, h->stream));
+  ++launches;
+  AGN_TRY_CUDA(cudaEventRecord(h->ev1, h->stream));
+  int flag = 0;
+  AGN_TRY_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, h->stream));
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  float ms = 0.f;
+  cudaEventElapsedTime(&ms, h->ev0, h->ev1);
+  h->stats[0] = (double)plan.waves.size();
+  h->stats[1] = (double)launches;
+  h->stats[2] = ms;
+  h->stats[3] = (double)k * h->lam;
+  h->V = V0 + k;
+  h->prev = plan.prev;
+  h->pulled_v = plan.pulled_v;
+  h->steps = plan.steps;
+  if (flag) {
+    AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), h->stream));
+    AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+    return Status::Err(AGN_E_NONFINITE, "a loss or a commit was not finite");
+  }
+  return Status::Ok();
+}
+
+Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t lambda,
+              double eta, uint64_t seed, const agn_options& o) {
+  if (!dims || n_dims < 2) return Status::Err(AGN_E_INVALID, "need at least two layer dims");
+  for (int i = 0; i < n_dims; ++i)
+    if (dims[i] <= 0) return Status::Err(AGN_E_INVALID, "layer dims must be positive");
+  if (n_workers < 1 || n_workers > agn::kMaxPullsPerLaunch)
+    return Status::Err(AGN_E_INVALID, "n_workers must be in [1, 256]");
+  if (lambda < 1) return Status::Err(AGN_E_INVALID, "lambda must be >= 1");
+  if (!(eta > 0.0) || !std::isfinite(eta)) return Status::Err(AGN_E_INVALID, "eta must be > 0");
+  if (o.precision != AGN_PREC_FP32 && o.precision != AGN_PREC_BF16)
+    return Status::Err(AGN_E_INVALID, "unknown precision");
+  if (o.batch < 1) return Status::Err(AGN_E_INVALID, "batch must be >= 1");
+  if (o.n_samples < n_workers) return Status::Err(AGN_E_INVALID, "need n_samples >= n_workers");
+  if (o.input_dist != AGN_DIST_UNIFORM && o.input_dist != AGN_DIST_NORMAL)
+    return Status::Err(AGN_E_INVALID, "unknown input distribution");
+  if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
+  if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
+    return Status::Err(AGN_E_INVALID, "unknown gemm backend");
+  if (o.gemm == AGN_GEMM_TCGEN05)
+    return Status::Err(AGN_E_UNSUPPORTED, "tcgen05 GEMM backend not built in this library");
+  h->dims.assign(dims, dims + n_dims);
+  h->L = n_dims - 1;
+  h->n = n_workers;
+  h->lam = lambda;
+  h->eta = eta;
+  h->seed = seed;
+  h->prec = o.precision;
+  h->m = o.batch;
+  h->N = o.n_samples;
+  h->S = o.n_samples / n_workers;
+  h->dist = o.input_dist;
+  h->normalize = o.normalize ? 1 : 0;
+  h->gemm = o.gemm;
+  h->tau_lo = o.tau_lo;
+  h->tau_hi = o.tau_hi;
+  if (o.teacher_dims && o.n_teacher_dims >= 2) {
+    h->tdims.assign(o.teacher_dims, o.teacher_dims + o.n_teacher_dims);
+    if (h->tdims.front() != dims[0] || h->tdims.back() != dims[n_dims - 1])
+      return Status::Err(AGN_E_INVALID, "teacher dims must start at d_0 and end at d_L");
+    for (int d : h->tdims)
+      if (d <= 0) return Status::Err(AGN_E_INVALID, "teacher dims must be positive");
+  } else {
+    h->tdims = {dims[0], 64, dims[n_dims - 1]};
+  }
+  // parameter layouts: flat (the ABI's order) and padded (device, 64-element aligned tensors)
+  int64_t off = 0, offp = 0;
+  h->maxd = 0;
+  for (int l = 1; l <= h->L; ++l) {
+    const int64_t fi = dims[l - 1], fo = dims[l];
+    h->woff_flat.push_back(off);
+    h->boff_flat.push_back(off + fo * fi);
+    off += fo * fi + fo;
+    offp = round_up(offp, 64);
+    h->woff.push_back(offp);
+    offp = round_up(offp + fo * fi, 64);
+    h->boff.push_back(offp);
+    offp += fo;
+    h->maxd = std::max<int>(h->maxd, (int)fo);
+  }
+  h->P = off;
+  h->P_pad = round_up(offp, 64);
+  h->prev.assign(h->n, -1);
+  h->pulled_v.assign(h->n, 0);
+  h->steps.assign(h->n, 0);
+
+  AGN_TRY_CUDA(cudaGetDevice(&h->device));
+  if (o.stream) {
+    h->stream = static_cast<cudaStream_t>(o.stream);
+  } else {
+    AGN_TRY_CUDA(cudaStreamCreateWithFlags(&h->stream, cudaStreamNonBlocking));
+    h->own_stream = true;
+  }
+  AGN_TRY_CUDA(cudaEventCreate(&h->ev0));
+  AGN_TRY_CUDA(cudaEventCreate(&h->ev1));
+
+  // host inputs
+  const int d0 = dims[0];
+  h->hX.resize((size_t)h->N * d0);
+  h->hy.resize((size_t)h->N);
+  h->htheta0.resize((size_t)h->P);
+  if (o.x_init) std::memcpy(h->hX.data(), o.x_init, h->hX.size() * sizeof(float));
+  else agn::gen_dataset(seed, d0, h->N, h->dist, h->hX.data());
+  if (o.y_init) {
+    std::memcpy(h->hy.data(), o.y_init, h->hy.size() * sizeof(int32_t));
+    for (int32_t v : h->hy)
+      if (v < 0 || v >= dims[n_dims - 1]) return Status::Err(AGN_E_INVALID, "label out of range");
+  } else {
+    auto Ws = agn::gen_teacher(seed, h->tdims);
+    agn::gen_teacher_labels(h->hX.data(), h->N, d0, h->dist, h->tdims, Ws, h->hy.data());
+  }
+  if (o.theta_init) std::memcpy(h->htheta0.data(), o.theta_init, h->htheta0.size() * sizeof(float));
+  else agn::gen_init(seed, h->dims, h->htheta0.data());
+
+  // device buffers
+  const size_t es = elem_size(h);
+  const int64_t n = h->n, m = h->m;
+  AGN_TRY(dalloc_t(h, &h->theta_c, (size_t)h->P_pad));
+  AGN_TRY(dalloc_t(h, &h->rep, (size_t)(n * h->P_pad)));
+  AGN_TRY(dalloc_t(h, &h->acc, (size_t)(n * h->P_pad)));
+  if (h->prec == AGN_PREC_BF16) AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(n * h->P_pad)));
+  AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
+  AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));
+  AGN_TRY(dalloc(h, &h->Xb, (size_t)(n * m * d0) * es));
+  AGN_TRY(dalloc_t(h, &h->yb, (size_t)(n * m)));
+  h->H.assign(h->L, nullptr);
+  for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->H[l], (size_t)(n * m * dims[l]) * es));
+  AGN_TRY(dalloc_t(h, &h->Z, (size_t)(n * m * dims[h->L])));
+  AGN_TRY(dalloc(h, &h->dz[0], (size_t)(n * m * h->maxd) * es));
+  AGN_TRY(dalloc(h, &h->dz[1], (size_t)(n * m * h->maxd) * es));
+  AGN_TRY(dalloc_t(h, &h->flag, 1));
+  h->grid = agn::commit_grid(h->P_pad);
+  AGN_TRY(dalloc_t(h, &h->partials, (size_t)agn::kMaxCommitsPerLaunch * h->grid));
+  AGN_TRY(dalloc_t(h, &h->pull_list, (size_t)n));
+  AGN_TRY(dalloc_t(h, &h->dnorm, 1024));
+  AGN_TRY(dalloc_t(h, &h->loss, 1024));
+  h->cap_commits = 1024;
+
+  // uploads
+  std::vector<float> tpad((size_t)h->P_pad, 0.f);
+  for (int l = 0; l < h->L; ++l) {
+    const int64_t fi = dims[l], fo = dims[l + 1];
+    std::memcpy(&tpad[h->woff[l]], &h->htheta0[h->woff_flat[l]], (size_t)(fo * fi) * sizeof(float));
+    std::memcpy(&tpad[h->boff[l]], &h->htheta0[h->boff_flat[l]], (size_t)fo * sizeof(float));
+  }
+  AGN_TRY_CUDA(cudaMemcpy(h->theta_c, tpad.data(), tpad.size() * sizeof(float),
+                          cudaMemcpyHostToDevice));
+  if (h->prec == AGN_PREC_BF16) {
+    std::vector<bf16> xb(h->hX.size());
+    for (size_t i = 0; i < xb.size(); ++i) xb[i] = __float2bfloat16_rn(h->hX[i]);
+    AGN_TRY_CUDA(cudaMemcpy(h->X, xb.data(), xb.size() * sizeof(bf16), cudaMemcpyHostToDevice));
+  } else {
+    AGN_TRY_CUDA(cudaMemcpy(h->X, h->hX.data(), h->hX.size() * sizeof(float),
+                            cudaMemcpyHostToDevice));
+  }
+  AGN_TRY_CUDA(cudaMemcpy(h->y, h->hy.data(), h->hy.size() * sizeof(int32_t),
+                          cudaMemcpyHostToDevice));
+  AGN_TRY_CUDA(cudaMemsetAsync(h->acc, 0, (size_t)(n * h->P_pad) * sizeof(float), h->stream));
+  AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), h->stream));
+  std::vector<int> all(n);
+  for (int w = 0; w < n; ++w) all[w] = w;
+  AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,
+                               h->stream));
+  AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
+                             (int)n, h->stream));   // every worker pulls version 0
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  return Status::Ok();
+}
+
+Status read_params(agn_handle* h, const float* dev, float* out, int64_t cap) {
+  if (!out || cap < h->P) return Status::Err(AGN_E_INVALID, "output buffer shorter than P");
+  std::vector<float> tpad((size_t)h->P_pad);
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  AGN_TRY_CUDA(cudaMemcpy(tpad.data(), dev, tpad.size() * sizeof(float), cudaMemcpyDeviceToHost));
+  for (int l = 0; l < h->L; ++l) {
+    const int64_t fi = h->dims[l], fo = h->dims[l + 1];
+    std::memcpy(out + h->woff_flat[l], &tpad[h->woff[l]], (size_t)(fo * fi) * sizeof(float));
+    std::memcpy(out + h->boff_flat[l], &tpad[h->boff[l]], (size_t)fo * sizeof(float));
+  }
+  return Status::Ok();
+}
+
+Status read_commit_array(agn_handle* h, const float* dev, float* out, int64_t cap) {
+  if (h->V > 0 && (!out || cap < h->V))
+    return Status::Err(AGN_E_INVALID, "output buffer shorter than the number of commits");
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  if (h->V > 0)
+    AGN_TRY_CUDA(cudaMemcpy(out, dev, (size_t)h->V * sizeof(float), cudaMemcpyDeviceToHost));
+  return Status::Ok();
+}
+
+// ---------------------------------------------------------------------------
+// Standalone commit + pull
+// ---------------------------------------------------------------------------
+
+Status commit_pull(float* theta_c, float* acc, float* reps, void* reps_b, int64_t P, int64_t ld,
+                   int n, int C, const int32_t* cw, const int32_t* po, const int32_t* pw,
+                   double eta, int lambda, int normalize, float* dnorm, cudaStream_t st) {
+  if (P < 1 || ld < P || ld % 4 != 0 || n < 1 || C < 0 || lambda < 1 || !(eta > 0.0))
+    return Status::Err(AGN_E_INVALID, "bad sizes (need P >= 1, ld >= P, ld % 4 == 0, n >= 1)");
+  if (!theta_c || !acc || (C > 0 && (!cw || !po)))
+    return Status::Err(AGN_E_INVALID, "null pointer");
+  auto misaligned = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) != 0; };
+  if (misaligned(theta_c) || misaligned(acc) || (reps && misaligned(reps)) ||
+      (reps_b && (reinterpret_cast<uintptr_t>(reps_b) & 7) != 0))
+    return Status::Err(AGN_E_INVALID, "device buffers must be 16-byte aligned");
+  if (C == 0) return Status::Ok();
+  if (po[0] != 0) return Status::Err(AGN_E_INVALID, "pull_offsets[0] must be 0");
+  for (int c = 0; c < C; ++c) {
+    if (cw[c] < 0 || cw[c] >= n) return Status::Err(AGN_E_INVALID, "commit worker out of range");
+    if (po[c + 1] < po[c]) return Status::Err(AGN_E_INVALID, "pull_offsets must not decrease");
+    for (int p = po[c]; p < po[c + 1]; ++p)
+      if (pw[p] < 0 || pw[p] >= n) return Status::Err(AGN_E_INVALID, "pull worker out of range");
+  }
+  if (po[C] > 0 && (!reps || !pw)) return Status::Err(AGN_E_INVALID, "pulls need replicas");
+  const float scale = (float)(normalize ? -(eta / (double)lambda) : -eta);
+  const int grid = agn::commit_grid(P);
+  double* partials = nullptr;
+  if (dnorm) AGN_TRY_CUDA(cudaMallocAsync((void**)&partials,
+                                          sizeof(double) * agn::kMaxCommitsPerLaunch * grid, st));
+  Status result = Status::Ok();
+  CommitPlan cp{};
+  std::vector<int> extra;            // pulls that did not fit into the launch
+  int* extra_dev = nullptr;
+  auto flush = [&]() -> Status {
+    if (cp.n_commits > 0)
+      AGN_TRY(agn::launch_commit_pull(cp, theta_c, acc, reps, static_cast<bf16*>(reps_b), P, ld,
+                                      scale, true, partials, grid, dnorm, nullptr, st));
+    if (!extra.empty()) {
+      if (!extra_dev) AGN_TRY_CUDA(cudaMallocAsync((void**)&extra_dev, sizeof(int) * n, st));
+      for (size_t b = 0; b < extra.size(); b += (size_t)n) {
+        const int cnt = (int)std::min<size_t>((size_t)n, extra.size() - b);
+        AGN_TRY_CUDA(cudaMemcpyAsync(extra_dev, extra.data() + b, sizeof(int) * cnt,
+                                     cudaMemcpyHostToDevice, st));
+        AGN_TRY(agn::pull_replicas(theta_c, reps, static_cast<bf16*>(reps_b), P, ld, extra_dev,
+                                   cnt, st));
+        // the host vector must outlive the copy
+        AGN_TRY_CUDA(cudaStreamSynchronize(st));
+      }
+      extra.clear();
+    }
+    cp = CommitPlan{};
+    return Status::Ok();
+  };
+  for (int c = 0; c < C && result.ok(); ++c) {
+    bool dup = false;
+    for (int i = 0; i < cp.n_commits; ++i) dup |= cp.worker[i] == cw[c];
+    const int np = po[c + 1] - po[c];
+    if (cp.n_commits == agn::kMaxCommitsPerLaunch || dup ||
+        (cp.n_commits > 0 && cp.pull_begin[cp.n_commits] + np > agn::kMaxPullsPerLaunch)) {
+      result = flush();
+      if (!result.ok()) break;
+    }
+    const int i = cp.n_commits;
+    cp.worker[i] = cw[c];
+    cp.norm_slot[i] = c;
+    int pb = cp.pull_begin[i];
+    int p = po[c];
+    for (; p < po[c + 1] && pb < agn::kMaxPullsPerLaunch; ++p) cp.pull_worker[pb++] = pw[p];
+    cp.pull_begin[i + 1] = pb;
+    cp.n_commits = i + 1;
+    if (p < po[c + 1]) {   // more pulls than one launch holds: finish them after it
+      for (; p < po[c + 1]; ++p) extra.push_back(pw[p]);
+      result = flush();
+    }
+  }
+  if (result.ok()) result = flush();
+  if (partials) cudaFreeAsync(partials, st);
+  if (extra_dev) cudaFreeAsync(extra_dev, st);
+  return result;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+extern "C" {
+
+void agn_default_options(agn_options* o) {
+  if (!o) return;
+  std::memset(o, 0, sizeof(*o));
+  o->precision = AGN_PREC_FP32;
+  o->batch = 32;
+  o->n_samples = 2048;
+  o->input_dist = AGN_DIST_UNIFORM;
+  o->normalize = 1;
+  o->gemm = AGN_GEMM_AUTO;
+  o->tau_lo = 0;
+  o->tau_hi = 0;
+}
+
+int agn_create(const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t lambda, double eta,
+               uint64_t seed, const agn_options* opt, agn_handle** out) {
+  if (!out) return fail(nullptr, AGN_E_INVALID, "out is null");
+  *out = nullptr;
+  agn_options o;
+  if (opt) o = *opt; else agn_default_options(&o);
+  agn_handle* h = new (std::nothrow) agn_handle();
+  if (!h) return fail(nullptr, AGN_E_OOM, "host allocation failed");
+  Status s;
+  try {
+    s = create(h, dims, n_dims, n_workers, lambda, eta, seed, o);
+  } catch (const std::bad_alloc&) {
+    s = Status::Err(AGN_E_OOM, "host allocation failed");
+  }
+  if (!s.ok()) {
+    g_error = s.msg;
+    agn_destroy(h);
+    return s.code;
+  }
+  *out = h;
+  return AGN_OK;
+}
+
+int agn_run(agn_handle* h, int32_t n_commits, const int32_t* worker, const int32_t* staleness,
+            int32_t n_schedule) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  DeviceGuard g(h->device);
+  if (n_commits < 0) return fail(h, AGN_E_INVALID, "n_commits < 0");
+  if (n_commits == 0) return AGN_OK;
+  std::vector<int32_t> w, t;
+  if (!worker && !staleness) {
+    const int64_t total = h->V + n_commits + h->n;
+    w.resize(total);
+    t.resize(total);
+    agn::gen_schedule(h->n, total, h->tau_lo, h->tau_hi, h->seed, w.data(), t.data());
+    worker = w.data() + h->V;
+    staleness = t.data() + h->V;
+    n_schedule = n_commits + h->n;
+  } else if (!worker || !staleness) {
+    return fail(h, AGN_E_INVALID, "give both schedule arrays or neither");
+  }
+  if (n_schedule < n_commits) return fail(h, AGN_E_INVALID, "n_schedule < n_commits");
+  try {
+    Status s = do_run(h, n_commits, worker, staleness, n_schedule);
+    if (!s.ok()) return fail(h, s);
+  } catch (const std::bad_alloc&) {
+    return fail(h, AGN_E_OOM, "host allocation failed");
+  }
+  return AGN_OK;
+}
+
+int agn_central(agn_handle* h, float* out, int64_t cap) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  DeviceGuard g(h->device);
+  Status s = read_params(h, h->theta_c, out, cap);
+  return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int agn_replica(agn_handle* h, int32_t k, float* out, int64_t cap) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  if (k < 0 || k >= h->n) return fail(h, AGN_E_INVALID, "replica index out of range");
+  DeviceGuard g(h->device);
+  Status s = read_params(h, h->rep + (int64_t)k * h->P_pad, out, cap);
+  return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int agn_loss(agn_handle* h, float* out, int64_t cap) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  DeviceGuard g(h->device);
+  Status s = read_commit_array(h, h->loss, out, cap);
+  return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int agn_delta_norm(agn_handle* h, float* out, int64_t cap) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  DeviceGuard g(h->device);
+  Status s = read_commit_array(h, h->dnorm, out, cap);
+  return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int64_t agn_num_params(const agn_handle* h) { return h ? h->P : -1; }
+int64_t agn_num_commits(const agn_handle* h) { return h ? h->V : -1; }
+
+int agn_last_run_stats(const agn_handle* h, double* out, int64_t cap) {
+  if (!h || !out || cap < 4) return fail(const_cast<agn_handle*>(h), AGN_E_INVALID, "need 4 slots");
+  for (int i = 0; i < 4; ++i) out[i] = h->stats[i];
+  return AGN_OK;
+}
+
+int agn_generate_inputs(const int32_t* dims, int32_t n_dims, int32_t input_dist,
+                        const int32_t* teacher_dims, int32_t n_teacher_dims, uint64_t seed,
+                        int64_t row0, int64_t n_rows, float* x, int32_t* y, float* theta0) {
+  if (!dims || n_dims < 2 || row0 < 0 || n_rows < 0 ||
+      (input_dist != AGN_DIST_UNIFORM && input_dist != AGN_DIST_NORMAL))
+    return fail(nullptr, AGN_E_INVALID, "bad arguments");
+  for (int i = 0; i < n_dims; ++i)
+    if (dims[i] <= 0) return fail(nullptr, AGN_E_INVALID, "layer dims must be positive");
+  std::vector<int> td;
+  if (teacher_dims && n_teacher_dims >= 2) td.assign(teacher_dims, teacher_dims + n_teacher_dims);
+  else td = {dims[0], 64, dims[n_dims - 1]};
+  if (td.front() != dims[0] || td.back() != dims[n_dims - 1])
+    return fail(nullptr, AGN_E_INVALID, "teacher dims must start at d_0 and end at d_L");
+  try {
+    std::vector<float> xs;
+    float* xp = x;
+    if (!xp && y) {
+      xs.resize((size_t)n_rows * dims[0]);
+      xp = xs.data();
+    }
+    if (xp) agn::gen_dataset_rows(seed, dims[0], row0, n_rows, input_dist, xp);
+    if (y) {
+      auto Ws = agn::gen_teacher(seed, td);
+      agn::gen_teacher_labels(xp, n_rows, dims[0], input_dist, td, Ws, y);
+    }
+    if (theta0) agn::gen_init(seed, std::vector<int>(dims, dims + n_dims), theta0);
+  } catch (const std::bad_alloc&) {
+    return fail(nullptr, AGN_E_OOM, "host allocation failed");
+  }
+  return AGN_OK;
+}
+
+int agn_export_inputs(agn_handle* h, float* x, int32_t* y, float* theta0) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  if (x) std::memcpy(x, h->hX.data(), h->hX.size() * sizeof(float));
+  if (y) std::memcpy(y, h->hy.data(), h->hy.size() * sizeof(int32_t));
+  if (theta0) std::memcpy(theta0, h->htheta0.data(), h->htheta0.size() * sizeof(float));
+  return AGN_OK;
+}
+
+const char* agn_last_error(const agn_handle* h) { return h ? h->err.c_str() : g_error.c_str(); }
+
+void agn_destroy(agn_handle* h) {
+  if (!h) return;
+  DeviceGuard g(h->device);
+  if (h->stream) cudaStreamSynchronize(h->stream);
+  for (void* p : h->allocs)
+    if (p) cudaFree(p);
+  if (h->ev0) cudaEventDestroy(h->ev0);
+  if (h->ev1) cudaEventDestroy(h->ev1);
+  if (h->own_stream && h->stream) cudaStreamDestroy(h->stream);
+  delete h;
+}
+
+int agn_make_schedule(int32_t n, int32_t n_commits, int32_t tau_lo, int32_t tau_hi, uint64_t seed,
+                      int32_t* worker_out, int32_t* tau_out) {
+  if (n < 1 || n_commits < 0 || tau_lo < 0 || tau_hi < tau_lo || (n_commits > 0 && (!worker_out || !tau_out)))
+    return fail(nullptr, AGN_E_INVALID, "bad schedule arguments");
+  agn::gen_schedule(n, n_commits, tau_lo, tau_hi, seed, worker_out, tau_out);
+  return AGN_OK;
+}
+
+int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_bf16, int64_t P,
+                    int64_t ld, int32_t n, int32_t C, const int32_t* commit_worker,
+                    const int32_t* pull_offsets, const int32_t* pull_workers, double eta,
+                    int32_t lambda, int32_t normalize, float* delta_norm, void* stream) {
+  Status s = commit_pull(theta_c, acc, replicas, replicas_bf16, P, ld, n, C, commit_worker,
+                         pull_offsets, pull_workers, eta, lambda, normalize, delta_norm,
+                         static_cast<cudaStream_t>(stream));
+  return s.ok() ? AGN_OK : fail(nullptr, s);
+}
+
+int agn_fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,
+                           int32_t n, uint64_t seed, void* stream) {
+  if (!theta_c || !acc || P < 1 || ld < P || n < 1)
+    return fail(nullptr, AGN_E_INVALID, "bad arguments");
+  Status s = agn::fill_commit_inputs(theta_c, acc, replicas, P, ld, n, seed,
+                                     static_cast<cudaStream_t>(stream));
+  return s.ok() ? AGN_OK : fail(nullptr, s);
+}
+
+}  // extern "C"

@@ -1,0 +1,317 @@
+// Kernel (c): fused commit + pull of the parameter server.
+//
+// For a run of consecutive commits (FIFO order, Eq. 2) the kernel streams the
+// parameter vector once: each thread keeps its slice of theta~ in registers,
+// and for every commit c of the launch reads the committing worker's
+// accumulator, forms Delta = fp32(a * s) with s = fp32(-eta/lambda) (Eq. 1;
+// the normalisation step of Algorithm 1), adds it to theta~ with a plain
+// round-to-nearest add (no FMA, so the sequence is bit-reproducible), zeroes
+// the accumulator (Algorithm 1 restarts a at 0) and writes theta~ into every
+// replica that pulls at the new version (Pull).  theta~ is written back once.
+// Bytes per launch: 8P (theta~) + C (4P read a + 4P zero a) + pulls * 4P
+// (+ 2P per pull for the bf16 working copy).
+//
+// Per-commit ||Delta||_2: per-thread double partial sums, a warp-shuffle
+// tree, a fixed-order sum over the warps of the block, one partial per block,
+// then a second kernel sums the block partials in a fixed order.  The result
+// is deterministic for a given grid size.
+#include "generator.cuh"
+#include "mlp.cuh"
+
+namespace agn {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 2;   // float4 per thread per iteration (memory-level parallelism)
+
+__device__ __forceinline__ float4 ld_stream(const float4* p) { return __ldcs(p); }
+__device__ __forceinline__ void st_stream(float4* p, float4 v) { __stcs(p, v); }
+
+__device__ __forceinline__ uint2 pack_bf16x4(float4 v) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y);
+  __nv_bfloat162 hi = __floats2bfloat162_rn(v.z, v.w);
+  uint2 r;
+  r.x = *reinterpret_cast<uint32_t*>(&lo);
+  r.y = *reinterpret_cast<uint32_t*>(&hi);
+  return r;
+}
+
+template <bool kBF16>
+__global__ void __launch_bounds__(kThreads)
+commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ theta_c,
+                   float* __restrict__ acc, float* __restrict__ replicas,
+                   bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, float s, int zero_acc,
+                   double* __restrict__ partials) {
+  const int nc = plan.n_commits;
+  double sq[kMaxCommitsPerLaunch];
+#pragma unroll
+  for (int c = 0; c < kMaxCommitsPerLaunch; ++c) sq[c] = 0.0;
+
+  const int64_t n4 = P / 4;
+  const int64_t stride = (int64_t)gridDim.x * kThreads * kUnroll;
+  float4* th4 = reinterpret_cast<float4*>(theta_c);
+  for (int64_t base = (int64_t)blockIdx.x * kThreads * kUnroll + threadIdx.x; base < n4;
+       base += stride) {
+    int64_t idx[kUnroll];
+    bool live[kUnroll];
+    float4 th[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      idx[u] = base + (int64_t)u * kThreads;
+      live[u] = idx[u] < n4;
+      if (live[u]) th[u] = th4[idx[u]];
+    }
+#pragma unroll
+    for (int c = 0; c < kMaxCommitsPerLaunch; ++c) {
+      if (c < nc) {
+        float4* arow = reinterpret_cast<float4*>(acc + (int64_t)plan.worker[c] * ld);
+        float4 a[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u)
+          if (live[u]) a[u] = ld_stream(arow + idx[u]);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          if (!live[u]) continue;
+          float4 d;
+          d.x = __fmul_rn(a[u].x, s);
+          d.y = __fmul_rn(a[u].y, s);
+          d.z = __fmul_rn(a[u].z, s);
+          d.w = __fmul_rn(a[u].w, s);
+          th[u].x = __fadd_rn(th[u].x, d.x);
+          th[u].y = __fadd_rn(th[u].y, d.y);
+          th[u].z = __fadd_rn(th[u].z, d.z);
+          th[u].w = __fadd_rn(th[u].w, d.w);
+          float q = d.x * d.x + d.y * d.y + d.z * d.z + d.w * d.w;
+          sq[c] += (double)q;
+          if (zero_acc) st_stream(arow + idx[u], make_float4(0.f, 0.f, 0.f, 0.f));
+        }
+        for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
+          const int64_t row = (int64_t)plan.pull_worker[p] * ld;
+          float4* rrow = reinterpret_cast<float4*>(replicas + row);
+#pragma unroll
+          for (int u = 0; u < kUnroll; ++u) {
+            if (!live[u]) continue;
+            rrow[idx[u]] = th[u];
+            if (kBF16) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      if (live[u]) th4[idx[u]] = th[u];
+  }
+
+  // Tail of P % 4 elements: block 0, one element per thread.
+  if (blockIdx.x == 0 && threadIdx.x < (int)(P - n4 * 4)) {
+    const int64_t i = n4 * 4 + threadIdx.x;
+    float t = theta_c[i];
+    for (int c = 0; c < nc; ++c) {
+      float* ap = acc + (int64_t)plan.worker[c] * ld + i;
+      float d = __fmul_rn(*ap, s);
+      t = __fadd_rn(t, d);
+#pragma unroll
+      for (int cc = 0; cc < kMaxCommitsPerLaunch; ++cc)
+        if (cc == c) sq[cc] += (double)(d * d);
+      if (zero_acc) *ap = 0.f;
+      for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
+        const int64_t row = (int64_t)plan.pull_worker[p] * ld;
+        replicas[row + i] = t;
+        if (kBF16) rep_bf16[row + i] = __float2bfloat16_rn(t);
+      }
+    }
+    theta_c[i] = t;
+  }
+
+  if (partials == nullptr) return;
+  __shared__ double red[kThreads / 32][kMaxCommitsPerLaunch];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int c = 0; c < kMaxCommitsPerLaunch; ++c) {
+    if (c < nc) {
+      double v = sq[c];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (lane == 0) red[warp][c] = v;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < nc) {
+    double v = 0.0;
+    for (int w = 0; w < kThreads / 32; ++w) v += red[w][threadIdx.x];
+    partials[(int64_t)threadIdx.x * gridDim.x + blockIdx.x] = v;
+  }
+}
+
+// norm[slot] = sqrt(sum_b partials[slot][b]) in a fixed order; one block per commit.
+__global__ void __launch_bounds__(kThreads)
+reduce_norms_kernel(const double* __restrict__ partials, int grid, const __grid_constant__ CommitPlan plan,
+                    float* __restrict__ norms, int* __restrict__ flag) {
+  const int c = blockIdx.x;
+  const int slot = plan.norm_slot[c];
+  const double* row = partials + (int64_t)c * grid;
+  double v = 0.0;
+  for (int b = threadIdx.x; b < grid; b += kThreads) v += row[b];
+  __shared__ double red[kThreads];
+  red[threadIdx.x] = v;
+  __syncthreads();
+  for (int w = kThreads / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    float nrm = (float)sqrt(red[0]);
+    if (norms) norms[slot] = nrm;
+    if (flag && !isfinite(nrm)) atomicExch(flag, 1);
+  }
+}
+
+int g_num_sms = 0;
+
+}  // namespace
+
+int commit_grid(int64_t P) {
+  if (g_num_sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (g_num_sms <= 0) g_num_sms = 148;
+  }
+  const int64_t need = ceil_div(std::max<int64_t>(P / 4, 1), (int64_t)kThreads * kUnroll);
+  const int64_t cap = (int64_t)g_num_sms * 4;
+  return (int)std::max<int64_t>(1, std::min(need, cap));
+}
+
+Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
+                          bf16* replicas_bf16, int64_t P, int64_t ld, float scale, bool zero_acc,
+                          double* partials, int grid, float* delta_norm, int* flag,
+                          cudaStream_t stream) {
+  if (plan.n_commits <= 0) return Status::Ok();
+  if (replicas_bf16)
+    commit_pull_kernel<true><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
+                                                             replicas_bf16, P, ld, scale,
+                                                             zero_acc ? 1 : 0, partials);
+  else
+    commit_pull_kernel<false><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
+                                                              nullptr, P, ld, scale,
+                                                              zero_acc ? 1 : 0, partials);
+  AGN_TRY_CUDA(cudaGetLastError());
+  if (partials && (delta_norm || flag)) {
+    reduce_norms_kernel<<<plan.n_commits, kThreads, 0, stream>>>(partials, grid, plan, delta_norm,
+                                                                 flag);
+    AGN_TRY_CUDA(cudaGetLastError());
+  }
+  return Status::Ok();
+}
+
+// ---------------------------------------------------------------------------
+// Pulls outside a commit (version 0 at create, or at the start of a run)
+// ---------------------------------------------------------------------------
+
+namespace {
+
+__global__ void __launch_bounds__(kThreads)
+pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
+            bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers) {
+  const int k = workers[blockIdx.y];
+  float* dst = replicas + (int64_t)k * ld;
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < P; i += stride) {
+    const float t = theta_c[i];
+    dst[i] = t;
+    if (rep_bf16) rep_bf16[(int64_t)k * ld + i] = __float2bfloat16_rn(t);
+  }
+}
+
+__global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda, int count,
+                                     float* __restrict__ loss) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= count) return;
+  float s = 0.f;
+  for (int i = 0; i < lambda; ++i) s += parts[(int64_t)c * lambda + i];
+  loss[c] = s / (float)lambda;
+}
+
+}  // namespace
+
+Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
+                     int64_t ld, const int* workers, int count, cudaStream_t st) {
+  if (count <= 0) return Status::Ok();
+  dim3 grid((unsigned)std::max(1, commit_grid(P) / std::max(1, count) + 1), (unsigned)count);
+  pull_kernel<<<grid, kThreads, 0, st>>>(theta_c, replicas, replicas_bf16, P, ld, workers);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st) {
+  if (count <= 0) return Status::Ok();
+  reduce_losses_kernel<<<(unsigned)ceil_div(count, 128), 128, 0, st>>>(parts, lambda, count, loss);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+// ---------------------------------------------------------------------------
+// Inputs of the standalone commit workload, on the device (float32 variates)
+// ---------------------------------------------------------------------------
+
+namespace {
+
+constexpr int kLnTermsF32 = 6;
+constexpr int kCosTermsF32 = 12;
+
+__device__ __forceinline__ float normal_f32(uint64_t k, uint64_t i) {
+  using namespace gen;
+  const float u1 = uniform_f32(draw(k, 2 * i));
+  const float u2 = uniform_f32(draw(k, 2 * i + 1));
+  const float x = __fsub_rn(1.0f, u1);
+  int e;
+  float f = frexpf(x, &e);
+  if (f < (float)kSqrtHalf) {
+    f = __fmul_rn(f, 2.0f);
+    e -= 1;
+  }
+  const float s = __fdiv_rn(__fsub_rn(f, 1.0f), __fadd_rn(f, 1.0f));
+  const float s2 = __fmul_rn(s, s);
+  float p = __fdiv_rn(1.0f, (float)(2 * (kLnTermsF32 - 1) + 1));
+  for (int j = kLnTermsF32 - 2; j >= 0; --j)
+    p = __fadd_rn(__fmul_rn(p, s2), __fdiv_rn(1.0f, (float)(2 * j + 1)));
+  const float ln = __fadd_rn(__fmul_rn((float)e, (float)kLn2), __fmul_rn(__fmul_rn(2.0f, s), p));
+  const float r = __fsqrt_rn(__fmul_rn(-2.0f, ln));
+  float c[kCosTermsF32];
+  c[0] = 1.0f;
+  for (int j = 1; j < kCosTermsF32; ++j) c[j] = __fdiv_rn(-c[j - 1], (float)((2 * j - 1) * (2 * j)));
+  const float th = __fsub_rn(__fmul_rn(u2, (float)kTwoPi), (float)kPi);
+  const float th2 = __fmul_rn(th, th);
+  float q = c[kCosTermsF32 - 1];
+  for (int j = kCosTermsF32 - 2; j >= 0; --j) q = __fadd_rn(__fmul_rn(q, th2), c[j]);
+  return __fmul_rn(r, -q);
+}
+
+__global__ void fill_commit_inputs_kernel(float* __restrict__ theta_c, float* __restrict__ acc,
+                                          float* __restrict__ replicas, int64_t P, int64_t ld,
+                                          int n, uint64_t key_theta, uint64_t key_acc) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < P; i += stride) {
+    const float t = normal_f32(key_theta, (uint64_t)i);
+    theta_c[i] = t;
+    for (int k = 0; k < n; ++k) {
+      acc[(int64_t)k * ld + i] = __fmul_rn(normal_f32(key_acc, (uint64_t)k * (uint64_t)P + i), 0.1f);
+      if (replicas) replicas[(int64_t)k * ld + i] = t;
+    }
+  }
+}
+
+}  // namespace
+
+Status fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,
+                          int n, uint64_t seed, cudaStream_t stream) {
+  const int grid = commit_grid(P) * 2;
+  fill_commit_inputs_kernel<<<grid, kThreads, 0, stream>>>(
+      theta_c, acc, replicas, P, ld, n, gen::key(seed, gen::kCommitTheta),
+      gen::key(seed, gen::kCommitAcc));
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+}  // namespace agn

@@ -1,0 +1,79 @@
+// Shared definitions of the AGN CUDA library (not part of the C ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstdint>
+#include <cstdio>
+#include <string>
+
+#include "../../include/agn.h"
+
+namespace agn {
+
+using bf16 = __nv_bfloat16;
+
+// Error carried from an internal call up to the C ABI.
+struct Status {
+  int code = AGN_OK;
+  std::string msg;
+  bool ok() const { return code == AGN_OK; }
+  static Status Ok() { return Status{}; }
+  static Status Err(int c, std::string m) { return Status{c, std::move(m)}; }
+};
+
+inline Status cuda_status(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return Status::Ok();
+  return Status::Err(e == cudaErrorMemoryAllocation ? AGN_E_OOM : AGN_E_CUDA,
+                     std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define AGN_TRY_CUDA(expr)                                  \
+  do {                                                      \
+    cudaError_t e__ = (expr);                               \
+    if (e__ != cudaSuccess) return ::agn::cuda_status(e__, #expr); \
+  } while (0)
+
+#define AGN_TRY(expr)             \
+  do {                            \
+    ::agn::Status s__ = (expr);   \
+    if (!s__.ok()) return s__;    \
+  } while (0)
+
+constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
+
+// ---------------------------------------------------------------------------
+// Standalone commit + pull (kernel c)
+// ---------------------------------------------------------------------------
+
+// Commits handled by one launch of the fused commit+pull kernel: theta~ stays
+// in registers across them and each keeps a per-thread norm accumulator.
+constexpr int kMaxCommitsPerLaunch = 16;
+// Pulls one launch may do in total.
+constexpr int kMaxPullsPerLaunch = 256;
+
+struct CommitPlan {
+  int32_t n_commits;                       // <= kMaxCommitsPerLaunch
+  int32_t worker[kMaxCommitsPerLaunch];    // accumulator committed by commit c
+  int32_t pull_begin[kMaxCommitsPerLaunch + 1];
+  int32_t pull_worker[kMaxPullsPerLaunch];
+  int32_t norm_slot[kMaxCommitsPerLaunch]; // index of commit c in the norm output
+};
+
+// Queue one fused launch for the commits of `plan` plus the partial-norm
+// reduction.  partials: device double [kMaxCommitsPerLaunch * grid] (null: no
+// norms); delta_norm: device float indexed by norm_slot (may be null).
+// flag: device int set to 1 when a Delta is not finite (may be null).
+Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
+                          bf16* replicas_bf16, int64_t P, int64_t ld, float scale,
+                          bool zero_acc, double* partials, int grid, float* delta_norm,
+                          int* flag, cudaStream_t stream);
+
+// Grid size used by the commit kernel for P parameters (a multiple of the SM
+// count, capped by the work).
+int commit_grid(int64_t P);
+
+}  // namespace agn

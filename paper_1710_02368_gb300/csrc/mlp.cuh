@@ -1,0 +1,70 @@
+// Batched MLP kernels (forward, softmax cross-entropy, backward with the
+// fused local update) shared by the host scheduler.
+#pragma once
+
+#include "common.cuh"
+
+namespace agn {
+
+enum { kEpiFwd = 0, kEpiDX = 1, kEpiDW = 2 };
+
+// One batched GEMM over the slots of a wave: C[M x N] = sum_k A(m,k) B(k,n).
+// Slot z reads operand X at X + (X_by_worker ? slot_worker[z] : z) * X_bstride.
+//   forward : A = H_{l-1} [m][d_{l-1}] (k-major), B = W_l [d_l][d_{l-1}]
+//             (k-major), M = m, N = d_l, K = d_{l-1};
+//             out[j][f] = act(C + b_l[f])                       (Eq. 1 inner term)
+//   dX      : A = dZ_l [m][d_l] (k-major), B = W_l (n-major), M = m,
+//             N = d_{l-1}, K = d_l; out = C * [H_{l-1} > 0]
+//   dW      : A = dZ_l (m-major: A(f,j) = dZ_l[j][f]), B = H_{l-1} (n-major),
+//             M = d_l, N = d_{l-1}, K = m; theta_k -= eta C, a_k += C
+//             (Algorithm 1's local step and accumulation; the bias gradient
+//             sum_j dZ_l[j][f] is folded into the first column tile)
+struct GemmArgs {
+  int64_t M, N, K;
+  const void* a;
+  int64_t lda, a_bstride;
+  int a_by_worker;
+  const void* b;
+  int64_t ldb, b_bstride;
+  int b_by_worker;
+  const int* slot_worker;
+  // epilogue
+  void* out;             // forward / dX output
+  int64_t ldo, out_bstride;
+  const void* mask;      // dX: H_{l-1}
+  int64_t mask_bstride;
+  int relu;
+  float* theta;          // fp32 master replicas [n][ld_param]
+  float* acc;            // accumulators [n][ld_param]
+  bf16* theta_bf16;      // bf16 working copies or null
+  int64_t ld_param;
+  int64_t woff, boff;    // offsets of W_l and b_l in a replica
+  float eta;
+};
+
+template <typename T>
+Status simt_forward(const GemmArgs& g, bool last, int slots, cudaStream_t st);
+template <typename T>
+Status simt_backward_dx(const GemmArgs& g, int slots, cudaStream_t st);
+template <typename T>
+Status simt_backward_dw(const GemmArgs& g, int slots, cudaStream_t st);
+// Loss of slot z at local step `step` goes to loss_parts[slot_commit[z] * lam + step].
+template <typename T>
+Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* loss_parts,
+                    const int* slot_commit, int lam, int step, int* flag, int slots,
+                    cudaStream_t st);
+template <typename T>
+Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
+                    const int* slot_worker, const long long* slot_t0, int step, int slots,
+                    cudaStream_t st);
+
+// Pull: copy theta~ into the replicas of `workers` (device list) and their bf16 copies.
+Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
+                     int64_t ld, const int* workers, int count, cudaStream_t st);
+// loss[c] = mean_i parts[c * lambda + i] for c < count.
+Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st);
+// Device-side standalone-commit input generator.
+Status fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,
+                          int n, uint64_t seed, cudaStream_t stream);
+
+}  // namespace agn

@@ -1,0 +1,271 @@
+// Kernels (a) and (b) on CUDA cores: the batched-over-workers MLP forward,
+// softmax cross-entropy, and backward with the fused local SGD step and
+// gradient accumulation of Algorithm 1 (g = grad L; theta_k -= eta g; a_k += g).
+//
+// One launch covers every worker of a wave: grid.z indexes the wave's slots,
+// and slot z reads and updates the replica of worker slot_worker[z].  All
+// three GEMM shapes use one tiled kernel (64x64 tile, 16-deep k slices, 4x4
+// outputs per thread); the element type T is float (fp32 mode) or bf16 (bf16
+// mode: operands bf16, accumulation fp32, master weights fp32).
+#include "mlp.cuh"
+
+namespace agn {
+
+namespace {
+
+constexpr int kBM = 64, kBN = 64, kBK = 16, kTM = 4, kTN = 4;
+constexpr int kThreads = (kBM / kTM) * (kBN / kTN);   // 256
+
+template <typename T>
+__device__ __forceinline__ float to_f(T v);
+template <>
+__device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f<bf16>(bf16 v) { return __bfloat162float(v); }
+
+template <typename T>
+__device__ __forceinline__ T from_f(float v);
+template <>
+__device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// C[M x N] (+)= sum_k A(m, k) B(k, n) for one slot; see GemmArgs for layouts.
+template <typename T, typename TO, bool kAKMajor, bool kBKMajor, int kEpi>
+__global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
+  __shared__ float As[kBK][kBM + 1];
+  __shared__ float Bs[kBK][kBN + 1];
+  const int z = blockIdx.z;
+  const int w = g.slot_worker[z];
+  const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * kBN;
+  const T* A = reinterpret_cast<const T*>(g.a) + (g.a_by_worker ? (int64_t)w : z) * g.a_bstride;
+  const T* B = reinterpret_cast<const T*>(g.b) + (g.b_by_worker ? (int64_t)w : z) * g.b_bstride;
+  const int tid = threadIdx.x;
+  const int tx = tid % (kBN / kTN), ty = tid / (kBN / kTN);
+
+  float acc[kTM][kTN];
+#pragma unroll
+  for (int i = 0; i < kTM; ++i)
+#pragma unroll
+    for (int j = 0; j < kTN; ++j) acc[i][j] = 0.f;
+  float bsum = 0.f;   // bias gradient (kEpi == kEpiDW, first column tile)
+  const bool do_bias = (kEpi == kEpiDW) && blockIdx.x == 0 && tid < kBM;
+
+  for (int64_t k0 = 0; k0 < g.K; k0 += kBK) {
+#pragma unroll
+    for (int r = 0; r < (kBM * kBK) / kThreads; ++r) {
+      const int e = tid + r * kThreads;
+      int mm, kk;
+      if (kAKMajor) { mm = e / kBK; kk = e % kBK; } else { kk = e / kBM; mm = e % kBM; }
+      const int64_t gm = m0 + mm, gk = k0 + kk;
+      float v = 0.f;
+      if (gm < g.M && gk < g.K) v = to_f(kAKMajor ? A[gm * g.lda + gk] : A[gk * g.lda + gm]);
+      As[kk][mm] = v;
+    }
+#pragma unroll
+    for (int r = 0; r < (kBN * kBK) / kThreads; ++r) {
+      const int e = tid + r * kThreads;
+      int nn, kk;
+      if (kBKMajor) { nn = e / kBK; kk = e % kBK; } else { kk = e / kBN; nn = e % kBN; }
+      const int64_t gn = n0 + nn, gk = k0 + kk;
+      float v = 0.f;
+      if (gn < g.N && gk < g.K) v = to_f(kBKMajor ? B[gn * g.ldb + gk] : B[gk * g.ldb + gn]);
+      Bs[kk][nn] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < kBK; ++kk) {
+      float a[kTM], b[kTN];
+#pragma unroll
+      for (int i = 0; i < kTM; ++i) a[i] = As[kk][ty + i * (kBM / kTM)];
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) b[j] = Bs[kk][tx + j * (kBN / kTN)];
+#pragma unroll
+      for (int i = 0; i < kTM; ++i)
+#pragma unroll
+        for (int j = 0; j < kTN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    if (do_bias) {
+#pragma unroll
+      for (int kk = 0; kk < kBK; ++kk) bsum += As[kk][tid];
+    }
+    __syncthreads();
+  }
+
+  // Epilogues.
+  float* theta = g.theta + (int64_t)w * g.ld_param;
+  if (kEpi == kEpiFwd) {
+    const float* bias = theta + g.boff;
+    TO* out = reinterpret_cast<TO*>(g.out) + (int64_t)z * g.out_bstride;
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+      const int64_t m = m0 + ty + i * (kBM / kTM);
+      if (m >= g.M) continue;
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) {
+        const int64_t n = n0 + tx + j * (kBN / kTN);
+        if (n >= g.N) continue;
+        float v = acc[i][j] + bias[n];
+        if (g.relu) v = fmaxf(v, 0.f);
+        out[m * g.ldo + n] = from_f<TO>(v);
+      }
+    }
+  } else if (kEpi == kEpiDX) {
+    const T* mask = reinterpret_cast<const T*>(g.mask) + (int64_t)z * g.mask_bstride;
+    TO* out = reinterpret_cast<TO*>(g.out) + (int64_t)z * g.out_bstride;
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+      const int64_t m = m0 + ty + i * (kBM / kTM);
+      if (m >= g.M) continue;
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) {
+        const int64_t n = n0 + tx + j * (kBN / kTN);
+        if (n >= g.N) continue;
+        const float h = to_f(mask[m * g.ldo + n]);
+        out[m * g.ldo + n] = from_f<TO>(h > 0.f ? acc[i][j] : 0.f);
+      }
+    }
+  } else {   // kEpiDW: theta_k -= eta g, a_k += g, bf16 copy refresh
+    float* a = g.acc + (int64_t)w * g.ld_param;
+    bf16* tb = g.theta_bf16 ? g.theta_bf16 + (int64_t)w * g.ld_param : nullptr;
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+      const int64_t m = m0 + ty + i * (kBM / kTM);
+      if (m >= g.M) continue;
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) {
+        const int64_t n = n0 + tx + j * (kBN / kTN);
+        if (n >= g.N) continue;
+        const int64_t p = g.woff + m * g.N + n;
+        const float gr = acc[i][j];
+        const float t = fmaf(-g.eta, gr, theta[p]);
+        theta[p] = t;
+        a[p] += gr;
+        if (tb) tb[p] = __float2bfloat16_rn(t);
+      }
+    }
+    if (do_bias && m0 + tid < g.M) {
+      const int64_t p = g.boff + m0 + tid;
+      const float t = fmaf(-g.eta, bsum, theta[p]);
+      theta[p] = t;
+      a[p] += bsum;
+      if (tb) tb[p] = __float2bfloat16_rn(t);
+    }
+  }
+}
+
+// Softmax cross-entropy on Z [m][C] (fp32) per slot: dZ = (softmax - onehot)/m,
+// loss = mean_j (logsumexp(z_j) - z_j[y_j]), summed over the block in a fixed
+// order.  One block per slot.
+template <typename T>
+__global__ void __launch_bounds__(128) softmax_xent_kernel(const float* __restrict__ Z,
+                                                           const int* __restrict__ yb, T* dZ,
+                                                           int m, int C, float* loss_parts,
+                                                           const int* slot_commit, int lam,
+                                                           int step, int* flag) {
+  const int z = blockIdx.x;
+  const float* Zs = Z + (int64_t)z * m * C;
+  T* dZs = dZ + (int64_t)z * m * C;
+  const int* ys = yb + (int64_t)z * m;
+  const float inv_m = 1.0f / (float)m;
+  float part = 0.f;
+  for (int j = threadIdx.x; j < m; j += blockDim.x) {
+    const float* zr = Zs + (int64_t)j * C;
+    float mx = zr[0];
+    for (int c = 1; c < C; ++c) mx = fmaxf(mx, zr[c]);
+    float s = 0.f;
+    for (int c = 0; c < C; ++c) s += expf(zr[c] - mx);
+    const int y = ys[j];
+    part += (logf(s) + mx) - zr[y];
+    const float inv_s = 1.0f / s;
+    for (int c = 0; c < C; ++c) {
+      float p = expf(zr[c] - mx) * inv_s;
+      if (c == y) p -= 1.0f;
+      dZs[(int64_t)j * C + c] = from_f<T>(p * inv_m);
+    }
+  }
+  __shared__ float red[128];
+  red[threadIdx.x] = part;
+  __syncthreads();
+  for (int s = 64; s > 0; s >>= 1) {
+    if (threadIdx.x < s) red[threadIdx.x] += red[threadIdx.x + s];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const float loss = red[0] * inv_m;
+    loss_parts[(int64_t)slot_commit[z] * lam + step] = loss;
+    if (!isfinite(loss)) atomicExch(flag, 1);
+  }
+}
+
+// Minibatch gather (FetchNextMiniBatch of Algorithm 1): slot z, row j reads
+// dataset row k S + ((t0 + i) m + j) mod S of worker k = slot_worker[z].
+template <typename T>
+__global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y, T* Xb, int* yb,
+                              int d0, int m, int64_t S, const int* slot_worker,
+                              const long long* slot_t0, int step) {
+  const int z = blockIdx.y, j = blockIdx.x;
+  const int w = slot_worker[z];
+  const long long t = slot_t0[z] + step;
+  const int64_t row = (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
+  const T* src = X + row * d0;
+  T* dst = Xb + ((int64_t)z * m + j) * d0;
+  for (int c = threadIdx.x; c < d0; c += blockDim.x) dst[c] = src[c];
+  if (threadIdx.x == 0) yb[(int64_t)z * m + j] = y[row];
+}
+
+template <typename T, typename TO, bool kAK, bool kBK, int kEpi>
+Status launch_gemm(const GemmArgs& g, int slots, cudaStream_t st) {
+  dim3 grid((unsigned)ceil_div(g.N, kBN), (unsigned)ceil_div(g.M, kBM), (unsigned)slots);
+  gemm_simt_kernel<T, TO, kAK, kBK, kEpi><<<grid, kThreads, 0, st>>>(g);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+}  // namespace
+
+template <typename T>
+Status simt_forward(const GemmArgs& g, bool last, int slots, cudaStream_t st) {
+  if (last) return launch_gemm<T, float, true, true, kEpiFwd>(g, slots, st);
+  return launch_gemm<T, T, true, true, kEpiFwd>(g, slots, st);
+}
+template <typename T>
+Status simt_backward_dx(const GemmArgs& g, int slots, cudaStream_t st) {
+  return launch_gemm<T, T, true, false, kEpiDX>(g, slots, st);
+}
+template <typename T>
+Status simt_backward_dw(const GemmArgs& g, int slots, cudaStream_t st) {
+  return launch_gemm<T, T, false, false, kEpiDW>(g, slots, st);
+}
+template <typename T>
+Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* loss_parts,
+                    const int* slot_commit, int lam, int step, int* flag, int slots,
+                    cudaStream_t st) {
+  softmax_xent_kernel<T><<<slots, 128, 0, st>>>(Z, yb, dZ, m, C, loss_parts, slot_commit, lam,
+                                                step, flag);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+template <typename T>
+Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
+                    const int* slot_worker, const long long* slot_t0, int step, int slots,
+                    cudaStream_t st) {
+  dim3 grid((unsigned)m, (unsigned)slots);
+  gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+#define AGN_INST(T)                                                                          \
+  template Status simt_forward<T>(const GemmArgs&, bool, int, cudaStream_t);                 \
+  template Status simt_backward_dx<T>(const GemmArgs&, int, cudaStream_t);                   \
+  template Status simt_backward_dw<T>(const GemmArgs&, int, cudaStream_t);                   \
+  template Status softmax_xent<T>(const float*, const int*, T*, int, int, float*, const int*, \
+                                  int, int, int*, int, cudaStream_t);                        \
+  template Status gather_batch<T>(const T*, const int*, T*, int*, int, int, int64_t,          \
+                                  const int*, const long long*, int, int, cudaStream_t);
+AGN_INST(float)
+AGN_INST(bf16)
+#undef AGN_INST
+
+}  // namespace agn

@@ -1,0 +1,106 @@
+"""The C ABI without a GPU: the library loads, exports every symbol that
+include/agn.h declares, its host-side generator reproduces agn_inputs bit for
+bit, and invalid arguments are rejected with the documented codes."""
+
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+import agn_inputs as I
+from agn_inputs import workloads as WL
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def agn():
+    import __graft_entry__ as g
+    g.build()
+    import paper_1710_02368_gb300 as agn
+    return agn
+
+
+def _declared_symbols():
+    syms = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            syms |= set(re.findall(r"\b(agn_\w+)\s*\(", text))
+    return syms
+
+
+def test_library_exports_every_declared_symbol(agn):
+    out = subprocess.run(["nm", "-D", "--defined-only", agn.library_path()],
+                         capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (agn_\w+)", out))
+    declared = _declared_symbols()
+    assert declared, "no declarations found"
+    assert declared <= exported, declared - exported
+    from paper_1710_02368_gb300 import _lib
+    assert declared <= set(_lib.SIGNATURES), declared - set(_lib.SIGNATURES)
+    lib = _lib.load()
+    for s in declared:
+        assert hasattr(lib, s)
+
+
+@pytest.mark.parametrize("n,C,lo,hi,seed", [(4, 50, 0, 2, I.DEFAULT_SEED),
+                                             (16, 2000, 0, 15, I.DEFAULT_SEED),
+                                             (32, 300, 31, 31, 5), (3, 100, 1, 7, 99)])
+def test_schedule_matches_python_generator(agn, n, C, lo, hi, seed):
+    w, t = agn.agn_make_schedule(n, C, lo, hi, seed)
+    pw, pt = I.make_schedule(n, C, lo, hi, seed)
+    assert np.array_equal(w, pw) and np.array_equal(t, pt)
+
+
+@pytest.mark.parametrize("w,rows", [
+    (WL.SMALL, (0, 2048)),
+    (WL.MNIST_SHAPED, (3750 * 5 - 7, 300)),
+    (WL.WIDE_BF16, (1562 * 3, 40)),
+    (WL.LARGE_BF16, (99000, 1000)),
+], ids=lambda v: getattr(v, "name", str(v)))
+def test_generated_inputs_match_python_generator(agn, w, rows):
+    row0, nr = rows
+    x, y, th = agn.agn_generate_inputs(w.dims, w.dist, I.DEFAULT_SEED, row0, nr,
+                                       teacher_dims=w.teacher_dims,
+                                       want_theta=(w.dims[1] <= 1000))
+    r = np.arange(row0, row0 + nr)
+    px = I.make_inputs_x(I.DEFAULT_SEED, w.dims[0], r, w.dist)
+    assert np.array_equal(x, px)
+    py = I.teacher_labels(px, I.teacher_params(I.DEFAULT_SEED, w.teacher_dims), w.dist)
+    assert np.array_equal(y, py)
+    if th is not None:
+        assert np.array_equal(th, I.init_params(I.DEFAULT_SEED, w.dims))
+
+
+def test_generate_inputs_rejects_bad_arguments(agn):
+    with pytest.raises(agn.AGNError) as e:
+        agn.agn_generate_inputs([784, 0, 10], 0, 1, 0, 4)
+    assert e.value.code == agn.AGN_E_INVALID
+    with pytest.raises(agn.AGNError) as e:
+        agn.agn_generate_inputs([784, 10], 0, 1, 0, 4, teacher_dims=[700, 10])
+    assert e.value.code == agn.AGN_E_INVALID
+
+
+def test_make_schedule_rejects_bad_arguments(agn):
+    for args in [(0, 10, 0, 0, 1), (4, 10, 3, 2, 1), (4, 10, -1, 2, 1)]:
+        with pytest.raises(agn.AGNError) as e:
+            agn.agn_make_schedule(*args)
+        assert e.value.code == agn.AGN_E_INVALID
+
+
+def test_create_validates_before_touching_the_device(agn):
+    for dims, n, lam, eta in [((784,), 4, 5, 0.1), ((784, 0, 10), 4, 5, 0.1),
+                              ((784, 10), 0, 5, 0.1), ((784, 10), 4, 0, 0.1),
+                              ((784, 10), 4, 5, -1.0), ((784, 10), 300, 5, 0.1)]:
+        with pytest.raises(agn.AGNError) as e:
+            agn.agn_create(dims, n, lam, eta, 1)
+        assert e.value.code == agn.AGN_E_INVALID
+    o = agn.agn_default_options()
+    o.precision = 7
+    with pytest.raises(agn.AGNError) as e:
+        agn.agn_create((8, 4), 2, 1, 0.1, 1, o)
+    assert e.value.code == agn.AGN_E_INVALID
