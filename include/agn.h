@@ -149,6 +149,27 @@ int agn_generate_inputs(const int32_t* dims, int32_t n_dims, int32_t input_dist,
                         const int32_t* teacher_dims, int32_t n_teacher_dims, uint64_t seed,
                         int64_t row0, int64_t n_rows, float* x, int32_t* y, float* theta0);
 
+/*
+ * Per-kernel profiling.  agn_profile(h, 1) makes every later agn_run record a
+ * CUDA event pair around each kernel launch (on the handle's stream) and
+ * accumulate, per kernel class, the launches, the device milliseconds and
+ * the algorithmic flops and DRAM bytes of those launches; agn_profile(h, 0)
+ * stops and agn_profile(h, 2) clears the totals.  agn_kernel_stats writes
+ * AGN_KERNEL_CLASSES rows of 4 doubles {launches, ms, flops, bytes}, row i
+ * for class i below, into out (cap >= 4 * AGN_KERNEL_CLASSES).
+ */
+#define AGN_K_GATHER 0       /* minibatch gather (FetchNextMiniBatch)            */
+#define AGN_K_FORWARD 1      /* forward GEMM + bias + ReLU                       */
+#define AGN_K_SOFTMAX 2      /* softmax cross-entropy                            */
+#define AGN_K_BACKWARD_DX 3  /* dX GEMM + ReLU mask                              */
+#define AGN_K_BACKWARD_DW 4  /* dW GEMM + local step + accumulation              */
+#define AGN_K_COMMIT 5       /* fused commit + pull                              */
+#define AGN_K_NORMS 6        /* per-commit norm reduction                        */
+#define AGN_K_OTHER 7        /* pulls outside commits, loss means                */
+#define AGN_KERNEL_CLASSES 8
+int agn_profile(agn_handle* h, int32_t mode);
+int agn_kernel_stats(const agn_handle* h, double* out, int64_t cap);
+
 /* Copy the generated inputs (host, caller-owned, any may be NULL):
    x [n_samples][d_0] fp32, y [n_samples] int32, theta0 [P] fp32 flat. */
 int agn_export_inputs(agn_handle* h, float* x, int32_t* y, float* theta0);

@@ -22,7 +22,7 @@ from ._lib import (AGN_DIST_NORMAL, AGN_DIST_UNIFORM, AGN_GEMM_AUTO, AGN_GEMM_SI
 __all__ = [
     "AGNError", "AGN", "agn_default_options", "agn_create", "agn_run", "agn_central",
     "agn_replica", "agn_loss", "agn_delta_norm", "agn_num_params", "agn_num_commits",
-    "agn_last_run_stats", "agn_generate_inputs", "agn_export_inputs", "agn_last_error",
+    "agn_last_run_stats", "agn_profile", "agn_kernel_stats", "agn_generate_inputs", "agn_export_inputs", "agn_last_error",
     "agn_destroy", "agn_make_schedule", "agn_commit_pull", "agn_fill_commit_inputs",
     "library_path",
 ]
@@ -133,6 +133,18 @@ def agn_last_run_stats(h) -> dict:
     out = (C.c_double * 4)()
     _check(_L().agn_last_run_stats(h, out, 4), h)
     return {"waves": out[0], "launches": out[1], "gpu_ms": out[2], "worker_steps": out[3]}
+
+
+def agn_profile(h, mode):
+    _check(_L().agn_profile(h, int(mode)), h)
+
+
+def agn_kernel_stats(h) -> dict:
+    n = len(_lib.KERNEL_CLASSES)
+    out = (C.c_double * (4 * n))()
+    _check(_L().agn_kernel_stats(h, out, 4 * n), h)
+    return {name: {"launches": out[4 * i], "ms": out[4 * i + 1], "flops": out[4 * i + 2],
+                   "bytes": out[4 * i + 3]} for i, name in enumerate(_lib.KERNEL_CLASSES)}
 
 
 def agn_generate_inputs(dims, input_dist, seed, row0, n_rows, teacher_dims=None,
@@ -249,6 +261,12 @@ class AGN:
 
     def last_run_stats(self):
         return agn_last_run_stats(self.h)
+
+    def profile(self, mode):
+        agn_profile(self.h, mode)
+
+    def kernel_stats(self):
+        return agn_kernel_stats(self.h)
 
     def export_inputs(self):
         return agn_export_inputs(self.h, self.n_samples, self.dims[0])

@@ -29,6 +29,9 @@ AGN_GEMM_AUTO = 0
 AGN_GEMM_SIMT = 1
 AGN_GEMM_TCGEN05 = 2
 
+KERNEL_CLASSES = ["gather", "forward", "softmax", "backward_dx", "backward_dw", "commit",
+                  "norms", "other"]
+
 ERROR_NAMES = {
     AGN_E_INVALID: "AGN_E_INVALID", AGN_E_SCHEDULE: "AGN_E_SCHEDULE", AGN_E_OOM: "AGN_E_OOM",
     AGN_E_CUDA: "AGN_E_CUDA", AGN_E_TIMEOUT: "AGN_E_TIMEOUT",
@@ -75,6 +78,8 @@ SIGNATURES = {
     "agn_generate_inputs": (C.c_int, [_I32P, C.c_int32, C.c_int32, _I32P, C.c_int32, C.c_uint64,
                                       C.c_int64, C.c_int64, _F32P, _I32P, _F32P]),
     "agn_export_inputs": (C.c_int, [C.c_void_p, _F32P, _I32P, _F32P]),
+    "agn_profile": (C.c_int, [C.c_void_p, C.c_int32]),
+    "agn_kernel_stats": (C.c_int, [C.c_void_p, _F64P, C.c_int64]),
     "agn_last_error": (C.c_char_p, [C.c_void_p]),
     "agn_destroy": (None, [C.c_void_p]),
     "agn_make_schedule": (C.c_int, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_uint64,

@@ -101,6 +101,17 @@ struct agn_handle {
   std::vector<int64_t> prev, pulled_v, steps;     // per worker
   std::string err;
   double stats[4] = {0, 0, 0, 0};
+  // per-kernel profiling (agn_profile)
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  struct Pending {
+    int cls;
+    size_t e0;
+    double flops, bytes;
+  };
+  std::vector<Pending> pend;
+  double kstats[AGN_KERNEL_CLASSES][4] = {};
 };
 
 namespace {
@@ -158,6 +169,57 @@ Status grow(agn_handle* h, Tp** p, int64_t* cap, int64_t need, int64_t keep) {
 
 size_t elem_size(const agn_handle* h) { return h->prec == AGN_PREC_BF16 ? 2 : 4; }
 
+// CUDA events around one launch when profiling is on; always counts it.
+class Launch {
+ public:
+  Launch(agn_handle* h, int cls, double flops, double bytes, int64_t* counter)
+      : h_(h), cls_(cls), flops_(flops), bytes_(bytes) {
+    ++*counter;
+    if (h_->prof) {
+      e0_ = next();
+      if (e0_ != kNone) cudaEventRecord(h_->ev_pool[e0_], h_->stream);
+    }
+  }
+  ~Launch() {
+    if (h_->prof && e0_ != kNone) {
+      size_t e1 = next();
+      if (e1 == kNone) return;
+      cudaEventRecord(h_->ev_pool[e1], h_->stream);
+      h_->pend.push_back({cls_, e0_, flops_, bytes_});
+    }
+  }
+
+ private:
+  static constexpr size_t kNone = ~size_t(0);
+  size_t next() {
+    if (h_->ev_used == h_->ev_pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return kNone;
+      h_->ev_pool.push_back(e);
+    }
+    return h_->ev_used++;
+  }
+  agn_handle* h_;
+  int cls_;
+  double flops_, bytes_;
+  size_t e0_ = kNone;
+};
+
+// After the stream has drained: fold the recorded event pairs into kstats.
+void collect_profile(agn_handle* h) {
+  for (const auto& p : h->pend) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, h->ev_pool[p.e0], h->ev_pool[p.e0 + 1]) == cudaSuccess) {
+      h->kstats[p.cls][0] += 1;
+      h->kstats[p.cls][1] += ms;
+      h->kstats[p.cls][2] += p.flops;
+      h->kstats[p.cls][3] += p.bytes;
+    }
+  }
+  h->pend.clear();
+  h->ev_used = 0;
+}
+
 // ---------------------------------------------------------------------------
 // One wave: lambda local steps of every slot (Algorithm 1's inner loop)
 // ---------------------------------------------------------------------------
@@ -172,10 +234,14 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   const T* W = h->prec == AGN_PREC_BF16 ? reinterpret_cast<const T*>(h->rep_b)
                                          : reinterpret_cast<const T*>(h->rep);
   const float eta = (float)h->eta;
+  const double es = (double)sizeof(T);
+  const double upd = h->prec == AGN_PREC_BF16 ? 18.0 : 16.0;   // theta RMW + a RMW (+ bf16 copy)
   for (int i = 0; i < h->lam; ++i) {
-    AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb), h->yb,
-                                 h->dims[0], m, h->S, sw, st0, i, s, h->stream));
-    ++*launches;
+    {
+      Launch k(h, AGN_K_GATHER, 0.0, (double)s * m * (2.0 * h->dims[0] * es + 8.0), launches);
+      AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb),
+                                   h->yb, h->dims[0], m, h->S, sw, st0, i, s, h->stream));
+    }
     // forward, l = 1..L
     for (int l = 1; l <= L; ++l) {
       agn::GemmArgs g{};
@@ -188,12 +254,17 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       g.ldo = fo; g.out_bstride = (int64_t)m * fo;
       g.relu = l < L;
       g.theta = h->rep; g.ld_param = h->P_pad; g.boff = h->boff[l - 1];
+      const double oes = l == L ? 4.0 : es;
+      Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
+               (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es + (double)m * fo * oes),
+               launches);
       AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
-      ++*launches;
     }
-    AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dz[0]), m, h->dims[L],
-                                 h->loss_parts, sc, h->lam, i, h->flag, s, h->stream));
-    ++*launches;
+    {
+      Launch k(h, AGN_K_SOFTMAX, 0.0, (double)s * m * (h->dims[L] * (4.0 + es) + 4.0), launches);
+      AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dz[0]), m, h->dims[L],
+                                   h->loss_parts, sc, h->lam, i, h->flag, s, h->stream));
+    }
     // backward, l = L..1: dX (reads W_l before its update), then dW + update
     int cur = 0;
     for (int l = L; l >= 1; --l) {
@@ -208,8 +279,10 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         g.out = h->dz[1 - cur]; g.ldo = fi; g.out_bstride = (int64_t)m * fi;
         g.mask = Hprev; g.mask_bstride = (int64_t)m * fi;
         g.theta = h->rep; g.ld_param = h->P_pad;
+        Launch k(h, AGN_K_BACKWARD_DX, 2.0 * s * m * fo * fi,
+                 (double)s * ((double)fo * fi * es + (double)m * fo * es + 2.0 * m * fi * es),
+                 launches);
         AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
-        ++*launches;
       }
       agn::GemmArgs g{};
       g.M = fo; g.N = fi; g.K = m;
@@ -218,8 +291,12 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       g.slot_worker = sw;
       g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
       g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
-      AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
-      ++*launches;
+      {
+        Launch k(h, AGN_K_BACKWARD_DW, 2.0 * s * m * fo * fi,
+                 (double)s * (((double)fo * fi + fo) * upd + (double)m * fo * es + (double)m * fi * es),
+                 launches);
+        AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+      }
       cur = 1 - cur;
     }
   }
@@ -393,29 +470,40 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, plan.start_pulls.data(),
                                  plan.start_pulls.size() * sizeof(int), cudaMemcpyHostToDevice,
                                  h->stream));
+    Launch k(h, AGN_K_OTHER, 0.0,
+             (double)h->P * (4.0 + plan.start_pulls.size() * (h->rep_b ? 6.0 : 4.0)), &launches);
     AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
                                (int)plan.start_pulls.size(), h->stream));
-    ++launches;
   }
   const float scale = (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
   for (const Wave& wv : plan.waves) {
     if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
     else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
     for (const CommitPlan& cp : wv.commits) {
-      AGN_TRY(agn::launch_commit_pull(cp, h->theta_c, h->acc, h->rep, h->rep_b, h->P_pad,
-                                      h->P_pad, scale, true, h->partials, h->grid, h->dnorm,
-                                      h->flag, h->stream));
-      launches += 2;
+      const double pulls = cp.pull_begin[cp.n_commits];
+      {
+        Launch kc(h, AGN_K_COMMIT, 2.0 * cp.n_commits * h->P,
+                  (double)h->P * (8.0 + 8.0 * cp.n_commits + pulls * (h->rep_b ? 6.0 : 4.0)),
+                  &launches);
+        AGN_TRY(agn::launch_commit_pull(cp, h->theta_c, h->acc, h->rep, h->rep_b, h->P_pad,
+                                        h->P_pad, scale, true, h->partials, h->grid, nullptr,
+                                        nullptr, h->stream, /*norms=*/false));
+      }
+      Launch kn(h, AGN_K_NORMS, 0.0, 8.0 * cp.n_commits * h->grid, &launches);
+      AGN_TRY(agn::launch_commit_norms(cp, h->partials, h->grid, h->dnorm, h->flag, h->stream));
     }
   }
-  AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, k, h->loss + V0, h->stream));
-  ++launches;
+  {
+    Launch kl(h, AGN_K_OTHER, 0.0, 4.0 * k * (h->lam + 1), &launches);
+    AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, k, h->loss + V0, h->stream));
+  }
   AGN_TRY_CUDA(cudaEventRecord(h->ev1, h->stream));
   int flag = 0;
   AGN_TRY_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, h->stream));
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
   float ms = 0.f;
   cudaEventElapsedTime(&ms, h->ev0, h->ev1);
+  if (h->prof) collect_profile(h);
   h->stats[0] = (double)plan.waves.size();
   h->stats[1] = (double)launches;
   h->stats[2] = ms;
@@ -833,6 +921,22 @@ int agn_export_inputs(agn_handle* h, float* x, int32_t* y, float* theta0) {
   return AGN_OK;
 }
 
+int agn_profile(agn_handle* h, int32_t mode) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  if (mode == 0) h->prof = false;
+  else if (mode == 1) h->prof = true;
+  else if (mode == 2) std::memset(h->kstats, 0, sizeof(h->kstats));
+  else return fail(h, AGN_E_INVALID, "mode must be 0, 1 or 2");
+  return AGN_OK;
+}
+
+int agn_kernel_stats(const agn_handle* h, double* out, int64_t cap) {
+  if (!h || !out || cap < 4 * AGN_KERNEL_CLASSES)
+    return fail(const_cast<agn_handle*>(h), AGN_E_INVALID, "need 4 * AGN_KERNEL_CLASSES slots");
+  std::memcpy(out, h->kstats, sizeof(h->kstats));
+  return AGN_OK;
+}
+
 const char* agn_last_error(const agn_handle* h) { return h ? h->err.c_str() : g_error.c_str(); }
 
 void agn_destroy(agn_handle* h) {
@@ -841,6 +945,7 @@ void agn_destroy(agn_handle* h) {
   if (h->stream) cudaStreamSynchronize(h->stream);
   for (void* p : h->allocs)
     if (p) cudaFree(p);
+  for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
   if (h->ev0) cudaEventDestroy(h->ev0);
   if (h->ev1) cudaEventDestroy(h->ev1);
   if (h->own_stream && h->stream) cudaStreamDestroy(h->stream);

@@ -186,7 +186,7 @@ int commit_grid(int64_t P) {
 Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale, bool zero_acc,
                           double* partials, int grid, float* delta_norm, int* flag,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, bool norms) {
   if (plan.n_commits <= 0) return Status::Ok();
   if (replicas_bf16)
     commit_pull_kernel<true><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
@@ -197,11 +197,17 @@ Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, fl
                                                               nullptr, P, ld, scale,
                                                               zero_acc ? 1 : 0, partials);
   AGN_TRY_CUDA(cudaGetLastError());
-  if (partials && (delta_norm || flag)) {
-    reduce_norms_kernel<<<plan.n_commits, kThreads, 0, stream>>>(partials, grid, plan, delta_norm,
-                                                                 flag);
-    AGN_TRY_CUDA(cudaGetLastError());
-  }
+  if (norms && partials && (delta_norm || flag))
+    return launch_commit_norms(plan, partials, grid, delta_norm, flag, stream);
+  return Status::Ok();
+}
+
+Status launch_commit_norms(const CommitPlan& plan, const double* partials, int grid,
+                           float* delta_norm, int* flag, cudaStream_t stream) {
+  if (plan.n_commits <= 0) return Status::Ok();
+  reduce_norms_kernel<<<plan.n_commits, kThreads, 0, stream>>>(partials, grid, plan, delta_norm,
+                                                               flag);
+  AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
 

@@ -70,7 +70,11 @@ struct CommitPlan {
 Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale,
                           bool zero_acc, double* partials, int grid, float* delta_norm,
-                          int* flag, cudaStream_t stream);
+                          int* flag, cudaStream_t stream, bool norms = true);
+// The per-commit norm reduction of one launch of launch_commit_pull (when
+// that launch was queued with norms = false).
+Status launch_commit_norms(const CommitPlan& plan, const double* partials, int grid,
+                           float* delta_norm, int* flag, cudaStream_t stream);
 
 // Grid size used by the commit kernel for P parameters (a multiple of the SM
 // count, capped by the work).
