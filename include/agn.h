@@ -214,6 +214,36 @@ int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_
                     int32_t normalize, float* delta_norm, void* stream);
 
 /*
+ * agn_commit_pull_noalloc: agn_commit_pull for callers that may not allocate
+ * device memory.  The paper has no counterpart; it is a deployment variant.
+ * Some callers cannot call cudaMalloc on this path: a host framework that
+ * owns all device memory through its own pool and forbids allocations
+ * outside it, or a latency-bound loop where an allocation, which can
+ * synchronise the device or fail under memory pressure, is not allowed.
+ * Same arguments, same kernels and bit-identical results as agn_commit_pull
+ * (theta~, accumulators, replicas, and the norms, which are reduced in the
+ * same fixed order).  It allocates nothing: its scratch (the per-block
+ * partial sums of the norms) is a fixed array of 16 x 1024 doubles
+ * (128 KiB) in device global memory that every GPU loading the library holds
+ * until the process exits.
+ *   - Limit: each commit may have at most 256 pulls (more gives
+ *     AGN_E_INVALID with a message saying so); P, C and n are otherwise free.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture.
+ *   - Every call shares the one array, which keeps the last call's contents
+ *     (nothing in it needs to start at zero).  Calls that overlap on the GPU
+ *     (other streams, other host threads) race on it and give wrong norms:
+ *     order them on one stream or with events.
+ * Errors: AGN_E_INVALID, AGN_E_CUDA, AGN_E_UNSUPPORTED (device ordinal > 63).
+ */
+int agn_commit_pull_noalloc(float* theta_c, float* acc, float* replicas, void* replicas_bf16,
+                            int64_t P, int64_t ld, int32_t n, int32_t C,
+                            const int32_t* commit_worker, const int32_t* pull_offsets,
+                            const int32_t* pull_workers, double eta, int32_t lambda,
+                            int32_t normalize, float* delta_norm, void* stream);
+
+/*
  * Fill the inputs of the standalone commit workload on the device with the
  * seeded generator: theta_c[i] = fp32(N(0,1) number i of the commit-theta
  * stream); acc[k][i] = fp32(0.1 * N(0,1) number k*P + i of the commit-acc

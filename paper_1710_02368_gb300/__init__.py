@@ -23,7 +23,8 @@ __all__ = [
     "AGNError", "AGN", "agn_default_options", "agn_create", "agn_run", "agn_central",
     "agn_replica", "agn_loss", "agn_delta_norm", "agn_num_params", "agn_num_commits",
     "agn_last_run_stats", "agn_profile", "agn_kernel_stats", "agn_generate_inputs", "agn_export_inputs", "agn_last_error",
-    "agn_destroy", "agn_make_schedule", "agn_commit_pull", "agn_fill_commit_inputs",
+    "agn_destroy", "agn_make_schedule", "agn_commit_pull", "agn_commit_pull_noalloc",
+    "agn_fill_commit_inputs",
     "library_path",
 ]
 
@@ -200,6 +201,20 @@ def agn_commit_pull(theta_c, acc, replicas, replicas_bf16, P, ld, n, commit_work
     _check(_L().agn_commit_pull(_ptr(theta_c), _ptr(acc), _ptr(replicas), _ptr(replicas_bf16),
                                 int(P), int(ld), int(n), len(cw), cwp, pop, pwp, float(eta),
                                 int(lam), int(normalize), _ptr(delta_norm), _ptr(stream)))
+
+
+def agn_commit_pull_noalloc(theta_c, acc, replicas, replicas_bf16, P, ld, n, commit_worker,
+                            pull_offsets, pull_workers, eta, lam, normalize=1, delta_norm=None,
+                            stream=None):
+    """agn_commit_pull without any device allocation (scratch in a fixed
+    device array); for callers that may not allocate on this path."""
+    cw, cwp = _i32(commit_worker)
+    po, pop = _i32(pull_offsets)
+    pw, pwp = _i32(pull_workers if len(pull_workers) else [0])
+    _check(_L().agn_commit_pull_noalloc(
+        _ptr(theta_c), _ptr(acc), _ptr(replicas), _ptr(replicas_bf16), int(P), int(ld), int(n),
+        len(cw), cwp, pop, pwp, float(eta), int(lam), int(normalize), _ptr(delta_norm),
+        _ptr(stream)))
 
 
 def agn_fill_commit_inputs(theta_c, acc, replicas, P, ld, n, seed, stream=None):

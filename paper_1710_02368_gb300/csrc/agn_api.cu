@@ -980,3 +980,8 @@ int agn_fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t 
 }
 
 }  // extern "C"
+
+namespace agn {
+// Message returned by agn_last_error(NULL) for entry points defined in other files.
+void set_global_error(const std::string& msg) { g_error = msg; }
+}  // namespace agn
