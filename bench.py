@@ -33,7 +33,9 @@ from agn_inputs import workloads as WL  # noqa: E402
 
 METRIC = "worker-samples/s (fwd+bwd+AGN commit) on 1 GB300; % tensor-pipe peak; commit HBM GB/s"
 UNIT = "worker-samples/s"
-COMMITS_PER_STEP = 100
+# commits per step: whole waves where the schedule allows (n or 2n commits)
+COMMITS_PER_STEP = {"mnist": 100, "small": 50, "wide": 64, "large": 128}
+GEMMS = {"auto": 0, "simt": 1, "tcgen05": 2}
 WORKLOADS = {"mnist": WL.MNIST_SHAPED, "small": WL.SMALL, "wide": WL.WIDE_BF16,
              "large": WL.LARGE_BF16}
 # FP32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flop x 2.07 GHz.
@@ -238,12 +240,13 @@ def run_agn(args, wl):
     dev = torch.device("cuda", local)
     st = torch.cuda.current_stream()
     seed = I.DEFAULT_SEED
-    per_step = args.commits_per_step
+    per_step = args.commits_per_step or (
+        COMMITS_PER_STEP[args.workload] if not args.workers else 2 * wl.n)
     total = (args.warmup + 2 * args.steps) * per_step + wl.n
     w, tau = agn.agn_make_schedule(wl.n, total, wl.tau_lo, wl.tau_hi, seed)
     h = agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, seed, precision=wl.precision, batch=wl.batch,
                 n_samples=wl.n_samples, input_dist=wl.dist, teacher_dims=wl.teacher_dims,
-                normalize=wl.normalize, gemm=agn.AGN_GEMM_SIMT, stream=st.cuda_stream)
+                normalize=wl.normalize, gemm=GEMMS[args.gemm], stream=st.cuda_stream)
 
     def barrier():
         if ws > 1:
@@ -275,6 +278,8 @@ def run_agn(args, wl):
     h.profile(0)
     ms = e0.elapsed_time(e1)
     kst = h.kernel_stats()
+    gemm_used = ("tcgen05 (hidden layers) + simt (output layer)"
+                 if wl.precision == WL.PREC_BF16 and args.gemm != "simt" else "simt")
     # timed region 2: end to end through the public API with host buffers
     barrier()
     t0 = time.perf_counter()
@@ -307,8 +312,17 @@ def run_agn(args, wl):
                     "peak": FP32_FMA_PEAK_TFLOPS, "unit": "TFLOP/s",
                     "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
         else:
-            roof = {"bound": "tensor", "achieved": d["flops"] / d["ms"] / 1e9, "peak": bf16,
-                    "unit": "TFLOP/s", "peak_source": f"{peak_src} bf16 burst"}
+            # bf16 GEMMs: the bound is set by the arithmetic intensity against
+            # the ridge point of the measured peaks (bf16 TFLOP/s / HBM GB/s)
+            ai = d["flops"] / max(d["bytes"], 1.0)
+            if ai >= bf16 * 1e12 / (hbm * 1e9):
+                roof = {"bound": "tensor", "achieved": d["flops"] / d["ms"] / 1e9, "peak": bf16,
+                        "unit": "TFLOP/s", "peak_source": f"{peak_src} bf16 burst"}
+            else:
+                roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
+                        "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
+            roof["tensor_pipe_frac_of_bf16_peak"] = d["flops"] / d["ms"] / 1e9 / bf16
+            roof["arithmetic_intensity_flop_per_byte"] = ai
     else:
         roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
                 "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
@@ -336,7 +350,9 @@ def run_agn(args, wl):
         "config": {"workload": wl.name, "commits_per_step": per_step,
                    "parallelism": "replicas" if ws > 1 else "single GPU",
                    "l2": "inputs larger than L2 (dataset 188 MB + replicas and accumulators "
-                         "230 MB vs 129 MB L2)", "gemm": "simt"},
+                         "230 MB vs 129 MB L2)" if args.workload == "mnist" else
+                         "inputs larger than L2 (replicas and accumulators of all workers)",
+                   "gemm": gemm_used},
         "roofline": roof,
         "kernels": kernels,
         "commit_pull_kernel": commit,
@@ -361,13 +377,24 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="agn", choices=["agn", "reference"])
     ap.add_argument("--workload", default="mnist", choices=sorted(WORKLOADS))
-    ap.add_argument("--commits-per-step", type=int, default=COMMITS_PER_STEP)
+    ap.add_argument("--commits-per-step", type=int, default=0)
+    ap.add_argument("--gemm", default="auto", choices=sorted(GEMMS))
+    ap.add_argument("--workers", type=int, default=0,
+                    help="override n (profiling captures of a smaller case)")
     ap.add_argument("--ref-commits", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-commit-bench", action="store_true")
     args = ap.parse_args()
     wl = WORKLOADS[args.workload]
+    if args.workers:
+        # a smaller copy of the workload (fewer workers, same shapes), for
+        # profiler captures that must stay small; not a benchmark line
+        import dataclasses
+        wl = dataclasses.replace(wl, name=f"{wl.name}-workers{args.workers}", n=args.workers,
+                                 n_samples=wl.shard * args.workers,
+                                 tau_lo=min(wl.tau_lo, args.workers - 1),
+                                 tau_hi=min(wl.tau_hi, args.workers - 1))
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_agn(args, wl)

@@ -52,9 +52,13 @@ extern "C" {
 #define AGN_DIST_UNIFORM 0     /* x ~ U[0,1)^d0 */
 #define AGN_DIST_NORMAL 1      /* x ~ N(0,1)^d0 */
 
-#define AGN_GEMM_AUTO 0        /* tensor cores where the build has them     */
-#define AGN_GEMM_SIMT 1        /* CUDA-core GEMM kernels                     */
-#define AGN_GEMM_TCGEN05 2     /* tcgen05/TMEM GEMM kernels (bf16 mode)      */
+#define AGN_GEMM_AUTO 0        /* tcgen05 where eligible, else CUDA cores   */
+#define AGN_GEMM_SIMT 1        /* CUDA-core GEMM kernels only                */
+#define AGN_GEMM_TCGEN05 2     /* tcgen05/TMEM GEMMs for the hidden layers;
+                                  needs bf16 mode, batch <= 256 and d_0 ..
+                                  d_{L-1} multiples of 8 (else
+                                  AGN_E_UNSUPPORTED); the d_L-wide output
+                                  layer always runs on CUDA cores          */
 
 typedef struct agn_handle agn_handle;
 
@@ -80,6 +84,9 @@ typedef struct agn_options {
   const float* x_init;
   const int32_t* y_init;
   const float* theta_init;
+  /* Diagnostic: which hidden-layer GEMMs use the tcgen05 kernels when they
+     are on (bit 0 forward, bit 1 dX, bit 2 dW); 0 = all. */
+  int32_t tc_mask;
 } agn_options;
 
 void agn_default_options(agn_options* opt);
@@ -113,7 +120,8 @@ int agn_create(const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t l
  * Cumulative: repeated calls continue the commit index and the step counters.
  * Queues the work on the handle's stream and waits for it.
  * Errors: AGN_E_INVALID, AGN_E_SCHEDULE (nothing run), AGN_E_CUDA,
- * AGN_E_NONFINITE (run completed; results readable).
+ * AGN_E_NONFINITE (run completed; results readable), AGN_E_TIMEOUT (a
+ * tensor-core kernel gave up on a bounded wait; results are not valid).
  */
 int agn_run(agn_handle* h, int32_t n_commits, const int32_t* worker,
             const int32_t* staleness, int32_t n_schedule);

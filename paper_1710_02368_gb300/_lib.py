@@ -55,6 +55,7 @@ class agn_options(C.Structure):
         ("x_init", C.POINTER(C.c_float)),
         ("y_init", C.POINTER(C.c_int32)),
         ("theta_init", C.POINTER(C.c_float)),
+        ("tc_mask", C.c_int32),
     ]
 
 

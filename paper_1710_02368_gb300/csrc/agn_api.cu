@@ -20,6 +20,7 @@
 
 #include "host_inputs.h"
 #include "mlp.cuh"
+#include "mlp_tc.cuh"
 
 using agn::bf16;
 using agn::CommitPlan;
@@ -81,8 +82,15 @@ struct agn_handle {
   std::vector<void*> H;       // H[l] [n][m][d_l] T, l = 1..L-1 (H[0] = Xb)
   float* Z = nullptr;         // [n][m][d_L]
   void* dz[2] = {nullptr, nullptr};   // [n][m][maxd] T
-  int* flag = nullptr;
+  int* flag = nullptr;        // [0] non-finite loss or commit, [1] bounded wait gave up
   double* partials = nullptr;
+  // tcgen05 path (bf16 mode): tensor maps per layer l = 1..L-1 (index l-1)
+  bool use_tc = false;
+  int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW
+  struct LayerMaps {
+    CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
+  };
+  std::vector<LayerMaps> tmaps;
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
   float* dnorm = nullptr;     // [cap_commits]
@@ -220,6 +228,41 @@ void collect_profile(agn_handle* h) {
   h->ev_used = 0;
 }
 
+// Layer l (1-based) runs on the tensor cores: bf16 mode, a hidden layer.
+bool tc_layer(const agn_handle* h, int l) { return h->use_tc && l < h->L; }
+
+agn::TcArgs tc_args(agn_handle* h, const int* sw) {
+  agn::TcArgs t{};
+  t.slot_worker = sw;
+  t.err = h->flag + 1;
+  t.theta = h->rep;
+  t.acc = h->acc;
+  t.theta_b = h->rep_b;
+  t.ld_param = h->P_pad;
+  return t;
+}
+
+// Tensor maps of the tcgen05 path (addresses are fixed for the handle's life).
+Status build_tc_maps(agn_handle* h) {
+  const int n = h->n, m = h->m, L = h->L;
+  const uint32_t bn = (uint32_t)agn::tc_bn(m);
+  h->tmaps.assign(L - 1, {});
+  for (int l = 1; l < L; ++l) {
+    const uint64_t fi = h->dims[l - 1], fo = h->dims[l];
+    auto& mp = h->tmaps[l - 1];
+    const bf16* W = h->rep_b + h->woff[l - 1];
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, 64, 128));
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 64, 64));
+    const void* Hin = l == 1 ? h->Xb : h->H[l - 1];
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, bn));
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_mn, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
+    const void* dZ = h->dz[(L - l) % 2];   // dZ_l: dz[0] for l = L, alternating downwards
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
+  }
+  return Status::Ok();
+}
+
 // ---------------------------------------------------------------------------
 // One wave: lambda local steps of every slot (Algorithm 1's inner loop)
 // ---------------------------------------------------------------------------
@@ -258,6 +301,16 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
                (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es + (double)m * fo * oes),
                launches);
+      if (tc_layer(h, l) && (h->tc_mask & 1)) {
+        agn::TcArgs t = tc_args(h, sw);
+        t.M = fo; t.N = m; t.K = fi;
+        t.a_by_worker = 1;
+        t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
+        t.relu = 1; t.boff = h->boff[l - 1];
+        const auto& mp = h->tmaps[l - 1];
+        AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream));
+        continue;
+      }
       AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
     }
     {
@@ -282,7 +335,17 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         Launch k(h, AGN_K_BACKWARD_DX, 2.0 * s * m * fo * fi,
                  (double)s * ((double)fo * fi * es + (double)m * fo * es + 2.0 * m * fi * es),
                  launches);
-        AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
+        if (tc_layer(h, l) && (h->tc_mask & 2)) {
+          agn::TcArgs t = tc_args(h, sw);
+          t.M = fi; t.N = m; t.K = fo;
+          t.a_by_worker = 1;
+          t.out = h->dz[1 - cur]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
+          t.mask = static_cast<const bf16*>(Hprev); t.mask_bstride = (int64_t)m * fi;
+          const auto& mp = h->tmaps[l - 1];
+          AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream));
+        } else {
+          AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
+        }
       }
       agn::GemmArgs g{};
       g.M = fo; g.N = fi; g.K = m;
@@ -295,7 +358,18 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         Launch k(h, AGN_K_BACKWARD_DW, 2.0 * s * m * fo * fi,
                  (double)s * (((double)fo * fi + fo) * upd + (double)m * fo * es + (double)m * fi * es),
                  launches);
-        AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+        if (tc_layer(h, l) && (h->tc_mask & 4)) {
+          agn::TcArgs t = tc_args(h, sw);
+          t.M = fi; t.N = fo; t.K = m;
+          t.woff = h->woff[l - 1]; t.eta = eta;
+          const auto& mp = h->tmaps[l - 1];
+          AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, t, s, h->stream));
+          AGN_TRY(agn::bias_update(static_cast<const bf16*>(h->dz[cur]), m, fo, (int64_t)m * fo, sw,
+                                   h->rep, h->acc, h->rep_b, h->P_pad, h->boff[l - 1], eta, s,
+                                   h->stream));
+        } else {
+          AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+        }
       }
       cur = 1 - cur;
     }
@@ -498,8 +572,8 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, k, h->loss + V0, h->stream));
   }
   AGN_TRY_CUDA(cudaEventRecord(h->ev1, h->stream));
-  int flag = 0;
-  AGN_TRY_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, h->stream));
+  int flags[2] = {0, 0};
+  AGN_TRY_CUDA(cudaMemcpyAsync(flags, h->flag, 2 * sizeof(int), cudaMemcpyDeviceToHost, h->stream));
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
   float ms = 0.f;
   cudaEventElapsedTime(&ms, h->ev0, h->ev1);
@@ -512,9 +586,11 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   h->prev = plan.prev;
   h->pulled_v = plan.pulled_v;
   h->steps = plan.steps;
-  if (flag) {
-    AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), h->stream));
+  if (flags[0] || flags[1]) {
+    AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
     AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+    if (flags[1])
+      return Status::Err(AGN_E_TIMEOUT, "a tensor-core GEMM gave up on a bounded wait");
     return Status::Err(AGN_E_NONFINITE, "a loss or a commit was not finite");
   }
   return Status::Ok();
@@ -538,8 +614,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.gemm == AGN_GEMM_TCGEN05)
-    return Status::Err(AGN_E_UNSUPPORTED, "tcgen05 GEMM backend not built in this library");
+  if (o.tc_mask < 0 || o.tc_mask > 7) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 7]");
   h->dims.assign(dims, dims + n_dims);
   h->L = n_dims - 1;
   h->n = n_workers;
@@ -581,6 +656,15 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   }
   h->P = off;
   h->P_pad = round_up(offp, 64);
+  // tcgen05 path: bf16 mode, m <= 256, every TMA row 16-byte aligned
+  bool tc_ok = h->prec == AGN_PREC_BF16 && h->m <= 256 && h->L >= 2;
+  for (int l = 0; l < h->L; ++l) tc_ok = tc_ok && dims[l] % 8 == 0;
+  if (o.gemm == AGN_GEMM_TCGEN05 && !tc_ok)
+    return Status::Err(AGN_E_UNSUPPORTED,
+                       "tcgen05 GEMMs need bf16 mode, batch <= 256, at least one hidden layer "
+                       "and d_0 .. d_{L-1} multiples of 8");
+  h->use_tc = tc_ok && o.gemm != AGN_GEMM_SIMT;
+  h->tc_mask = o.tc_mask == 0 ? 7 : o.tc_mask;
   h->prev.assign(h->n, -1);
   h->pulled_v.assign(h->n, 0);
   h->steps.assign(h->n, 0);
@@ -629,7 +713,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY(dalloc_t(h, &h->Z, (size_t)(n * m * dims[h->L])));
   AGN_TRY(dalloc(h, &h->dz[0], (size_t)(n * m * h->maxd) * es));
   AGN_TRY(dalloc(h, &h->dz[1], (size_t)(n * m * h->maxd) * es));
-  AGN_TRY(dalloc_t(h, &h->flag, 1));
+  AGN_TRY(dalloc_t(h, &h->flag, 2));
   h->grid = agn::commit_grid(h->P_pad);
   AGN_TRY(dalloc_t(h, &h->partials, (size_t)agn::kMaxCommitsPerLaunch * h->grid));
   AGN_TRY(dalloc_t(h, &h->pull_list, (size_t)n));
@@ -657,7 +741,8 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY_CUDA(cudaMemcpy(h->y, h->hy.data(), h->hy.size() * sizeof(int32_t),
                           cudaMemcpyHostToDevice));
   AGN_TRY_CUDA(cudaMemsetAsync(h->acc, 0, (size_t)(n * h->P_pad) * sizeof(float), h->stream));
-  AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), h->stream));
+  AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
+  if (h->use_tc) AGN_TRY(build_tc_maps(h));
   std::vector<int> all(n);
   for (int w = 0; w < n; ++w) all[w] = w;
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,

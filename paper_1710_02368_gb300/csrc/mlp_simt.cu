@@ -128,6 +128,23 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
   } else {   // kEpiDW: theta_k -= eta g, a_k += g, bf16 copy refresh
     float* a = g.acc + (int64_t)w * g.ld_param;
     bf16* tb = g.theta_bf16 ? g.theta_bf16 + (int64_t)w * g.ld_param : nullptr;
+    // loads of all 16 outputs first, then the updates (memory-level parallelism)
+    const float* __restrict__ th_in = theta;
+    const float* __restrict__ a_in = a;
+    float th[kTM][kTN], av[kTM][kTN];
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+      const int64_t m = m0 + ty + i * (kBM / kTM);
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) {
+        const int64_t n = n0 + tx + j * (kBN / kTN);
+        if (m < g.M && n < g.N) {
+          const int64_t p = g.woff + m * g.N + n;
+          th[i][j] = __ldcs(th_in + p);
+          av[i][j] = __ldcs(a_in + p);
+        }
+      }
+    }
 #pragma unroll
     for (int i = 0; i < kTM; ++i) {
       const int64_t m = m0 + ty + i * (kBM / kTM);
@@ -138,9 +155,9 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         if (n >= g.N) continue;
         const int64_t p = g.woff + m * g.N + n;
         const float gr = acc[i][j];
-        const float t = fmaf(-g.eta, gr, theta[p]);
+        const float t = fmaf(-g.eta, gr, th[i][j]);
         theta[p] = t;
-        a[p] += gr;
+        a[p] = av[i][j] + gr;
         if (tb) tb[p] = __float2bfloat16_rn(t);
       }
     }
