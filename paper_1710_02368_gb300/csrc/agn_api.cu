@@ -91,6 +91,12 @@ struct agn_handle {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
   };
   std::vector<LayerMaps> tmaps;
+  // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
+  bool split = false;
+  int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
+  std::vector<bf16*> Hs;          // pieces of H_l, l = 0..L-2: [3][n][m][d_l]
+  bf16* dZs = nullptr;            // pieces of the current dZ_l: [3][n][m][maxd]
+  int64_t dzs_plane = 0;
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
   float* dnorm = nullptr;     // [cap_commits]
@@ -239,6 +245,7 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.acc = h->acc;
   t.theta_b = h->rep_b;
   t.ld_param = h->P_pad;
+  t.piece_plane = h->piece_plane;
   return t;
 }
 
@@ -250,6 +257,20 @@ Status build_tc_maps(agn_handle* h) {
   for (int l = 1; l < L; ++l) {
     const uint64_t fi = h->dims[l - 1], fo = h->dims[l];
     auto& mp = h->tmaps[l - 1];
+    if (h->split) {   // 4D maps over the three piece planes
+      const bf16* W = h->rep_b + h->woff[l - 1];
+      const uint64_t wp = (uint64_t)h->piece_plane;
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, wp, 64, 128));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, wp, 64, 64));
+      const bf16* Hp = h->Hs[l - 1];
+      const uint64_t hp = (uint64_t)n * m * fi;
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
+      const uint64_t dp = (uint64_t)h->dzs_plane;
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
+      continue;
+    }
     const bf16* W = h->rep_b + h->woff[l - 1];
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, 64, 128));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 64, 64));
@@ -261,6 +282,16 @@ Status build_tc_maps(agn_handle* h) {
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
   }
   return Status::Ok();
+}
+
+// Pieces of an fp32 activation buffer [slots][m][d] (planes `plane` apart,
+// default n m d) for the tensor-core GEMMs of the fp32 mode.
+Status split_act(agn_handle* h, const void* src, bf16* dst, int d, int slots, int64_t* launches,
+                 int64_t plane = -1) {
+  const int64_t count = (int64_t)slots * h->m * d;
+  const int64_t pl = plane >= 0 ? plane : (int64_t)h->n * h->m * d;
+  Launch k(h, AGN_K_OTHER, 0.0, (double)count * 10.0, launches);
+  return agn::split_pieces(static_cast<const float*>(src), dst, count, pl, h->stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -285,6 +316,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb),
                                    h->yb, h->dims[0], m, h->S, sw, st0, i, s, h->stream));
     }
+    if (h->split) AGN_TRY(split_act(h, h->Xb, h->Hs[0], h->dims[0], s, launches));
     // forward, l = 1..L
     for (int l = 1; l <= L; ++l) {
       agn::GemmArgs g{};
@@ -308,10 +340,13 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
         t.relu = 1; t.boff = h->boff[l - 1];
         const auto& mp = h->tmaps[l - 1];
-        AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream));
-        continue;
+        AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split));
+      } else {
+        AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
       }
-      AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
+      // pieces of a hidden activation that the next tensor-core GEMMs read
+      // (the forward of layer l + 1 and the dW of layer l + 1)
+      if (h->split && l + 1 < L) AGN_TRY(split_act(h, h->H[l], h->Hs[l], fo, s, launches));
     }
     {
       Launch k(h, AGN_K_SOFTMAX, 0.0, (double)s * m * (h->dims[L] * (4.0 + es) + 4.0), launches);
@@ -323,6 +358,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     for (int l = L; l >= 1; --l) {
       const int fi = h->dims[l - 1], fo = h->dims[l];
       const void* Hprev = l == 1 ? h->Xb : h->H[l - 1];
+      if (h->split && tc_layer(h, l))
+        AGN_TRY(split_act(h, h->dz[cur], h->dZs, fo, s, launches, h->dzs_plane));
       if (l > 1) {
         agn::GemmArgs g{};
         g.M = m; g.N = fi; g.K = fo;
@@ -340,9 +377,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.M = fi; t.N = m; t.K = fo;
           t.a_by_worker = 1;
           t.out = h->dz[1 - cur]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
-          t.mask = static_cast<const bf16*>(Hprev); t.mask_bstride = (int64_t)m * fi;
+          t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
           const auto& mp = h->tmaps[l - 1];
-          AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream));
+          AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream, h->split));
         } else {
           AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
         }
@@ -353,6 +390,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       g.b = Hprev; g.ldb = fi; g.b_bstride = (int64_t)m * fi;
       g.slot_worker = sw;
       g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
+      g.piece_plane = h->piece_plane;
       g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
       {
         Launch k(h, AGN_K_BACKWARD_DW, 2.0 * s * m * fo * fi,
@@ -363,10 +401,10 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.M = fi; t.N = fo; t.K = m;
           t.woff = h->woff[l - 1]; t.eta = eta;
           const auto& mp = h->tmaps[l - 1];
-          AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, t, s, h->stream));
-          AGN_TRY(agn::bias_update(static_cast<const bf16*>(h->dz[cur]), m, fo, (int64_t)m * fo, sw,
-                                   h->rep, h->acc, h->rep_b, h->P_pad, h->boff[l - 1], eta, s,
-                                   h->stream));
+          AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, t, s, h->stream, h->split));
+          AGN_TRY(agn::bias_update(h->dz[cur], m, fo, (int64_t)m * fo, sw, h->rep, h->acc,
+                                   h->rep_b, h->P_pad, h->boff[l - 1], eta, s, h->stream,
+                                   h->split, h->piece_plane));
         } else {
           AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
         }
@@ -547,7 +585,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     Launch k(h, AGN_K_OTHER, 0.0,
              (double)h->P * (4.0 + plan.start_pulls.size() * (h->rep_b ? 6.0 : 4.0)), &launches);
     AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
-                               (int)plan.start_pulls.size(), h->stream));
+                               (int)plan.start_pulls.size(), h->stream, h->piece_plane));
   }
   const float scale = (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
   for (const Wave& wv : plan.waves) {
@@ -556,12 +594,13 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     for (const CommitPlan& cp : wv.commits) {
       const double pulls = cp.pull_begin[cp.n_commits];
       {
+        const double copy_b = h->split ? 6.0 : h->rep_b ? 2.0 : 0.0;
         Launch kc(h, AGN_K_COMMIT, 2.0 * cp.n_commits * h->P,
-                  (double)h->P * (8.0 + 8.0 * cp.n_commits + pulls * (h->rep_b ? 6.0 : 4.0)),
+                  (double)h->P * (8.0 + 8.0 * cp.n_commits + pulls * (4.0 + copy_b)),
                   &launches);
         AGN_TRY(agn::launch_commit_pull(cp, h->theta_c, h->acc, h->rep, h->rep_b, h->P_pad,
                                         h->P_pad, scale, true, h->partials, h->grid, nullptr,
-                                        nullptr, h->stream, /*norms=*/false));
+                                        nullptr, h->stream, /*norms=*/false, h->piece_plane));
       }
       Launch kn(h, AGN_K_NORMS, 0.0, 8.0 * cp.n_commits * h->grid, &launches);
       AGN_TRY(agn::launch_commit_norms(cp, h->partials, h->grid, h->dnorm, h->flag, h->stream));
@@ -656,14 +695,17 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   }
   h->P = off;
   h->P_pad = round_up(offp, 64);
-  // tcgen05 path: bf16 mode, m <= 256, every TMA row 16-byte aligned
-  bool tc_ok = h->prec == AGN_PREC_BF16 && h->m <= 256 && h->L >= 2;
+  // tcgen05 path: m <= 256, a hidden layer, every TMA row 16-byte aligned.
+  // bf16 mode feeds bf16 operands; fp32 mode feeds each fp32 operand as three
+  // exact bf16 pieces (split mode).
+  bool tc_ok = h->m <= 256 && h->L >= 2;
   for (int l = 0; l < h->L; ++l) tc_ok = tc_ok && dims[l] % 8 == 0;
   if (o.gemm == AGN_GEMM_TCGEN05 && !tc_ok)
     return Status::Err(AGN_E_UNSUPPORTED,
-                       "tcgen05 GEMMs need bf16 mode, batch <= 256, at least one hidden layer "
+                       "tcgen05 GEMMs need batch <= 256, at least one hidden layer "
                        "and d_0 .. d_{L-1} multiples of 8");
   h->use_tc = tc_ok && o.gemm != AGN_GEMM_SIMT;
+  h->split = h->use_tc && h->prec == AGN_PREC_FP32;
   h->tc_mask = o.tc_mask == 0 ? 7 : o.tc_mask;
   h->prev.assign(h->n, -1);
   h->pulled_v.assign(h->n, 0);
@@ -704,6 +746,19 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY(dalloc_t(h, &h->rep, (size_t)(n * h->P_pad)));
   AGN_TRY(dalloc_t(h, &h->acc, (size_t)(n * h->P_pad)));
   if (h->prec == AGN_PREC_BF16) AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(n * h->P_pad)));
+  if (h->split) {   // three piece planes of every replica, and of the activations
+    h->piece_plane = n * h->P_pad;
+    AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));
+    h->Hs.assign(h->L - 1, nullptr);
+    int maxh = 0;
+    for (int l = 0; l + 1 < h->L; ++l) {
+      AGN_TRY(dalloc_t(h, &h->Hs[l], (size_t)(3 * n * m * dims[l])));
+      if (l > 0) maxh = std::max(maxh, dims[l]);
+    }
+    maxh = std::max(maxh, dims[h->L - 1]);
+    h->dzs_plane = n * m * maxh;
+    AGN_TRY(dalloc_t(h, &h->dZs, (size_t)(3 * h->dzs_plane)));
+  }
   AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
   AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));
   AGN_TRY(dalloc(h, &h->Xb, (size_t)(n * m * d0) * es));
@@ -748,7 +803,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,
                                h->stream));
   AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
-                             (int)n, h->stream));   // every worker pulls version 0
+                             (int)n, h->stream, h->piece_plane));   // every worker pulls version 0
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
   return Status::Ok();
 }

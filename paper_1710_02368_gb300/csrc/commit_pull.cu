@@ -37,12 +37,36 @@ __device__ __forceinline__ uint2 pack_bf16x4(float4 v) {
   return r;
 }
 
-template <bool kBF16>
+// Three exact bf16 pieces of four floats, one uint2 per piece plane.
+__device__ __forceinline__ void pack_pieces_x4(float4 v, uint2& p0, uint2& p1, uint2& p2) {
+  const float x[4] = {v.x, v.y, v.z, v.w};
+  bf16 q[3][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    q[0][i] = __float2bfloat16_rn(x[i]);
+    const float r1 = __fsub_rn(x[i], __bfloat162float(q[0][i]));
+    q[1][i] = __float2bfloat16_rn(r1);
+    q[2][i] = __float2bfloat16_rn(__fsub_rn(r1, __bfloat162float(q[1][i])));
+  }
+  uint2* out[3] = {&p0, &p1, &p2};
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    __nv_bfloat162 lo = __halves2bfloat162(q[k][0], q[k][1]);
+    __nv_bfloat162 hi = __halves2bfloat162(q[k][2], q[k][3]);
+    out[k]->x = *reinterpret_cast<uint32_t*>(&lo);
+    out[k]->y = *reinterpret_cast<uint32_t*>(&hi);
+  }
+}
+
+// kCopy: 0 = fp32 replicas only, 1 = plus a bf16 copy, 3 = plus the three
+// exact bf16 pieces (planes `plane` elements apart) of the fp32 mode's
+// tensor-core operands.
+template <int kCopy>
 __global__ void __launch_bounds__(kThreads)
 commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ theta_c,
                    float* __restrict__ acc, float* __restrict__ replicas,
                    bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, float s, int zero_acc,
-                   double* __restrict__ partials) {
+                   double* __restrict__ partials, int64_t plane) {
   const int nc = plan.n_commits;
   double sq[kMaxCommitsPerLaunch];
 #pragma unroll
@@ -93,7 +117,14 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
           for (int u = 0; u < kUnroll; ++u) {
             if (!live[u]) continue;
             rrow[idx[u]] = th[u];
-            if (kBF16) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
+            if (kCopy == 1) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
+            if (kCopy == 3) {
+              uint2 q0, q1, q2;
+              pack_pieces_x4(th[u], q0, q1, q2);
+              reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = q0;
+              reinterpret_cast<uint2*>(rep_bf16 + plane + row)[idx[u]] = q1;
+              reinterpret_cast<uint2*>(rep_bf16 + 2 * plane + row)[idx[u]] = q2;
+            }
           }
         }
       }
@@ -118,7 +149,15 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
       for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
         const int64_t row = (int64_t)plan.pull_worker[p] * ld;
         replicas[row + i] = t;
-        if (kBF16) rep_bf16[row + i] = __float2bfloat16_rn(t);
+        if (kCopy == 1) rep_bf16[row + i] = __float2bfloat16_rn(t);
+        if (kCopy == 3) {
+          const bf16 q0 = __float2bfloat16_rn(t);
+          const float r1 = __fsub_rn(t, __bfloat162float(q0));
+          const bf16 q1 = __float2bfloat16_rn(r1);
+          rep_bf16[row + i] = q0;
+          rep_bf16[plane + row + i] = q1;
+          rep_bf16[2 * plane + row + i] = __float2bfloat16_rn(__fsub_rn(r1, __bfloat162float(q1)));
+        }
       }
     }
     theta_c[i] = t;
@@ -186,16 +225,20 @@ int commit_grid(int64_t P) {
 Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale, bool zero_acc,
                           double* partials, int grid, float* delta_norm, int* flag,
-                          cudaStream_t stream, bool norms) {
+                          cudaStream_t stream, bool norms, int64_t piece_plane) {
   if (plan.n_commits <= 0) return Status::Ok();
-  if (replicas_bf16)
-    commit_pull_kernel<true><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
-                                                             replicas_bf16, P, ld, scale,
-                                                             zero_acc ? 1 : 0, partials);
+  const int z = zero_acc ? 1 : 0;
+  if (replicas_bf16 && piece_plane > 0)
+    commit_pull_kernel<3><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
+                                                          replicas_bf16, P, ld, scale, z, partials,
+                                                          piece_plane);
+  else if (replicas_bf16)
+    commit_pull_kernel<1><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
+                                                          replicas_bf16, P, ld, scale, z, partials,
+                                                          0);
   else
-    commit_pull_kernel<false><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
-                                                              nullptr, P, ld, scale,
-                                                              zero_acc ? 1 : 0, partials);
+    commit_pull_kernel<0><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas, nullptr, P,
+                                                          ld, scale, z, partials, 0);
   AGN_TRY_CUDA(cudaGetLastError());
   if (norms && partials && (delta_norm || flag))
     return launch_commit_norms(plan, partials, grid, delta_norm, flag, stream);
@@ -219,14 +262,26 @@ namespace {
 
 __global__ void __launch_bounds__(kThreads)
 pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
-            bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers) {
+            bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers,
+            int64_t plane) {
   const int k = workers[blockIdx.y];
   float* dst = replicas + (int64_t)k * ld;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < P; i += stride) {
     const float t = theta_c[i];
     dst[i] = t;
-    if (rep_bf16) rep_bf16[(int64_t)k * ld + i] = __float2bfloat16_rn(t);
+    if (rep_bf16) {
+      const int64_t o = (int64_t)k * ld + i;
+      if (plane > 0) {
+        bf16 q0, q1, q2;
+        split3(t, q0, q1, q2);
+        rep_bf16[o] = q0;
+        rep_bf16[plane + o] = q1;
+        rep_bf16[2 * plane + o] = q2;
+      } else {
+        rep_bf16[o] = __float2bfloat16_rn(t);
+      }
+    }
   }
 }
 
@@ -242,10 +297,12 @@ __global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda
 }  // namespace
 
 Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
-                     int64_t ld, const int* workers, int count, cudaStream_t st) {
+                     int64_t ld, const int* workers, int count, cudaStream_t st,
+                     int64_t piece_plane) {
   if (count <= 0) return Status::Ok();
   dim3 grid((unsigned)std::max(1, commit_grid(P) / std::max(1, count) + 1), (unsigned)count);
-  pull_kernel<<<grid, kThreads, 0, st>>>(theta_c, replicas, replicas_bf16, P, ld, workers);
+  pull_kernel<<<grid, kThreads, 0, st>>>(theta_c, replicas, replicas_bf16, P, ld, workers,
+                                         piece_plane);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

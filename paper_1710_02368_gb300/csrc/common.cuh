@@ -45,6 +45,19 @@ inline Status cuda_status(cudaError_t e, const char* what) {
 constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
 
+// x = q0 + q1 + q2 exactly, each a bf16 (round to nearest even): q0 keeps the
+// leading 8 significant bits of x, q1 the next 8, q2 the last 8.  The two
+// residuals are exact float subtractions (Sterbenz); x must not be so small
+// that a piece falls below the smallest normal float.  The fp32 mode feeds
+// the tensor cores with these pieces.
+__device__ __forceinline__ void split3(float x, bf16& q0, bf16& q1, bf16& q2) {
+  q0 = __float2bfloat16_rn(x);
+  const float r1 = __fsub_rn(x, __bfloat162float(q0));
+  q1 = __float2bfloat16_rn(r1);
+  const float r2 = __fsub_rn(r1, __bfloat162float(q1));
+  q2 = __float2bfloat16_rn(r2);
+}
+
 // ---------------------------------------------------------------------------
 // Standalone commit + pull (kernel c)
 // ---------------------------------------------------------------------------
@@ -70,7 +83,8 @@ struct CommitPlan {
 Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale,
                           bool zero_acc, double* partials, int grid, float* delta_norm,
-                          int* flag, cudaStream_t stream, bool norms = true);
+                          int* flag, cudaStream_t stream, bool norms = true,
+                          int64_t piece_plane = 0);   // > 0: pulls write 3 pieces
 // The per-commit norm reduction of one launch of launch_commit_pull (when
 // that launch was queued with norms = false).
 Status launch_commit_norms(const CommitPlan& plan, const double* partials, int grid,

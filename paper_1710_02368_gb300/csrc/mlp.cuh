@@ -37,6 +37,7 @@ struct GemmArgs {
   float* theta;          // fp32 master replicas [n][ld_param]
   float* acc;            // accumulators [n][ld_param]
   bf16* theta_bf16;      // bf16 working copies or null
+  int64_t piece_plane;   // > 0: theta_bf16 holds three exact bf16 pieces, planes this far apart
   int64_t ld_param;
   int64_t woff, boff;    // offsets of W_l and b_l in a replica
   float eta;
@@ -59,8 +60,10 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
                     cudaStream_t st);
 
 // Pull: copy theta~ into the replicas of `workers` (device list) and their bf16 copies.
+// piece_plane > 0: replicas_bf16 holds three piece planes (fp32 mode on tensor cores).
 Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
-                     int64_t ld, const int* workers, int count, cudaStream_t st);
+                     int64_t ld, const int* workers, int count, cudaStream_t st,
+                     int64_t piece_plane = 0);
 // loss[c] = mean_i parts[c * lambda + i] for c < count.
 Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st);
 // Device-side standalone-commit input generator.

@@ -30,6 +30,20 @@ __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
 
+// The low-precision copy of an updated weight: one bf16, or its three exact
+// pieces (fp32 mode on tensor cores).
+__device__ __forceinline__ void write_copy(bf16* tb, int64_t plane, int64_t p, float t) {
+  if (plane > 0) {
+    bf16 q0, q1, q2;
+    split3(t, q0, q1, q2);
+    tb[p] = q0;
+    tb[plane + p] = q1;
+    tb[2 * plane + p] = q2;
+  } else {
+    tb[p] = __float2bfloat16_rn(t);
+  }
+}
+
 // C[M x N] (+)= sum_k A(m, k) B(k, n) for one slot; see GemmArgs for layouts.
 template <typename T, typename TO, bool kAKMajor, bool kBKMajor, int kEpi>
 __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
@@ -158,7 +172,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         const float t = fmaf(-g.eta, gr, th[i][j]);
         theta[p] = t;
         a[p] = av[i][j] + gr;
-        if (tb) tb[p] = __float2bfloat16_rn(t);
+        if (tb) write_copy(tb, g.piece_plane, p, t);
       }
     }
     if (do_bias && m0 + tid < g.M) {
@@ -166,7 +180,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       const float t = fmaf(-g.eta, bsum, theta[p]);
       theta[p] = t;
       a[p] += bsum;
-      if (tb) tb[p] = __float2bfloat16_rn(t);
+      if (tb) write_copy(tb, g.piece_plane, p, t);
     }
   }
 }

@@ -17,39 +17,51 @@ struct TcArgs {
   int* err;                // set to 1 when a bounded wait gives up
   void* out;               // forward / dX output (bf16) [slots][N rows][ldo]
   int64_t ldo, out_bstride;
-  const bf16* mask;        // dX: H_{l-1}, same layout as out
+  const void* mask;        // dX: H_{l-1}, same layout and type as out
   int64_t mask_bstride;
   int relu;
   float* theta;            // fp32 master replicas [n][ld_param]
   float* acc;              // accumulators [n][ld_param]
-  bf16* theta_b;           // bf16 working copies [n][ld_param]
+  bf16* theta_b;           // bf16 working copies [n][ld_param] (split mode: piece 0 of
+                           // three planes [3][n][ld_param])
   int64_t ld_param, woff, boff;
+  int64_t piece_plane;     // split mode: elements between weight piece planes
   float eta;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
 // must have this many rows (K-major) or 64-element chunks summing to it.
 inline int tc_bn(int N) { return N <= 64 ? 64 : N <= 128 ? 128 : 256; }
-constexpr int kTcDwBN = 256;
+constexpr int kTcDwBN = 256;        // dW column tile, bf16 mode
+constexpr int kTcDwBNSplit = 128;   // dW column tile, split (fp32) mode
 
 Status tc_init();
 // 3D bf16 tensor map (inner, rows, batch), 128-byte swizzle, zero fill.
 Status make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                          uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
                          uint32_t box_inner, uint32_t box_rows);
+// 4D bf16 tensor map (inner, rows, batch, piece) over three piece planes.
+Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                         uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
+                         uint64_t piece_stride_elems, uint32_t box_inner, uint32_t box_rows);
 
+// split = false: bf16 operands (3D maps), bf16 activations.
+// split = true : fp32 operands as three exact bf16 pieces (4D maps), fp32
+//                activations; dW writes the three pieces of the new weights.
 // forward: w_k box {64, 128} over W (K-major); h_k box {64, tc_bn(m)} over H_{l-1}.
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
-                  cudaStream_t st);
+                  cudaStream_t st, bool split);
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, tc_bn(m)} over dZ_l.
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
-                      int slots, cudaStream_t st);
+                      int slots, cudaStream_t st, bool split);
 // dW: h_mn box {64, 64} over H_{l-1}; dz_mn box {64, 64} over dZ_l.
 Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
-                      int slots, cudaStream_t st);
-// Bias gradient of a hidden layer and its local update.
-Status bias_update(const bf16* dz, int m, int d, int64_t dz_bstride, const int* slot_worker,
+                      int slots, cudaStream_t st, bool split);
+// Bias gradient of a hidden layer and its local update (dz: bf16, or fp32 when split).
+Status bias_update(const void* dz, int m, int d, int64_t dz_bstride, const int* slot_worker,
                    float* theta, float* acc, bf16* theta_b, int64_t ld_param, int64_t boff,
-                   float eta, int slots, cudaStream_t st);
+                   float eta, int slots, cudaStream_t st, bool split, int64_t piece_plane);
+// out[p * plane + i] = piece p of x[i], p < 3.
+Status split_pieces(const float* x, bf16* out, int64_t count, int64_t plane, cudaStream_t st);
 
 }  // namespace agn
