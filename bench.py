@@ -278,8 +278,13 @@ def run_agn(args, wl):
     h.profile(0)
     ms = e0.elapsed_time(e1)
     kst = h.kernel_stats()
-    gemm_used = ("tcgen05 (hidden layers) + simt (output layer)"
-                 if wl.precision == WL.PREC_BF16 and args.gemm != "simt" else "simt")
+    tc_ok = wl.batch <= 256 and all(d % 8 == 0 for d in wl.dims[:-1])
+    if args.gemm != "simt" and tc_ok:
+        gemm_used = ("tcgen05 bf16" if wl.precision == WL.PREC_BF16 else
+                     "tcgen05 fp32 as three exact bf16 pieces") + \
+                    " (hidden layers); fused output layer on CUDA cores"
+    else:
+        gemm_used = "CUDA-core GEMMs; fused output layer"
     # timed region 2: end to end through the public API with host buffers
     barrier()
     t0 = time.perf_counter()

@@ -20,7 +20,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB_NAME = "libagn_gb300.so"
 LIB_PATH = os.path.join(BUILD, LIB_NAME)
 
-SOURCES = ["agn_api.cu", "commit_pull.cu", "commit_pull_noalloc.cu", "mlp_simt.cu",
+SOURCES = ["agn_api.cu", "commit_pull.cu", "commit_pull_noalloc.cu", "mlp_simt.cu", "mlp_head.cu",
            "mlp_tc.cu", "host_inputs.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "--expt-relaxed-constexpr",

@@ -97,6 +97,10 @@ struct agn_handle {
   std::vector<bf16*> Hs;          // pieces of H_l, l = 0..L-2: [3][n][m][d_l]
   bf16* dZs = nullptr;            // pieces of the current dZ_l: [3][n][m][maxd]
   int64_t dzs_plane = 0;
+  // output layer fused into one kernel (forward + softmax-CE + dX) when narrow
+  bool use_head = false;
+  float* ce_partial = nullptr;    // [n][ceil(m / 8)]
+  int* head_counter = nullptr;    // [n]
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
   float* dnorm = nullptr;     // [cap_commits]
@@ -319,6 +323,23 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     if (h->split) AGN_TRY(split_act(h, h->Xb, h->Hs[0], h->dims[0], s, launches));
     // forward, l = 1..L
     for (int l = 1; l <= L; ++l) {
+      if (l == L && h->use_head) {   // output layer: forward + softmax-CE + dX, one kernel
+        agn::HeadArgs a{};
+        const int fi = h->dims[L - 1], C = h->dims[L];
+        a.H = L == 1 ? h->Xb : h->H[L - 1];
+        a.W = W; a.theta = h->rep; a.ld_param = h->P_pad;
+        a.woff = h->woff[L - 1]; a.boff = h->boff[L - 1];
+        a.K = fi; a.C = C; a.m = m;
+        a.slot_worker = sw; a.yb = h->yb;
+        a.dZL = h->dz[0]; a.dH = L > 1 ? h->dz[1] : nullptr;
+        a.ce_partial = h->ce_partial; a.counter = h->head_counter;
+        a.loss_parts = h->loss_parts; a.slot_commit = sc; a.lam = h->lam; a.step = i;
+        a.flag = h->flag;
+        Launch k(h, AGN_K_SOFTMAX, 4.0 * s * m * fi * C,
+                 (double)s * ((double)C * fi * es + 2.0 * m * fi * es + (double)m * C * es), launches);
+        AGN_TRY(agn::head_forward_backward<T>(a, s, h->stream));
+        continue;
+      }
       agn::GemmArgs g{};
       const int fi = h->dims[l - 1], fo = h->dims[l];
       g.M = m; g.N = fo; g.K = fi;
@@ -348,7 +369,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       // (the forward of layer l + 1 and the dW of layer l + 1)
       if (h->split && l + 1 < L) AGN_TRY(split_act(h, h->H[l], h->Hs[l], fo, s, launches));
     }
-    {
+    if (!h->use_head) {
       Launch k(h, AGN_K_SOFTMAX, 0.0, (double)s * m * (h->dims[L] * (4.0 + es) + 4.0), launches);
       AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dz[0]), m, h->dims[L],
                                    h->loss_parts, sc, h->lam, i, h->flag, s, h->stream));
@@ -360,7 +381,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       const void* Hprev = l == 1 ? h->Xb : h->H[l - 1];
       if (h->split && tc_layer(h, l))
         AGN_TRY(split_act(h, h->dz[cur], h->dZs, fo, s, launches, h->dzs_plane));
-      if (l > 1) {
+      if (l > 1 && !(l == L && h->use_head)) {   // the head already wrote dZ_{L-1}
         agn::GemmArgs g{};
         g.M = m; g.N = fi; g.K = fo;
         g.a = h->dz[cur]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
@@ -769,6 +790,11 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY(dalloc(h, &h->dz[0], (size_t)(n * m * h->maxd) * es));
   AGN_TRY(dalloc(h, &h->dz[1], (size_t)(n * m * h->maxd) * es));
   AGN_TRY(dalloc_t(h, &h->flag, 2));
+  h->use_head = h->prec == AGN_PREC_BF16 ? agn::head_fits<bf16>(dims[h->L - 1], dims[h->L])
+                                         : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
+  AGN_TRY(dalloc_t(h, &h->ce_partial, (size_t)(n * ceil_div(m, 8))));
+  AGN_TRY(dalloc_t(h, &h->head_counter, (size_t)n));
+  AGN_TRY_CUDA(cudaMemsetAsync(h->head_counter, 0, (size_t)n * sizeof(int), h->stream));
   h->grid = agn::commit_grid(h->P_pad);
   AGN_TRY(dalloc_t(h, &h->partials, (size_t)agn::kMaxCommitsPerLaunch * h->grid));
   AGN_TRY(dalloc_t(h, &h->pull_list, (size_t)n));

@@ -59,6 +59,32 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
                     cudaStream_t st);
 
+// Output layer fused (mlp_head.cu): forward, softmax cross-entropy and dX of
+// layer L for d_L <= kHeadMaxClasses; one warp per sample.
+constexpr int kHeadMaxClasses = 16;
+struct HeadArgs {
+  const void* H;           // H_{L-1} [slots][m][K] (T)
+  const void* W;           // replica operand base [n][ld_param] (T); W_L at woff, [C][K]
+  const float* theta;      // fp32 masters (bias b_L at boff)
+  int64_t ld_param, woff, boff;
+  int K, C, m;
+  const int* slot_worker;
+  const int* yb;           // labels [slots][m]
+  void* dZL;               // out: dZ_L [slots][m][C] (T)
+  void* dH;                // out: dZ_{L-1} [slots][m][K] (T)
+  float* ce_partial;       // [slots][ceil(m / 8)] scratch
+  int* counter;            // [slots], zero between launches
+  float* loss_parts;
+  const int* slot_commit;
+  int lam, step;
+  int* flag;
+};
+template <typename T>
+Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st);
+// The fused head takes this output layer (classes and shared-memory staging fit).
+template <typename T>
+bool head_fits(int K, int C);
+
 // Pull: copy theta~ into the replicas of `workers` (device list) and their bf16 copies.
 // piece_plane > 0: replicas_bf16 holds three piece planes (fp32 mode on tensor cores).
 Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,

@@ -34,15 +34,17 @@ def agn():
 
 
 @pytest.mark.skipif(not os.path.exists(golden.OUT), reason="golden reference not generated")
-def test_mnist_shaped_workload_2000_commits(agn):
+@pytest.mark.parametrize("gemm", ["simt", "tcgen05"])
+def test_mnist_shaped_workload_2000_commits(agn, gemm):
     wl = WL.MNIST_SHAPED
     seed = I.DEFAULT_SEED
     idx, loss_ref, dn_ref, cps = golden.load()
     w, tau = I.make_schedule(wl.n, wl.commits, wl.tau_lo, wl.tau_hi, seed)
     bounds = sorted(set([0] + [c + 1 for c in cps] + [wl.commits]))
     got = {}
+    backend = agn.AGN_GEMM_SIMT if gemm == "simt" else agn.AGN_GEMM_TCGEN05
     with agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, seed, batch=wl.batch, n_samples=wl.n_samples,
-                 gemm=agn.AGN_GEMM_SIMT) as h:
+                 gemm=backend) as h:
         for a, b in zip(bounds[:-1], bounds[1:]):
             h.run(b - a, w[a:], tau[a:])
             got[b - 1] = h.central()
