@@ -89,7 +89,9 @@ struct agn_handle {
   int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
+    CUtensorMap h_k64, dz_k64;   // 64-row boxes: 64-wide column tiles for small waves
   };
+  int num_sms = 148;
   std::vector<LayerMaps> tmaps;
   // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
   bool split = false;
@@ -273,6 +275,8 @@ Status build_tc_maps(agn_handle* h) {
       const uint64_t dp = (uint64_t)h->dzs_plane;
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k64, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k64, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       continue;
     }
     const bf16* W = h->rep_b + h->woff[l - 1];
@@ -284,8 +288,18 @@ Status build_tc_maps(agn_handle* h) {
     const void* dZ = h->dz[(L - l) % 2];   // dZ_l: dz[0] for l = L, alternating downwards
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k64, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
+    AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k64, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
   }
   return Status::Ok();
+}
+
+// Column tile of a forward or dX GEMM with M rows and N = m columns over s
+// slots: the full tile, unless that leaves SMs idle (small waves), then 64.
+int pick_bn(const agn_handle* h, int M, int s) {
+  const int bn = agn::tc_bn(h->m);
+  const int64_t ctas = ceil_div(M, 128) * ceil_div(h->m, bn) * (int64_t)s;
+  return (bn > 64 && ctas < h->num_sms) ? 64 : bn;
 }
 
 // Pieces of an fp32 activation buffer [slots][m][d] (planes `plane` apart,
@@ -361,7 +375,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
         t.relu = 1; t.boff = h->boff[l - 1];
         const auto& mp = h->tmaps[l - 1];
-        AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split));
+        const int bn = pick_bn(h, fo, s);
+        AGN_TRY(agn::tc_forward(mp.w_k, bn == 64 ? mp.h_k64 : mp.h_k, t, s, h->stream, h->split,
+                                bn));
       } else {
         AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
       }
@@ -400,7 +416,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.out = h->dz[1 - cur]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
           t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
           const auto& mp = h->tmaps[l - 1];
-          AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream, h->split));
+          const int bn = pick_bn(h, fi, s);
+          AGN_TRY(agn::tc_backward_dx(mp.w_mn, bn == 64 ? mp.dz_k64 : mp.dz_k, t, s, h->stream,
+                                      h->split, bn));
         } else {
           AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
         }
@@ -733,6 +751,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->steps.assign(h->n, 0);
 
   AGN_TRY_CUDA(cudaGetDevice(&h->device));
+  AGN_TRY_CUDA(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
   if (o.stream) {
     h->stream = static_cast<cudaStream_t>(o.stream);
   } else {

@@ -351,19 +351,30 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 }
 
 // Bias gradient and update for a hidden layer: g_b[f] = sum_j dZ[j][f];
-// b -= eta g_b, a_b += g_b, and the bf16 copy (or its three pieces).  One
-// thread per (f, slot).
+// b -= eta g_b, a_b += g_b, and the bf16 copy (or its three pieces).  A block
+// covers 32 features of one slot: its 8 warps sum interleaved sample groups
+// (coalesced rows of dZ), then one warp adds the 8 partials in a fixed order.
+constexpr int kBiasGroups = 8;
 template <typename TD, int kSplit>
-__global__ void bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
-                                   const int* __restrict__ slot_worker, float* theta, float* acc,
-                                   bf16* theta_b, int64_t ld_param, int64_t boff, float eta,
-                                   int64_t piece_plane) {
-  const int f = blockIdx.x * blockDim.x + threadIdx.x;
+__global__ void __launch_bounds__(32 * kBiasGroups)
+bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
+                   const int* __restrict__ slot_worker, float* theta, float* acc,
+                   bf16* theta_b, int64_t ld_param, int64_t boff, float eta,
+                   int64_t piece_plane) {
+  __shared__ float red[kBiasGroups][32];
+  const int fx = threadIdx.x & 31, gy = threadIdx.x >> 5;
+  const int f = blockIdx.x * 32 + fx;
   const int z = blockIdx.y;
-  if (f >= d) return;
   const TD* col = dz + (int64_t)z * dz_bstride + f;
+  float part = 0.f;
+  if (f < d)
+    for (int j = gy; j < m; j += kBiasGroups) part += from_act(col[(int64_t)j * d]);
+  red[gy][fx] = part;
+  __syncthreads();
+  if (gy != 0 || f >= d) return;
   float s = 0.f;
-  for (int j = 0; j < m; ++j) s += from_act(col[(int64_t)j * d]);
+#pragma unroll
+  for (int q = 0; q < kBiasGroups; ++q) s += red[q][fx];
   const int64_t p = (int64_t)slot_worker[z] * ld_param + boff + f;
   const float t = fmaf(-eta, s, theta[p]);
   theta[p] = t;
@@ -478,8 +489,7 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
 }
 
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
-                  cudaStream_t st, bool split) {
-  const int bn = tc_bn(args.N);
+                  cudaStream_t st, bool split, int bn) {
   if (split) {
     if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 3, 3>(w_k, h_k, args, slots, st);
     if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 2, 3>(w_k, h_k, args, slots, st);
@@ -491,8 +501,7 @@ Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& 
 }
 
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
-                      int slots, cudaStream_t st, bool split) {
-  const int bn = tc_bn(args.N);
+                      int slots, cudaStream_t st, bool split, int bn) {
   if (split) {
     if (bn == 64) return launch_tc<64, true, false, kEpiDX, 3, 3>(w_mn, dz_k, args, slots, st);
     if (bn == 128) return launch_tc<128, true, false, kEpiDX, 2, 3>(w_mn, dz_k, args, slots, st);
@@ -512,15 +521,18 @@ Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const T
 Status bias_update(const void* dz, int m, int d, int64_t dz_bstride, const int* slot_worker,
                    float* theta, float* acc, bf16* theta_b, int64_t ld_param, int64_t boff,
                    float eta, int slots, cudaStream_t st, bool split, int64_t piece_plane) {
-  dim3 grid((unsigned)ceil_div(d, 128), (unsigned)slots);
+  dim3 grid((unsigned)ceil_div(d, 32), (unsigned)slots);
+  const int threads = 32 * kBiasGroups;
   if (split)
-    bias_update_kernel<float, 3><<<grid, 128, 0, st>>>(static_cast<const float*>(dz), m, d,
-                                                       dz_bstride, slot_worker, theta, acc,
-                                                       theta_b, ld_param, boff, eta, piece_plane);
+    bias_update_kernel<float, 3><<<grid, threads, 0, st>>>(static_cast<const float*>(dz), m, d,
+                                                           dz_bstride, slot_worker, theta, acc,
+                                                           theta_b, ld_param, boff, eta,
+                                                           piece_plane);
   else
-    bias_update_kernel<bf16, 1><<<grid, 128, 0, st>>>(static_cast<const bf16*>(dz), m, d,
-                                                      dz_bstride, slot_worker, theta, acc, theta_b,
-                                                      ld_param, boff, eta, piece_plane);
+    bias_update_kernel<bf16, 1><<<grid, threads, 0, st>>>(static_cast<const bf16*>(dz), m, d,
+                                                          dz_bstride, slot_worker, theta, acc,
+                                                          theta_b, ld_param, boff, eta,
+                                                          piece_plane);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -48,12 +48,14 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
 // split = false: bf16 operands (3D maps), bf16 activations.
 // split = true : fp32 operands as three exact bf16 pieces (4D maps), fp32
 //                activations; dW writes the three pieces of the new weights.
-// forward: w_k box {64, 128} over W (K-major); h_k box {64, tc_bn(m)} over H_{l-1}.
+// forward: w_k box {64, 128} over W (K-major); h_k box {64, bn} over H_{l-1},
+// bn in {64, 128, 256} the column tile (>= N unless a smaller tile is chosen
+// to give a small wave more CTAs).
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
-                  cudaStream_t st, bool split);
-// dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, tc_bn(m)} over dZ_l.
+                  cudaStream_t st, bool split, int bn);
+// dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
-                      int slots, cudaStream_t st, bool split);
+                      int slots, cudaStream_t st, bool split, int bn);
 // dW: h_mn box {64, 64} over H_{l-1}; dz_mn box {64, 64} over dZ_l.
 Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
                       int slots, cudaStream_t st, bool split);
