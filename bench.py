@@ -311,8 +311,9 @@ def run_agn(args, wl):
     dom = max(("forward", "backward_dx", "backward_dw", "commit", "softmax", "gather"),
               key=lambda k: kst[k]["ms"])
     d = kst[dom]
+    on_tc = args.gemm != "simt" and tc_ok
     if dom in ("forward", "backward_dx", "backward_dw"):
-        if wl.precision == WL.PREC_FP32:
+        if wl.precision == WL.PREC_FP32 and not on_tc:
             roof = {"bound": "alu", "achieved": d["flops"] / d["ms"] / 1e9,
                     "peak": FP32_FMA_PEAK_TFLOPS, "unit": "TFLOP/s",
                     "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
@@ -326,7 +327,9 @@ def run_agn(args, wl):
             else:
                 roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
                         "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
-            roof["tensor_pipe_frac_of_bf16_peak"] = d["flops"] / d["ms"] / 1e9 / bf16
+            # fp32 mode on tensor cores issues six bf16 piece products per fp32 product
+            mma_per_flop = 6.0 if wl.precision == WL.PREC_FP32 else 1.0
+            roof["tensor_pipe_frac_of_bf16_peak"] = mma_per_flop * d["flops"] / d["ms"] / 1e9 / bf16
             roof["arithmetic_intensity_flop_per_byte"] = ai
     else:
         roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,

@@ -97,7 +97,7 @@ struct agn_handle {
   bool split = false;
   int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
   std::vector<bf16*> Hs;          // pieces of H_l, l = 0..L-2: [3][n][m][d_l]
-  bf16* dZs = nullptr;            // pieces of the current dZ_l: [3][n][m][maxd]
+  bf16* dZs[2] = {nullptr, nullptr};   // pieces of dZ_l in dZs[l % 2]: [3][n][m][maxd]
   int64_t dzs_plane = 0;
   // output layer fused into one kernel (forward + softmax-CE + dX) when narrow
   bool use_head = false;
@@ -273,10 +273,11 @@ Status build_tc_maps(agn_handle* h) {
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
       const uint64_t dp = (uint64_t)h->dzs_plane;
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
+      const bf16* dZp = h->dZs[l % 2];
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k64, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k64, h->dZs, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k64, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       continue;
     }
     const bf16* W = h->rep_b + h->woff[l - 1];
@@ -322,19 +323,30 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   const int* sw = h->plan_worker + wv.offset;
   const int* sc = h->plan_commit + wv.offset;
   const long long* st0 = h->plan_t0 + wv.offset;
-  const int m = h->m, L = h->L;
+  const int m = h->m, L = h->L, n = h->n;
   const T* W = h->prec == AGN_PREC_BF16 ? reinterpret_cast<const T*>(h->rep_b)
                                          : reinterpret_cast<const T*>(h->rep);
   const float eta = (float)h->eta;
   const double es = (double)sizeof(T);
-  const double upd = h->prec == AGN_PREC_BF16 ? 18.0 : 16.0;   // theta RMW + a RMW (+ bf16 copy)
+  // bytes per parameter of the local step + accumulation: theta RMW, a RMW, and
+  // the low-precision copy (one bf16, or three pieces in the split mode)
+  const double upd = 16.0 + (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
+  // pieces of dZ_l in the split mode go to dZs[l % 2], so that dX of layer l
+  // can write dZ_{l-1}'s pieces while dW of layer l still reads dZ_l's
+  auto dz_pieces = [&](int l) -> bf16* {
+    return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZs[l % 2] : nullptr;
+  };
   for (int i = 0; i < h->lam; ++i) {
     {
-      Launch k(h, AGN_K_GATHER, 0.0, (double)s * m * (2.0 * h->dims[0] * es + 8.0), launches);
+      Launch k(h, AGN_K_GATHER, 0.0,
+               (double)s * m * (2.0 * h->dims[0] * es + 8.0 + (h->split ? 6.0 * h->dims[0] : 0.0)),
+               launches);
       AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb),
-                                   h->yb, h->dims[0], m, h->S, sw, st0, i, s, h->stream));
+                                   h->yb, h->dims[0], m, h->S, sw, st0, i, s, h->stream,
+                                   h->split ? h->Hs[0] : nullptr,
+                                   (int64_t)n * m * h->dims[0]));
     }
-    if (h->split) AGN_TRY(split_act(h, h->Xb, h->Hs[0], h->dims[0], s, launches));
+    bool dz_ready = false;   // pieces of the next layer's dZ already written by its producer
     // forward, l = 1..L
     for (int l = 1; l <= L; ++l) {
       if (l == L && h->use_head) {   // output layer: forward + softmax-CE + dX, one kernel
@@ -346,12 +358,15 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         a.K = fi; a.C = C; a.m = m;
         a.slot_worker = sw; a.yb = h->yb;
         a.dZL = h->dz[0]; a.dH = L > 1 ? h->dz[1] : nullptr;
+        a.dH_pieces = L > 1 ? dz_pieces(L - 1) : nullptr;
+        a.dH_plane = h->dzs_plane;
         a.ce_partial = h->ce_partial; a.counter = h->head_counter;
         a.loss_parts = h->loss_parts; a.slot_commit = sc; a.lam = h->lam; a.step = i;
         a.flag = h->flag;
         Launch k(h, AGN_K_SOFTMAX, 4.0 * s * m * fi * C,
                  (double)s * ((double)C * fi * es + 2.0 * m * fi * es + (double)m * C * es), launches);
         AGN_TRY(agn::head_forward_backward<T>(a, s, h->stream));
+        dz_ready = a.dH_pieces != nullptr;
         continue;
       }
       agn::GemmArgs g{};
@@ -365,25 +380,32 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       g.relu = l < L;
       g.theta = h->rep; g.ld_param = h->P_pad; g.boff = h->boff[l - 1];
       const double oes = l == L ? 4.0 : es;
-      Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
-               (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es + (double)m * fo * oes),
-               launches);
-      if (tc_layer(h, l) && (h->tc_mask & 1)) {
-        agn::TcArgs t = tc_args(h, sw);
-        t.M = fo; t.N = m; t.K = fi;
-        t.a_by_worker = 1;
-        t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
-        t.relu = 1; t.boff = h->boff[l - 1];
-        const auto& mp = h->tmaps[l - 1];
-        const int bn = pick_bn(h, fo, s);
-        AGN_TRY(agn::tc_forward(mp.w_k, bn == 64 ? mp.h_k64 : mp.h_k, t, s, h->stream, h->split,
-                                bn));
-      } else {
-        AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
-      }
       // pieces of a hidden activation that the next tensor-core GEMMs read
       // (the forward of layer l + 1 and the dW of layer l + 1)
-      if (h->split && l + 1 < L) AGN_TRY(split_act(h, h->H[l], h->Hs[l], fo, s, launches));
+      bf16* h_pieces = (h->split && l + 1 < L) ? h->Hs[l] : nullptr;
+      bool pieces_done = false;
+      {
+        Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
+                 (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es +
+                              (double)m * fo * (oes + (h_pieces ? 6.0 : 0.0))),
+                 launches);
+        if (tc_layer(h, l) && (h->tc_mask & 1)) {
+          agn::TcArgs t = tc_args(h, sw);
+          t.M = fo; t.N = m; t.K = fi;
+          t.a_by_worker = 1;
+          t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
+          t.relu = 1; t.boff = h->boff[l - 1];
+          t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
+          const auto& mp = h->tmaps[l - 1];
+          const int bn = pick_bn(h, fo, s);
+          AGN_TRY(agn::tc_forward(mp.w_k, bn == 64 ? mp.h_k64 : mp.h_k, t, s, h->stream,
+                                  h->split, bn));
+          pieces_done = true;
+        } else {
+          AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
+        }
+      }
+      if (h_pieces && !pieces_done) AGN_TRY(split_act(h, h->H[l], h_pieces, fo, s, launches));
     }
     if (!h->use_head) {
       Launch k(h, AGN_K_SOFTMAX, 0.0, (double)s * m * (h->dims[L] * (4.0 + es) + 4.0), launches);
@@ -395,8 +417,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     for (int l = L; l >= 1; --l) {
       const int fi = h->dims[l - 1], fo = h->dims[l];
       const void* Hprev = l == 1 ? h->Xb : h->H[l - 1];
-      if (h->split && tc_layer(h, l))
-        AGN_TRY(split_act(h, h->dz[cur], h->dZs, fo, s, launches, h->dzs_plane));
+      if (dz_pieces(l) && !(dz_ready && l < L))
+        AGN_TRY(split_act(h, h->dz[cur], dz_pieces(l), fo, s, launches, h->dzs_plane));
+      bool next_ready = false;
       if (l > 1 && !(l == L && h->use_head)) {   // the head already wrote dZ_{L-1}
         agn::GemmArgs g{};
         g.M = m; g.N = fi; g.K = fo;
@@ -406,8 +429,10 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         g.out = h->dz[1 - cur]; g.ldo = fi; g.out_bstride = (int64_t)m * fi;
         g.mask = Hprev; g.mask_bstride = (int64_t)m * fi;
         g.theta = h->rep; g.ld_param = h->P_pad;
+        bf16* next_pieces = dz_pieces(l - 1);
         Launch k(h, AGN_K_BACKWARD_DX, 2.0 * s * m * fo * fi,
-                 (double)s * ((double)fo * fi * es + (double)m * fo * es + 2.0 * m * fi * es),
+                 (double)s * ((double)fo * fi * es + (double)m * fo * es +
+                              (double)m * fi * (2.0 * es + (next_pieces ? 6.0 : 0.0))),
                  launches);
         if (tc_layer(h, l) && (h->tc_mask & 2)) {
           agn::TcArgs t = tc_args(h, sw);
@@ -415,13 +440,17 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.a_by_worker = 1;
           t.out = h->dz[1 - cur]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
           t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
+          t.out_pieces = next_pieces; t.out_plane = h->dzs_plane;
           const auto& mp = h->tmaps[l - 1];
           const int bn = pick_bn(h, fi, s);
           AGN_TRY(agn::tc_backward_dx(mp.w_mn, bn == 64 ? mp.dz_k64 : mp.dz_k, t, s, h->stream,
                                       h->split, bn));
+          next_ready = next_pieces != nullptr;
         } else {
           AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
         }
+      } else if (l == L && h->use_head) {
+        next_ready = dz_ready;
       }
       agn::GemmArgs g{};
       g.M = fo; g.N = fi; g.K = m;
@@ -448,6 +477,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
         }
       }
+      dz_ready = next_ready;
       cur = 1 - cur;
     }
   }
@@ -797,7 +827,8 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
     }
     maxh = std::max(maxh, dims[h->L - 1]);
     h->dzs_plane = n * m * maxh;
-    AGN_TRY(dalloc_t(h, &h->dZs, (size_t)(3 * h->dzs_plane)));
+    AGN_TRY(dalloc_t(h, &h->dZs[0], (size_t)(3 * h->dzs_plane)));
+    AGN_TRY(dalloc_t(h, &h->dZs[1], (size_t)(3 * h->dzs_plane)));
   }
   AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
   AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));

@@ -57,7 +57,7 @@ Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* l
 template <typename T>
 Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
-                    cudaStream_t st);
+                    cudaStream_t st, bf16* pieces = nullptr, int64_t plane = 0);
 
 // Output layer fused (mlp_head.cu): forward, softmax cross-entropy and dX of
 // layer L for d_L <= kHeadMaxClasses; one warp per sample.
@@ -72,6 +72,8 @@ struct HeadArgs {
   const int* yb;           // labels [slots][m]
   void* dZL;               // out: dZ_L [slots][m][C] (T)
   void* dH;                // out: dZ_{L-1} [slots][m][K] (T)
+  bf16* dH_pieces;         // fp32 T only: also its three exact bf16 pieces (planes
+  int64_t dH_plane;        // dH_plane apart) for tensor-core GEMMs; null = no
   float* ce_partial;       // [slots][ceil(m / 8)] scratch
   int* counter;            // [slots], zero between launches
   float* loss_parts;

@@ -111,12 +111,21 @@ __global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a)
     // dZ_{L-1}[j][k] = sum_c dZ_L[j][c] W_L[c][k], masked by h > 0 (W before its
     // update); skipped when the output layer is the only layer (dH null)
     T* dh = a.dH ? static_cast<T*>(a.dH) + ((int64_t)z * m + j) * K : nullptr;
+    bf16* dp = a.dH_pieces ? a.dH_pieces + ((int64_t)z * m + j) * K : nullptr;
     for (int k = lane; dh && k < K; k += 32) {
       float v = 0.f;
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
         if (c < C) v = fmaf(g[c], cvt(Ws[(int64_t)c * Kp + k]), v);
-      dh[k] = st_f<T>(cvt(h[k]) > 0.f ? v : 0.f);
+      const T out = st_f<T>(cvt(h[k]) > 0.f ? v : 0.f);
+      dh[k] = out;
+      if (dp) {
+        bf16 q0, q1, q2;
+        split3(cvt(out), q0, q1, q2);
+        dp[k] = q0;
+        dp[a.dH_plane + k] = q1;
+        dp[2 * a.dH_plane + k] = q2;
+      }
     }
   }
   if (lane == 0) ce_warp[warp] = ce;

@@ -231,17 +231,30 @@ __global__ void __launch_bounds__(128) softmax_xent_kernel(const float* __restri
 
 // Minibatch gather (FetchNextMiniBatch of Algorithm 1): slot z, row j reads
 // dataset row k S + ((t0 + i) m + j) mod S of worker k = slot_worker[z].
+// With `pieces` (fp32 mode on tensor cores) the rows are also written as three
+// exact bf16 pieces, planes `plane` apart.
 template <typename T>
 __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y, T* Xb, int* yb,
                               int d0, int m, int64_t S, const int* slot_worker,
-                              const long long* slot_t0, int step) {
+                              const long long* slot_t0, int step, bf16* pieces, int64_t plane) {
   const int z = blockIdx.y, j = blockIdx.x;
   const int w = slot_worker[z];
   const long long t = slot_t0[z] + step;
   const int64_t row = (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
   const T* src = X + row * d0;
-  T* dst = Xb + ((int64_t)z * m + j) * d0;
-  for (int c = threadIdx.x; c < d0; c += blockDim.x) dst[c] = src[c];
+  const int64_t o = ((int64_t)z * m + j) * d0;
+  T* dst = Xb + o;
+  for (int c = threadIdx.x; c < d0; c += blockDim.x) {
+    const T v = src[c];
+    dst[c] = v;
+    if (pieces) {
+      bf16 q0, q1, q2;
+      split3(to_f(v), q0, q1, q2);
+      pieces[o + c] = q0;
+      pieces[plane + o + c] = q1;
+      pieces[2 * plane + o + c] = q2;
+    }
+  }
   if (threadIdx.x == 0) yb[(int64_t)z * m + j] = y[row];
 }
 
@@ -280,9 +293,10 @@ Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* l
 template <typename T>
 Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
-                    cudaStream_t st) {
+                    cudaStream_t st, bf16* pieces, int64_t plane) {
   dim3 grid((unsigned)m, (unsigned)slots);
-  gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step);
+  gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
+                                         pieces, plane);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -294,7 +308,8 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
   template Status softmax_xent<T>(const float*, const int*, T*, int, int, float*, const int*, \
                                   int, int, int*, int, cudaStream_t);                        \
   template Status gather_batch<T>(const T*, const int*, T*, int*, int, int, int64_t,          \
-                                  const int*, const long long*, int, int, cudaStream_t);
+                                  const int*, const long long*, int, int, cudaStream_t,       \
+                                  bf16*, int64_t);
 AGN_INST(float)
 AGN_INST(bf16)
 #undef AGN_INST

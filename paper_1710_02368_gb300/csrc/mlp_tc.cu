@@ -63,6 +63,17 @@ __device__ __forceinline__ float to_act<float>(float v) { return v; }
 __device__ __forceinline__ float from_act(bf16 v) { return __bfloat162float(v); }
 __device__ __forceinline__ float from_act(float v) { return v; }
 
+// Three exact bf16 pieces of an fp32 output element (slot, offset o within
+// the slot), written to the out_pieces planes for the next tensor-core GEMM.
+__device__ __forceinline__ void write_pieces(const TcArgs& a, int slot, int64_t o, float v) {
+  bf16 q0, q1, q2;
+  split3(v, q0, q1, q2);
+  bf16* p = a.out_pieces + (int64_t)slot * a.out_bstride + o;
+  p[0] = q0;
+  p[a.out_plane] = q1;
+  p[2 * a.out_plane] = q2;
+}
+
 // Wait that also gives up when another role has aborted.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity,
                                               volatile int* abort_flag) {
@@ -243,7 +254,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (j < args.N) {
               float v = __uint_as_float(r[i]) + bias;
               if (args.relu) v = fmaxf(v, 0.f);
-              out[(int64_t)j * args.ldo + row] = to_act<TAct>(v);
+              const int64_t o = (int64_t)j * args.ldo + row;
+              out[o] = to_act<TAct>(v);
+              if (kSplit == 3 && args.out_pieces) write_pieces(args, slot, o, v);
             }
           }
         }
@@ -271,7 +284,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (j < args.N) {
               const int64_t o = (int64_t)j * args.ldo + row;
               const float h = from_act(mask[o]);
-              out[o] = to_act<TAct>(h > 0.f ? __uint_as_float(r[i]) : 0.f);
+              const float v = h > 0.f ? __uint_as_float(r[i]) : 0.f;
+              out[o] = to_act<TAct>(v);
+              if (kSplit == 3 && args.out_pieces) write_pieces(args, slot, o, v);
             }
           }
         }

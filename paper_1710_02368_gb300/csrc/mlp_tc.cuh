@@ -27,6 +27,8 @@ struct TcArgs {
   int64_t ld_param, woff, boff;
   int64_t piece_plane;     // split mode: elements between weight piece planes
   float eta;
+  bf16* out_pieces;        // split mode, forward / dX: also write the output's three
+  int64_t out_plane;       // pieces here (same index, planes out_plane apart); null = no
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
