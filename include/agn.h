@@ -85,7 +85,9 @@ typedef struct agn_options {
   const int32_t* y_init;
   const float* theta_init;
   /* Diagnostic: which hidden-layer GEMMs use the tcgen05 kernels when they
-     are on (bit 0 forward, bit 1 dX, bit 2 dW); 0 = all. */
+     are on (bit 0 forward, bit 1 dX, bit 2 dW; 0 = bits 0-2).  Bit 3 runs the
+     dW GEMMs on the earlier non-persistent tcgen05 kernel (one tile per CTA)
+     instead of the persistent one, for comparison. */
   int32_t tc_mask;
 } agn_options;
 
@@ -168,7 +170,8 @@ int agn_generate_inputs(const int32_t* dims, int32_t n_dims, int32_t input_dist,
  */
 #define AGN_K_GATHER 0       /* minibatch gather (FetchNextMiniBatch)            */
 #define AGN_K_FORWARD 1      /* forward GEMM + bias + ReLU                       */
-#define AGN_K_SOFTMAX 2      /* softmax cross-entropy                            */
+#define AGN_K_SOFTMAX 2      /* softmax cross-entropy; with a narrow output layer
+                                the fused output head (forward, softmax-CE, dX)  */
 #define AGN_K_BACKWARD_DX 3  /* dX GEMM + ReLU mask                              */
 #define AGN_K_BACKWARD_DW 4  /* dW GEMM + local step + accumulation              */
 #define AGN_K_COMMIT 5       /* fused commit + pull                              */

@@ -90,6 +90,7 @@ struct agn_handle {
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
     CUtensorMap h_k64, dz_k64;   // 64-row boxes: 64-wide column tiles for small waves
+    CUtensorMap theta, acc;      // fp32 W_l of every replica / accumulator, box {128, 32}
   };
   int num_sms = 148;
   std::vector<LayerMaps> tmaps;
@@ -263,6 +264,10 @@ Status build_tc_maps(agn_handle* h) {
   for (int l = 1; l < L; ++l) {
     const uint64_t fi = h->dims[l - 1], fo = h->dims[l];
     auto& mp = h->tmaps[l - 1];
+    AGN_TRY(agn::make_tmap_f32_3d(&mp.theta, h->rep + h->woff[l - 1], fi, fo, n, fi, h->P_pad,
+                                  128, 32));
+    AGN_TRY(agn::make_tmap_f32_3d(&mp.acc, h->acc + h->woff[l - 1], fi, fo, n, fi, h->P_pad,
+                                  128, 32));
     if (h->split) {   // 4D maps over the three piece planes
       const bf16* W = h->rep_b + h->woff[l - 1];
       const uint64_t wp = (uint64_t)h->piece_plane;
@@ -469,7 +474,11 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.M = fi; t.N = fo; t.K = m;
           t.woff = h->woff[l - 1]; t.eta = eta;
           const auto& mp = h->tmaps[l - 1];
-          AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, t, s, h->stream, h->split));
+          if (h->tc_mask & 8)
+            AGN_TRY(agn::tc_backward_dw_tiled(mp.h_mn, mp.dz_mn, t, s, h->stream, h->split));
+          else
+            AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, mp.theta, mp.acc, t, s, h->stream,
+                                        h->split, h->num_sms));
           AGN_TRY(agn::bias_update(h->dz[cur], m, fo, (int64_t)m * fo, sw, h->rep, h->acc,
                                    h->rep_b, h->P_pad, h->boff[l - 1], eta, s, h->stream,
                                    h->split, h->piece_plane));
@@ -722,7 +731,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 7) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 7]");
+  if (o.tc_mask < 0 || o.tc_mask > 15) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 15]");
   h->dims.assign(dims, dims + n_dims);
   h->L = n_dims - 1;
   h->n = n_workers;

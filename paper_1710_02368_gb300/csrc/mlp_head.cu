@@ -4,8 +4,8 @@
 //
 // The output layer is narrow (d_L classes, at most 16 here), so a GEMM tile
 // would leave the GPU idle; instead one warp takes one sample.  A block first
-// stages W_L and its samples' input rows in shared memory with 16-byte loads
-// (all in flight at once), then each warp's lanes stride over the d_{L-1}
+// stages W_L and its samples' input rows in shared memory with asynchronous
+// 16-byte copies (all in flight at once), then each warp's lanes stride over the d_{L-1}
 // inputs, keep one partial dot product per class and combine them with a
 // fixed shuffle tree, so results are deterministic.  The per-slot loss (mean
 // over the minibatch) is summed in a fixed order by the last block of the
@@ -27,8 +27,10 @@ __device__ __forceinline__ float st_f<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ bf16 st_f<bf16>(float v) { return __float2bfloat16_rn(v); }
 
-// Copy `count` elements of T from global to shared memory with 16-byte loads
-// where both ends are aligned, element loads elsewhere.
+// Start copying `count` elements of T from global to shared memory: 16-byte
+// asynchronous copies (cp.async, no register round trip, so every row of the
+// block is in flight at once) where both ends are aligned, element copies
+// elsewhere.  The caller waits with cp.async.wait_all before its barrier.
 template <typename T>
 __device__ __forceinline__ void stage(T* dst, const T* src, int64_t count) {
   constexpr int kVec = 16 / sizeof(T);
@@ -37,11 +39,18 @@ __device__ __forceinline__ void stage(T* dst, const T* src, int64_t count) {
     const int64_t nv = count / kVec;
     const uint4* s = reinterpret_cast<const uint4*>(src);
     uint4* d = reinterpret_cast<uint4*>(dst);
-    for (int64_t i = threadIdx.x; i < nv; i += blockDim.x) d[i] = __ldg(s + i);
+    for (int64_t i = threadIdx.x; i < nv; i += blockDim.x)
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                       static_cast<uint32_t>(__cvta_generic_to_shared(d + i))),
+                   "l"(s + i)
+                   : "memory");
     for (int64_t i = nv * kVec + threadIdx.x; i < count; i += blockDim.x) dst[i] = src[i];
   } else {
     for (int64_t i = threadIdx.x; i < count; i += blockDim.x) dst[i] = src[i];
   }
+}
+__device__ __forceinline__ void stage_wait() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 template <typename T, int kMaxC>
@@ -60,6 +69,7 @@ __global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a)
   const T* Hg = static_cast<const T*>(a.H) + ((int64_t)z * m + j0) * K;
   for (int c = 0; c < C; ++c) stage(Ws + c * Kp, Wg + (int64_t)c * K, K);
   for (int q = 0; q < nj; ++q) stage(Hs + q * Kp, Hg + (int64_t)q * K, K);
+  stage_wait();
   __syncthreads();
 
   const float* bias = a.theta + (int64_t)w * a.ld_param + a.boff;

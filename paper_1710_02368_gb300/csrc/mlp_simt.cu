@@ -7,6 +7,8 @@
 // three GEMM shapes use one tiled kernel (64x64 tile, 16-deep k slices, 4x4
 // outputs per thread); the element type T is float (fp32 mode) or bf16 (bf16
 // mode: operands bf16, accumulation fp32, master weights fp32).
+#include <algorithm>
+
 #include "mlp.cuh"
 
 namespace agn {
@@ -258,6 +260,41 @@ __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y
   if (threadIdx.x == 0) yb[(int64_t)z * m + j] = y[row];
 }
 
+// The same gather, four consecutive elements per thread (d_0 a multiple of
+// 4): one 16-byte (fp32) or 8-byte (bf16) load and store, and 8-byte piece
+// stores; a grid-stride loop over (slot, sample, element group).
+template <typename T>
+__global__ void gather4_kernel(const T* __restrict__ X, const int* __restrict__ y, T* Xb, int* yb,
+                               int d0, int m, int64_t S, const int* slot_worker,
+                               const long long* slot_t0, int step, bf16* pieces, int64_t plane,
+                               int64_t total) {
+  struct alignas(4 * sizeof(T)) Vec { T v[4]; };
+  struct alignas(8) Piece4 { bf16 v[4]; };
+  const int g4 = d0 / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+    const int64_t r = i / g4;             // slot * m + j
+    const int c = (int)(i - r * g4) * 4;
+    const int z = (int)(r / m), j = (int)(r - (int64_t)z * m);
+    const int w = slot_worker[z];
+    const long long t = slot_t0[z] + step;
+    const int64_t row =
+        (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
+    const Vec v = *reinterpret_cast<const Vec*>(X + row * d0 + c);
+    const int64_t o = r * d0 + c;
+    *reinterpret_cast<Vec*>(Xb + o) = v;
+    if (pieces) {
+      Piece4 p0, p1, p2;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) split3(to_f(v.v[e]), p0.v[e], p1.v[e], p2.v[e]);
+      *reinterpret_cast<Piece4*>(pieces + o) = p0;
+      *reinterpret_cast<Piece4*>(pieces + plane + o) = p1;
+      *reinterpret_cast<Piece4*>(pieces + 2 * plane + o) = p2;
+    }
+    if (c == 0) yb[r] = y[row];
+  }
+}
+
 template <typename T, typename TO, bool kAK, bool kBK, int kEpi>
 Status launch_gemm(const GemmArgs& g, int slots, cudaStream_t st) {
   dim3 grid((unsigned)ceil_div(g.N, kBN), (unsigned)ceil_div(g.M, kBM), (unsigned)slots);
@@ -294,9 +331,20 @@ template <typename T>
 Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
                     cudaStream_t st, bf16* pieces, int64_t plane) {
-  dim3 grid((unsigned)m, (unsigned)slots);
-  gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
-                                         pieces, plane);
+  const bool vec = d0 % 4 == 0 && plane % 4 == 0 &&
+                   ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(Xb) |
+                     reinterpret_cast<uintptr_t>(pieces)) & 15) == 0;
+  if (slots <= 0 || m <= 0) return Status::Ok();
+  if (vec) {
+    const int64_t total = (int64_t)slots * m * (d0 / 4);
+    const int grid = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 16);
+    gather4_kernel<T><<<grid, 256, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
+                                            pieces, plane, total);
+  } else {
+    dim3 grid((unsigned)m, (unsigned)slots);
+    gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
+                                           pieces, plane);
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

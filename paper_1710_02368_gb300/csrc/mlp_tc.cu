@@ -77,15 +77,7 @@ __device__ __forceinline__ void write_pieces(const TcArgs& a, int slot, int64_t 
 // Wait that also gives up when another role has aborted.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity,
                                               volatile int* abort_flag) {
-  if (tc::mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = tc::globaltimer_ns();
-  for (uint32_t it = 0;; ++it) {
-    if (tc::mbar_try_wait(bar, parity)) return true;
-    if ((it & 63) == 63) {
-      if (*abort_flag) return false;
-      if (tc::globaltimer_ns() - t0 > kWaitNs) return false;
-    }
-  }
+  return tc::wait_or_abort(bar, parity, abort_flag, kWaitNs);
 }
 
 // The dW kernel is bound by its epilogue's DRAM traffic: two CTAs per SM
@@ -449,18 +441,22 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 Status encode(CUtensorMap* map, int rank, const void* base, const cuuint64_t* dims,
-              const cuuint64_t* strides_bytes, const cuuint32_t* box) {
+              const cuuint64_t* strides_bytes, const cuuint32_t* box,
+              CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, int esize = 2,
+              CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   AGN_TRY(tc_init());
   if (reinterpret_cast<uintptr_t>(base) & 15)
     return Status::Err(AGN_E_UNSUPPORTED, "tensor map base not 16-byte aligned");
-  if ((dims[0] * 2) % 16) return Status::Err(AGN_E_UNSUPPORTED, "tensor map rows not 16-byte aligned");
+  if ((dims[0] * esize) % 16)
+    return Status::Err(AGN_E_UNSUPPORTED, "tensor map rows not 16-byte aligned");
+  if ((box[0] * esize) % 16)
+    return Status::Err(AGN_E_UNSUPPORTED, "tensor map box rows not a multiple of 16 bytes");
   for (int i = 0; i < rank - 1; ++i)
     if (strides_bytes[i] % 16)
       return Status::Err(AGN_E_UNSUPPORTED, "tensor map stride not a multiple of 16 bytes");
   cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims,
-                        strides_bytes, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  CUresult r = g_encode(map, dtype, rank, const_cast<void*>(base), dims, strides_bytes, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return Status::Err(AGN_E_CUDA, "cuTensorMapEncodeTiled failed with code " + std::to_string(r));
@@ -503,6 +499,16 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
   return encode(map, 4, base, dims, strides, box);
 }
 
+Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                        uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
+                        uint32_t box_inner, uint32_t box_rows) {
+  cuuint64_t dims[3] = {inner, rows, batch};
+  cuuint64_t strides[2] = {row_stride_elems * 4, batch_stride_elems * 4};
+  cuuint32_t box[3] = {box_inner, box_rows, 1};
+  return encode(map, 3, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4,
+                CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
                   cudaStream_t st, bool split, int bn) {
   if (split) {
@@ -527,8 +533,8 @@ Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const Tc
   return launch_tc<256, true, false, kEpiDX, 4, 1>(w_mn, dz_k, args, slots, st);
 }
 
-Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
-                      int slots, cudaStream_t st, bool split) {
+Status tc_backward_dw_tiled(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
+                            int slots, cudaStream_t st, bool split) {
   if (split) return launch_tc<kTcDwBNSplit, true, true, kEpiDW, 1, 3>(h_mn, dz_mn, args, slots, st);
   return launch_tc<kTcDwBN, true, true, kEpiDW, 2, 1>(h_mn, dz_mn, args, slots, st);
 }

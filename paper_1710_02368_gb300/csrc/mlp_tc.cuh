@@ -42,6 +42,10 @@ Status tc_init();
 Status make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                          uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
                          uint32_t box_inner, uint32_t box_rows);
+// 3D fp32 tensor map (inner, rows, batch), no swizzle, zero fill.
+Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                        uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
+                        uint32_t box_inner, uint32_t box_rows);
 // 4D bf16 tensor map (inner, rows, batch, piece) over three piece planes.
 Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                          uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
@@ -58,9 +62,17 @@ Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& 
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
                       int slots, cudaStream_t st, bool split, int bn);
-// dW: h_mn box {64, 64} over H_{l-1}; dz_mn box {64, 64} over dZ_l.
-Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
-                      int slots, cudaStream_t st, bool split);
+// dW (mlp_tc_dw.cu, persistent, grid min(tiles, num_sms)): h_mn box {64, 64}
+// over H_{l-1}; dz_mn box {64, 64} over dZ_l; theta_map / acc_map fp32 maps
+// (d_{l-1}, d_l, n) over the layer's weights in the replicas and the
+// accumulators, box {128, 32}, no swizzle.
+Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn,
+                      const CUtensorMap& theta_map, const CUtensorMap& acc_map,
+                      const TcArgs& args, int slots, cudaStream_t st, bool split, int num_sms);
+// The earlier non-persistent dW kernel (mlp_tc.cu): one 128 x BN tile per CTA,
+// two CTAs per SM, theta_k and a_k loaded into registers by the epilogue.
+Status tc_backward_dw_tiled(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,
+                            int slots, cudaStream_t st, bool split);
 // Bias gradient of a hidden layer and its local update (dz: bf16, or fp32 when split).
 Status bias_update(const void* dz, int m, int d, int64_t dz_bstride, const int* slot_worker,
                    float* theta, float* acc, bf16* theta_b, int64_t ld_param, int64_t boff,
