@@ -81,7 +81,7 @@ struct agn_handle {
   int* yb = nullptr;          // [n][m]
   std::vector<void*> H;       // H[l] [n][m][d_l] T, l = 1..L-1 (H[0] = Xb)
   float* Z = nullptr;         // [n][m][d_L]
-  void* dz[2] = {nullptr, nullptr};   // [n][m][maxd] T
+  std::vector<void*> dZ;      // dZ[l] [n][m][d_l] T, l = 1..L
   int* flag = nullptr;        // [0] non-finite loss or commit, [1] bounded wait gave up
   double* partials = nullptr;
   // tcgen05 path (bf16 mode): tensor maps per layer l = 1..L-1 (index l-1)
@@ -98,11 +98,10 @@ struct agn_handle {
   bool split = false;
   int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
   std::vector<bf16*> Hs;          // pieces of H_l, l = 0..L-2: [3][n][m][d_l]
-  bf16* dZs[2] = {nullptr, nullptr};   // pieces of dZ_l in dZs[l % 2]: [3][n][m][maxd]
-  int64_t dzs_plane = 0;
+  std::vector<bf16*> dZp;         // pieces of dZ_l, l = 1..L-1: [3][n][m][d_l]
   // output layer fused into one kernel (forward + softmax-CE + dX) when narrow
   bool use_head = false;
-  float* ce_partial = nullptr;    // [n][ceil(m / 8)]
+  float* ce_partial = nullptr;    // [n][ceil(m / kHeadSamples)]
   int* head_counter = nullptr;    // [n]
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
@@ -277,8 +276,8 @@ Status build_tc_maps(agn_handle* h) {
       const uint64_t hp = (uint64_t)n * m * fi;
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
-      const uint64_t dp = (uint64_t)h->dzs_plane;
-      const bf16* dZp = h->dZs[l % 2];
+      const uint64_t dp = (uint64_t)n * m * fo;
+      const bf16* dZp = h->dZp[l];
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k64, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
@@ -291,7 +290,7 @@ Status build_tc_maps(agn_handle* h) {
     const void* Hin = l == 1 ? h->Xb : h->H[l - 1];
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_mn, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
-    const void* dZ = h->dz[(L - l) % 2];   // dZ_l: dz[0] for l = L, alternating downwards
+    const void* dZ = h->dZ[l];
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k64, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
@@ -336,11 +335,11 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   // bytes per parameter of the local step + accumulation: theta RMW, a RMW, and
   // the low-precision copy (one bf16, or three pieces in the split mode)
   const double upd = 16.0 + (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
-  // pieces of dZ_l in the split mode go to dZs[l % 2], so that dX of layer l
-  // can write dZ_{l-1}'s pieces while dW of layer l still reads dZ_l's
+  // pieces of dZ_l (split mode, hidden tensor-core layers), planes n m d_l apart
   auto dz_pieces = [&](int l) -> bf16* {
-    return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZs[l % 2] : nullptr;
+    return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZp[l] : nullptr;
   };
+  auto dz_plane = [&](int l) -> int64_t { return (int64_t)n * m * h->dims[l]; };
   for (int i = 0; i < h->lam; ++i) {
     {
       Launch k(h, AGN_K_GATHER, 0.0,
@@ -362,9 +361,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         a.woff = h->woff[L - 1]; a.boff = h->boff[L - 1];
         a.K = fi; a.C = C; a.m = m;
         a.slot_worker = sw; a.yb = h->yb;
-        a.dZL = h->dz[0]; a.dH = L > 1 ? h->dz[1] : nullptr;
+        a.dZL = h->dZ[L]; a.dH = L > 1 ? h->dZ[L - 1] : nullptr;
         a.dH_pieces = L > 1 ? dz_pieces(L - 1) : nullptr;
-        a.dH_plane = h->dzs_plane;
+        a.dH_plane = L > 1 ? dz_plane(L - 1) : 0;
         a.ce_partial = h->ce_partial; a.counter = h->head_counter;
         a.loss_parts = h->loss_parts; a.slot_commit = sc; a.lam = h->lam; a.step = i;
         a.flag = h->flag;
@@ -414,80 +413,111 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     }
     if (!h->use_head) {
       Launch k(h, AGN_K_SOFTMAX, 0.0, (double)s * m * (h->dims[L] * (4.0 + es) + 4.0), launches);
-      AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dz[0]), m, h->dims[L],
+      AGN_TRY(agn::softmax_xent<T>(h->Z, h->yb, static_cast<T*>(h->dZ[L]), m, h->dims[L],
                                    h->loss_parts, sc, h->lam, i, h->flag, s, h->stream));
     }
-    // backward, l = L..1: dX (reads W_l before its update), then dW + update
-    int cur = 0;
+    // backward: dX for l = L..2 (each reads W_l before its update), then the
+    // weight and bias gradients with the local step of every layer
+    std::vector<char> have_pieces(L + 1, 0);   // pieces of dZ_l written by its producer
+    if (L > 1) have_pieces[L - 1] = dz_ready;
+    auto ensure_pieces = [&](int l) -> Status {
+      if (dz_pieces(l) && !have_pieces[l]) {
+        AGN_TRY(split_act(h, h->dZ[l], dz_pieces(l), h->dims[l], s, launches, dz_plane(l)));
+        have_pieces[l] = 1;
+      }
+      return Status::Ok();
+    };
+    for (int l = L; l >= 2; --l) {
+      if (l == L && h->use_head) continue;   // the head already wrote dZ_{L-1}
+      const int fi = h->dims[l - 1], fo = h->dims[l];
+      const void* Hprev = h->H[l - 1];
+      bf16* next_pieces = dz_pieces(l - 1);
+      Launch k(h, AGN_K_BACKWARD_DX, 2.0 * s * m * fo * fi,
+               (double)s * ((double)fo * fi * es + (double)m * fo * es +
+                            (double)m * fi * (2.0 * es + (next_pieces ? 6.0 : 0.0))),
+               launches);
+      if (tc_layer(h, l) && (h->tc_mask & 2)) {
+        AGN_TRY(ensure_pieces(l));
+        agn::TcArgs t = tc_args(h, sw);
+        t.M = fi; t.N = m; t.K = fo;
+        t.a_by_worker = 1;
+        t.out = h->dZ[l - 1]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
+        t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
+        t.out_pieces = next_pieces; t.out_plane = dz_plane(l - 1);
+        const auto& mp = h->tmaps[l - 1];
+        const int bn = pick_bn(h, fi, s);
+        AGN_TRY(agn::tc_backward_dx(mp.w_mn, bn == 64 ? mp.dz_k64 : mp.dz_k, t, s, h->stream,
+                                    h->split, bn));
+        have_pieces[l - 1] = next_pieces != nullptr;
+      } else {
+        agn::GemmArgs g{};
+        g.M = m; g.N = fi; g.K = fo;
+        g.a = h->dZ[l]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
+        g.b = W + h->woff[l - 1]; g.ldb = fi; g.b_bstride = h->P_pad; g.b_by_worker = 1;
+        g.slot_worker = sw;
+        g.out = h->dZ[l - 1]; g.ldo = fi; g.out_bstride = (int64_t)m * fi;
+        g.mask = Hprev; g.mask_bstride = (int64_t)m * fi;
+        g.theta = h->rep; g.ld_param = h->P_pad;
+        AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
+      }
+    }
+    // dW: the output layer, then the hidden layers (on the tensor cores, all
+    // in one persistent launch)
+    std::vector<agn::DwLayerMaps> tc_dw;
+    double tc_flops = 0.0, tc_bytes = 0.0;
     for (int l = L; l >= 1; --l) {
       const int fi = h->dims[l - 1], fo = h->dims[l];
       const void* Hprev = l == 1 ? h->Xb : h->H[l - 1];
-      if (dz_pieces(l) && !(dz_ready && l < L))
-        AGN_TRY(split_act(h, h->dz[cur], dz_pieces(l), fo, s, launches, h->dzs_plane));
-      bool next_ready = false;
-      if (l > 1 && !(l == L && h->use_head)) {   // the head already wrote dZ_{L-1}
-        agn::GemmArgs g{};
-        g.M = m; g.N = fi; g.K = fo;
-        g.a = h->dz[cur]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
-        g.b = W + h->woff[l - 1]; g.ldb = fi; g.b_bstride = h->P_pad; g.b_by_worker = 1;
-        g.slot_worker = sw;
-        g.out = h->dz[1 - cur]; g.ldo = fi; g.out_bstride = (int64_t)m * fi;
-        g.mask = Hprev; g.mask_bstride = (int64_t)m * fi;
-        g.theta = h->rep; g.ld_param = h->P_pad;
-        bf16* next_pieces = dz_pieces(l - 1);
-        Launch k(h, AGN_K_BACKWARD_DX, 2.0 * s * m * fo * fi,
-                 (double)s * ((double)fo * fi * es + (double)m * fo * es +
-                              (double)m * fi * (2.0 * es + (next_pieces ? 6.0 : 0.0))),
-                 launches);
-        if (tc_layer(h, l) && (h->tc_mask & 2)) {
-          agn::TcArgs t = tc_args(h, sw);
-          t.M = fi; t.N = m; t.K = fo;
-          t.a_by_worker = 1;
-          t.out = h->dz[1 - cur]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
-          t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
-          t.out_pieces = next_pieces; t.out_plane = h->dzs_plane;
-          const auto& mp = h->tmaps[l - 1];
-          const int bn = pick_bn(h, fi, s);
-          AGN_TRY(agn::tc_backward_dx(mp.w_mn, bn == 64 ? mp.dz_k64 : mp.dz_k, t, s, h->stream,
-                                      h->split, bn));
-          next_ready = next_pieces != nullptr;
-        } else {
-          AGN_TRY(agn::simt_backward_dx<T>(g, s, h->stream));
-        }
-      } else if (l == L && h->use_head) {
-        next_ready = dz_ready;
-      }
-      agn::GemmArgs g{};
-      g.M = fo; g.N = fi; g.K = m;
-      g.a = h->dz[cur]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
-      g.b = Hprev; g.ldb = fi; g.b_bstride = (int64_t)m * fi;
-      g.slot_worker = sw;
-      g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
-      g.piece_plane = h->piece_plane;
-      g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
-      {
-        Launch k(h, AGN_K_BACKWARD_DW, 2.0 * s * m * fo * fi,
-                 (double)s * (((double)fo * fi + fo) * upd + (double)m * fo * es + (double)m * fi * es),
-                 launches);
-        if (tc_layer(h, l) && (h->tc_mask & 4)) {
+      const double flops = 2.0 * s * m * fo * fi;
+      const double bytes =
+          (double)s * (((double)fo * fi + fo) * upd + (double)m * fo * es + (double)m * fi * es);
+      if (tc_layer(h, l) && (h->tc_mask & 4)) {
+        AGN_TRY(ensure_pieces(l));
+        if (h->tc_mask & 8) {   // the earlier one-tile-per-CTA kernel, layer by layer
+          Launch k(h, AGN_K_BACKWARD_DW, flops, bytes, launches);
           agn::TcArgs t = tc_args(h, sw);
           t.M = fi; t.N = fo; t.K = m;
           t.woff = h->woff[l - 1]; t.eta = eta;
           const auto& mp = h->tmaps[l - 1];
-          if (h->tc_mask & 8)
-            AGN_TRY(agn::tc_backward_dw_tiled(mp.h_mn, mp.dz_mn, t, s, h->stream, h->split));
-          else
-            AGN_TRY(agn::tc_backward_dw(mp.h_mn, mp.dz_mn, mp.theta, mp.acc, t, s, h->stream,
-                                        h->split, h->num_sms));
-          AGN_TRY(agn::bias_update(h->dz[cur], m, fo, (int64_t)m * fo, sw, h->rep, h->acc,
+          AGN_TRY(agn::tc_backward_dw_tiled(mp.h_mn, mp.dz_mn, t, s, h->stream, h->split));
+          AGN_TRY(agn::bias_update(h->dZ[l], m, fo, (int64_t)m * fo, sw, h->rep, h->acc,
                                    h->rep_b, h->P_pad, h->boff[l - 1], eta, s, h->stream,
                                    h->split, h->piece_plane));
         } else {
-          AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+          const auto& mp = h->tmaps[l - 1];
+          tc_dw.push_back({&mp.h_mn, &mp.dz_mn, &mp.theta, &mp.acc, fi, fo, h->woff[l - 1],
+                           h->boff[l - 1]});
+          tc_flops += flops;
+          tc_bytes += bytes;
         }
+        continue;
       }
-      dz_ready = next_ready;
-      cur = 1 - cur;
+      Launch k(h, AGN_K_BACKWARD_DW, flops, bytes, launches);
+      if (l == L && h->use_head) {   // narrow output layer
+        agn::HeadDwArgs d{};
+        d.H = Hprev; d.dZL = h->dZ[l]; d.slot_worker = sw;
+        d.theta = h->rep; d.acc = h->acc; d.theta_b = h->rep_b; d.piece_plane = h->piece_plane;
+        d.ld_param = h->P_pad; d.woff = h->woff[l - 1]; d.boff = h->boff[l - 1];
+        d.K = fi; d.C = fo; d.m = m; d.eta = eta;
+        AGN_TRY(agn::head_backward_dw<T>(d, s, h->stream));
+      } else {
+        agn::GemmArgs g{};
+        g.M = fo; g.N = fi; g.K = m;
+        g.a = h->dZ[l]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
+        g.b = Hprev; g.ldb = fi; g.b_bstride = (int64_t)m * fi;
+        g.slot_worker = sw;
+        g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
+        g.piece_plane = h->piece_plane;
+        g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
+        AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
+      }
+    }
+    if (!tc_dw.empty()) {
+      Launch k(h, AGN_K_BACKWARD_DW, tc_flops, tc_bytes, launches);
+      agn::TcArgs t = tc_args(h, sw);
+      t.K = m; t.eta = eta;
+      AGN_TRY(agn::tc_backward_dw(tc_dw.data(), (int)tc_dw.size(), t, s, h->stream, h->split,
+                                  h->num_sms));
     }
   }
   return Status::Ok();
@@ -829,15 +859,10 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
     h->piece_plane = n * h->P_pad;
     AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));
     h->Hs.assign(h->L - 1, nullptr);
-    int maxh = 0;
-    for (int l = 0; l + 1 < h->L; ++l) {
+    for (int l = 0; l + 1 < h->L; ++l)
       AGN_TRY(dalloc_t(h, &h->Hs[l], (size_t)(3 * n * m * dims[l])));
-      if (l > 0) maxh = std::max(maxh, dims[l]);
-    }
-    maxh = std::max(maxh, dims[h->L - 1]);
-    h->dzs_plane = n * m * maxh;
-    AGN_TRY(dalloc_t(h, &h->dZs[0], (size_t)(3 * h->dzs_plane)));
-    AGN_TRY(dalloc_t(h, &h->dZs[1], (size_t)(3 * h->dzs_plane)));
+    h->dZp.assign(h->L, nullptr);
+    for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc_t(h, &h->dZp[l], (size_t)(3 * n * m * dims[l])));
   }
   AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
   AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));
@@ -846,12 +871,12 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->H.assign(h->L, nullptr);
   for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->H[l], (size_t)(n * m * dims[l]) * es));
   AGN_TRY(dalloc_t(h, &h->Z, (size_t)(n * m * dims[h->L])));
-  AGN_TRY(dalloc(h, &h->dz[0], (size_t)(n * m * h->maxd) * es));
-  AGN_TRY(dalloc(h, &h->dz[1], (size_t)(n * m * h->maxd) * es));
+  h->dZ.assign(h->L + 1, nullptr);
+  for (int l = 1; l <= h->L; ++l) AGN_TRY(dalloc(h, &h->dZ[l], (size_t)(n * m * dims[l]) * es));
   AGN_TRY(dalloc_t(h, &h->flag, 2));
   h->use_head = h->prec == AGN_PREC_BF16 ? agn::head_fits<bf16>(dims[h->L - 1], dims[h->L])
                                          : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
-  AGN_TRY(dalloc_t(h, &h->ce_partial, (size_t)(n * ceil_div(m, 8))));
+  AGN_TRY(dalloc_t(h, &h->ce_partial, (size_t)(n * ceil_div(m, agn::kHeadSamples))));
   AGN_TRY(dalloc_t(h, &h->head_counter, (size_t)n));
   AGN_TRY_CUDA(cudaMemsetAsync(h->head_counter, 0, (size_t)n * sizeof(int), h->stream));
   h->grid = agn::commit_grid(h->P_pad);

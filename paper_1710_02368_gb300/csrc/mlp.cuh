@@ -60,8 +60,9 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
                     cudaStream_t st, bf16* pieces = nullptr, int64_t plane = 0);
 
 // Output layer fused (mlp_head.cu): forward, softmax cross-entropy and dX of
-// layer L for d_L <= kHeadMaxClasses; one warp per sample.
+// layer L for d_L <= kHeadMaxClasses; kHeadSamples samples per block.
 constexpr int kHeadMaxClasses = 16;
+constexpr int kHeadSamples = 2;
 struct HeadArgs {
   const void* H;           // H_{L-1} [slots][m][K] (T)
   const void* W;           // replica operand base [n][ld_param] (T); W_L at woff, [C][K]
@@ -74,7 +75,7 @@ struct HeadArgs {
   void* dH;                // out: dZ_{L-1} [slots][m][K] (T)
   bf16* dH_pieces;         // fp32 T only: also its three exact bf16 pieces (planes
   int64_t dH_plane;        // dH_plane apart) for tensor-core GEMMs; null = no
-  float* ce_partial;       // [slots][ceil(m / 8)] scratch
+  float* ce_partial;       // [slots][ceil(m / kHeadSamples)] scratch
   int* counter;            // [slots], zero between launches
   float* loss_parts;
   const int* slot_commit;
@@ -83,6 +84,21 @@ struct HeadArgs {
 };
 template <typename T>
 Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st);
+// dW of the output layer with its local update and accumulation (mlp_head.cu).
+struct HeadDwArgs {
+  const void* H;           // H_{L-1} [slots][m][K] (T)
+  const void* dZL;         // dZ_L [slots][m][C] (T)
+  const int* slot_worker;
+  float* theta;            // fp32 master replicas [n][ld_param]
+  float* acc;              // accumulators [n][ld_param]
+  bf16* theta_b;           // bf16 copies (or piece 0 of three planes), or null
+  int64_t piece_plane;     // > 0: three piece planes this far apart
+  int64_t ld_param, woff, boff;
+  int K, C, m;
+  float eta;
+};
+template <typename T>
+Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st);
 // The fused head takes this output layer (classes and shared-memory staging fit).
 template <typename T>
 bool head_fits(int K, int C);

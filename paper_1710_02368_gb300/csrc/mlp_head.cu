@@ -3,20 +3,29 @@
 // and the output layer's dX, dZ_{L-1} = (dZ_L W_L) [h > 0].
 //
 // The output layer is narrow (d_L classes, at most 16 here), so a GEMM tile
-// would leave the GPU idle; instead one warp takes one sample.  A block first
-// stages W_L and its samples' input rows in shared memory with asynchronous
-// 16-byte copies (all in flight at once), then each warp's lanes stride over the d_{L-1}
-// inputs, keep one partial dot product per class and combine them with a
-// fixed shuffle tree, so results are deterministic.  The per-slot loss (mean
-// over the minibatch) is summed in a fixed order by the last block of the
-// slot to finish.
+// would leave the GPU idle.  Instead a block takes two samples with four warps
+// each: it first stages W_L and the two input rows in shared memory with
+// asynchronous 16-byte copies (all in flight at once); warp q of a sample then
+// takes the inputs k = 32 q + lane (mod 128), keeps one partial dot product
+// per class and folds it with a fixed shuffle tree; the four partials of a
+// class are added in a fixed order by every warp of the sample, so all four
+// hold the same z, softmax and dZ_L, and each writes its own inputs of
+// dZ_{L-1}.  Results are deterministic.  The per-slot loss (mean over the
+// minibatch) is summed in a fixed order by the last block of the slot to
+// finish.
+#include <mutex>
+#include <set>
+#include <utility>
+
 #include "mlp.cuh"
 
 namespace agn {
 
 namespace {
 
-constexpr int kHeadWarps = 8;   // samples per block
+constexpr int kHeadSplit = 4;                          // warps per sample
+constexpr int kHeadSmemCap = 200 * 1024;               // dynamic shared memory per block
+constexpr int kHeadThreads = 32 * kHeadSplit * kHeadSamples;
 
 __device__ __forceinline__ float cvt(float v) { return v; }
 __device__ __forceinline__ float cvt(bf16 v) { return __bfloat162float(v); }
@@ -54,45 +63,60 @@ __device__ __forceinline__ void stage_wait() {
 }
 
 template <typename T, int kMaxC>
-__global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a) {
+__global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   extern __shared__ __align__(16) uint8_t head_smem[];
+  __shared__ float red[kHeadSamples][kHeadSplit][kMaxC];
+  __shared__ float ce_s[kHeadSamples];
   const int z = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j0 = blockIdx.x * kHeadWarps;
+  const int sj = warp / kHeadSplit, q = warp % kHeadSplit;   // sample in block, input quarter
+  const int j0 = blockIdx.x * kHeadSamples;
   const int K = a.K, C = a.C, m = a.m;
-  const int nj = min(kHeadWarps, m - j0);
+  const int nj = min(kHeadSamples, m - j0);
   const int w = a.slot_worker[z];
   const int64_t Kp = (K + 7) / 8 * 8;   // padded row length in shared memory
   T* Ws = reinterpret_cast<T*>(head_smem);                  // [C][Kp]
-  T* Hs = Ws + (int64_t)C * Kp;                             // [kHeadWarps][Kp]
+  T* Hs = Ws + (int64_t)C * Kp;                             // [kHeadSamples][Kp]
   const T* Wg = static_cast<const T*>(a.W) + (int64_t)w * a.ld_param + a.woff;
   const T* Hg = static_cast<const T*>(a.H) + ((int64_t)z * m + j0) * K;
   for (int c = 0; c < C; ++c) stage(Ws + c * Kp, Wg + (int64_t)c * K, K);
-  for (int q = 0; q < nj; ++q) stage(Hs + q * Kp, Hg + (int64_t)q * K, K);
+  for (int r = 0; r < nj; ++r) stage(Hs + r * Kp, Hg + (int64_t)r * K, K);
   stage_wait();
   __syncthreads();
 
-  const float* bias = a.theta + (int64_t)w * a.ld_param + a.boff;
-  __shared__ float ce_warp[kHeadWarps];
-  float ce = 0.f;
-  const int j = j0 + warp;
-  if (warp < nj) {
-    const T* h = Hs + (int64_t)warp * Kp;
+  const bool active = sj < nj;
+  const T* h = Hs + (int64_t)sj * Kp;
+  constexpr int kStride = 32 * kHeadSplit;
+  if (active) {
     float part[kMaxC];
 #pragma unroll
     for (int c = 0; c < kMaxC; ++c) part[c] = 0.f;
-    for (int k = lane; k < K; k += 32) {
+    for (int k = 32 * q + lane; k < K; k += kStride) {
       const float hv = cvt(h[k]);
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
         if (c < C) part[c] = fmaf(hv, cvt(Ws[(int64_t)c * Kp + k]), part[c]);
     }
-    float zc[kMaxC];
 #pragma unroll
     for (int c = 0; c < kMaxC; ++c) {
       float v = part[c];
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (lane == 0) red[sj][q][c] = v;
+    }
+  }
+  __syncthreads();
+
+  float ce = 0.f;
+  if (active) {
+    const int j = j0 + sj;
+    const float* bias = a.theta + (int64_t)w * a.ld_param + a.boff;
+    float zc[kMaxC];
+#pragma unroll
+    for (int c = 0; c < kMaxC; ++c) {
+      float v = 0.f;
+#pragma unroll
+      for (int r = 0; r < kHeadSplit; ++r) v += red[sj][r][c < C ? c : 0];
       zc[c] = c < C ? v + bias[c] : -INFINITY;
     }
     const int y = a.yb[(int64_t)z * m + j];
@@ -114,15 +138,17 @@ __global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a)
       if (c == y) p -= 1.0f;
       g[c] = p * inv_m;
     }
-    T* dzl = static_cast<T*>(a.dZL) + ((int64_t)z * m + j) * C;
+    if (q == 0) {
+      T* dzl = static_cast<T*>(a.dZL) + ((int64_t)z * m + j) * C;
 #pragma unroll
-    for (int c = 0; c < kMaxC; ++c)
-      if (c < C && lane == c) dzl[c] = st_f<T>(g[c]);
+      for (int c = 0; c < kMaxC; ++c)
+        if (c < C && lane == c) dzl[c] = st_f<T>(g[c]);
+    }
     // dZ_{L-1}[j][k] = sum_c dZ_L[j][c] W_L[c][k], masked by h > 0 (W before its
     // update); skipped when the output layer is the only layer (dH null)
     T* dh = a.dH ? static_cast<T*>(a.dH) + ((int64_t)z * m + j) * K : nullptr;
     bf16* dp = a.dH_pieces ? a.dH_pieces + ((int64_t)z * m + j) * K : nullptr;
-    for (int k = lane; dh && k < K; k += 32) {
+    for (int k = 32 * q + lane; dh && k < K; k += kStride) {
       float v = 0.f;
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
@@ -138,11 +164,11 @@ __global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a)
       }
     }
   }
-  if (lane == 0) ce_warp[warp] = ce;
+  if (q == 0 && lane == 0) ce_s[sj] = ce;
   __syncthreads();
   if (threadIdx.x == 0) {
     float part = 0.f;
-    for (int q = 0; q < kHeadWarps; ++q) part += ce_warp[q];
+    for (int r = 0; r < kHeadSamples; ++r) part += ce_s[r];
     const int nblk = gridDim.x;
     a.ce_partial[(int64_t)z * nblk + blockIdx.x] = part;
     __threadfence();
@@ -159,28 +185,143 @@ __global__ void __launch_bounds__(kHeadWarps * 32) head_kernel(const HeadArgs a)
   }
 }
 
+// The output layer's weight gradient and local update:
+//   g[c][k] = sum_j dZ_L[j][c] h[j][k],   g_b[c] = sum_j dZ_L[j][c],
+//   theta_k -= eta g, a_k += g, and the bf16 copy (or its three pieces).
+// A block covers 32 inputs k of one slot; its four warps take the samples
+// j = w (mod 4), each lane one input, with dZ_L of the whole minibatch staged
+// in shared memory; the four partials are added in a fixed order.  The
+// bias gradient is summed (fixed order) by the first block of the slot.
+constexpr int kDwGroups = 4;
+template <typename T, int kMaxC>
+__global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArgs a) {
+  extern __shared__ __align__(16) uint8_t dw_smem[];
+  float* dz = reinterpret_cast<float*>(dw_smem);           // [m][C]
+  float* red = dz + (int64_t)a.m * a.C;                     // [kDwGroups][kMaxC][32]
+  const int z = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = a.K, C = a.C, m = a.m;
+  const T* dzg = static_cast<const T*>(a.dZL) + (int64_t)z * m * C;
+  for (int i = threadIdx.x; i < m * C; i += blockDim.x) dz[i] = cvt(dzg[i]);
+  __syncthreads();
+  const int w = a.slot_worker[z];
+  const int k = blockIdx.x * 32 + lane;
+  const T* hg = static_cast<const T*>(a.H) + (int64_t)z * m * K + k;
+  float g[kMaxC];
+#pragma unroll
+  for (int c = 0; c < kMaxC; ++c) g[c] = 0.f;
+  if (k < K) {
+    int j = warp;
+    for (; j + 3 * kDwGroups < m; j += 4 * kDwGroups) {   // four loads in flight
+      float hv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) hv[u] = cvt(hg[(int64_t)(j + u * kDwGroups) * K]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float* dzj = dz + (j + u * kDwGroups) * C;
+#pragma unroll
+        for (int c = 0; c < kMaxC; ++c)
+          if (c < C) g[c] = fmaf(dzj[c], hv[u], g[c]);
+      }
+    }
+    for (; j < m; j += kDwGroups) {
+      const float hv = cvt(hg[(int64_t)j * K]);
+      const float* dzj = dz + j * C;
+#pragma unroll
+      for (int c = 0; c < kMaxC; ++c)
+        if (c < C) g[c] = fmaf(dzj[c], hv, g[c]);
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < kMaxC; ++c) red[(warp * kMaxC + c) * 32 + lane] = g[c];
+  __syncthreads();
+  float* theta = a.theta + (int64_t)w * a.ld_param;
+  float* acc = a.acc + (int64_t)w * a.ld_param;
+  bf16* tb = a.theta_b ? a.theta_b + (int64_t)w * a.ld_param : nullptr;
+  auto update = [&](int64_t p, float gr) {
+    const float t = fmaf(-a.eta, gr, theta[p]);
+    theta[p] = t;
+    acc[p] += gr;
+    if (tb) {
+      if (a.piece_plane > 0) {
+        bf16 q0, q1, q2;
+        split3(t, q0, q1, q2);
+        tb[p] = q0;
+        tb[a.piece_plane + p] = q1;
+        tb[2 * a.piece_plane + p] = q2;
+      } else {
+        tb[p] = __float2bfloat16_rn(t);
+      }
+    }
+  };
+  if (warp == 0 && k < K) {
+    for (int c = 0; c < C; ++c) {
+      float s = 0.f;
+#pragma unroll
+      for (int r = 0; r < kDwGroups; ++r) s += red[(r * kMaxC + c) * 32 + lane];
+      update(a.woff + (int64_t)c * K + k, s);
+    }
+  }
+  if (blockIdx.x == 0 && warp == 1 && lane < C) {
+    float s = 0.f;
+    for (int j = 0; j < m; ++j) s += dz[j * C + lane];
+    update(a.boff + lane, s);
+  }
+}
+
 template <typename T>
 size_t head_smem_bytes(int K, int C) {
   const size_t kp = (size_t)(K + 7) / 8 * 8;
-  return (size_t)(C + kHeadWarps) * kp * sizeof(T);
+  return (size_t)(C + kHeadSamples) * kp * sizeof(T);
+}
+
+// Opt a kernel in to the full dynamic shared-memory budget of the fused
+// head (static shared memory comes on top, so the 48 KB default can fail
+// even below 48 KB of dynamic memory); once per kernel and device.
+Status allow_smem(const void* kern) {
+  static std::mutex mu;
+  static std::set<std::pair<int, const void*>> done;
+  int dev = 0;
+  AGN_TRY_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> lock(mu);
+  if (done.count({dev, kern})) return Status::Ok();
+  AGN_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kHeadSmemCap));
+  done.insert({dev, kern});
+  return Status::Ok();
 }
 
 }  // namespace
 
 template <typename T>
 bool head_fits(int K, int C) {
-  return C <= kHeadMaxClasses && head_smem_bytes<T>(K, C) <= 200 * 1024;
+  return C <= kHeadMaxClasses && head_smem_bytes<T>(K, C) <= (size_t)kHeadSmemCap;
 }
 
 template <typename T>
 Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st) {
   if (!head_fits<T>(a.K, a.C)) return Status::Err(AGN_E_UNSUPPORTED, "output layer too wide");
   const size_t smem = head_smem_bytes<T>(a.K, a.C);
-  auto kern = head_kernel<T, kHeadMaxClasses>;
-  if (smem > 48 * 1024)
-    AGN_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  dim3 grid((unsigned)ceil_div(a.m, kHeadWarps), (unsigned)slots);
-  kern<<<grid, kHeadWarps * 32, smem, st>>>(a);
+  // ten classes (the MNIST-shaped workloads) get an exact instantiation
+  auto kern = a.C == 10 ? head_kernel<T, 10> : head_kernel<T, kHeadMaxClasses>;
+  AGN_TRY(allow_smem(reinterpret_cast<const void*>(kern)));
+  dim3 grid((unsigned)ceil_div(a.m, kHeadSamples), (unsigned)slots);
+  kern<<<grid, kHeadThreads, smem, st>>>(a);
+  AGN_TRY_CUDA(cudaGetLastError());
+  return Status::Ok();
+}
+
+template <typename T>
+Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st) {
+  if (a.C > kHeadMaxClasses) return Status::Err(AGN_E_UNSUPPORTED, "output layer too wide");
+  const size_t smem = (size_t)a.m * a.C * sizeof(float) +
+                      (size_t)kDwGroups * kHeadMaxClasses * 32 * sizeof(float);
+  if (smem > (size_t)kHeadSmemCap)
+    return Status::Err(AGN_E_UNSUPPORTED, "minibatch too large for the output dW");
+  auto kern = a.C == 10 ? head_dw_kernel<T, 10> : head_dw_kernel<T, kHeadMaxClasses>;
+  AGN_TRY(allow_smem(reinterpret_cast<const void*>(kern)));
+  dim3 grid((unsigned)ceil_div(a.K, 32), (unsigned)slots);
+  kern<<<grid, 32 * kDwGroups, smem, st>>>(a);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -189,5 +330,7 @@ template bool head_fits<float>(int, int);
 template bool head_fits<bf16>(int, int);
 template Status head_forward_backward<float>(const HeadArgs&, int, cudaStream_t);
 template Status head_forward_backward<bf16>(const HeadArgs&, int, cudaStream_t);
+template Status head_backward_dw<float>(const HeadDwArgs&, int, cudaStream_t);
+template Status head_backward_dw<bf16>(const HeadDwArgs&, int, cudaStream_t);
 
 }  // namespace agn

@@ -62,13 +62,21 @@ Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& 
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
                       int slots, cudaStream_t st, bool split, int bn);
-// dW (mlp_tc_dw.cu, persistent, grid min(tiles, num_sms)): h_mn box {64, 64}
-// over H_{l-1}; dz_mn box {64, 64} over dZ_l; theta_map / acc_map fp32 maps
-// (d_{l-1}, d_l, n) over the layer's weights in the replicas and the
-// accumulators, box {128, 32}, no swizzle.
-Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn,
-                      const CUtensorMap& theta_map, const CUtensorMap& acc_map,
-                      const TcArgs& args, int slots, cudaStream_t st, bool split, int num_sms);
+// One hidden layer of a dW launch: h_mn box {64, 64} over H_{l-1}; dz_mn box
+// {64, 64} over dZ_l; theta / acc fp32 maps (d_{l-1}, d_l, n) over the
+// layer's weights in the replicas and the accumulators, box {128, 32}, no
+// swizzle.  M = d_{l-1}, N = d_l.
+struct DwLayerMaps {
+  const CUtensorMap *h_mn, *dz_mn, *theta, *acc;
+  int M, N;
+  int64_t woff, boff;
+};
+// dW with the local step and accumulation of the weights and biases of all
+// `layers` in one persistent launch (mlp_tc_dw.cu, grid min(tiles, num_sms)).
+// args supplies slot_worker, err, theta, acc, theta_b, ld_param, piece_plane,
+// eta and K = m; its per-layer fields are ignored.
+Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& args, int slots,
+                      cudaStream_t st, bool split, int num_sms);
 // The earlier non-persistent dW kernel (mlp_tc.cu): one 128 x BN tile per CTA,
 // two CTAs per SM, theta_k and a_k loaded into registers by the epilogue.
 Status tc_backward_dw_tiled(const CUtensorMap& h_mn, const CUtensorMap& dz_mn, const TcArgs& args,

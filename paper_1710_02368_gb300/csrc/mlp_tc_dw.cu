@@ -1,6 +1,7 @@
 // Kernel (b), weight-gradient half, on the tensor cores: D = H_{l-1}^T dZ_l
-// for every slot of a wave, fused with Algorithm 1's local step and
-// accumulation (theta_k -= eta g, a_k += g, and the bf16 copy of theta_k).
+// for every slot of a wave and every hidden layer in one launch, fused with
+// Algorithm 1's local step and accumulation (theta_k -= eta g, a_k += g, the
+// bf16 copy of theta_k) for the weights and the biases.
 //
 // The GEMM is tiny next to its epilogue (K = m samples against 18-22 bytes
 // of fp32 master weight and accumulator traffic per parameter), so the kernel
@@ -20,17 +21,26 @@
 //              at a time, takes theta_k and a_k from shared memory and stores
 //              the new values coalesced (32 consecutive k per feature row).
 //
-// The kernel is persistent (one CTA per SM: the rings take 192 KB of shared
-// memory and the accumulators all 512 TMEM columns); tiles (slot, feature
-// tile, input tile) are dealt out round-robin with input tiles fastest, so
-// neighbouring CTAs stream neighbouring parts of the same weight rows.
-// Every wait is bounded (2 s of global time): on expiry the CTA sets *err,
-// stops issuing, drains its own copies and MMAs (bounded), frees TMEM and
-// returns.
+// Bias gradients ride along: a layer with d_{l-1} = M inputs gets M + 1 GEMM
+// rows, row M of H^T being all ones (written into the staged A tile by the
+// MMA warp, over the zero fill of the out-of-range row), so D[M][f] =
+// sum_j dZ_l[j][f] = g_b[f]; the epilogue thread of that row updates b_l and
+// its accumulator, whose 32 values per chunk the producer copies in with the
+// chunk.
+//
+// The kernel is persistent (one CTA per SM: the rings take 194 KB of shared
+// memory and the accumulators all 512 TMEM columns); tiles (layer, slot,
+// feature tile, input tile) are dealt out round-robin with input tiles
+// fastest, so neighbouring CTAs stream neighbouring parts of the same weight
+// rows.  Every wait is bounded (2 s of global time): on expiry the CTA sets
+// *err, stops issuing, drains its own copies and MMAs (bounded), frees TMEM
+// and returns.
 #include <cuda.h>
 
 #include <algorithm>
+#include <cstring>
 #include <mutex>
+#include <set>
 
 #include "mlp.cuh"
 #include "mlp_tc.cuh"
@@ -46,6 +56,8 @@ constexpr int kBK = 64;                        // K (samples) per stage
 constexpr int kABytes = 128 * 128;             // A box pair: 128 inputs x 64 samples, bf16
 constexpr int kCF = 32;                        // output features per parameter chunk
 constexpr int kChunkBytes = kCF * 128 * 4;     // one fp32 chunk: 32 rows x 128 inputs
+constexpr int kBiasBytes = 2 * kCF * 4;       // b_l and its accumulator for one chunk
+constexpr int kSlotBytes = 2 * kChunkBytes + kBiasBytes;   // one ring slot
 constexpr int kRing = 3;                       // chunks (theta and a) in flight
 constexpr uint64_t kWaitNs = 2000000000ull;    // 2 s
 
@@ -59,7 +71,7 @@ struct DwCfg {
   static constexpr uint32_t kTmemCols = 2 * kAccCols;
   static constexpr int kChunks = BN / kCF;
   static constexpr size_t kRingOff = (size_t)kStages * kStageBytes;
-  static constexpr size_t kBarOff = kRingOff + (size_t)kRing * 2 * kChunkBytes;
+  static constexpr size_t kBarOff = kRingOff + (size_t)kRing * kSlotBytes;
   static constexpr size_t kSmem = kBarOff + 256 + 1024;   // barriers, alignment slack
 };
 
@@ -67,23 +79,50 @@ struct DwCfg {
 __device__ __forceinline__ int pair_a(int q) { return q == 2 || q == 4 ? 1 : q == 5 ? 2 : 0; }
 __device__ __forceinline__ int pair_b(int q) { return q == 1 || q == 4 ? 1 : q == 3 ? 2 : 0; }
 
-struct TileIdx {
-  int m_tile, n_tile, slot;
+constexpr int kMaxDwLayers = 8;   // layers per launch (more are split into launches)
+struct DwLayer {
+  int M, N;          // inputs d_{l-1}, outputs d_l
+  int mt, nt;        // input tiles (M / 128 + 1: the last holds the bias row), feature tiles
+  int tile_begin;    // first tile of this layer in the launch
+  int64_t woff, boff;
 };
-__device__ __forceinline__ TileIdx decode(int t, int mt, int nt) {
+struct DwBatch {
+  CUtensorMap a[kMaxDwLayers], b[kMaxDwLayers], th[kMaxDwLayers], ac[kMaxDwLayers];
+  DwLayer layer[kMaxDwLayers];
+  int n_layers, total_tiles;
+};
+
+struct TileIdx {
+  int layer, m_tile, n_tile, slot;
+};
+__device__ __forceinline__ TileIdx decode(const DwBatch& B, int t) {
+  int i = 0;
+  while (i + 1 < B.n_layers && t >= B.layer[i + 1].tile_begin) ++i;
+  const DwLayer& L = B.layer[i];
+  const int u = t - L.tile_begin;
   TileIdx r;
-  r.m_tile = t % mt;
-  const int rest = t / mt;
-  r.n_tile = rest % nt;
-  r.slot = rest / nt;
+  r.layer = i;
+  r.m_tile = u % L.mt;
+  const int rest = u / L.mt;
+  r.n_tile = rest % L.nt;
+  r.slot = rest / L.nt;
   return r;
+}
+
+// Row r (< 128) of H^T set to one in every sample of an A stage: two 64-input
+// boxes, 128-byte rows (one per sample), 16-byte chunks swizzled by row % 8.
+__device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
+  uint8_t* box = sa + (r >> 6) * 8192;
+  const int i = r & 63;
+  for (int j = 0; j < kBK; ++j) {
+    const int off = j * 128 + ((((i >> 3) ^ (j & 7))) << 4) + (i & 7) * 2;
+    *reinterpret_cast<uint16_t*>(box + off) = 0x3F80;   // bf16 1.0
+  }
 }
 
 template <int BN, int kSplit, int kStages>
 __global__ void __launch_bounds__(kThreads, 1)
-tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-             const __grid_constant__ CUtensorMap tmTheta,
-             const __grid_constant__ CUtensorMap tmAcc, const TcArgs args, int slots) {
+tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   using Cfg = DwCfg<BN, kSplit, kStages>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -104,9 +143,7 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
   if (s_skip != 0) return;   // an earlier launch gave up: uniform across the CTA
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int M = args.M, N = args.N;
-  const int mt = (M + 127) / 128, nt = (N + BN - 1) / BN;
-  const int T = mt * nt * slots;
+  const int T = B.total_tiles;
   const int KT = (args.K + kBK - 1) / kBK;
 
   if (threadIdx.x == 0) {
@@ -125,10 +162,12 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
     tc::mbar_init(fin, 1);
     *abort_flag = 0;
     tc::fence_mbar_init();
-    tc::tma_prefetch_desc(&tmA);
-    tc::tma_prefetch_desc(&tmB);
-    tc::tma_prefetch_desc(&tmTheta);
-    tc::tma_prefetch_desc(&tmAcc);
+    for (int i = 0; i < B.n_layers; ++i) {
+      tc::tma_prefetch_desc(&B.a[i]);
+      tc::tma_prefetch_desc(&B.b[i]);
+      tc::tma_prefetch_desc(&B.th[i]);
+      tc::tma_prefetch_desc(&B.ac[i]);
+    }
   }
   if (warp == 1) {
     tc::tmem_alloc(tmem_holder, Cfg::kTmemCols);
@@ -144,7 +183,10 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
       uint32_t ml = 0, ch = 0;   // stage fills and chunk fills issued
       bool ok = true;
       for (int t = blockIdx.x; ok && t < T; t += gridDim.x) {
-        const TileIdx ti = decode(t, mt, nt);
+        const TileIdx ti = decode(B, t);
+        const DwLayer& L = B.layer[ti.layer];
+        const CUtensorMap* tmA = &B.a[ti.layer];
+        const CUtensorMap* tmB = &B.b[ti.layer];
         const int worker = args.slot_worker[ti.slot];
         for (int kt = 0; kt < KT; ++kt) {
           const int s = ml % kStages;
@@ -161,26 +203,27 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
             uint8_t* sa = sa0 + p * kABytes;
             uint8_t* sb = sb0 + p * Cfg::kBBytes;
             if (kSplit == 1) {
-              tc::tma_load_3d(sa, &tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
-              tc::tma_load_3d(sa + 8192, &tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
+              tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
+              tc::tma_load_3d(sa + 8192, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
 #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_3d(sb + c * 8192, &tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                tc::tma_load_3d(sb + c * 8192, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
                                 ti.slot);
             } else {
-              tc::tma_load_4d(sa, &tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
-              tc::tma_load_4d(sa + 8192, &tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
+              tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
+              tc::tma_load_4d(sa + 8192, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
                               p);
 #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_4d(sb + c * 8192, &tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                tc::tma_load_4d(sb + c * 8192, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
                                 ti.slot, p);
             }
           }
           ++ml;
         }
         if (!ok) break;
-        const int nch = min(Cfg::kChunks, (N - ti.n_tile * BN + kCF - 1) / kCF);
+        const bool bias_tile = ti.m_tile == L.M / 128;
+        const int nch = min(Cfg::kChunks, (L.N - ti.n_tile * BN + kCF - 1) / kCF);
         for (int c = 0; c < nch; ++c) {
           const int r = ch % kRing;
           if (ch >= kRing &&
@@ -188,11 +231,18 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
             ok = false;
             break;
           }
-          uint8_t* dst = smem + Cfg::kRingOff + (size_t)r * 2 * kChunkBytes;
+          uint8_t* dst = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
           const int f0 = ti.n_tile * BN + c * kCF;
-          tc::mbar_arrive_expect_tx(&cfull[r], 2 * kChunkBytes);
-          tc::tma_load_3d(dst, &tmTheta, &cfull[r], ti.m_tile * 128, f0, worker);
-          tc::tma_load_3d(dst + kChunkBytes, &tmAcc, &cfull[r], ti.m_tile * 128, f0, worker);
+          tc::mbar_arrive_expect_tx(&cfull[r], 2 * kChunkBytes + (bias_tile ? kBiasBytes : 0));
+          tc::tma_load_3d(dst, &B.th[ti.layer], &cfull[r], ti.m_tile * 128, f0, worker);
+          tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
+                          worker);
+          if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
+            const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
+            tc::bulk_load(dst + 2 * kChunkBytes, args.theta + pb, kBiasBytes / 2, &cfull[r]);
+            tc::bulk_load(dst + 2 * kChunkBytes + kBiasBytes / 2, args.acc + pb, kBiasBytes / 2,
+                          &cfull[r]);
+          }
           ++ch;
         }
       }
@@ -212,6 +262,8 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
       bool ok = true;
       int it = 0;
       for (int t = blockIdx.x; ok && t < T; t += gridDim.x, ++it) {
+        const TileIdx ti = decode(B, t);
+        const DwLayer& L = B.layer[ti.layer];
         const int b = it & 1;
         if (it >= 2 && !tc::wait_or_abort(&tempty[b], ((it >> 1) - 1) & 1, abort_flag, kWaitNs)) {
           ok = false;
@@ -219,6 +271,7 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
         }
         tc::tc_fence_after();
         const uint32_t dbase = tmem + (uint32_t)b * Cfg::kAccCols;
+        const int ones_row = L.M - ti.m_tile * 128;   // < 128 on the bias tile
         for (int kt = 0; kt < KT; ++kt) {
           const int s = ml % kStages;
           if (!tc::wait_or_abort(&full[s], (ml / kStages) & 1, abort_flag, kWaitNs)) {
@@ -226,6 +279,10 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
             break;
           }
           tc::tc_fence_after();
+          if (ones_row < 128) {   // piece 0 of the out-of-range row := 1 (pieces 1, 2 stay 0)
+            write_ones_row(smem + s * Cfg::kStageBytes, ones_row);
+            tc::fence_proxy_async_smem();
+          }
           const uint32_t sa0 = tc::smem_u32(smem + s * Cfg::kStageBytes);
           const uint32_t sb0 = sa0 + kSplit * kABytes;
           constexpr int kPairs = kSplit == 1 ? 1 : 6;
@@ -263,8 +320,25 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
     uint32_t ch = 0;
     bool ok = true;
     int it = 0;
+    auto update = [&](float* theta, float* acc, bf16* tb, int64_t p, float gr, float th,
+                      float ac) {
+      const float tn = fmaf(-eta, gr, th);
+      theta[p] = tn;
+      acc[p] = ac + gr;
+      if (kSplit == 1) {
+        tb[p] = __float2bfloat16_rn(tn);
+      } else {
+        bf16 q0, q1, q2;
+        split3(tn, q0, q1, q2);
+        tb[p] = q0;
+        tb[args.piece_plane + p] = q1;
+        tb[2 * args.piece_plane + p] = q2;
+      }
+    };
     for (int t = blockIdx.x; ok && t < T; t += gridDim.x, ++it) {
-      const TileIdx ti = decode(t, mt, nt);
+      const TileIdx ti = decode(B, t);
+      const DwLayer& L = B.layer[ti.layer];
+      const int M = L.M, N = L.N;
       const int worker = args.slot_worker[ti.slot];
       const int b = it & 1;
       // waits are warp-uniform: a lane that gave up takes its whole warp out
@@ -274,12 +348,12 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
       if (!ok) break;
       tc::tc_fence_after();
       const int row = ti.m_tile * 128 + 32 * g + lane;   // input index k of this thread
-      const bool row_ok = row < M;
+      const bool row_ok = row < M, bias_row = row == M;
       const uint32_t tbase = tmem + ((uint32_t)(32 * g) << 16) + (uint32_t)b * Cfg::kAccCols;
-      const int64_t wbase = (int64_t)worker * args.ld_param + args.woff + row;
-      float* theta = args.theta + wbase;
-      float* acc = args.acc + wbase;
-      bf16* tb = args.theta_b + wbase;
+      const int64_t rbase = (int64_t)worker * args.ld_param;
+      float* theta = args.theta + rbase;
+      float* acc = args.acc + rbase;
+      bf16* tb = args.theta_b + rbase;
       const int nch = min(Cfg::kChunks, (N - ti.n_tile * BN + kCF - 1) / kCF);
       for (int c = 0; c < nch; ++c) {
         const int r = ch % kRing;
@@ -298,31 +372,26 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
         ok = __all_sync(0xffffffffu,
                         tc::wait_or_abort(&cfull[r], (ch / kRing) & 1, abort_flag, kWaitNs));
         if (!ok) break;
-        const float* sT = reinterpret_cast<const float*>(smem + Cfg::kRingOff +
-                                                         (size_t)r * 2 * kChunkBytes) +
-                          32 * g + lane;
-        const float* sA = sT + kChunkBytes / 4;
+        const uint8_t* slot = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
         const int f0 = ti.n_tile * BN + c * kCF;
-        const int nf = row_ok ? min(kCF, N - f0) : 0;
+        if (row_ok) {
+          const float* sT = reinterpret_cast<const float*>(slot) + 32 * g + lane;
+          const float* sA = sT + kChunkBytes / 4;
+          const int nf = min(kCF, N - f0);
+          const int64_t pw = L.woff + (int64_t)f0 * M + row;
 #pragma unroll
-        for (int i = 0; i < kCF; ++i) {
-          if (i < nf) {
-            const float gr = __uint_as_float(v[i]);
-            const float tn = fmaf(-eta, gr, sT[i * 128]);
-            const float an = sA[i * 128] + gr;
-            const int64_t p = (int64_t)(f0 + i) * M;
-            theta[p] = tn;
-            acc[p] = an;
-            if (kSplit == 1) {
-              tb[p] = __float2bfloat16_rn(tn);
-            } else {
-              bf16 q0, q1, q2;
-              split3(tn, q0, q1, q2);
-              tb[p] = q0;
-              tb[args.piece_plane + p] = q1;
-              tb[2 * args.piece_plane + p] = q2;
-            }
-          }
+          for (int i = 0; i < kCF; ++i)
+            if (i < nf)
+              update(theta, acc, tb, pw + (int64_t)i * M, __uint_as_float(v[i]), sT[i * 128],
+                     sA[i * 128]);
+        } else if (bias_row) {
+          const float* sTb = reinterpret_cast<const float*>(slot + 2 * kChunkBytes);
+          const float* sAb = sTb + kCF;
+          const int nf = min(kCF, N - f0);
+          const int64_t pb = L.boff + f0;
+#pragma unroll
+          for (int i = 0; i < kCF; ++i)
+            if (i < nf) update(theta, acc, tb, pb + i, __uint_as_float(v[i]), sTb[i], sAb[i]);
         }
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&cempty[r]);
@@ -343,39 +412,65 @@ tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CU
 }
 
 template <int BN, int kSplit, int kStages>
-Status launch_dw(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& th,
-                 const CUtensorMap& ac, const TcArgs& args, int slots, int num_sms,
-                 cudaStream_t st) {
+Status launch_dw(const DwBatch& batch, const TcArgs& args, int num_sms, cudaStream_t st) {
   using Cfg = DwCfg<BN, kSplit, kStages>;
   static_assert(Cfg::kSmem <= 232448, "shared memory");
   static_assert(Cfg::kSmem > 232448 / 2, "one CTA per SM (all 512 TMEM columns)");
   static_assert(Cfg::kTmemCols == 512, "TMEM columns");
   auto kern = tc_dw_kernel<BN, kSplit, kStages>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)Cfg::kSmem);
-  });
-  AGN_TRY_CUDA(attr_err);
-  const int64_t tiles = (int64_t)ceil_div(args.M, 128) * ceil_div(args.N, BN) * slots;
-  if (tiles <= 0) return Status::Ok();
-  if (tiles > INT32_MAX) return Status::Err(AGN_E_UNSUPPORTED, "dW tile count overflows");
-  const int grid = (int)std::min<int64_t>(tiles, num_sms);
-  kern<<<grid, kThreads, Cfg::kSmem, st>>>(a, b, th, ac, args, slots);
+  static std::mutex mu;
+  static std::set<int> done;
+  {
+    int dev = 0;
+    AGN_TRY_CUDA(cudaGetDevice(&dev));
+    std::lock_guard<std::mutex> lock(mu);
+    if (!done.count(dev)) {
+      AGN_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)Cfg::kSmem));
+      done.insert(dev);
+    }
+  }
+  if (batch.total_tiles <= 0) return Status::Ok();
+  const int grid = std::min(batch.total_tiles, num_sms);
+  kern<<<grid, kThreads, Cfg::kSmem, st>>>(batch, args);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
 
 }  // namespace
 
-Status tc_backward_dw(const CUtensorMap& h_mn, const CUtensorMap& dz_mn,
-                      const CUtensorMap& theta_map, const CUtensorMap& acc_map,
-                      const TcArgs& args, int slots, cudaStream_t st, bool split, int num_sms) {
-  if (split)
-    return launch_dw<kTcDwBNSplit, 3, 1>(h_mn, dz_mn, theta_map, acc_map, args, slots, num_sms,
-                                         st);
-  return launch_dw<kTcDwBN, 1, 2>(h_mn, dz_mn, theta_map, acc_map, args, slots, num_sms, st);
+Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& args, int slots,
+                      cudaStream_t st, bool split, int num_sms) {
+  const int bn = split ? kTcDwBNSplit : kTcDwBN;
+  for (int l0 = 0; l0 < n_layers; l0 += kMaxDwLayers) {
+    DwBatch batch;
+    std::memset(&batch, 0, sizeof(batch));
+    int64_t tiles = 0;
+    batch.n_layers = std::min(kMaxDwLayers, n_layers - l0);
+    for (int i = 0; i < batch.n_layers; ++i) {
+      const DwLayerMaps& d = layers[l0 + i];
+      if (d.M <= 0 || d.N <= 0) return Status::Err(AGN_E_INVALID, "empty dW layer");
+      batch.a[i] = *d.h_mn;
+      batch.b[i] = *d.dz_mn;
+      batch.th[i] = *d.theta;
+      batch.ac[i] = *d.acc;
+      DwLayer& L = batch.layer[i];
+      L.M = d.M;
+      L.N = d.N;
+      L.woff = d.woff;
+      L.boff = d.boff;
+      L.mt = d.M / 128 + 1;          // rows 0 .. M, row M the bias
+      L.nt = (d.N + bn - 1) / bn;
+      L.tile_begin = (int)tiles;
+      tiles += (int64_t)L.mt * L.nt * slots;
+      if (tiles > INT32_MAX) return Status::Err(AGN_E_UNSUPPORTED, "dW tile count overflows");
+    }
+    batch.total_tiles = (int)tiles;
+    Status r = split ? launch_dw<kTcDwBNSplit, 3, 1>(batch, args, num_sms, st)
+                     : launch_dw<kTcDwBN, 1, 2>(batch, args, num_sms, st);
+    if (!r.ok()) return r;
+  }
+  return Status::Ok();
 }
 
 }  // namespace agn
