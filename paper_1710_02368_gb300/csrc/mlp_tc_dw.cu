@@ -16,19 +16,20 @@
 //   warp 1     MMA issuer (one thread) and TMEM owner.  Two accumulators
 //              (double buffer): the GEMM of the next tile runs while the
 //              epilogue drains this one.
-//   warps 2-5  epilogue.  Warp w reads TMEM lanes 32 (w % 4) .. + 31, i.e.
-//              32 consecutive inputs k of the tile, one chunk of 32 features
-//              at a time, takes theta_k and a_k from shared memory and stores
-//              the new values coalesced (32 consecutive k per feature row).
+//   warps 2-9  epilogue.  Warp w reads TMEM lanes 32 (w % 4) .. + 31, i.e.
+//              32 consecutive inputs k of the tile, and 16 of the 32 features
+//              of a chunk; it transposes them through shared memory so that
+//              each lane updates four consecutive inputs of a feature at a
+//              time (16-byte reads of theta_k and a_k from the chunk, 16-byte
+//              coalesced stores).
 //
 // Bias gradients ride along: a layer with d_{l-1} = M inputs gets M + 1 GEMM
 // rows, row M of H^T being all ones (written into the staged A tile by the
 // MMA warp, over the zero fill of the out-of-range row), so D[M][f] =
-// sum_j dZ_l[j][f] = g_b[f]; the epilogue thread of that row updates b_l and
-// its accumulator, whose 32 values per chunk the producer copies in with the
-// chunk.
+// sum_j dZ_l[j][f] = g_b[f]; the epilogue updates b_l and its accumulator
+// from that row, with their 32 values per chunk copied in by the producer.
 //
-// The kernel is persistent (one CTA per SM: the rings take 194 KB of shared
+// The kernel is persistent (one CTA per SM: the rings take 210 KB of shared
 // memory and the accumulators all 512 TMEM columns); tiles (layer, slot,
 // feature tile, input tile) are dealt out round-robin with input tiles
 // fastest, so neighbouring CTAs stream neighbouring parts of the same weight
@@ -50,7 +51,8 @@ namespace agn {
 
 namespace {
 
-constexpr int kWarps = 6;
+constexpr int kWarps = 10;
+constexpr int kEpiWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kBK = 64;                        // K (samples) per stage
 constexpr int kABytes = 128 * 128;             // A box pair: 128 inputs x 64 samples, bf16
@@ -71,9 +73,34 @@ struct DwCfg {
   static constexpr uint32_t kTmemCols = 2 * kAccCols;
   static constexpr int kChunks = BN / kCF;
   static constexpr size_t kRingOff = (size_t)kStages * kStageBytes;
-  static constexpr size_t kBarOff = kRingOff + (size_t)kRing * kSlotBytes;
+  static constexpr size_t kGOff = kRingOff + (size_t)kRing * kSlotBytes;   // gradient staging
+  static constexpr size_t kBarOff = kGOff + (size_t)kEpiWarps * 16 * 32 * 4;
   static constexpr size_t kSmem = kBarOff + 256 + 1024;   // barriers, alignment slack
 };
+
+// Four floats as four bf16 (round to nearest even), packed for one 8-byte store.
+__device__ __forceinline__ uint2 bf16x4(const float (&x)[4]) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(x[0], x[1]);
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(x[2], x[3]);
+  return make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+}
+// The three exact bf16 pieces of four floats (split3 of each), packed.
+__device__ __forceinline__ void split3_x4(const float (&x)[4], uint2& q0, uint2& q1, uint2& q2) {
+  float r[4];
+  q0 = bf16x4(x);
+  const __nv_bfloat162* p0 = reinterpret_cast<const __nv_bfloat162*>(&q0);
+  r[0] = __fsub_rn(x[0], __low2float(p0[0]));
+  r[1] = __fsub_rn(x[1], __high2float(p0[0]));
+  r[2] = __fsub_rn(x[2], __low2float(p0[1]));
+  r[3] = __fsub_rn(x[3], __high2float(p0[1]));
+  q1 = bf16x4(r);
+  const __nv_bfloat162* p1 = reinterpret_cast<const __nv_bfloat162*>(&q1);
+  r[0] = __fsub_rn(r[0], __low2float(p1[0]));
+  r[1] = __fsub_rn(r[1], __high2float(p1[0]));
+  r[2] = __fsub_rn(r[2], __low2float(p1[1]));
+  r[3] = __fsub_rn(r[3], __high2float(p1[1]));
+  q2 = bf16x4(r);
+}
 
 // Piece pairs (i, j), i + j <= 2, of the split product (pair 0 = a0 b0).
 __device__ __forceinline__ int pair_a(int q) { return q == 2 || q == 4 ? 1 : q == 5 ? 2 : 0; }
@@ -130,9 +157,9 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Cfg::kBarOff);
   uint64_t* empty = full + kStages;
   uint64_t* cfull = empty + kStages;     // parameter chunk landed
-  uint64_t* cempty = cfull + kRing;      // parameter chunk consumed (4 epilogue warps)
+  uint64_t* cempty = cfull + kRing;      // parameter chunk consumed (8 epilogue warps)
   uint64_t* tfull = cempty + kRing;      // accumulator b complete
-  uint64_t* tempty = tfull + 2;          // accumulator b drained (4 epilogue warps)
+  uint64_t* tempty = tfull + 2;          // accumulator b drained (8 epilogue warps)
   uint64_t* fin = tempty + 2;            // MMA drain on abort
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(fin + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
@@ -153,11 +180,11 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
     }
     for (int r = 0; r < kRing; ++r) {
       tc::mbar_init(&cfull[r], 1);
-      tc::mbar_init(&cempty[r], 4);
+      tc::mbar_init(&cempty[r], kEpiWarps);
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(&tfull[b], 1);
-      tc::mbar_init(&tempty[b], 4);
+      tc::mbar_init(&tempty[b], kEpiWarps);
     }
     tc::mbar_init(fin, 1);
     *abort_flag = 0;
@@ -314,27 +341,18 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
       }
     }
   } else {
-    // epilogue warps 2..5 -> TMEM lane quadrants 2, 3, 0, 1
-    const int g = warp & 3;
+    // epilogue warps 2..9: warp w reads TMEM lane quadrant w % 4 (inputs
+    // 32 (w % 4) .. + 31 of the tile) and columns 16 hf .. + 15 of each chunk,
+    // hf = (w - 2) / 4.  It stages its 16 x 32 gradients in shared memory
+    // (feature-major), then each lane updates four consecutive inputs of four
+    // features with 16-byte shared loads and 16-byte global stores.
+    const int g = warp & 3, hf = (warp - 2) >> 2;
+    float* gS = reinterpret_cast<float*>(smem + Cfg::kGOff) + (warp - 2) * (16 * 32);
     const float eta = args.eta;
     uint32_t ch = 0;
     bool ok = true;
     int it = 0;
-    auto update = [&](float* theta, float* acc, bf16* tb, int64_t p, float gr, float th,
-                      float ac) {
-      const float tn = fmaf(-eta, gr, th);
-      theta[p] = tn;
-      acc[p] = ac + gr;
-      if (kSplit == 1) {
-        tb[p] = __float2bfloat16_rn(tn);
-      } else {
-        bf16 q0, q1, q2;
-        split3(tn, q0, q1, q2);
-        tb[p] = q0;
-        tb[args.piece_plane + p] = q1;
-        tb[2 * args.piece_plane + p] = q2;
-      }
-    };
+    const int k4 = (lane & 7) * 4, i0 = lane >> 3;   // phase-2 position of this lane
     for (int t = blockIdx.x; ok && t < T; t += gridDim.x, ++it) {
       const TileIdx ti = decode(B, t);
       const DwLayer& L = B.layer[ti.layer];
@@ -347,9 +365,11 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
                                                       kWaitNs));
       if (!ok) break;
       tc::tc_fence_after();
-      const int row = ti.m_tile * 128 + 32 * g + lane;   // input index k of this thread
-      const bool row_ok = row < M, bias_row = row == M;
-      const uint32_t tbase = tmem + ((uint32_t)(32 * g) << 16) + (uint32_t)b * Cfg::kAccCols;
+      const int k0 = ti.m_tile * 128 + 32 * g;            // first input of this quadrant
+      const bool quad_ok = k0 + k4 < M;                   // M % 8 == 0: all four or none
+      const int kb = M - k0;                              // bias row, if 0 <= kb < 32
+      const uint32_t tbase = tmem + ((uint32_t)(32 * g) << 16) + (uint32_t)b * Cfg::kAccCols +
+                             (uint32_t)(16 * hf);
       const int64_t rbase = (int64_t)worker * args.ld_param;
       float* theta = args.theta + rbase;
       float* acc = args.acc + rbase;
@@ -357,41 +377,75 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
       const int nch = min(Cfg::kChunks, (N - ti.n_tile * BN + kCF - 1) / kCF);
       for (int c = 0; c < nch; ++c) {
         const int r = ch % kRing;
-        uint32_t v[32];
-        tc::tmem_ld_32x32b_x32(tbase + (uint32_t)(c * kCF), v);
+        uint32_t v[16];
+        tc::tmem_ld_32x32b_x16(tbase + (uint32_t)(c * kCF), v);
         if (kSplit == 3) {
-          uint32_t v2[32];
-          tc::tmem_ld_32x32b_x32(tbase + (uint32_t)(BN + c * kCF), v2);
+          uint32_t v2[16];
+          tc::tmem_ld_32x32b_x16(tbase + (uint32_t)(BN + c * kCF), v2);
           tc::tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
+          for (int i = 0; i < 16; ++i)
             v[i] = __float_as_uint(__fadd_rn(__uint_as_float(v[i]), __uint_as_float(v2[i])));
         } else {
           tc::tmem_ld_wait();
         }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) gS[i * 32 + lane] = __uint_as_float(v[i]);
         ok = __all_sync(0xffffffffu,
                         tc::wait_or_abort(&cfull[r], (ch / kRing) & 1, abort_flag, kWaitNs));
         if (!ok) break;
+        __syncwarp();
         const uint8_t* slot = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
-        const int f0 = ti.n_tile * BN + c * kCF;
-        if (row_ok) {
-          const float* sT = reinterpret_cast<const float*>(slot) + 32 * g + lane;
-          const float* sA = sT + kChunkBytes / 4;
-          const int nf = min(kCF, N - f0);
-          const int64_t pw = L.woff + (int64_t)f0 * M + row;
+        const int fbase = ti.n_tile * BN + c * kCF + 16 * hf;   // first feature of this warp
+        if (quad_ok) {
 #pragma unroll
-          for (int i = 0; i < kCF; ++i)
-            if (i < nf)
-              update(theta, acc, tb, pw + (int64_t)i * M, __uint_as_float(v[i]), sT[i * 128],
-                     sA[i * 128]);
-        } else if (bias_row) {
+          for (int u = 0; u < 4; ++u) {
+            const int i = i0 + 4 * u;                           // feature fbase + i
+            if (fbase + i < N) {
+              const float4 gv = *reinterpret_cast<const float4*>(gS + i * 32 + k4);
+              const int so = (16 * hf + i) * 128 + 32 * g + k4;   // in the fp32 chunks
+              const float4 tv = *reinterpret_cast<const float4*>(
+                  reinterpret_cast<const float*>(slot) + so);
+              const float4 av = *reinterpret_cast<const float4*>(
+                  reinterpret_cast<const float*>(slot + kChunkBytes) + so);
+              float tn[4];
+              tn[0] = fmaf(-eta, gv.x, tv.x);
+              tn[1] = fmaf(-eta, gv.y, tv.y);
+              tn[2] = fmaf(-eta, gv.z, tv.z);
+              tn[3] = fmaf(-eta, gv.w, tv.w);
+              const float4 an = make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w);
+              const int64_t p = L.woff + (int64_t)(fbase + i) * M + k0 + k4;
+              *reinterpret_cast<float4*>(theta + p) = make_float4(tn[0], tn[1], tn[2], tn[3]);
+              *reinterpret_cast<float4*>(acc + p) = an;
+              if (kSplit == 1) {
+                *reinterpret_cast<uint2*>(tb + p) = bf16x4(tn);
+              } else {
+                uint2 q0, q1, q2;
+                split3_x4(tn, q0, q1, q2);
+                *reinterpret_cast<uint2*>(tb + p) = q0;
+                *reinterpret_cast<uint2*>(tb + args.piece_plane + p) = q1;
+                *reinterpret_cast<uint2*>(tb + 2 * args.piece_plane + p) = q2;
+              }
+            }
+          }
+        }
+        if (kb >= 0 && kb < 32 && lane < 16 && fbase + lane < N) {   // bias row: b_l[f]
           const float* sTb = reinterpret_cast<const float*>(slot + 2 * kChunkBytes);
           const float* sAb = sTb + kCF;
-          const int nf = min(kCF, N - f0);
-          const int64_t pb = L.boff + f0;
-#pragma unroll
-          for (int i = 0; i < kCF; ++i)
-            if (i < nf) update(theta, acc, tb, pb + i, __uint_as_float(v[i]), sTb[i], sAb[i]);
+          const float gb = gS[lane * 32 + kb];
+          const int64_t pb = L.boff + fbase + lane;
+          const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
+          theta[pb] = tn;
+          acc[pb] = sAb[16 * hf + lane] + gb;
+          if (kSplit == 1) {
+            tb[pb] = __float2bfloat16_rn(tn);
+          } else {
+            bf16 q0, q1, q2;
+            split3(tn, q0, q1, q2);
+            tb[pb] = q0;
+            tb[args.piece_plane + pb] = q1;
+            tb[2 * args.piece_plane + pb] = q2;
+          }
         }
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&cempty[r]);
