@@ -89,10 +89,11 @@ struct agn_handle {
   int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
-    CUtensorMap h_k64, dz_k64;   // 64-row boxes: 64-wide column tiles for small waves
     CUtensorMap theta, acc;      // fp32 W_l of every replica / accumulator, box {128, 32}
   };
   int num_sms = 148;
+  float* tc_part = nullptr;     // split-K partial sums: [SMs][BN <= 256][128]
+  int* tc_counter = nullptr;    // split-K arrival count per output tile: [SMs]
   std::vector<LayerMaps> tmaps;
   // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
   bool split = false;
@@ -246,6 +247,9 @@ bool tc_layer(const agn_handle* h, int l) { return h->use_tc && l < h->L; }
 agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   agn::TcArgs t{};
   t.slot_worker = sw;
+  t.ksplit = 1;
+  t.part = h->tc_part;
+  t.counter = h->tc_counter;
   t.err = h->flag + 1;
   t.theta = h->rep;
   t.acc = h->acc;
@@ -280,8 +284,6 @@ Status build_tc_maps(agn_handle* h) {
       const bf16* dZp = h->dZp[l];
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k64, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k64, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       continue;
     }
     const bf16* W = h->rep_b + h->woff[l - 1];
@@ -293,18 +295,22 @@ Status build_tc_maps(agn_handle* h) {
     const void* dZ = h->dZ[l];
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
-    AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k64, Hin, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
-    AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k64, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
   }
   return Status::Ok();
 }
 
-// Column tile of a forward or dX GEMM with M rows and N = m columns over s
-// slots: the full tile, unless that leaves SMs idle (small waves), then 64.
-int pick_bn(const agn_handle* h, int M, int s) {
-  const int bn = agn::tc_bn(h->m);
-  const int64_t ctas = ceil_div(M, 128) * ceil_div(h->m, bn) * (int64_t)s;
-  return (bn > 64 && ctas < h->num_sms) ? 64 : bn;
+// Split K of a forward or dX GEMM with M rows, N = m columns and K inner
+// over s slots: one CTA per output tile, unless the tiles leave SMs idle
+// (small waves); then ks CTAs share each tile, with ks <= SMs / tiles and
+// every CTA's range of 64-deep k steps non-empty.
+int pick_ksplit(const agn_handle* h, int M, int K, int s) {
+  const int64_t tiles = ceil_div(M, 128) * ceil_div(h->m, agn::tc_bn(h->m)) * (int64_t)s;
+  if (tiles >= h->num_sms) return 1;
+  const int kt = (int)ceil_div(K, 64);
+  int ks = (int)std::min<int64_t>(kt, h->num_sms / tiles);
+  if (ks <= 1) return 1;
+  const int per = (int)ceil_div(kt, ks);
+  return (int)ceil_div(kt, per);
 }
 
 // Pieces of an fp32 activation buffer [slots][m][d] (planes `plane` apart,
@@ -401,9 +407,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.relu = 1; t.boff = h->boff[l - 1];
           t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
           const auto& mp = h->tmaps[l - 1];
-          const int bn = pick_bn(h, fo, s);
-          AGN_TRY(agn::tc_forward(mp.w_k, bn == 64 ? mp.h_k64 : mp.h_k, t, s, h->stream,
-                                  h->split, bn));
+          t.ksplit = pick_ksplit(h, fo, fi, s);
+          AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split, agn::tc_bn(m)));
           pieces_done = true;
         } else {
           AGN_TRY(agn::simt_forward<T>(g, l == L, s, h->stream));
@@ -445,9 +450,9 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         t.mask = Hprev; t.mask_bstride = (int64_t)m * fi;
         t.out_pieces = next_pieces; t.out_plane = dz_plane(l - 1);
         const auto& mp = h->tmaps[l - 1];
-        const int bn = pick_bn(h, fi, s);
-        AGN_TRY(agn::tc_backward_dx(mp.w_mn, bn == 64 ? mp.dz_k64 : mp.dz_k, t, s, h->stream,
-                                    h->split, bn));
+        t.ksplit = pick_ksplit(h, fi, fo, s);
+        AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream, h->split,
+                                    agn::tc_bn(m)));
         have_pieces[l - 1] = next_pieces != nullptr;
       } else {
         agn::GemmArgs g{};
@@ -735,6 +740,8 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   h->steps = plan.steps;
   if (flags[0] || flags[1]) {
     AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
+    if (flags[1] && h->tc_counter)   // CTAs that gave up may have left tiles unfinished
+      AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)h->num_sms * sizeof(int), h->stream));
     AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
     if (flags[1])
       return Status::Err(AGN_E_TIMEOUT, "a tensor-core GEMM gave up on a bounded wait");
@@ -907,7 +914,12 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
                           cudaMemcpyHostToDevice));
   AGN_TRY_CUDA(cudaMemsetAsync(h->acc, 0, (size_t)(n * h->P_pad) * sizeof(float), h->stream));
   AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
-  if (h->use_tc) AGN_TRY(build_tc_maps(h));
+  if (h->use_tc) {
+    AGN_TRY(build_tc_maps(h));
+    AGN_TRY(dalloc_t(h, &h->tc_part, (size_t)h->num_sms * 256 * 128));
+    AGN_TRY(dalloc_t(h, &h->tc_counter, (size_t)h->num_sms));
+    AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)h->num_sms * sizeof(int), h->stream));
+  }
   std::vector<int> all(n);
   for (int w = 0; w < n; ++w) all[w] = w;
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,

@@ -36,6 +36,7 @@ constexpr int kThreads = 256;
 constexpr int kBK = 64;                       // K per stage: 64 bf16 = one 128-byte row
 constexpr int kABytes = 128 * 128;            // 128 rows x 128 bytes
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s
+constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles (end of ring)
 
 // A stage holds kSplit A pieces then kSplit B pieces (kSplit = 3 in the fp32
 // mode, where every fp32 operand is the exact sum of three bf16 pieces).
@@ -54,24 +55,44 @@ struct TileCfg {
 __device__ __constant__ const int kPairA[6] = {0, 0, 1, 0, 1, 2};
 __device__ __constant__ const int kPairB[6] = {0, 1, 0, 2, 1, 0};
 
-template <typename T>
-__device__ __forceinline__ T to_act(float v);
-template <>
-__device__ __forceinline__ bf16 to_act<bf16>(float v) { return __float2bfloat16_rn(v); }
-template <>
-__device__ __forceinline__ float to_act<float>(float v) { return v; }
 __device__ __forceinline__ float from_act(bf16 v) { return __bfloat162float(v); }
 __device__ __forceinline__ float from_act(float v) { return v; }
 
-// Three exact bf16 pieces of an fp32 output element (slot, offset o within
-// the slot), written to the out_pieces planes for the next tensor-core GEMM.
-__device__ __forceinline__ void write_pieces(const TcArgs& a, int slot, int64_t o, float v) {
-  bf16 q0, q1, q2;
-  split3(v, q0, q1, q2);
-  bf16* p = a.out_pieces + (int64_t)slot * a.out_bstride + o;
-  p[0] = q0;
-  p[a.out_plane] = q1;
-  p[2 * a.out_plane] = q2;
+// Four consecutive activations (16-byte aligned fp32, or 8-byte aligned bf16).
+__device__ __forceinline__ float4 load4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 load4(const bf16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+  const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+  return make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
+}
+__device__ __forceinline__ uint2 bf16x4(const float (&x)[4]) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(x[0], x[1]);
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(x[2], x[3]);
+  return make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+}
+__device__ __forceinline__ void store4(float* p, const float (&v)[4]) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ void store4(bf16* p, const float (&v)[4]) {
+  *reinterpret_cast<uint2*>(p) = bf16x4(v);
+}
+// The three exact bf16 pieces of four floats (split3 of each), packed.
+__device__ __forceinline__ void split3_x4(const float (&x)[4], uint2& q0, uint2& q1, uint2& q2) {
+  float r[4];
+  q0 = bf16x4(x);
+  const __nv_bfloat162* p0 = reinterpret_cast<const __nv_bfloat162*>(&q0);
+  r[0] = __fsub_rn(x[0], __low2float(p0[0]));
+  r[1] = __fsub_rn(x[1], __high2float(p0[0]));
+  r[2] = __fsub_rn(x[2], __low2float(p0[1]));
+  r[3] = __fsub_rn(x[3], __high2float(p0[1]));
+  q1 = bf16x4(r);
+  const __nv_bfloat162* p1 = reinterpret_cast<const __nv_bfloat162*>(&q1);
+  r[0] = __fsub_rn(r[0], __low2float(p1[0]));
+  r[1] = __fsub_rn(r[1], __high2float(p1[0]));
+  r[2] = __fsub_rn(r[2], __low2float(p1[1]));
+  r[3] = __fsub_rn(r[3], __high2float(p1[1]));
+  q2 = bf16x4(r);
 }
 
 // Wait that also gives up when another role has aborted.
@@ -98,7 +119,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * Cfg::kStageBytes);
   uint64_t* empty = full + kStages;
   uint64_t* done = empty + kStages;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* red = done + 1;              // split K: the other ranks' partial sums landed
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(red + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   // A CTA that gave up earlier in this launch (or run) makes the rest return
@@ -108,9 +130,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __syncthreads();
   if (s_skip != 0) return;   // uniform across the CTA
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tile = blockIdx.x, n_tile = blockIdx.y, slot = blockIdx.z;
+  const int ks = kEpi == kEpiDW ? 1 : args.ksplit;   // CTAs sharing one output tile
+  const int m_tile = blockIdx.x, n_tile = blockIdx.y;
+  const int slot = blockIdx.z / ks, sk = blockIdx.z % ks;
   const int worker = args.slot_worker[slot];
-  const int KT = (args.K + kBK - 1) / kBK;
+  // k steps [kt0, kt0 + KT) of this CTA (the host picks ks so that none is empty)
+  const int KT_all = (args.K + kBK - 1) / kBK;
+  const int kt_per = (KT_all + ks - 1) / ks;
+  const int kt0 = sk * kt_per;
+  const int KT = min(KT_all, kt0 + kt_per) - kt0;
   const int a_z = args.a_by_worker ? worker : slot;
   const int b_z = args.b_by_worker ? worker : slot;
 
@@ -120,6 +148,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       tc::mbar_init(&empty[s], 1);
     }
     tc::mbar_init(done, 1);
+    tc::mbar_init(red, 1);
     *abort_flag = 0;
     tc::fence_mbar_init();
     tc::tma_prefetch_desc(&tmA);
@@ -156,18 +185,19 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int p = 0; p < kSplit; ++p) {
           uint8_t* sa = sa0 + p * kABytes;
           uint8_t* sb = sb0 + p * Cfg::kBBytes;
+          const int kc = (kt0 + kt) * kBK;
           if (!kAMN) {
-            load(sa, &tmA, kt * kBK, m_tile * 128, a_z, p);
+            load(sa, &tmA, kc, m_tile * 128, a_z, p);
           } else {
-            load(sa, &tmA, m_tile * 128, kt * kBK, a_z, p);
-            load(sa + 8192, &tmA, m_tile * 128 + 64, kt * kBK, a_z, p);
+            load(sa, &tmA, m_tile * 128, kc, a_z, p);
+            load(sa + 8192, &tmA, m_tile * 128 + 64, kc, a_z, p);
           }
           if (!kBMN) {
-            load(sb, &tmB, kt * kBK, n_tile * BN, b_z, p);
+            load(sb, &tmB, kc, n_tile * BN, b_z, p);
           } else {
 #pragma unroll
             for (int c = 0; c < BN / 64; ++c)
-              load(sb + c * 8192, &tmB, n_tile * BN + c * 64, kt * kBK, b_z, p);
+              load(sb + c * 8192, &tmB, n_tile * BN + c * 64, kc, b_z, p);
           }
         }
       }
@@ -213,7 +243,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   }
   __syncwarp();
 
-  const bool ok = wait_or_abort(done, 0, abort_flag) && !*abort_flag;
+  // block-uniform, so that the epilogue's barriers and warp-wide TMEM loads
+  // are reached by every thread or by none
+  const bool ok = __syncthreads_and(wait_or_abort(done, 0, abort_flag) && !*abort_flag) != 0;
   tc::tc_fence_after();
   if (!ok) {
     if (threadIdx.x == 0) atomicExch(args.err, 1);
@@ -223,65 +255,153 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const bool row_ok = row < args.M;
     const uint32_t lane_base = (uint32_t)(32 * g) << 16;
     float* theta = args.theta + (int64_t)worker * args.ld_param;
-    if (kEpi == kEpiFwd) {
-      const float bias = row_ok ? theta[args.boff + row] : 0.f;
-      TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
+    // Accumulated values of this thread's row for columns c0 .. c0 + 31: from
+    // TMEM (the sum of the two accumulators in the split mode), or, with
+    // split K, the partial sums of all ks CTAs of the tile in rank order.
+    const int64_t tile_id = ((int64_t)slot * gridDim.y + n_tile) * gridDim.x + m_tile;
+    const int trow = 32 * g + lane;
+    auto tmem_vals = [&](int c0, uint32_t (&r)[32]) {
+      tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)c0, r);
+      if (kSplit == 3) {
+        uint32_t r2[32];
+        tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(BN + c0), r2);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
+      }
+      tc::tmem_ld_wait();
+    };
+    bool last = true;
+    const float* red_smem = reinterpret_cast<const float*>(smem);   // the free stage ring
+    if (kEpi != kEpiDW && ks > 1) {
+      // every CTA of the tile stores its partial sums ([column][row], rows
+      // contiguous); the last to finish copies the others' into its stage
+      // ring (TMA bulk copies, all in flight at once) and adds them in rank
+      // order, its own from TMEM
+      float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
 #pragma unroll 1
       for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
         uint32_t r[32];
-        tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)c0, r);
-        if (kSplit == 3) {
-          uint32_t r2[32];
-          tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(BN + c0), r2);
-          tc::tmem_ld_wait();
+        tmem_vals(c0, r);
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
-        }
-        tc::tmem_ld_wait();
-        if (row_ok) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int j = n_tile * BN + c0 + i;
-            if (j < args.N) {
-              float v = __uint_as_float(r[i]) + bias;
-              if (args.relu) v = fmaxf(v, 0.f);
-              const int64_t o = (int64_t)j * args.ldo + row;
-              out[o] = to_act<TAct>(v);
-              if (kSplit == 3 && args.out_pieces) write_pieces(args, slot, o, v);
-            }
+        for (int i = 0; i < 32; ++i) __stcg(mine + (int64_t)(c0 + i) * 128 + trow, __uint_as_float(r[i]));
+      }
+      // the CTA's stores, ordered by the barrier, are released by one
+      // acquire-release arrival; the last arrival acquires the others'
+      __shared__ int s_last;
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        const int prev = tc::atomic_add_acq_rel_gpu(args.counter + tile_id, 1);
+        s_last = prev == ks - 1;
+        if (s_last) {
+          args.counter[tile_id] = 0;   // ready for the next launch
+          tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
+          constexpr uint32_t kPart = 128u * BN * 4u;
+          tc::mbar_arrive_expect_tx(red, kPart * (uint32_t)(ks - 1));
+          for (int q = 0, d = 0; q < ks; ++q) {
+            if (q == sk) continue;
+            tc::bulk_load(smem + (size_t)d * kPart,
+                          args.part + (tile_id * ks + q) * (int64_t)(128 * BN), kPart, red);
+            ++d;
           }
         }
       }
-    } else if (kEpi == kEpiDX) {
+      __syncthreads();
+      last = s_last != 0;
+      if (last && !__syncthreads_and(wait_or_abort(red, 0, abort_flag))) {
+        last = false;   // gave up: report, skip the epilogue
+        if (threadIdx.x == 0) atomicExch(args.err, 1);
+      }
+    }
+    auto vals = [&](int c0, uint32_t (&r)[32]) {
+      tmem_vals(c0, r);
+      if (kEpi == kEpiDW || ks == 1) return;
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = 0.f;
+      for (int q = 0, d = 0; q < ks; ++q) {
+        if (q == sk) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
+        } else {
+          const float* pq = red_smem + (size_t)d * (128 * BN) + (size_t)c0 * 128 + trow;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += pq[i * 128];
+          ++d;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(v[i]);
+    };
+    // Forward and dX epilogues: the warp's 32 rows x 32 columns go through a
+    // warp-private shared-memory tile (column-major) so that each lane then
+    // handles four consecutive rows (features, contiguous in memory) of
+    // eight columns: 16-byte bias / mask loads, 16-byte stores of the output
+    // and 8-byte stores of each bf16 piece.
+    float* tT = reinterpret_cast<float*>(smem + (size_t)kStages * Cfg::kStageBytes - kEpiTBytes) +
+                warp * (32 * 32);
+    const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
+    const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
+    const bool row4_ok = row4 < args.M;                      // M % 4 == 0: all four or none
+    if (!last) {
+      // another CTA of this tile finishes it
+    } else if (kEpi == kEpiFwd || kEpi == kEpiDX) {
       TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
-      const TAct* mask = static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride;
+      const TAct* mask = kEpi == kEpiDX
+                             ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
+                             : nullptr;
+      float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kEpi == kEpiFwd && row4_ok) bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
 #pragma unroll 1
       for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
         uint32_t r[32];
-        tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)c0, r);
-        if (kSplit == 3) {
-          uint32_t r2[32];
-          tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(BN + c0), r2);
-          tc::tmem_ld_wait();
+        vals(c0, r);
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
-        }
-        tc::tmem_ld_wait();
-        if (row_ok) {
+        for (int i = 0; i < 32; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
+        __syncwarp();
+        if (row4_ok) {
+          float4 hm[8];
+          if (kEpi == kEpiDX) {   // all mask loads in flight before any store
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int j = n_tile * BN + c0 + i;
+            for (int u = 0; u < 8; ++u) {
+              const int j = n_tile * BN + c0 + jl + 4 * u;
+              hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int jc = jl + 4 * u;
+            const int j = n_tile * BN + c0 + jc;
             if (j < args.N) {
-              const int64_t o = (int64_t)j * args.ldo + row;
-              const float h = from_act(mask[o]);
-              const float v = h > 0.f ? __uint_as_float(r[i]) : 0.f;
-              out[o] = to_act<TAct>(v);
-              if (kSplit == 3 && args.out_pieces) write_pieces(args, slot, o, v);
+              const float4 a = *reinterpret_cast<const float4*>(tT + jc * 32 + r4);
+              float v[4] = {a.x, a.y, a.z, a.w};
+              if (kEpi == kEpiFwd) {
+                v[0] += bias4.x; v[1] += bias4.y; v[2] += bias4.z; v[3] += bias4.w;
+                if (args.relu) {
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) v[e] = fmaxf(v[e], 0.f);
+                }
+              } else {
+                const float hv[4] = {hm[u].x, hm[u].y, hm[u].z, hm[u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) v[e] = hv[e] > 0.f ? v[e] : 0.f;
+              }
+              const int64_t o = (int64_t)j * args.ldo + row4;
+              store4(out + o, v);
+              if (kSplit == 3 && args.out_pieces) {
+                uint2 q0, q1, q2;
+                split3_x4(v, q0, q1, q2);
+                bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o;
+                *reinterpret_cast<uint2*>(pp) = q0;
+                *reinterpret_cast<uint2*>(pp + args.out_plane) = q1;
+                *reinterpret_cast<uint2*>(pp + 2 * args.out_plane) = q2;
+              }
             }
           }
         }
+        __syncwarp();
       }
     } else {   // kEpiDW
       float* acc = args.acc + (int64_t)worker * args.ld_param;
@@ -432,8 +552,23 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   });
   AGN_TRY_CUDA(attr_err);
-  dim3 grid((unsigned)ceil_div(args.M, 128), (unsigned)ceil_div(args.N, BN), (unsigned)slots);
-  kern<<<grid, kThreads, smem, st>>>(a, b, args);
+  // split K: at most as many other ranks' partial sums as the stage ring
+  // holds, every rank with a non-empty range of k steps
+  int ks = kEpi == kEpiDW ? 1 : std::max(1, args.ksplit);
+  if (ks > 1) {
+    const int ring = kStages * TileCfg<BN, kSplit>::kStageBytes - kEpiTBytes;
+    ks = std::min(ks, 1 + ring / (128 * BN * 4));
+    const int kt = (args.K + kBK - 1) / kBK;
+    ks = std::min(ks, kt);
+    if (ks > 1) ks = (kt + (kt + ks - 1) / ks - 1) / ((kt + ks - 1) / ks);
+  }
+  if (ks > 1 && (!args.part || !args.counter))
+    return Status::Err(AGN_E_INVALID, "split-K GEMM without workspace");
+  dim3 grid((unsigned)ceil_div(args.M, 128), (unsigned)ceil_div(args.N, BN),
+            (unsigned)(slots * ks));
+  TcArgs a2 = args;
+  a2.ksplit = ks;
+  kern<<<grid, kThreads, smem, st>>>(a, b, a2);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

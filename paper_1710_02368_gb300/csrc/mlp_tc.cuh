@@ -29,6 +29,14 @@ struct TcArgs {
   float eta;
   bf16* out_pieces;        // split mode, forward / dX: also write the output's three
   int64_t out_plane;       // pieces here (same index, planes out_plane apart); null = no
+  // forward / dX split K: ksplit CTAs share an output tile, each a contiguous
+  // range of ceil(KT / ksplit) k steps (none empty); each stores its partial
+  // sums to part ([tile][rank][BN][128] fp32) and the last to arrive (counter
+  // per tile, zero between launches) adds them in rank order and runs the
+  // epilogue.  ksplit <= 1: one CTA per tile.
+  int ksplit;
+  float* part;
+  int* counter;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
@@ -55,8 +63,7 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
 // split = true : fp32 operands as three exact bf16 pieces (4D maps), fp32
 //                activations; dW writes the three pieces of the new weights.
 // forward: w_k box {64, 128} over W (K-major); h_k box {64, bn} over H_{l-1},
-// bn in {64, 128, 256} the column tile (>= N unless a smaller tile is chosen
-// to give a small wave more CTAs).
+// bn = tc_bn(N) the column tile.  Small waves split K instead (args.ksplit).
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
                   cudaStream_t st, bool split, int bn);
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
