@@ -108,14 +108,18 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def _traffic_for(kernel_class, workload):
+def _traffic_for(kernel_class, workload, on_tc):
     """ncu DRAM bytes per launch of a kernel class, if a summary for the current
     source of that kernel exists under profiles/ (else None)."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
     if not os.path.exists(path):
         return None
-    src = {"forward": "mlp_simt.cu", "backward_dx": "mlp_simt.cu", "backward_dw": "mlp_simt.cu",
-           "commit": "commit_pull.cu"}.get(kernel_class)
+    if on_tc:
+        src = {"forward": "mlp_tc.cu", "backward_dx": "mlp_tc.cu", "backward_dw": "mlp_tc_dw.cu",
+               "softmax": "mlp_head.cu", "commit": "commit_pull.cu"}.get(kernel_class)
+    else:
+        src = {"forward": "mlp_simt.cu", "backward_dx": "mlp_simt.cu",
+               "backward_dw": "mlp_simt.cu", "commit": "commit_pull.cu"}.get(kernel_class)
     if src is None:
         return None
     digest = hashlib.sha256(open(os.path.join(ROOT, "paper_1710_02368_gb300", "csrc", src),
@@ -242,7 +246,7 @@ def run_agn(args, wl):
     seed = I.DEFAULT_SEED
     per_step = args.commits_per_step or (
         COMMITS_PER_STEP[args.workload] if not args.workers else 2 * wl.n)
-    total = (args.warmup + 2 * args.steps) * per_step + wl.n
+    total = (args.warmup + 3 * args.steps) * per_step + wl.n
     w, tau = agn.agn_make_schedule(wl.n, total, wl.tau_lo, wl.tau_hi, seed)
     h = agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, seed, precision=wl.precision, batch=wl.batch,
                 n_samples=wl.n_samples, input_dist=wl.dist, teacher_dims=wl.teacher_dims,
@@ -262,9 +266,8 @@ def run_agn(args, wl):
 
     for i in range(args.warmup):
         step(i)
-    # timed region 1: device-resident inputs, kernel profiling on
-    h.profile(2)
-    h.profile(1)
+    # timed region 1: device-resident inputs, no per-kernel events (the
+    # headline value)
     launches = 0
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -275,8 +278,22 @@ def run_agn(args, wl):
             launches += int(h.last_run_stats()["launches"])
         e1.record(st)
         barrier()
-    h.profile(0)
     ms = e0.elapsed_time(e1)
+    # timed region 2: the next steps of the same run with CUDA events around
+    # every kernel launch on the launching stream (per-kernel durations for
+    # the roofline and the shares; the events themselves cost some time, so
+    # this region is not the headline)
+    h.profile(2)
+    h.profile(1)
+    barrier()
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(st)
+    for i in range(args.warmup + args.steps, args.warmup + 2 * args.steps):
+        step(i)
+    p1.record(st)
+    barrier()
+    h.profile(0)
+    prof_ms = p0.elapsed_time(p1)
     kst = h.kernel_stats()
     tc_ok = wl.batch <= 256 and all(d % 8 == 0 for d in wl.dims[:-1])
     if args.gemm != "simt" and tc_ok:
@@ -292,7 +309,7 @@ def run_agn(args, wl):
     e3 = torch.cuda.Event(enable_timing=True)
     e2.record(st)
     d2h = 0
-    for i in range(args.warmup + args.steps, args.warmup + 2 * args.steps):
+    for i in range(args.warmup + 2 * args.steps, args.warmup + 3 * args.steps):
         losses = step(i, e2e=True)
         d2h += losses.nbytes
     e3.record(st)
@@ -335,10 +352,11 @@ def run_agn(args, wl):
         roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
                 "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    tr = _traffic_for(dom, wl.name)
+    tr = _traffic_for(dom, wl.name, on_tc)
     roof["traffic"] = tr
     roof["kernel"] = dom
     roof["avg_launch_us"] = 1e3 * d["ms"] / max(d["launches"], 1)
+    roof["events_region_ms_per_step"] = prof_ms / args.steps
     roof["algorithmic_per_launch"] = {"flops": d["flops"] / max(d["launches"], 1),
                                       "bytes": d["bytes"] / max(d["launches"], 1)}
     kernels = {k: {"launches": int(v["launches"]), "ms": round(v["ms"], 3),
