@@ -90,6 +90,7 @@ struct agn_handle {
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
     CUtensorMap theta, acc;      // fp32 W_l of every replica / accumulator, box {128, 32}
+    CUtensorMap h_mn32, dz_mn32; // split mode: 32-sample boxes for the dW kernel
   };
   int num_sms = 148;
   float* tc_part = nullptr;     // split-K partial sums: [SMs][BN <= 256][128]
@@ -284,6 +285,8 @@ Status build_tc_maps(agn_handle* h) {
       const bf16* dZp = h->dZp[l];
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 32));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn32, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 32));
       continue;
     }
     const bf16* W = h->rep_b + h->woff[l - 1];
@@ -490,8 +493,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
                                    h->split, h->piece_plane));
         } else {
           const auto& mp = h->tmaps[l - 1];
-          tc_dw.push_back({&mp.h_mn, &mp.dz_mn, &mp.theta, &mp.acc, fi, fo, h->woff[l - 1],
-                           h->boff[l - 1]});
+          tc_dw.push_back({h->split ? &mp.h_mn32 : &mp.h_mn, h->split ? &mp.dz_mn32 : &mp.dz_mn,
+                           &mp.theta, &mp.acc, fi, fo, h->woff[l - 1], h->boff[l - 1]});
           tc_flops += flops;
           tc_bytes += bytes;
         }

@@ -166,43 +166,58 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   }
   if (q == 0 && lane == 0) ce_s[sj] = ce;
   __syncthreads();
+  // per-slot loss: the last block of the slot to finish sums the blocks'
+  // partials with a fixed assignment (thread t takes blocks t, t + 256, ...)
+  // and a fixed shuffle tree, so the result does not depend on timing
+  __shared__ int s_last;
+  __shared__ float warp_sum[kHeadThreads / 32];
+  const int nblk = gridDim.x;
   if (threadIdx.x == 0) {
     float part = 0.f;
     for (int r = 0; r < kHeadSamples; ++r) part += ce_s[r];
-    const int nblk = gridDim.x;
     a.ce_partial[(int64_t)z * nblk + blockIdx.x] = part;
     __threadfence();
-    const int done = atomicAdd(a.counter + z, 1);
-    if (done == nblk - 1) {   // last block of this slot: fixed-order sum
-      __threadfence();
-      float tot = 0.f;
-      for (int b = 0; b < nblk; ++b) tot += *(volatile float*)(a.ce_partial + (int64_t)z * nblk + b);
-      const float loss = tot / (float)m;
-      a.loss_parts[(int64_t)a.slot_commit[z] * a.lam + a.step] = loss;
-      if (!isfinite(loss)) atomicExch(a.flag, 1);
-      a.counter[z] = 0;
-    }
+    s_last = atomicAdd(a.counter + z, 1) == nblk - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;   // uniform across the block
+  __threadfence();
+  float v = 0.f;
+  for (int b = threadIdx.x; b < nblk; b += blockDim.x) v += __ldcg(a.ce_partial + (int64_t)z * nblk + b);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  if (lane == 0) warp_sum[warp] = v;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float tot = 0.f;
+    for (int q = 0; q < kHeadThreads / 32; ++q) tot += warp_sum[q];
+    const float loss = tot / (float)m;
+    a.loss_parts[(int64_t)a.slot_commit[z] * a.lam + a.step] = loss;
+    if (!isfinite(loss)) atomicExch(a.flag, 1);
+    a.counter[z] = 0;
   }
 }
 
 // The output layer's weight gradient and local update:
 //   g[c][k] = sum_j dZ_L[j][c] h[j][k],   g_b[c] = sum_j dZ_L[j][c],
 //   theta_k -= eta g, a_k += g, and the bf16 copy (or its three pieces).
-// A block covers 32 inputs k of one slot; its four warps take the samples
-// j = w (mod 4), each lane one input, with dZ_L of the whole minibatch staged
-// in shared memory; the four partials are added in a fixed order.  The
-// bias gradient is summed (fixed order) by the first block of the slot.
-constexpr int kDwGroups = 4;
+// A block covers 32 inputs k of one slot with eight warps: dZ_L of the whole
+// minibatch is staged in shared memory (asynchronous copies); warp w takes
+// the samples j = w (mod 8), eight loads of h in flight per lane; the eight
+// partials are added in a fixed order by the warp that owns the class
+// (c = w mod 8), which then updates theta_k and a_k.  The bias gradient is
+// summed by the last warp of the slot's first block (fixed shuffle tree).
+constexpr int kDwGroups = 8;
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArgs a) {
   extern __shared__ __align__(16) uint8_t dw_smem[];
-  float* dz = reinterpret_cast<float*>(dw_smem);           // [m][C]
-  float* red = dz + (int64_t)a.m * a.C;                     // [kDwGroups][kMaxC][32]
+  float* red = reinterpret_cast<float*>(dw_smem);                      // [kDwGroups][kMaxC][32]
+  T* dz = reinterpret_cast<T*>(red + kDwGroups * kMaxC * 32);           // [m][C]
   const int z = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, C = a.C, m = a.m;
-  const T* dzg = static_cast<const T*>(a.dZL) + (int64_t)z * m * C;
-  for (int i = threadIdx.x; i < m * C; i += blockDim.x) dz[i] = cvt(dzg[i]);
+  stage(dz, static_cast<const T*>(a.dZL) + (int64_t)z * m * C, (int64_t)m * C);
+  stage_wait();
   __syncthreads();
   const int w = a.slot_worker[z];
   const int k = blockIdx.x * 32 + lane;
@@ -211,25 +226,26 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
 #pragma unroll
   for (int c = 0; c < kMaxC; ++c) g[c] = 0.f;
   if (k < K) {
+    constexpr int kU = 8;   // loads in flight per lane
     int j = warp;
-    for (; j + 3 * kDwGroups < m; j += 4 * kDwGroups) {   // four loads in flight
-      float hv[4];
+    for (; j + (kU - 1) * kDwGroups < m; j += kU * kDwGroups) {
+      float hv[kU];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) hv[u] = cvt(hg[(int64_t)(j + u * kDwGroups) * K]);
+      for (int u = 0; u < kU; ++u) hv[u] = cvt(hg[(int64_t)(j + u * kDwGroups) * K]);
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float* dzj = dz + (j + u * kDwGroups) * C;
+      for (int u = 0; u < kU; ++u) {
+        const T* dzj = dz + (j + u * kDwGroups) * C;
 #pragma unroll
         for (int c = 0; c < kMaxC; ++c)
-          if (c < C) g[c] = fmaf(dzj[c], hv[u], g[c]);
+          if (c < C) g[c] = fmaf(cvt(dzj[c]), hv[u], g[c]);
       }
     }
     for (; j < m; j += kDwGroups) {
       const float hv = cvt(hg[(int64_t)j * K]);
-      const float* dzj = dz + j * C;
+      const T* dzj = dz + j * C;
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
-        if (c < C) g[c] = fmaf(dzj[c], hv, g[c]);
+        if (c < C) g[c] = fmaf(cvt(dzj[c]), hv, g[c]);
     }
   }
 #pragma unroll
@@ -238,10 +254,10 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
   float* theta = a.theta + (int64_t)w * a.ld_param;
   float* acc = a.acc + (int64_t)w * a.ld_param;
   bf16* tb = a.theta_b ? a.theta_b + (int64_t)w * a.ld_param : nullptr;
-  auto update = [&](int64_t p, float gr) {
-    const float t = fmaf(-a.eta, gr, theta[p]);
+  auto update = [&](int64_t p, float gr, float th, float ac) {
+    const float t = fmaf(-a.eta, gr, th);
     theta[p] = t;
-    acc[p] += gr;
+    acc[p] = ac + gr;
     if (tb) {
       if (a.piece_plane > 0) {
         bf16 q0, q1, q2;
@@ -254,18 +270,36 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       }
     }
   };
-  if (warp == 0 && k < K) {
-    for (int c = 0; c < C; ++c) {
-      float s = 0.f;
+  if (k < K) {
+    constexpr int kPer = (kMaxC + kDwGroups - 1) / kDwGroups;   // classes per warp
+    float th[kPer], ac[kPer], gs[kPer];
 #pragma unroll
-      for (int r = 0; r < kDwGroups; ++r) s += red[(r * kMaxC + c) * 32 + lane];
-      update(a.woff + (int64_t)c * K + k, s);
+    for (int e = 0; e < kPer; ++e) {   // loads first, all in flight
+      const int c = warp + e * kDwGroups;
+      if (c < C) {
+        const int64_t p = a.woff + (int64_t)c * K + k;
+        th[e] = theta[p];
+        ac[e] = acc[p];
+        float v = 0.f;
+#pragma unroll
+        for (int r = 0; r < kDwGroups; ++r) v += red[(r * kMaxC + c) * 32 + lane];
+        gs[e] = v;
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      const int c = warp + e * kDwGroups;
+      if (c < C) update(a.woff + (int64_t)c * K + k, gs[e], th[e], ac[e]);
     }
   }
-  if (blockIdx.x == 0 && warp == 1 && lane < C) {
-    float s = 0.f;
-    for (int j = 0; j < m; ++j) s += dz[j * C + lane];
-    update(a.boff + lane, s);
+  if (blockIdx.x == 0 && warp == kDwGroups - 1) {
+    for (int c = 0; c < C; ++c) {
+      float v = 0.f;
+      for (int j = lane; j < m; j += 32) v += cvt(dz[j * C + c]);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (lane == 0) update(a.boff + c, v, theta[a.boff + c], acc[a.boff + c]);
+    }
   }
 }
 
@@ -314,8 +348,8 @@ Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st) {
 template <typename T>
 Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st) {
   if (a.C > kHeadMaxClasses) return Status::Err(AGN_E_UNSUPPORTED, "output layer too wide");
-  const size_t smem = (size_t)a.m * a.C * sizeof(float) +
-                      (size_t)kDwGroups * kHeadMaxClasses * 32 * sizeof(float);
+  const size_t smem = (size_t)kDwGroups * kHeadMaxClasses * 32 * sizeof(float) +
+                      (size_t)a.m * a.C * sizeof(T);
   if (smem > (size_t)kHeadSmemCap)
     return Status::Err(AGN_E_UNSUPPORTED, "minibatch too large for the output dW");
   auto kern = a.C == 10 ? head_dw_kernel<T, 10> : head_dw_kernel<T, kHeadMaxClasses>;

@@ -261,38 +261,38 @@ __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y
 }
 
 // The same gather, four consecutive elements per thread (d_0 a multiple of
-// 4): one 16-byte (fp32) or 8-byte (bf16) load and store, and 8-byte piece
-// stores; a grid-stride loop over (slot, sample, element group).
+// 4): a block per minibatch row, one 16-byte (fp32) or 8-byte (bf16) load and
+// store per thread and group, and 8-byte piece stores.
 template <typename T>
-__global__ void gather4_kernel(const T* __restrict__ X, const int* __restrict__ y, T* Xb, int* yb,
-                               int d0, int m, int64_t S, const int* slot_worker,
-                               const long long* slot_t0, int step, bf16* pieces, int64_t plane,
-                               int64_t total) {
+__global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
+                                                      const int* __restrict__ y, T* Xb, int* yb,
+                                                      int d0, int m, int64_t S,
+                                                      const int* slot_worker,
+                                                      const long long* slot_t0, int step,
+                                                      bf16* pieces, int64_t plane) {
   struct alignas(4 * sizeof(T)) Vec { T v[4]; };
   struct alignas(8) Piece4 { bf16 v[4]; };
-  const int g4 = d0 / 4;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
-    const int64_t r = i / g4;             // slot * m + j
-    const int c = (int)(i - r * g4) * 4;
-    const int z = (int)(r / m), j = (int)(r - (int64_t)z * m);
-    const int w = slot_worker[z];
-    const long long t = slot_t0[z] + step;
-    const int64_t row =
-        (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
-    const Vec v = *reinterpret_cast<const Vec*>(X + row * d0 + c);
-    const int64_t o = r * d0 + c;
-    *reinterpret_cast<Vec*>(Xb + o) = v;
+  const int r = blockIdx.x;                 // slot * m + j
+  const int z = r / m, j = r - z * m;
+  const int w = slot_worker[z];
+  const long long t = slot_t0[z] + step;
+  const int64_t row =
+      (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
+  const T* src = X + row * d0;
+  const int64_t o = (int64_t)r * d0;
+  for (int c = threadIdx.x * 4; c < d0; c += blockDim.x * 4) {
+    const Vec v = *reinterpret_cast<const Vec*>(src + c);
+    *reinterpret_cast<Vec*>(Xb + o + c) = v;
     if (pieces) {
       Piece4 p0, p1, p2;
 #pragma unroll
       for (int e = 0; e < 4; ++e) split3(to_f(v.v[e]), p0.v[e], p1.v[e], p2.v[e]);
-      *reinterpret_cast<Piece4*>(pieces + o) = p0;
-      *reinterpret_cast<Piece4*>(pieces + plane + o) = p1;
-      *reinterpret_cast<Piece4*>(pieces + 2 * plane + o) = p2;
+      *reinterpret_cast<Piece4*>(pieces + o + c) = p0;
+      *reinterpret_cast<Piece4*>(pieces + plane + o + c) = p1;
+      *reinterpret_cast<Piece4*>(pieces + 2 * plane + o + c) = p2;
     }
-    if (c == 0) yb[r] = y[row];
   }
+  if (threadIdx.x == 0) yb[r] = y[row];
 }
 
 template <typename T, typename TO, bool kAK, bool kBK, int kEpi>
@@ -336,10 +336,9 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
                      reinterpret_cast<uintptr_t>(pieces)) & 15) == 0;
   if (slots <= 0 || m <= 0) return Status::Ok();
   if (vec) {
-    const int64_t total = (int64_t)slots * m * (d0 / 4);
-    const int grid = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 16);
-    gather4_kernel<T><<<grid, 256, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
-                                            pieces, plane, total);
+    const int threads = (int)std::min<int64_t>(256, round_up((int64_t)d0 / 4, 32));
+    gather4_kernel<T><<<slots * m, threads, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker,
+                                                     slot_t0, step, pieces, plane);
   } else {
     dim3 grid((unsigned)m, (unsigned)slots);
     gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,

@@ -69,8 +69,9 @@ Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& 
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
                       int slots, cudaStream_t st, bool split, int bn);
-// One hidden layer of a dW launch: h_mn box {64, 64} over H_{l-1}; dz_mn box
-// {64, 64} over dZ_l; theta / acc fp32 maps (d_{l-1}, d_l, n) over the
+// One hidden layer of a dW launch: h_mn box {64, kBK} over H_{l-1}; dz_mn box
+// {64, kBK} over dZ_l (kBK = 64 samples, 32 in the split mode); theta / acc
+// fp32 maps (d_{l-1}, d_l, n) over the
 // layer's weights in the replicas and the accumulators, box {128, 32}, no
 // swizzle.  M = d_{l-1}, N = d_l.
 struct DwLayerMaps {

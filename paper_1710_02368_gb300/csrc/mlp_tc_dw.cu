@@ -54,8 +54,6 @@ namespace {
 constexpr int kWarps = 10;
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 32 * kWarps;
-constexpr int kBK = 64;                        // K (samples) per stage
-constexpr int kABytes = 128 * 128;             // A box pair: 128 inputs x 64 samples, bf16
 constexpr int kCF = 32;                        // output features per parameter chunk
 constexpr int kChunkBytes = kCF * 128 * 4;     // one fp32 chunk: 32 rows x 128 inputs
 constexpr int kBiasBytes = 2 * kCF * 4;       // b_l and its accumulator for one chunk
@@ -63,9 +61,15 @@ constexpr int kSlotBytes = 2 * kChunkBytes + kBiasBytes;   // one ring slot
 constexpr int kRing = 3;                       // chunks (theta and a) in flight
 constexpr uint64_t kWaitNs = 2000000000ull;    // 2 s
 
-template <int BN, int kSplit, int kStages>
+// kBK samples per stage: one TMA box is 64 MN-elements x kBK samples of bf16
+// (kBK rows of 128 bytes, 128-byte swizzle); A = two boxes (128 inputs),
+// B = BN / 64 boxes.
+template <int BN, int kSplit, int kStages, int kBKs>
 struct DwCfg {
-  static constexpr int kBBytes = BN * 128;
+  static constexpr int kBK = kBKs;
+  static constexpr int kBox = kBK * 128;
+  static constexpr int kABytes = 2 * kBox;
+  static constexpr int kBBytes = (BN / 64) * kBox;
   static constexpr int kStageBytes = kSplit * (kABytes + kBBytes);
   // one accumulator: BN columns, or two of BN in the split mode (the leading
   // piece products and the five smaller pairs, kept apart for accuracy)
@@ -137,9 +141,11 @@ __device__ __forceinline__ TileIdx decode(const DwBatch& B, int t) {
 }
 
 // Row r (< 128) of H^T set to one in every sample of an A stage: two 64-input
-// boxes, 128-byte rows (one per sample), 16-byte chunks swizzled by row % 8.
+// boxes of kBK 128-byte rows (one per sample), 16-byte chunks swizzled by
+// row % 8.
+template <int kBK>
 __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
-  uint8_t* box = sa + (r >> 6) * 8192;
+  uint8_t* box = sa + (r >> 6) * (kBK * 128);
   const int i = r & 63;
   for (int j = 0; j < kBK; ++j) {
     const int off = j * 128 + ((((i >> 3) ^ (j & 7))) << 4) + (i & 7) * 2;
@@ -147,10 +153,11 @@ __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
   }
 }
 
-template <int BN, int kSplit, int kStages>
+template <int BN, int kSplit, int kStages, int kBKs>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
-  using Cfg = DwCfg<BN, kSplit, kStages>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs>;
+  constexpr int kBK = Cfg::kBK, kABytes = Cfg::kABytes, kBox = Cfg::kBox;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -231,18 +238,18 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
             uint8_t* sb = sb0 + p * Cfg::kBBytes;
             if (kSplit == 1) {
               tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
-              tc::tma_load_3d(sa + 8192, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
+              tc::tma_load_3d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
 #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_3d(sb + c * 8192, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                tc::tma_load_3d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
                                 ti.slot);
             } else {
               tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
-              tc::tma_load_4d(sa + 8192, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
+              tc::tma_load_4d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
                               p);
 #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_4d(sb + c * 8192, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                tc::tma_load_4d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
                                 ti.slot, p);
             }
           }
@@ -307,7 +314,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           }
           tc::tc_fence_after();
           if (ones_row < 128) {   // piece 0 of the out-of-range row := 1 (pieces 1, 2 stay 0)
-            write_ones_row(smem + s * Cfg::kStageBytes, ones_row);
+            write_ones_row<kBK>(smem + s * Cfg::kStageBytes, ones_row);
             tc::fence_proxy_async_smem();
           }
           const uint32_t sa0 = tc::smem_u32(smem + s * Cfg::kStageBytes);
@@ -319,8 +326,8 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
             for (int q = 0; q < kPairs; ++q) {
               const uint32_t sa = sa0 + (kSplit == 1 ? 0 : pair_a(q)) * kABytes;
               const uint32_t sb = sb0 + (kSplit == 1 ? 0 : pair_b(q)) * Cfg::kBBytes;
-              const uint64_t ad = tc::smem_desc_sw128(sa + kk * 2048, 8192, 1024);
-              const uint64_t bd = tc::smem_desc_sw128(sb + kk * 2048, 8192, 1024);
+              const uint64_t ad = tc::smem_desc_sw128(sa + kk * 2048, kBox, 1024);
+              const uint64_t bd = tc::smem_desc_sw128(sb + kk * 2048, kBox, 1024);
               const uint32_t dcol = (kSplit == 3 && q > 0) ? (uint32_t)BN : 0u;
               const bool acc_on = kSplit == 1 ? (kt | kk | q) != 0
                                               : (q == 0 ? (kt | kk) != 0
@@ -465,13 +472,13 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   if (warp == 1) tc::tmem_dealloc(tmem, Cfg::kTmemCols);
 }
 
-template <int BN, int kSplit, int kStages>
+template <int BN, int kSplit, int kStages, int kBKs>
 Status launch_dw(const DwBatch& batch, const TcArgs& args, int num_sms, cudaStream_t st) {
-  using Cfg = DwCfg<BN, kSplit, kStages>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs>;
   static_assert(Cfg::kSmem <= 232448, "shared memory");
   static_assert(Cfg::kSmem > 232448 / 2, "one CTA per SM (all 512 TMEM columns)");
   static_assert(Cfg::kTmemCols == 512, "TMEM columns");
-  auto kern = tc_dw_kernel<BN, kSplit, kStages>;
+  auto kern = tc_dw_kernel<BN, kSplit, kStages, kBKs>;
   static std::mutex mu;
   static std::set<int> done;
   {
@@ -520,8 +527,10 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
       if (tiles > INT32_MAX) return Status::Err(AGN_E_UNSUPPORTED, "dW tile count overflows");
     }
     batch.total_tiles = (int)tiles;
-    Status r = split ? launch_dw<kTcDwBNSplit, 3, 1>(batch, args, num_sms, st)
-                     : launch_dw<kTcDwBN, 1, 2>(batch, args, num_sms, st);
+    // split mode: 32 samples per stage, so that two stages fit beside the
+    // parameter ring (the next tile's operands land while this one multiplies)
+    Status r = split ? launch_dw<kTcDwBNSplit, 3, 2, 32>(batch, args, num_sms, st)
+                     : launch_dw<kTcDwBN, 1, 2, 64>(batch, args, num_sms, st);
     if (!r.ok()) return r;
   }
   return Status::Ok();
