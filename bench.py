@@ -175,7 +175,7 @@ def run_reference(args, wl):
 
     def step():
         O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:per_step], tau[:per_step], ds, wl.batch,
-                  wl.shard, dtype=dtype)
+                  wl.shard, dtype=dtype, staleness_scaled=args.commit_rule == "dynsgd")
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
@@ -189,6 +189,7 @@ def run_reference(args, wl):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64" if dtype == np.float64 else "f32", "data": "synthetic",
         "config": {"workload": wl.name, "commits_per_step": per_step,
+                   "commit_rule": args.commit_rule,
                    "sample": f"each step re-runs the first {per_step} commits on the CPU"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
                          "kind": "oracle",
@@ -250,7 +251,9 @@ def run_agn(args, wl):
     w, tau = agn.agn_make_schedule(wl.n, total, wl.tau_lo, wl.tau_hi, seed)
     h = agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, seed, precision=wl.precision, batch=wl.batch,
                 n_samples=wl.n_samples, input_dist=wl.dist, teacher_dims=wl.teacher_dims,
-                normalize=wl.normalize, gemm=GEMMS[args.gemm], stream=st.cuda_stream)
+                normalize=wl.normalize, gemm=GEMMS[args.gemm], stream=st.cuda_stream,
+                commit_rule=agn.AGN_COMMIT_DYNSGD if args.commit_rule == "dynsgd"
+                else agn.AGN_COMMIT_AGN)
 
     def barrier():
         if ws > 1:
@@ -374,6 +377,7 @@ def run_agn(args, wl):
         "dtype": "f32" if wl.precision == WL.PREC_FP32 else "bf16",
         "data": "synthetic (seeded MNIST-shaped teacher-labelled set; MNIST itself unavailable)",
         "config": {"workload": wl.name, "commits_per_step": per_step,
+                   "commit_rule": args.commit_rule,
                    "parallelism": "replicas" if ws > 1 else "single GPU",
                    "l2": "inputs larger than L2 (dataset 188 MB + replicas and accumulators "
                          "230 MB vs 129 MB L2)" if args.workload == "mnist" else
@@ -405,6 +409,8 @@ def main():
     ap.add_argument("--workload", default="mnist", choices=sorted(WORKLOADS))
     ap.add_argument("--commits-per-step", type=int, default=0)
     ap.add_argument("--gemm", default="auto", choices=sorted(GEMMS))
+    ap.add_argument("--commit-rule", default="agn", choices=["agn", "dynsgd"],
+                    help="AGN's commit (Eq. 1) or the DynSGD-style staleness-scaled commit")
     ap.add_argument("--workers", type=int, default=0,
                     help="override n (profiling captures of a smaller case)")
     ap.add_argument("--ref-commits", type=int, default=2)

@@ -60,6 +60,10 @@ extern "C" {
                                   AGN_E_UNSUPPORTED); the d_L-wide output
                                   layer always runs on CUDA cores          */
 
+/* Commit rules (agn_options.commit_rule) */
+#define AGN_COMMIT_AGN 0       /* Delta = -eta a / lambda (Eq. 1)            */
+#define AGN_COMMIT_DYNSGD 1    /* Delta = -eta a / (tau_c + 1), Section 4     */
+
 typedef struct agn_handle agn_handle;
 
 /* Options of agn_create.  Fill with agn_default_options, then override. */
@@ -89,6 +93,12 @@ typedef struct agn_options {
      dW GEMMs on the earlier non-persistent tcgen05 kernel (one tile per CTA)
      instead of the persistent one, for comparison. */
   int32_t tc_mask;
+  /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
+     Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);
+     AGN_COMMIT_DYNSGD commits the accumulated update scaled by staleness,
+     Delta = -eta a / (tau_c + 1), tau_c the schedule's staleness of commit c
+     (the DynSGD comparison of Section 4; normalize is ignored). */
+  int32_t commit_rule;
 } agn_options;
 
 void agn_default_options(agn_options* opt);

@@ -207,7 +207,8 @@ class AGNResult:
 
 
 def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
-            normalize=True, snapshot_at=(), keep_locals=(), dtype=np.float64):
+            normalize=True, snapshot_at=(), keep_locals=(), dtype=np.float64,
+            staleness_scaled=False):
     """Run the commits of one schedule through the FIFO parameter server.
 
     model      : object with loss_grad(theta, X, y) -> (loss, grad)
@@ -220,6 +221,11 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
     v_c commits (its Pull); it takes lambda local steps (Algorithm 1):
         g = -eta * grad;  a = a + g;  theta = theta + g
     then a = a / lambda (skipped when normalize is False) and theta~ += a.
+
+    staleness_scaled: the DynSGD-style commit the paper compares against
+    (Section 4): the accumulated update divided by tau_c + 1, where
+    tau_c = c - v_c is the number of commits between the worker's pull and
+    its commit, instead of by lambda (`normalize` is then ignored).
     """
     worker = np.asarray(worker, dtype=np.int64)
     v = schedule_versions(n, worker, tau)
@@ -261,7 +267,9 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
             losses.append(li)
             if iterates is not None:
                 iterates.append(theta.copy())
-        if normalize:
+        if staleness_scaled:
+            a = a / dtype(c - vc + 1)                   # DynSGD: 1 / (tau_c + 1)
+        elif normalize:
             a = a / dtype(lam)                          # normalisation step
         theta_c = theta_c + a                           # Eq. 2
         loss[c] = float(np.mean(losses))

@@ -14,7 +14,8 @@ import ctypes as C
 import numpy as np
 
 from . import _lib
-from ._lib import (AGN_DIST_NORMAL, AGN_DIST_UNIFORM, AGN_GEMM_AUTO, AGN_GEMM_SIMT,  # noqa: F401
+from ._lib import (AGN_COMMIT_AGN, AGN_COMMIT_DYNSGD,  # noqa: F401
+                   AGN_DIST_NORMAL, AGN_DIST_UNIFORM, AGN_GEMM_AUTO, AGN_GEMM_SIMT,  # noqa: F401
                    AGN_GEMM_TCGEN05, AGN_PREC_BF16, AGN_PREC_FP32, AGN_OK, AGN_E_INVALID,
                    AGN_E_SCHEDULE, AGN_E_OOM, AGN_E_CUDA, AGN_E_TIMEOUT, AGN_E_NONFINITE,
                    AGN_E_UNSUPPORTED, agn_options)
@@ -228,12 +229,13 @@ class AGN:
     def __init__(self, dims, n_workers, lam, eta, seed, *, precision=AGN_PREC_FP32, batch=32,
                  n_samples=2048, input_dist=AGN_DIST_UNIFORM, teacher_dims=None, normalize=1,
                  gemm=AGN_GEMM_AUTO, tau_lo=0, tau_hi=0, stream=None, x=None, y=None,
-                 theta0=None, tc_mask=0):
+                 theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN):
         o = agn_default_options()
         o.precision, o.batch, o.n_samples = int(precision), int(batch), int(n_samples)
         o.input_dist, o.normalize, o.gemm = int(input_dist), int(normalize), int(gemm)
         o.tau_lo, o.tau_hi = int(tau_lo), int(tau_hi)
         o.tc_mask = int(tc_mask)
+        o.commit_rule = int(commit_rule)
         keep = []
         if teacher_dims is not None:
             td, tdp = _i32(teacher_dims)

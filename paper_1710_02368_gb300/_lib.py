@@ -25,6 +25,8 @@ AGN_PREC_FP32 = 0
 AGN_PREC_BF16 = 1
 AGN_DIST_UNIFORM = 0
 AGN_DIST_NORMAL = 1
+AGN_COMMIT_AGN = 0
+AGN_COMMIT_DYNSGD = 1
 AGN_GEMM_AUTO = 0
 AGN_GEMM_SIMT = 1
 AGN_GEMM_TCGEN05 = 2
@@ -56,6 +58,7 @@ class agn_options(C.Structure):
         ("y_init", C.POINTER(C.c_int32)),
         ("theta_init", C.POINTER(C.c_float)),
         ("tc_mask", C.c_int32),
+        ("commit_rule", C.c_int32),
     ]
 
 

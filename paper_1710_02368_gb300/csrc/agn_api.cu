@@ -58,6 +58,7 @@ struct agn_handle {
   double eta = 0.0;
   uint64_t seed = 0;
   int prec = AGN_PREC_FP32, m = 32, dist = AGN_DIST_UNIFORM, normalize = 1, gemm = 0;
+  int commit_rule = AGN_COMMIT_AGN;
   int tau_lo = 0, tau_hi = 0;
   int64_t N = 0, S = 0;
   std::vector<int> tdims;
@@ -647,6 +648,10 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
       const int c = cp.n_commits;
       cp.worker[c] = worker[i];
       cp.norm_slot[c] = (int)(V0 + i);
+      if (h->commit_rule == AGN_COMMIT_DYNSGD) {   // Delta = -eta a / (tau_c + 1)
+        cp.per_commit_scale = 1;
+        cp.scale[c] = (float)(-(h->eta / (double)(tau[i] + 1)));
+      }
       int pb = cp.pull_begin[c];
       for (int p : pulls_at[i + 1]) cp.pull_worker[pb++] = p;
       cp.pull_begin[c + 1] = pb;
@@ -772,6 +777,8 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
   if (o.tc_mask < 0 || o.tc_mask > 15) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 15]");
+  if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
+    return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   h->dims.assign(dims, dims + n_dims);
   h->L = n_dims - 1;
   h->n = n_workers;
@@ -784,6 +791,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->S = o.n_samples / n_workers;
   h->dist = o.input_dist;
   h->normalize = o.normalize ? 1 : 0;
+  h->commit_rule = o.commit_rule;
   h->gemm = o.gemm;
   h->tau_lo = o.tau_lo;
   h->tau_hi = o.tau_hi;
@@ -1055,6 +1063,7 @@ void agn_default_options(agn_options* o) {
   o->gemm = AGN_GEMM_AUTO;
   o->tau_lo = 0;
   o->tau_hi = 0;
+  o->commit_rule = AGN_COMMIT_AGN;
 }
 
 int agn_create(const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t lambda, double eta,

@@ -4,7 +4,8 @@
 // parameter vector once: each thread keeps its slice of theta~ in registers,
 // and for every commit c of the launch reads the committing worker's
 // accumulator, forms Delta = fp32(a * s) with s = fp32(-eta/lambda) (Eq. 1;
-// the normalisation step of Algorithm 1), adds it to theta~ with a plain
+// the normalisation step of Algorithm 1; or a per-commit s = fp32(-eta /
+// (tau_c + 1)) for the DynSGD rule), adds it to theta~ with a plain
 // round-to-nearest add (no FMA, so the sequence is bit-reproducible), zeroes
 // the accumulator (Algorithm 1 restarts a at 0) and writes theta~ into every
 // replica that pulls at the new version (Pull).  theta~ is written back once.
@@ -94,14 +95,15 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u)
           if (live[u]) a[u] = ld_stream(arow + idx[u]);
+        const float sc = plan.per_commit_scale ? plan.scale[c] : s;
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) {
           if (!live[u]) continue;
           float4 d;
-          d.x = __fmul_rn(a[u].x, s);
-          d.y = __fmul_rn(a[u].y, s);
-          d.z = __fmul_rn(a[u].z, s);
-          d.w = __fmul_rn(a[u].w, s);
+          d.x = __fmul_rn(a[u].x, sc);
+          d.y = __fmul_rn(a[u].y, sc);
+          d.z = __fmul_rn(a[u].z, sc);
+          d.w = __fmul_rn(a[u].w, sc);
           th[u].x = __fadd_rn(th[u].x, d.x);
           th[u].y = __fadd_rn(th[u].y, d.y);
           th[u].z = __fadd_rn(th[u].z, d.z);
@@ -140,7 +142,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
     float t = theta_c[i];
     for (int c = 0; c < nc; ++c) {
       float* ap = acc + (int64_t)plan.worker[c] * ld + i;
-      float d = __fmul_rn(*ap, s);
+      float d = __fmul_rn(*ap, plan.per_commit_scale ? plan.scale[c] : s);
       t = __fadd_rn(t, d);
 #pragma unroll
       for (int cc = 0; cc < kMaxCommitsPerLaunch; ++cc)

@@ -74,6 +74,8 @@ struct CommitPlan {
   int32_t pull_begin[kMaxCommitsPerLaunch + 1];
   int32_t pull_worker[kMaxPullsPerLaunch];
   int32_t norm_slot[kMaxCommitsPerLaunch]; // index of commit c in the norm output
+  int32_t per_commit_scale;                // 1: commit c uses scale[c], else the launch's
+  float scale[kMaxCommitsPerLaunch];
 };
 
 // Queue one fused launch for the commits of `plan` plus the partial-norm

@@ -104,3 +104,9 @@ def test_create_validates_before_touching_the_device(agn):
     with pytest.raises(agn.AGNError) as e:
         agn.agn_create((8, 4), 2, 1, 0.1, 1, o)
     assert e.value.code == agn.AGN_E_INVALID
+    o = agn.agn_default_options()
+    assert o.commit_rule == agn.AGN_COMMIT_AGN
+    o.commit_rule = 5
+    with pytest.raises(agn.AGNError) as e:
+        agn.agn_create((8, 4), 2, 1, 0.1, 1, o)
+    assert e.value.code == agn.AGN_E_INVALID

@@ -297,6 +297,80 @@ def test_staleness_reads_the_scheduled_version():
         assert np.allclose(r.snapshots[c], V[-1], rtol=0, atol=1e-15)
 
 
+# ----------------------------------------------------------------------------
+# DynSGD-style staleness-scaled commit (Section 4's comparison)
+# ----------------------------------------------------------------------------
+
+def _local_sum(mlp, theta_start, X, y, k, t0, lam, eta, m, S):
+    theta = theta_start.copy()
+    a = np.zeros_like(theta)
+    for i in range(lam):
+        rows = k * S + ((t0 + i) * m + np.arange(m)) % S
+        _, g = mlp.loss_grad(theta, X[rows], y[rows])
+        a -= eta * g
+        theta -= eta * g
+    return a
+
+
+def test_dynsgd_scales_each_commit_by_its_staleness():
+    """Commit c adds the worker's accumulated update divided by tau_c + 1,
+    tau_c = c - v_c (an independent step-by-step loop)."""
+    rng = np.random.default_rng(7)
+    dims, m, S, lam, eta, n = (4, 3, 3), 2, 5, 3, 0.25, 3
+    mlp = O.MLP(dims)
+    X, y = rng.uniform(size=(n * S, dims[0])), rng.integers(0, dims[-1], n * S)
+    th0 = rng.normal(0, 0.5, mlp.num_params)
+    worker = [0, 1, 2, 0, 1, 2, 1]
+    tau = [0, 1, 2, 2, 1, 2, 0]
+    r = O.agn_run(mlp, th0, n, lam, eta, worker, tau, _ListData(X, y), m, S,
+                  snapshot_at=range(len(worker)), staleness_scaled=True)
+    V = [th0]
+    steps = [0] * n
+    for c, (w, t) in enumerate(zip(worker, tau)):
+        d = _local_sum(mlp, V[c - t], X, y, w, steps[w], lam, eta, m, S) / (t + 1)
+        steps[w] += lam
+        V.append(V[-1] + d)
+        assert np.allclose(r.snapshots[c], V[-1], rtol=0, atol=1e-15)
+
+
+def test_dynsgd_without_staleness_is_the_unnormalised_ablation():
+    rng = np.random.default_rng(8)
+    dims, m, S, lam = (5, 4, 3), 3, 9, 4
+    mlp = O.MLP(dims)
+    X, y = rng.uniform(size=(S, dims[0])), rng.integers(0, dims[-1], S)
+    th0 = rng.normal(0, 0.4, mlp.num_params)
+    d = _ListData(X, y)
+    w, tau = [0, 0, 0], [0, 0, 0]
+    r_dyn = O.agn_run(mlp, th0, 1, lam, 0.1, w, tau, d, m, S, staleness_scaled=True)
+    r_un = O.agn_run(mlp, th0, 1, lam, 0.1, w, tau, d, m, S, normalize=False)
+    assert np.array_equal(r_dyn.theta, r_un.theta)
+
+
+def test_dynsgd_commits_from_one_version_scale_as_one_over_tau_plus_one():
+    """The first n commits all read version 0 (tau_c = c), so every rule
+    computes the same accumulated updates a_c; DynSGD adds a_c / (c + 1) where
+    the un-normalised ablation adds a_c."""
+    rng = np.random.default_rng(9)
+    n = 4
+    dims, m, S, lam = (4, 3, 3), 2, 6, 3
+    mlp = O.MLP(dims)
+    X, y = rng.uniform(size=(n * S, dims[0])), rng.integers(0, dims[-1], n * S)
+    th0 = rng.normal(0, 0.4, mlp.num_params)
+    d = _ListData(X, y)
+    w, tau = list(range(n)), list(range(n))
+    r_dyn = O.agn_run(mlp, th0, n, lam, 0.2, w, tau, d, m, S, staleness_scaled=True,
+                      snapshot_at=range(n))
+    r_un = O.agn_run(mlp, th0, n, lam, 0.2, w, tau, d, m, S, normalize=False,
+                     snapshot_at=range(n))
+    prev_un, expect = th0, th0.copy()
+    for c in range(n):
+        a_c = r_un.snapshots[c] - prev_un
+        prev_un = r_un.snapshots[c]
+        expect = expect + a_c / (c + 1)
+        assert np.allclose(r_dyn.snapshots[c], expect, rtol=0, atol=1e-15)
+        assert math.isclose(r_dyn.delta_norm[c] * (c + 1), r_un.delta_norm[c], rel_tol=1e-12)
+
+
 def test_schedule_feasibility():
     v = O.schedule_versions(3, [0, 1, 2, 0, 1, 2], [0, 1, 2, 2, 2, 2])
     assert list(v) == [0, 0, 0, 1, 2, 3]
