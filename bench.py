@@ -175,7 +175,8 @@ def run_reference(args, wl):
 
     def step():
         O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:per_step], tau[:per_step], ds, wl.batch,
-                  wl.shard, dtype=dtype, staleness_scaled=args.commit_rule == "dynsgd")
+                  wl.shard, dtype=dtype, staleness_scaled=args.commit_rule == "dynsgd",
+                  elide_accumulator=args.elide_accumulator)
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
@@ -253,7 +254,7 @@ def run_agn(args, wl):
                 n_samples=wl.n_samples, input_dist=wl.dist, teacher_dims=wl.teacher_dims,
                 normalize=wl.normalize, gemm=GEMMS[args.gemm], stream=st.cuda_stream,
                 commit_rule=agn.AGN_COMMIT_DYNSGD if args.commit_rule == "dynsgd"
-                else agn.AGN_COMMIT_AGN)
+                else agn.AGN_COMMIT_AGN, elide_accumulator=int(args.elide_accumulator))
 
     def barrier():
         if ws > 1:
@@ -378,6 +379,7 @@ def run_agn(args, wl):
         "data": "synthetic (seeded MNIST-shaped teacher-labelled set; MNIST itself unavailable)",
         "config": {"workload": wl.name, "commits_per_step": per_step,
                    "commit_rule": args.commit_rule,
+                   "accumulator": "elided" if args.elide_accumulator else "kept",
                    "parallelism": "replicas" if ws > 1 else "single GPU",
                    "l2": "inputs larger than L2 (dataset 188 MB + replicas and accumulators "
                          "230 MB vs 129 MB L2)" if args.workload == "mnist" else
@@ -411,6 +413,8 @@ def main():
     ap.add_argument("--gemm", default="auto", choices=sorted(GEMMS))
     ap.add_argument("--commit-rule", default="agn", choices=["agn", "dynsgd"],
                     help="AGN's commit (Eq. 1) or the DynSGD-style staleness-scaled commit")
+    ap.add_argument("--elide-accumulator", action="store_true",
+                    help="keep no gradient accumulator; commit from the pulled parameters")
     ap.add_argument("--workers", type=int, default=0,
                     help="override n (profiling captures of a smaller case)")
     ap.add_argument("--ref-commits", type=int, default=2)

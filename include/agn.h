@@ -99,6 +99,13 @@ typedef struct agn_options {
      Delta = -eta a / (tau_c + 1), tau_c the schedule's staleness of commit c
      (the DynSGD comparison of Section 4; normalize is ignored). */
   int32_t commit_rule;
+  /* 1: keep no gradient accumulator.  Each worker keeps the theta~ it
+     pulled (theta_pull) and a commit adds (theta_k - theta_pull) scaled by
+     1/lambda (1/(tau_c + 1) for DynSGD, 1 without normalisation), which
+     equals -eta a / lambda in exact arithmetic (the sum of the local updates,
+     Algorithm 1).  Saves the accumulator's 8 bytes per parameter and local
+     step; the paper has no such variant.  Not with tc_mask bit 3. */
+  int32_t elide_accumulator;
 } agn_options;
 
 void agn_default_options(agn_options* opt);

@@ -208,7 +208,7 @@ class AGNResult:
 
 def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
             normalize=True, snapshot_at=(), keep_locals=(), dtype=np.float64,
-            staleness_scaled=False):
+            staleness_scaled=False, elide_accumulator=False):
     """Run the commits of one schedule through the FIFO parameter server.
 
     model      : object with loss_grad(theta, X, y) -> (loss, grad)
@@ -226,6 +226,11 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
     (Section 4): the accumulated update divided by tau_c + 1, where
     tau_c = c - v_c is the number of commits between the worker's pull and
     its commit, instead of by lambda (`normalize` is then ignored).
+
+    elide_accumulator: no accumulator; the commit is formed from the local
+    iterate and the pulled parameters, (theta_lambda - theta_pull) scaled the
+    same way.  Equal to the accumulated form in exact arithmetic (the
+    accumulated updates telescope).
     """
     worker = np.asarray(worker, dtype=np.int64)
     v = schedule_versions(n, worker, tau)
@@ -251,6 +256,7 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
         k = int(worker[c])
         vc = int(v[c])
         theta = snaps[vc].copy()                       # Pull
+        snaps_pull = theta.copy() if elide_accumulator else None
         readers[vc].remove(c)
         if not readers[vc]:
             del snaps[vc]
@@ -267,6 +273,8 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
             losses.append(li)
             if iterates is not None:
                 iterates.append(theta.copy())
+        if elide_accumulator:
+            a = theta - snaps_pull                      # sum of the local updates
         if staleness_scaled:
             a = a / dtype(c - vc + 1)                   # DynSGD: 1 / (tau_c + 1)
         elif normalize:

@@ -229,13 +229,14 @@ class AGN:
     def __init__(self, dims, n_workers, lam, eta, seed, *, precision=AGN_PREC_FP32, batch=32,
                  n_samples=2048, input_dist=AGN_DIST_UNIFORM, teacher_dims=None, normalize=1,
                  gemm=AGN_GEMM_AUTO, tau_lo=0, tau_hi=0, stream=None, x=None, y=None,
-                 theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN):
+                 theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN, elide_accumulator=0):
         o = agn_default_options()
         o.precision, o.batch, o.n_samples = int(precision), int(batch), int(n_samples)
         o.input_dist, o.normalize, o.gemm = int(input_dist), int(normalize), int(gemm)
         o.tau_lo, o.tau_hi = int(tau_lo), int(tau_hi)
         o.tc_mask = int(tc_mask)
         o.commit_rule = int(commit_rule)
+        o.elide_accumulator = int(elide_accumulator)
         keep = []
         if teacher_dims is not None:
             td, tdp = _i32(teacher_dims)

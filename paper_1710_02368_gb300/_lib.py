@@ -59,6 +59,7 @@ class agn_options(C.Structure):
         ("theta_init", C.POINTER(C.c_float)),
         ("tc_mask", C.c_int32),
         ("commit_rule", C.c_int32),
+        ("elide_accumulator", C.c_int32),
     ]
 
 

@@ -59,6 +59,9 @@ struct agn_handle {
   uint64_t seed = 0;
   int prec = AGN_PREC_FP32, m = 32, dist = AGN_DIST_UNIFORM, normalize = 1, gemm = 0;
   int commit_rule = AGN_COMMIT_AGN;
+  // accumulator elided: `acc` holds each worker's theta at its last pull and
+  // a commit adds (theta_k - theta_pull) scaled by 1/lambda (or 1/(tau+1), 1)
+  bool elide = false;
   int tau_lo = 0, tau_hi = 0;
   int64_t N = 0, S = 0;
   std::vector<int> tdims;
@@ -254,7 +257,7 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.counter = h->tc_counter;
   t.err = h->flag + 1;
   t.theta = h->rep;
-  t.acc = h->acc;
+  t.acc = h->elide ? nullptr : h->acc;
   t.theta_b = h->rep_b;
   t.ld_param = h->P_pad;
   t.piece_plane = h->piece_plane;
@@ -344,7 +347,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   const double es = (double)sizeof(T);
   // bytes per parameter of the local step + accumulation: theta RMW, a RMW, and
   // the low-precision copy (one bf16, or three pieces in the split mode)
-  const double upd = 16.0 + (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
+  const double upd = (h->elide ? 8.0 : 16.0) +
+                     (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
   // pieces of dZ_l (split mode, hidden tensor-core layers), planes n m d_l apart
   auto dz_pieces = [&](int l) -> bf16* {
     return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZp[l] : nullptr;
@@ -505,7 +509,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       if (l == L && h->use_head) {   // narrow output layer
         agn::HeadDwArgs d{};
         d.H = Hprev; d.dZL = h->dZ[l]; d.slot_worker = sw;
-        d.theta = h->rep; d.acc = h->acc; d.theta_b = h->rep_b; d.piece_plane = h->piece_plane;
+        d.theta = h->rep; d.acc = h->elide ? nullptr : h->acc; d.theta_b = h->rep_b;
+        d.piece_plane = h->piece_plane;
         d.ld_param = h->P_pad; d.woff = h->woff[l - 1]; d.boff = h->boff[l - 1];
         d.K = fi; d.C = fo; d.m = m; d.eta = eta;
         AGN_TRY(agn::head_backward_dw<T>(d, s, h->stream));
@@ -515,7 +520,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         g.a = h->dZ[l]; g.lda = fo; g.a_bstride = (int64_t)m * fo;
         g.b = Hprev; g.ldb = fi; g.b_bstride = (int64_t)m * fi;
         g.slot_worker = sw;
-        g.theta = h->rep; g.acc = h->acc; g.theta_bf16 = h->rep_b; g.ld_param = h->P_pad;
+        g.theta = h->rep; g.acc = h->elide ? nullptr : h->acc; g.theta_bf16 = h->rep_b;
+        g.ld_param = h->P_pad;
         g.piece_plane = h->piece_plane;
         g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
         AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
@@ -650,7 +656,8 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
       cp.norm_slot[c] = (int)(V0 + i);
       if (h->commit_rule == AGN_COMMIT_DYNSGD) {   // Delta = -eta a / (tau_c + 1)
         cp.per_commit_scale = 1;
-        cp.scale[c] = (float)(-(h->eta / (double)(tau[i] + 1)));
+        cp.scale[c] = h->elide ? (float)(1.0 / (double)(tau[i] + 1))
+                               : (float)(-(h->eta / (double)(tau[i] + 1)));
       }
       int pb = cp.pull_begin[c];
       for (int p : pulls_at[i + 1]) cp.pull_worker[pb++] = p;
@@ -706,9 +713,14 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     Launch k(h, AGN_K_OTHER, 0.0,
              (double)h->P * (4.0 + plan.start_pulls.size() * (h->rep_b ? 6.0 : 4.0)), &launches);
     AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
-                               (int)plan.start_pulls.size(), h->stream, h->piece_plane));
+                               (int)plan.start_pulls.size(), h->stream, h->piece_plane,
+                               h->elide ? h->acc : nullptr));
   }
-  const float scale = (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
+  // commit scale: of the raw gradient sum a (-eta / lambda, or -eta without
+  // normalisation), or, with the accumulator elided, of theta_k - theta_pull
+  // (which already carries -eta): 1 / lambda, or 1
+  const float scale = h->elide ? (float)(h->normalize ? 1.0 / (double)h->lam : 1.0)
+                               : (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
   for (const Wave& wv : plan.waves) {
     if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
     else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
@@ -717,11 +729,13 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
       {
         const double copy_b = h->split ? 6.0 : h->rep_b ? 2.0 : 0.0;
         Launch kc(h, AGN_K_COMMIT, 2.0 * cp.n_commits * h->P,
-                  (double)h->P * (8.0 + 8.0 * cp.n_commits + pulls * (4.0 + copy_b)),
+                  (double)h->P * (8.0 + 8.0 * cp.n_commits +
+                                  pulls * (4.0 + copy_b + (h->elide ? 4.0 : 0.0))),
                   &launches);
         AGN_TRY(agn::launch_commit_pull(cp, h->theta_c, h->acc, h->rep, h->rep_b, h->P_pad,
                                         h->P_pad, scale, true, h->partials, h->grid, nullptr,
-                                        nullptr, h->stream, /*norms=*/false, h->piece_plane));
+                                        nullptr, h->stream, /*norms=*/false, h->piece_plane,
+                                        h->elide));
       }
       Launch kn(h, AGN_K_NORMS, 0.0, 8.0 * cp.n_commits * h->grid, &launches);
       AGN_TRY(agn::launch_commit_norms(cp, h->partials, h->grid, h->dnorm, h->flag, h->stream));
@@ -779,6 +793,9 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tc_mask < 0 || o.tc_mask > 15) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 15]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
+  if (o.elide_accumulator && (o.tc_mask & 8))
+    return Status::Err(AGN_E_UNSUPPORTED,
+                       "the one-tile-per-CTA dW kernel (tc_mask bit 3) keeps the accumulator");
   h->dims.assign(dims, dims + n_dims);
   h->L = n_dims - 1;
   h->n = n_workers;
@@ -792,6 +809,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->dist = o.input_dist;
   h->normalize = o.normalize ? 1 : 0;
   h->commit_rule = o.commit_rule;
+  h->elide = o.elide_accumulator != 0;
   h->gemm = o.gemm;
   h->tau_lo = o.tau_lo;
   h->tau_hi = o.tau_hi;
@@ -936,7 +954,8 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,
                                h->stream));
   AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
-                             (int)n, h->stream, h->piece_plane));   // every worker pulls version 0
+                             (int)n, h->stream, h->piece_plane,
+                             h->elide ? h->acc : nullptr));   // every worker pulls version 0
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
   return Status::Ok();
 }

@@ -62,7 +62,11 @@ __device__ __forceinline__ void pack_pieces_x4(float4 v, uint2& p0, uint2& p1, u
 // kCopy: 0 = fp32 replicas only, 1 = plus a bf16 copy, 3 = plus the three
 // exact bf16 pieces (planes `plane` elements apart) of the fp32 mode's
 // tensor-core operands.
-template <int kCopy>
+// kElide: no accumulators.  `acc` then holds each worker's snapshot theta_pull
+// of its last pull, the committed quantity is fp32(theta_k - theta_pull) (the
+// sum of the local updates) with s = fp32(1/lambda) (or fp32(1/(tau_c + 1)),
+// or 1), and every pull also refreshes the snapshot.
+template <int kCopy, bool kElide>
 __global__ void __launch_bounds__(kThreads)
 commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ theta_c,
                    float* __restrict__ acc, float* __restrict__ replicas,
@@ -92,9 +96,21 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
       if (c < nc) {
         float4* arow = reinterpret_cast<float4*>(acc + (int64_t)plan.worker[c] * ld);
         float4 a[kUnroll];
+        if (kElide) {
+          const float4* krow =
+              reinterpret_cast<const float4*>(replicas + (int64_t)plan.worker[c] * ld);
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u)
-          if (live[u]) a[u] = ld_stream(arow + idx[u]);
+          for (int u = 0; u < kUnroll; ++u) {
+            if (!live[u]) continue;
+            const float4 tk = ld_stream(krow + idx[u]), tp = ld_stream(arow + idx[u]);
+            a[u] = make_float4(__fsub_rn(tk.x, tp.x), __fsub_rn(tk.y, tp.y),
+                               __fsub_rn(tk.z, tp.z), __fsub_rn(tk.w, tp.w));
+          }
+        } else {
+#pragma unroll
+          for (int u = 0; u < kUnroll; ++u)
+            if (live[u]) a[u] = ld_stream(arow + idx[u]);
+        }
         const float sc = plan.per_commit_scale ? plan.scale[c] : s;
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) {
@@ -110,7 +126,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
           th[u].w = __fadd_rn(th[u].w, d.w);
           float q = d.x * d.x + d.y * d.y + d.z * d.z + d.w * d.w;
           sq[c] += (double)q;
-          if (zero_acc) st_stream(arow + idx[u], make_float4(0.f, 0.f, 0.f, 0.f));
+          if (!kElide && zero_acc) st_stream(arow + idx[u], make_float4(0.f, 0.f, 0.f, 0.f));
         }
         for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
           const int64_t row = (int64_t)plan.pull_worker[p] * ld;
@@ -119,6 +135,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
           for (int u = 0; u < kUnroll; ++u) {
             if (!live[u]) continue;
             rrow[idx[u]] = th[u];
+            if (kElide) reinterpret_cast<float4*>(acc + row)[idx[u]] = th[u];
             if (kCopy == 1) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
             if (kCopy == 3) {
               uint2 q0, q1, q2;
@@ -142,15 +159,17 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
     float t = theta_c[i];
     for (int c = 0; c < nc; ++c) {
       float* ap = acc + (int64_t)plan.worker[c] * ld + i;
-      float d = __fmul_rn(*ap, plan.per_commit_scale ? plan.scale[c] : s);
+      const float av = kElide ? __fsub_rn(replicas[(int64_t)plan.worker[c] * ld + i], *ap) : *ap;
+      float d = __fmul_rn(av, plan.per_commit_scale ? plan.scale[c] : s);
       t = __fadd_rn(t, d);
 #pragma unroll
       for (int cc = 0; cc < kMaxCommitsPerLaunch; ++cc)
         if (cc == c) sq[cc] += (double)(d * d);
-      if (zero_acc) *ap = 0.f;
+      if (!kElide && zero_acc) *ap = 0.f;
       for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
         const int64_t row = (int64_t)plan.pull_worker[p] * ld;
         replicas[row + i] = t;
+        if (kElide) acc[row + i] = t;
         if (kCopy == 1) rep_bf16[row + i] = __float2bfloat16_rn(t);
         if (kCopy == 3) {
           const bf16 q0 = __float2bfloat16_rn(t);
@@ -227,20 +246,22 @@ int commit_grid(int64_t P) {
 Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, float* replicas,
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale, bool zero_acc,
                           double* partials, int grid, float* delta_norm, int* flag,
-                          cudaStream_t stream, bool norms, int64_t piece_plane) {
+                          cudaStream_t stream, bool norms, int64_t piece_plane, bool elide) {
   if (plan.n_commits <= 0) return Status::Ok();
   const int z = zero_acc ? 1 : 0;
+  auto go = [&](auto kern, bf16* rb, int64_t plane) {
+    kern<<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas, rb, P, ld, scale, z,
+                                        partials, plane);
+  };
   if (replicas_bf16 && piece_plane > 0)
-    commit_pull_kernel<3><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
-                                                          replicas_bf16, P, ld, scale, z, partials,
-                                                          piece_plane);
+    elide ? go(commit_pull_kernel<3, true>, replicas_bf16, piece_plane)
+          : go(commit_pull_kernel<3, false>, replicas_bf16, piece_plane);
   else if (replicas_bf16)
-    commit_pull_kernel<1><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas,
-                                                          replicas_bf16, P, ld, scale, z, partials,
-                                                          0);
+    elide ? go(commit_pull_kernel<1, true>, replicas_bf16, 0)
+          : go(commit_pull_kernel<1, false>, replicas_bf16, 0);
   else
-    commit_pull_kernel<0><<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas, nullptr, P,
-                                                          ld, scale, z, partials, 0);
+    elide ? go(commit_pull_kernel<0, true>, nullptr, 0)
+          : go(commit_pull_kernel<0, false>, nullptr, 0);
   AGN_TRY_CUDA(cudaGetLastError());
   if (norms && partials && (delta_norm || flag))
     return launch_commit_norms(plan, partials, grid, delta_norm, flag, stream);
@@ -265,13 +286,15 @@ namespace {
 __global__ void __launch_bounds__(kThreads)
 pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
             bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers,
-            int64_t plane) {
+            int64_t plane, float* __restrict__ snapshot) {
   const int k = workers[blockIdx.y];
   float* dst = replicas + (int64_t)k * ld;
+  float* snap = snapshot ? snapshot + (int64_t)k * ld : nullptr;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < P; i += stride) {
     const float t = theta_c[i];
     dst[i] = t;
+    if (snap) snap[i] = t;
     if (rep_bf16) {
       const int64_t o = (int64_t)k * ld + i;
       if (plane > 0) {
@@ -300,11 +323,11 @@ __global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda
 
 Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
                      int64_t ld, const int* workers, int count, cudaStream_t st,
-                     int64_t piece_plane) {
+                     int64_t piece_plane, float* snapshot) {
   if (count <= 0) return Status::Ok();
   dim3 grid((unsigned)std::max(1, commit_grid(P) / std::max(1, count) + 1), (unsigned)count);
   pull_kernel<<<grid, kThreads, 0, st>>>(theta_c, replicas, replicas_bf16, P, ld, workers,
-                                         piece_plane);
+                                         piece_plane, snapshot);
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -86,7 +86,8 @@ Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, fl
                           bf16* replicas_bf16, int64_t P, int64_t ld, float scale,
                           bool zero_acc, double* partials, int grid, float* delta_norm,
                           int* flag, cudaStream_t stream, bool norms = true,
-                          int64_t piece_plane = 0);   // > 0: pulls write 3 pieces
+                          int64_t piece_plane = 0,   // > 0: pulls write 3 pieces
+                          bool elide = false);       // acc holds pull snapshots (no accumulators)
 // The per-commit norm reduction of one launch of launch_commit_pull (when
 // that launch was queued with norms = false).
 Status launch_commit_norms(const CommitPlan& plan, const double* partials, int grid,

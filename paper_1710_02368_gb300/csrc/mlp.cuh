@@ -35,7 +35,7 @@ struct GemmArgs {
   int64_t mask_bstride;
   int relu;
   float* theta;          // fp32 master replicas [n][ld_param]
-  float* acc;            // accumulators [n][ld_param]
+  float* acc;            // accumulators [n][ld_param], or null (accumulator elided)
   bf16* theta_bf16;      // bf16 working copies or null
   int64_t piece_plane;   // > 0: theta_bf16 holds three exact bf16 pieces, planes this far apart
   int64_t ld_param;
@@ -90,7 +90,7 @@ struct HeadDwArgs {
   const void* dZL;         // dZ_L [slots][m][C] (T)
   const int* slot_worker;
   float* theta;            // fp32 master replicas [n][ld_param]
-  float* acc;              // accumulators [n][ld_param]
+  float* acc;              // accumulators [n][ld_param], or null (accumulator elided)
   bf16* theta_b;           // bf16 copies (or piece 0 of three planes), or null
   int64_t piece_plane;     // > 0: three piece planes this far apart
   int64_t ld_param, woff, boff;
@@ -105,9 +105,10 @@ bool head_fits(int K, int C);
 
 // Pull: copy theta~ into the replicas of `workers` (device list) and their bf16 copies.
 // piece_plane > 0: replicas_bf16 holds three piece planes (fp32 mode on tensor cores).
+// snapshot (accumulator elided): also copy theta~ into the workers' rows there.
 Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16, int64_t P,
                      int64_t ld, const int* workers, int count, cudaStream_t st,
-                     int64_t piece_plane = 0);
+                     int64_t piece_plane = 0, float* snapshot = nullptr);
 // loss[c] = mean_i parts[c * lambda + i] for c < count.
 Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st);
 // Device-side standalone-commit input generator.

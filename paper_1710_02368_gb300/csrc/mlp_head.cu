@@ -252,12 +252,12 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
   for (int c = 0; c < kMaxC; ++c) red[(warp * kMaxC + c) * 32 + lane] = g[c];
   __syncthreads();
   float* theta = a.theta + (int64_t)w * a.ld_param;
-  float* acc = a.acc + (int64_t)w * a.ld_param;
+  float* acc = a.acc ? a.acc + (int64_t)w * a.ld_param : nullptr;   // null: elided
   bf16* tb = a.theta_b ? a.theta_b + (int64_t)w * a.ld_param : nullptr;
   auto update = [&](int64_t p, float gr, float th, float ac) {
     const float t = fmaf(-a.eta, gr, th);
     theta[p] = t;
-    acc[p] = ac + gr;
+    if (acc) acc[p] = ac + gr;
     if (tb) {
       if (a.piece_plane > 0) {
         bf16 q0, q1, q2;
@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       if (c < C) {
         const int64_t p = a.woff + (int64_t)c * K + k;
         th[e] = theta[p];
-        ac[e] = acc[p];
+        ac[e] = acc ? acc[p] : 0.f;
         float v = 0.f;
 #pragma unroll
         for (int r = 0; r < kDwGroups; ++r) v += red[(r * kMaxC + c) * 32 + lane];
@@ -298,7 +298,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       for (int j = lane; j < m; j += 32) v += cvt(dz[j * C + c]);
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (lane == 0) update(a.boff + c, v, theta[a.boff + c], acc[a.boff + c]);
+      if (lane == 0) update(a.boff + c, v, theta[a.boff + c], acc ? acc[a.boff + c] : 0.f);
     }
   }
 }

@@ -141,8 +141,9 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         out[m * g.ldo + n] = from_f<TO>(h > 0.f ? acc[i][j] : 0.f);
       }
     }
-  } else {   // kEpiDW: theta_k -= eta g, a_k += g, bf16 copy refresh
-    float* a = g.acc + (int64_t)w * g.ld_param;
+  } else {   // kEpiDW: theta_k -= eta g, a_k += g (unless elided), bf16 copy refresh
+    const bool has_a = g.acc != nullptr;
+    float* a = has_a ? g.acc + (int64_t)w * g.ld_param : theta;
     bf16* tb = g.theta_bf16 ? g.theta_bf16 + (int64_t)w * g.ld_param : nullptr;
     // loads of all 16 outputs first, then the updates (memory-level parallelism)
     const float* __restrict__ th_in = theta;
@@ -157,7 +158,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         if (m < g.M && n < g.N) {
           const int64_t p = g.woff + m * g.N + n;
           th[i][j] = __ldcs(th_in + p);
-          av[i][j] = __ldcs(a_in + p);
+          av[i][j] = has_a ? __ldcs(a_in + p) : 0.f;
         }
       }
     }
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         const float gr = acc[i][j];
         const float t = fmaf(-g.eta, gr, th[i][j]);
         theta[p] = t;
-        a[p] = av[i][j] + gr;
+        if (has_a) a[p] = av[i][j] + gr;
         if (tb) write_copy(tb, g.piece_plane, p, t);
       }
     }
@@ -181,7 +182,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       const int64_t p = g.boff + m0 + tid;
       const float t = fmaf(-g.eta, bsum, theta[p]);
       theta[p] = t;
-      a[p] += bsum;
+      if (has_a) a[p] += bsum;
       if (tb) write_copy(tb, g.piece_plane, p, t);
     }
   }

@@ -56,16 +56,19 @@ constexpr int kEpiWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kCF = 32;                        // output features per parameter chunk
 constexpr int kChunkBytes = kCF * 128 * 4;     // one fp32 chunk: 32 rows x 128 inputs
-constexpr int kBiasBytes = 2 * kCF * 4;       // b_l and its accumulator for one chunk
-constexpr int kSlotBytes = 2 * kChunkBytes + kBiasBytes;   // one ring slot
-constexpr int kRing = 3;                       // chunks (theta and a) in flight
+constexpr int kBiasHalf = kCF * 4;            // b_l (or its accumulator) for one chunk
 constexpr uint64_t kWaitNs = 2000000000ull;    // 2 s
 
 // kBK samples per stage: one TMA box is 64 MN-elements x kBK samples of bf16
 // (kBK rows of 128 bytes, 128-byte swizzle); A = two boxes (128 inputs),
 // B = BN / 64 boxes.
-template <int BN, int kSplit, int kStages, int kBKs>
+// kAcc: theta_k and a_k per chunk (3 slots in flight); without the
+// accumulator (elided, commits from a pull snapshot) theta_k alone (6 slots).
+template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
 struct DwCfg {
+  static constexpr int kArrays = kAcc ? 2 : 1;
+  static constexpr int kSlotBytes = kArrays * (kChunkBytes + kBiasHalf);
+  static constexpr int kRing = kAcc ? 3 : 6;
   static constexpr int kBK = kBKs;
   static constexpr int kBox = kBK * 128;
   static constexpr int kABytes = 2 * kBox;
@@ -153,10 +156,11 @@ __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
   }
 }
 
-template <int BN, int kSplit, int kStages, int kBKs>
+template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
-  using Cfg = DwCfg<BN, kSplit, kStages, kBKs>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kAcc>;
+  constexpr int kRing = Cfg::kRing, kSlotBytes = Cfg::kSlotBytes;
   constexpr int kBK = Cfg::kBK, kABytes = Cfg::kABytes, kBox = Cfg::kBox;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -267,15 +271,18 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           }
           uint8_t* dst = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
           const int f0 = ti.n_tile * BN + c * kCF;
-          tc::mbar_arrive_expect_tx(&cfull[r], 2 * kChunkBytes + (bias_tile ? kBiasBytes : 0));
+          constexpr int kA = Cfg::kArrays;
+          tc::mbar_arrive_expect_tx(&cfull[r], kA * (kChunkBytes + (bias_tile ? kBiasHalf : 0)));
           tc::tma_load_3d(dst, &B.th[ti.layer], &cfull[r], ti.m_tile * 128, f0, worker);
-          tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
-                          worker);
+          if (kAcc)
+            tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
+                            worker);
           if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
             const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
-            tc::bulk_load(dst + 2 * kChunkBytes, args.theta + pb, kBiasBytes / 2, &cfull[r]);
-            tc::bulk_load(dst + 2 * kChunkBytes + kBiasBytes / 2, args.acc + pb, kBiasBytes / 2,
-                          &cfull[r]);
+            tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
+            if (kAcc)
+              tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
+                            &cfull[r]);
           }
           ++ch;
         }
@@ -379,7 +386,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
                              (uint32_t)(16 * hf);
       const int64_t rbase = (int64_t)worker * args.ld_param;
       float* theta = args.theta + rbase;
-      float* acc = args.acc + rbase;
+      float* acc = kAcc ? args.acc + rbase : nullptr;
       bf16* tb = args.theta_b + rbase;
       const int nch = min(Cfg::kChunks, (N - ti.n_tile * BN + kCF - 1) / kCF);
       for (int c = 0; c < nch; ++c) {
@@ -413,17 +420,19 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
               const int so = (16 * hf + i) * 128 + 32 * g + k4;   // in the fp32 chunks
               const float4 tv = *reinterpret_cast<const float4*>(
                   reinterpret_cast<const float*>(slot) + so);
-              const float4 av = *reinterpret_cast<const float4*>(
-                  reinterpret_cast<const float*>(slot + kChunkBytes) + so);
               float tn[4];
               tn[0] = fmaf(-eta, gv.x, tv.x);
               tn[1] = fmaf(-eta, gv.y, tv.y);
               tn[2] = fmaf(-eta, gv.z, tv.z);
               tn[3] = fmaf(-eta, gv.w, tv.w);
-              const float4 an = make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w);
               const int64_t p = L.woff + (int64_t)(fbase + i) * M + k0 + k4;
               *reinterpret_cast<float4*>(theta + p) = make_float4(tn[0], tn[1], tn[2], tn[3]);
-              *reinterpret_cast<float4*>(acc + p) = an;
+              if (kAcc) {
+                const float4 av = *reinterpret_cast<const float4*>(
+                    reinterpret_cast<const float*>(slot + kChunkBytes) + so);
+                *reinterpret_cast<float4*>(acc + p) =
+                    make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w);
+              }
               if (kSplit == 1) {
                 *reinterpret_cast<uint2*>(tb + p) = bf16x4(tn);
               } else {
@@ -437,13 +446,13 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           }
         }
         if (kb >= 0 && kb < 32 && lane < 16 && fbase + lane < N) {   // bias row: b_l[f]
-          const float* sTb = reinterpret_cast<const float*>(slot + 2 * kChunkBytes);
-          const float* sAb = sTb + kCF;
+          const float* sTb =
+              reinterpret_cast<const float*>(slot + Cfg::kArrays * kChunkBytes);
           const float gb = gS[lane * 32 + kb];
           const int64_t pb = L.boff + fbase + lane;
           const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
           theta[pb] = tn;
-          acc[pb] = sAb[16 * hf + lane] + gb;
+          if (kAcc) acc[pb] = sTb[kCF + 16 * hf + lane] + gb;
           if (kSplit == 1) {
             tb[pb] = __float2bfloat16_rn(tn);
           } else {
@@ -472,13 +481,13 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   if (warp == 1) tc::tmem_dealloc(tmem, Cfg::kTmemCols);
 }
 
-template <int BN, int kSplit, int kStages, int kBKs>
+template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
 Status launch_dw(const DwBatch& batch, const TcArgs& args, int num_sms, cudaStream_t st) {
-  using Cfg = DwCfg<BN, kSplit, kStages, kBKs>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kAcc>;
   static_assert(Cfg::kSmem <= 232448, "shared memory");
   static_assert(Cfg::kSmem > 232448 / 2, "one CTA per SM (all 512 TMEM columns)");
   static_assert(Cfg::kTmemCols == 512, "TMEM columns");
-  auto kern = tc_dw_kernel<BN, kSplit, kStages, kBKs>;
+  auto kern = tc_dw_kernel<BN, kSplit, kStages, kBKs, kAcc>;
   static std::mutex mu;
   static std::set<int> done;
   {
@@ -529,8 +538,11 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
     batch.total_tiles = (int)tiles;
     // split mode: 32 samples per stage, so that two stages fit beside the
     // parameter ring (the next tile's operands land while this one multiplies)
-    Status r = split ? launch_dw<kTcDwBNSplit, 3, 2, 32>(batch, args, num_sms, st)
-                     : launch_dw<kTcDwBN, 1, 2, 64>(batch, args, num_sms, st);
+    const bool acc = args.acc != nullptr;   // null: accumulator elided
+    Status r = split ? (acc ? launch_dw<kTcDwBNSplit, 3, 2, 32, true>(batch, args, num_sms, st)
+                            : launch_dw<kTcDwBNSplit, 3, 2, 32, false>(batch, args, num_sms, st))
+                     : (acc ? launch_dw<kTcDwBN, 1, 2, 64, true>(batch, args, num_sms, st)
+                            : launch_dw<kTcDwBN, 1, 2, 64, false>(batch, args, num_sms, st));
     if (!r.ok()) return r;
   }
   return Status::Ok();

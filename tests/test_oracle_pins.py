@@ -371,6 +371,47 @@ def test_dynsgd_commits_from_one_version_scale_as_one_over_tau_plus_one():
         assert math.isclose(r_dyn.delta_norm[c] * (c + 1), r_un.delta_norm[c], rel_tol=1e-12)
 
 
+# ----------------------------------------------------------------------------
+# Accumulator elision: commit from the pulled parameters
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("rule", ["agn", "unnormalised", "dynsgd"])
+def test_elided_commit_equals_accumulated_commit(rule):
+    """(theta_lambda - theta_pull) = sum of the local updates (they telescope),
+    so committing from the pull snapshot equals committing the accumulator,
+    up to float64 rounding, under every commit rule."""
+    rng = np.random.default_rng(12)
+    dims, m, S, lam, eta, n = (5, 4, 3), 3, 7, 4, 0.2, 3
+    mlp = O.MLP(dims)
+    X, y = rng.uniform(size=(n * S, dims[0])), rng.integers(0, dims[-1], n * S)
+    th0 = rng.normal(0, 0.5, mlp.num_params)
+    worker = [0, 1, 2, 0, 1, 2, 0, 1]
+    tau = [0, 1, 2, 2, 1, 2, 0, 2]
+    kw = dict(normalize=rule != "unnormalised", staleness_scaled=rule == "dynsgd",
+              snapshot_at=range(len(worker)))
+    r_acc = O.agn_run(mlp, th0, n, lam, eta, worker, tau, _ListData(X, y), m, S, **kw)
+    r_eli = O.agn_run(mlp, th0, n, lam, eta, worker, tau, _ListData(X, y), m, S,
+                      elide_accumulator=True, **kw)
+    for c in range(len(worker)):
+        d_acc = r_acc.snapshots[c] - (r_acc.snapshots[c - 1] if c else th0)
+        assert np.max(np.abs(r_eli.snapshots[c] - r_acc.snapshots[c])) <= 1e-12 * np.max(np.abs(d_acc))
+    assert not np.array_equal(r_eli.theta, th0)
+
+
+def test_elided_least_squares_commit_closed_form():
+    """The elided commit against the closed form of the local iteration."""
+    lsq, X, Y, theta0, A, Theta0, Theta_star = _lsq_setup()
+    eta, lam = 0.3, 17
+    S = X.shape[0]
+    r = O.agn_run(lsq, theta0, 1, lam, eta, [0], [0], _ListData(X, Y), S, S,
+                  elide_accumulator=True)
+    ev, Q = np.linalg.eigh(A)
+    Mlam = Q @ np.diag((1 - eta * ev) ** lam) @ Q.T
+    Delta = (Theta0 - Theta_star) @ (Mlam - np.eye(A.shape[0])) / lam
+    expect = _theta_to_flat(Theta0 + Delta, X.shape[1])
+    assert np.max(np.abs(r.theta - expect)) <= 1e-10 * max(1.0, np.max(np.abs(expect)))
+
+
 def test_schedule_feasibility():
     v = O.schedule_versions(3, [0, 1, 2, 0, 1, 2], [0, 1, 2, 2, 2, 2])
     assert list(v) == [0, 0, 0, 1, 2, 3]
