@@ -106,6 +106,10 @@ typedef struct agn_options {
      Algorithm 1).  Saves the accumulator's 8 bytes per parameter and local
      step; the paper has no such variant.  Not with tc_mask bit 3. */
   int32_t elide_accumulator;
+  /* Held-out evaluation set for agn_evaluate: rows [N, N + n_eval) of the
+     seeded generator, labelled by the same teacher (0 = none; not with
+     x_init / y_init). */
+  int64_t n_eval;
 } agn_options;
 
 void agn_default_options(agn_options* opt);
@@ -153,6 +157,29 @@ int agn_replica(agn_handle* h, int32_t k, float* out, int64_t cap);
 
 /* Per commit so far: the mean of its lambda minibatch losses (host out[C]). */
 int agn_loss(agn_handle* h, float* out, int64_t cap);
+
+/*
+ * Loss and accuracy of the current theta~ on the held-out set (the training-
+ * accuracy curves of Section 4): softmax cross-entropy mean and the fraction
+ * of samples whose argmax (lowest index on ties) is the label.  Forward pass in
+ * fp32 on the device (CUDA-core GEMMs), fixed-order reductions; blocks until
+ * done.  loss, accuracy: host floats (nullable); pred: host int32 [n_eval]
+ * predictions (nullable), cap its length.  AGN_E_INVALID without an
+ * evaluation set or with a short pred buffer.  No counterpart call in the
+ * paper, which reports these metrics.
+ */
+int agn_evaluate(agn_handle* h, float* loss, float* accuracy, int32_t* pred, int64_t cap);
+
+/*
+ * Temporal efficiency, Eq. 4: E(a, b) = int_0^m f_a dt / int_0^m f_b dt with m
+ * the shorter of the two curves' end times.  Curve x is sampled at times
+ * tx[0..nx) (non-decreasing, >= 0) with values fx; it is the piecewise-linear
+ * interpolation of its samples, constant at fx[0] on [0, tx[0]] (the paper
+ * does not fix the quadrature).  Host arrays; result in *out.  AGN_E_INVALID
+ * for empty or decreasing curves, no shared time, or a zero denominator.
+ */
+int agn_temporal_efficiency(const double* ta, const double* fa, int64_t na, const double* tb,
+                            const double* fb, int64_t nb, double* out);
 
 /* Per commit so far: ||Delta_c||_2 (host out[C]). */
 int agn_delta_norm(agn_handle* h, float* out, int64_t cap);

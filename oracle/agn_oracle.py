@@ -49,7 +49,7 @@ import numpy as np
 __all__ = [
     "ScheduleError", "MLP", "LeastSquares", "softmax_xent", "batch_rows",
     "schedule_versions", "agn_run", "AGNResult", "commit_pull_fp32",
-    "commit_scale_fp32",
+    "commit_scale_fp32", "evaluate", "temporal_efficiency",
 ]
 
 
@@ -331,3 +331,55 @@ def commit_pull_fp32(theta_c, accs, order, pulls, eta, lam, normalize=True,
         for p in pulls[c]:
             replicas[int(p)] = theta_c.copy()
     return theta_c, accs, replicas, norms
+
+
+# ----------------------------------------------------------------------------
+# Evaluation and temporal efficiency (Section 4, Eq. 4)
+# ----------------------------------------------------------------------------
+
+def evaluate(model, theta, X, y, dtype=np.float64):
+    """(mean softmax cross-entropy, accuracy, predictions) of parameters theta
+    on the rows of X: the forward pass of the model, log-sum-exp with the row
+    maximum subtracted, prediction = argmax with the lowest index on ties."""
+    h = np.asarray(X, dtype=dtype)
+    params = model.unpack(np.asarray(theta, dtype=dtype))
+    for l, (W, b) in enumerate(params):
+        h = h @ W.T + b
+        if l + 1 < len(params):
+            h = np.maximum(h, 0)
+    y = np.asarray(y, dtype=np.int64)
+    zmax = h.max(axis=1, keepdims=True)
+    lse = np.log(np.exp(h - zmax).sum(axis=1)) + zmax[:, 0]
+    loss = float(np.mean(lse - h[np.arange(len(y)), y]))
+    pred = np.argmax(h, axis=1)          # first maximum: the lowest index on ties
+    return loss, float(np.mean(pred == y)), pred
+
+
+def _curve_integral(t, f, m):
+    """Integral over [0, m] of the piecewise-linear interpolation of (t, f),
+    held at f[0] on [0, t[0]]."""
+    t = np.asarray(t, dtype=np.float64)
+    f = np.asarray(f, dtype=np.float64)
+    total = f[0] * min(t[0], m)
+    for i in range(len(t) - 1):
+        t0, t1 = t[i], t[i + 1]
+        if t0 >= m:
+            break
+        if t1 <= t0:
+            continue
+        if t1 > m:                       # the segment is cut at m
+            f_m = f[i] + (f[i + 1] - f[i]) * (m - t0) / (t1 - t0)
+            total += 0.5 * (f[i] + f_m) * (m - t0)
+            break
+        total += 0.5 * (f[i] + f[i + 1]) * (t1 - t0)
+    return total
+
+
+def temporal_efficiency(ta, fa, tb, fb):
+    """Eq. 4: E(a, b) = int_0^m f_a dt / int_0^m f_b dt, m the minimal shared
+    training time (the shorter curve's end).  Each curve is the piecewise-
+    linear interpolation of its samples (the paper leaves the quadrature open)."""
+    m = min(float(ta[-1]), float(tb[-1]))
+    if not m > 0:
+        raise ValueError("no shared training time")
+    return _curve_integral(ta, fa, m) / _curve_integral(tb, fb, m)

@@ -123,6 +123,31 @@ def agn_delta_norm(h) -> np.ndarray:
     return _read_commits(_L().agn_delta_norm, h)
 
 
+def agn_evaluate(h, pred=None):
+    """(loss, accuracy) of theta~ on the handle's held-out set; `pred`, an int32
+    array of n_eval entries, also receives the predictions."""
+    loss, acc = C.c_float(), C.c_float()
+    pp, cap = None, 0
+    if pred is not None:
+        if pred.dtype != np.int32 or not pred.flags.c_contiguous:
+            raise ValueError("pred must be a contiguous int32 array")
+        pp, cap = pred.ctypes.data_as(_lib._I32P), len(pred)
+    _check(_L().agn_evaluate(h, C.byref(loss), C.byref(acc), pp, cap), h)
+    return loss.value, acc.value
+
+
+def agn_temporal_efficiency(ta, fa, tb, fb) -> float:
+    """Eq. 4 on two sampled curves (times non-decreasing, >= 0)."""
+    arrs = [np.ascontiguousarray(x, dtype=np.float64) for x in (ta, fa, tb, fb)]
+    if arrs[0].shape != arrs[1].shape or arrs[2].shape != arrs[3].shape:
+        raise ValueError("each curve needs as many values as times")
+    out = C.c_double()
+    p = [a.ctypes.data_as(_lib._F64P) for a in arrs]
+    _check(_L().agn_temporal_efficiency(p[0], p[1], len(arrs[0]), p[2], p[3], len(arrs[2]),
+                                        C.byref(out)))
+    return out.value
+
+
 def agn_num_params(h) -> int:
     return int(_L().agn_num_params(h))
 
@@ -229,7 +254,8 @@ class AGN:
     def __init__(self, dims, n_workers, lam, eta, seed, *, precision=AGN_PREC_FP32, batch=32,
                  n_samples=2048, input_dist=AGN_DIST_UNIFORM, teacher_dims=None, normalize=1,
                  gemm=AGN_GEMM_AUTO, tau_lo=0, tau_hi=0, stream=None, x=None, y=None,
-                 theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN, elide_accumulator=0):
+                 theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN, elide_accumulator=0,
+                 n_eval=0):
         o = agn_default_options()
         o.precision, o.batch, o.n_samples = int(precision), int(batch), int(n_samples)
         o.input_dist, o.normalize, o.gemm = int(input_dist), int(normalize), int(gemm)
@@ -237,6 +263,8 @@ class AGN:
         o.tc_mask = int(tc_mask)
         o.commit_rule = int(commit_rule)
         o.elide_accumulator = int(elide_accumulator)
+        o.n_eval = int(n_eval)
+        self.n_eval = int(n_eval)
         keep = []
         if teacher_dims is not None:
             td, tdp = _i32(teacher_dims)
@@ -254,6 +282,14 @@ class AGN:
         self.dims = tuple(int(v) for v in dims)
         self.n_samples = int(n_samples)
         self.h = agn_create(dims, n_workers, lam, eta, seed, o)
+
+    def evaluate(self, with_pred=False):
+        """(loss, accuracy[, predictions]) of theta~ on the held-out set."""
+        if not with_pred:
+            return agn_evaluate(self.h)
+        pred = np.empty(self.n_eval, dtype=np.int32)
+        loss, acc = agn_evaluate(self.h, pred)
+        return loss, acc, pred
 
     def run(self, n_commits, worker=None, staleness=None):
         agn_run(self.h, n_commits, worker, staleness)

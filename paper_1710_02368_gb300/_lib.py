@@ -60,6 +60,7 @@ class agn_options(C.Structure):
         ("tc_mask", C.c_int32),
         ("commit_rule", C.c_int32),
         ("elide_accumulator", C.c_int32),
+        ("n_eval", C.c_int64),
     ]
 
 
@@ -77,6 +78,9 @@ SIGNATURES = {
     "agn_replica": (C.c_int, [C.c_void_p, C.c_int32, _F32P, C.c_int64]),
     "agn_loss": (C.c_int, [C.c_void_p, _F32P, C.c_int64]),
     "agn_delta_norm": (C.c_int, [C.c_void_p, _F32P, C.c_int64]),
+    "agn_evaluate": (C.c_int, [C.c_void_p, _F32P, _F32P, _I32P, C.c_int64]),
+    "agn_temporal_efficiency": (C.c_int, [_F64P, _F64P, C.c_int64, _F64P, _F64P, C.c_int64,
+                                          _F64P]),
     "agn_num_params": (C.c_int64, [C.c_void_p]),
     "agn_num_commits": (C.c_int64, [C.c_void_p]),
     "agn_last_run_stats": (C.c_int, [C.c_void_p, _F64P, C.c_int64]),

@@ -62,6 +62,18 @@ struct agn_handle {
   // accumulator elided: `acc` holds each worker's theta at its last pull and
   // a commit adds (theta_k - theta_pull) scaled by 1/lambda (or 1/(tau+1), 1)
   bool elide = false;
+  // held-out evaluation set (rows [N, N + n_eval) of the generator) and the
+  // buffers of its forward pass, chunk rows at a time
+  int64_t n_eval = 0, eval_chunk = 0;
+  float* Xe = nullptr;        // [n_eval][d0] fp32
+  int* ye = nullptr;          // [n_eval]
+  float* He[2] = {nullptr, nullptr};   // [eval_chunk][max hidden d]
+  float* Ze = nullptr;        // [eval_chunk][d_L]
+  float* e_loss = nullptr;    // [n_eval]
+  int* e_correct = nullptr;   // [n_eval]
+  int* e_pred = nullptr;      // [n_eval]
+  float* e_out = nullptr;     // [2]: mean loss, accuracy
+  int* e_sw = nullptr;        // [1] = {0}
   int tau_lo = 0, tau_hi = 0;
   int64_t N = 0, S = 0;
   std::vector<int> tdims;
@@ -793,6 +805,11 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tc_mask < 0 || o.tc_mask > 15) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 15]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
+  if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)
+    return Status::Err(AGN_E_INVALID, "n_eval must be in [0, 2^31]");
+  if (o.n_eval > 0 && (o.x_init || o.y_init))
+    return Status::Err(AGN_E_INVALID,
+                       "the evaluation set is generated: not with caller-supplied inputs");
   if (o.elide_accumulator && (o.tc_mask & 8))
     return Status::Err(AGN_E_UNSUPPORTED,
                        "the one-tile-per-CTA dW kernel (tc_mask bit 3) keeps the accumulator");
@@ -883,6 +900,16 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   }
   if (o.theta_init) std::memcpy(h->htheta0.data(), o.theta_init, h->htheta0.size() * sizeof(float));
   else agn::gen_init(seed, h->dims, h->htheta0.data());
+  std::vector<float> hXe;
+  std::vector<int32_t> hye;
+  if (o.n_eval > 0) {   // held-out rows of the same generator, labelled by the same teacher
+    h->n_eval = o.n_eval;
+    hXe.resize((size_t)(o.n_eval * d0));
+    hye.resize((size_t)o.n_eval);
+    agn::gen_dataset_rows(seed, d0, h->N, o.n_eval, h->dist, hXe.data());
+    auto Ws = agn::gen_teacher(seed, h->tdims);
+    agn::gen_teacher_labels(hXe.data(), o.n_eval, d0, h->dist, h->tdims, Ws, hye.data());
+  }
 
   // device buffers
   const size_t es = elem_size(h);
@@ -914,6 +941,25 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
                                          : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
   AGN_TRY(dalloc_t(h, &h->ce_partial, (size_t)(n * ceil_div(m, agn::kHeadSamples))));
   AGN_TRY(dalloc_t(h, &h->head_counter, (size_t)n));
+  if (h->n_eval > 0) {
+    const int64_t E = h->n_eval;
+    h->eval_chunk = std::min<int64_t>(E, 4096);
+    int maxh = 1;
+    for (int l = 1; l < h->L; ++l) maxh = std::max(maxh, dims[l]);
+    AGN_TRY(dalloc_t(h, &h->Xe, (size_t)(E * d0)));
+    AGN_TRY(dalloc_t(h, &h->ye, (size_t)E));
+    AGN_TRY(dalloc_t(h, &h->He[0], (size_t)(h->eval_chunk * maxh)));
+    AGN_TRY(dalloc_t(h, &h->He[1], (size_t)(h->eval_chunk * maxh)));
+    AGN_TRY(dalloc_t(h, &h->Ze, (size_t)(h->eval_chunk * dims[h->L])));
+    AGN_TRY(dalloc_t(h, &h->e_loss, (size_t)E));
+    AGN_TRY(dalloc_t(h, &h->e_correct, (size_t)E));
+    AGN_TRY(dalloc_t(h, &h->e_pred, (size_t)E));
+    AGN_TRY(dalloc_t(h, &h->e_out, 2));
+    AGN_TRY(dalloc_t(h, &h->e_sw, 1));
+    AGN_TRY_CUDA(cudaMemcpy(h->Xe, hXe.data(), hXe.size() * sizeof(float), cudaMemcpyHostToDevice));
+    AGN_TRY_CUDA(cudaMemcpy(h->ye, hye.data(), hye.size() * sizeof(int32_t), cudaMemcpyHostToDevice));
+    AGN_TRY_CUDA(cudaMemset(h->e_sw, 0, sizeof(int)));
+  }
   AGN_TRY_CUDA(cudaMemsetAsync(h->head_counter, 0, (size_t)n * sizeof(int), h->stream));
   h->grid = agn::commit_grid(h->P_pad);
   AGN_TRY(dalloc_t(h, &h->partials, (size_t)agn::kMaxCommitsPerLaunch * h->grid));
@@ -957,6 +1003,46 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
                              (int)n, h->stream, h->piece_plane,
                              h->elide ? h->acc : nullptr));   // every worker pulls version 0
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  return Status::Ok();
+}
+
+// Loss and accuracy of theta~ on the held-out set: the forward pass on the
+// CUDA-core fp32 GEMMs (theta~ as every row block's weights), then per-sample
+// log-sum-exp / argmax and fixed-order means.
+Status evaluate(agn_handle* h, float* loss, float* accuracy, int32_t* pred, int64_t cap) {
+  if (h->n_eval <= 0)
+    return Status::Err(AGN_E_INVALID, "the handle has no evaluation set (agn_options.n_eval)");
+  if (pred && cap < h->n_eval) return Status::Err(AGN_E_INVALID, "pred shorter than n_eval");
+  const int L = h->L, C = h->dims[L];
+  for (int64_t r0 = 0; r0 < h->n_eval; r0 += h->eval_chunk) {
+    const int rows = (int)std::min<int64_t>(h->eval_chunk, h->n_eval - r0);
+    const float* in = h->Xe + r0 * h->dims[0];
+    for (int l = 1; l <= L; ++l) {
+      const int fi = h->dims[l - 1], fo = h->dims[l];
+      agn::GemmArgs g{};
+      g.M = rows; g.N = fo; g.K = fi;
+      g.a = in; g.lda = fi;
+      g.b = h->theta_c + h->woff[l - 1]; g.ldb = fi;   // b_bstride 0: one weight set
+      g.slot_worker = h->e_sw;
+      float* out = l == L ? h->Ze : h->He[l % 2];
+      g.out = out; g.ldo = fo;
+      g.relu = l < L;
+      g.theta = h->theta_c; g.ld_param = 0; g.boff = h->boff[l - 1];
+      AGN_TRY(agn::simt_forward<float>(g, l == L, 1, h->stream));
+      in = out;
+    }
+    AGN_TRY(agn::eval_logits(h->Ze, h->ye + r0, rows, C, h->e_loss + r0, h->e_correct + r0,
+                             h->e_pred + r0, h->stream));
+  }
+  AGN_TRY(agn::eval_reduce(h->e_loss, h->e_correct, h->n_eval, h->e_out, h->stream));
+  float o2[2];
+  AGN_TRY_CUDA(cudaMemcpyAsync(o2, h->e_out, sizeof(o2), cudaMemcpyDeviceToHost, h->stream));
+  if (pred)
+    AGN_TRY_CUDA(cudaMemcpyAsync(pred, h->e_pred, (size_t)h->n_eval * sizeof(int32_t),
+                                 cudaMemcpyDeviceToHost, h->stream));
+  AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  if (loss) *loss = o2[0];
+  if (accuracy) *accuracy = o2[1];
   return Status::Ok();
 }
 
@@ -1156,6 +1242,19 @@ int agn_loss(agn_handle* h, float* out, int64_t cap) {
   DeviceGuard g(h->device);
   Status s = read_commit_array(h, h->loss, out, cap);
   return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int agn_evaluate(agn_handle* h, float* loss, float* accuracy, int32_t* pred, int64_t cap) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  DeviceGuard g(h->device);
+  Status s = evaluate(h, loss, accuracy, pred, cap);
+  return s.ok() ? AGN_OK : fail(h, s);
+}
+
+int agn_temporal_efficiency(const double* ta, const double* fa, int64_t na, const double* tb,
+                            const double* fb, int64_t nb, double* out) {
+  Status s = agn::temporal_efficiency(ta, fa, na, tb, fb, nb, out);
+  return s.ok() ? AGN_OK : fail(nullptr, s);
 }
 
 int agn_delta_norm(agn_handle* h, float* out, int64_t cap) {

@@ -103,6 +103,17 @@ Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st);
 template <typename T>
 bool head_fits(int K, int C);
 
+// Evaluation (mlp_eval.cu): per-sample loss / correctness / prediction of
+// fp32 logits Z [rows][C] against labels y, and their fixed-order means
+// (out[0] loss, out[1] accuracy).
+Status eval_logits(const float* Z, const int* y, int rows, int C, float* loss, int* correct,
+                   int* pred, cudaStream_t st);
+Status eval_reduce(const float* loss, const int* correct, int64_t E, float* out,
+                   cudaStream_t st);
+// Eq. 4 on two sampled curves (host).
+Status temporal_efficiency(const double* ta, const double* fa, int64_t na, const double* tb,
+                           const double* fb, int64_t nb, double* out);
+
 // Pull: copy theta~ into the replicas of `workers` (device list) and their bf16 copies.
 // piece_plane > 0: replicas_bf16 holds three piece planes (fp32 mode on tensor cores).
 // snapshot (accumulator elided): also copy theta~ into the workers' rows there.

@@ -2,6 +2,7 @@
 include/agn.h declares, its host-side generator reproduces agn_inputs bit for
 bit, and invalid arguments are rejected with the documented codes."""
 
+import math
 import os
 import re
 import subprocess
@@ -110,3 +111,21 @@ def test_create_validates_before_touching_the_device(agn):
     with pytest.raises(agn.AGNError) as e:
         agn.agn_create((8, 4), 2, 1, 0.1, 1, o)
     assert e.value.code == agn.AGN_E_INVALID
+
+
+def test_temporal_efficiency_through_the_abi(agn):
+    """Eq. 4 in the library (host code) against the oracle's restatement."""
+    import oracle as O
+    rng = np.random.default_rng(5)
+    for _ in range(20):
+        na, nb = rng.integers(1, 12, 2)
+        ta = np.sort(rng.uniform(0, 10, na)); ta[-1] = max(ta[-1], 0.5)
+        tb = np.sort(rng.uniform(0, 10, nb)); tb[-1] = max(tb[-1], 0.5)
+        fa, fb = rng.uniform(0.1, 1, na), rng.uniform(0.1, 1, nb)
+        got = agn.agn_temporal_efficiency(ta, fa, tb, fb)
+        assert math.isclose(got, O.temporal_efficiency(ta, fa, tb, fb), rel_tol=1e-12)
+    for bad in [([], [], [0, 1], [1, 1]), ([0, 2, 1], [1, 1, 1], [0, 1], [1, 1]),
+                ([0, 1], [1, 1], [0, 1], [0, 0])]:
+        with pytest.raises(agn.AGNError) as e:
+            agn.agn_temporal_efficiency(*bad)
+        assert e.value.code == agn.AGN_E_INVALID

@@ -476,3 +476,66 @@ def test_commit_fp32_matches_exact_rounding():
 
 def test_commit_fp32_unnormalised_scale():
     assert np.float32(O.commit_scale_fp32(0.01, 10, normalize=False)) == np.float32(-0.01)
+
+
+# ----------------------------------------------------------------------------
+# Evaluation and temporal efficiency (Section 4, Eq. 4)
+# ----------------------------------------------------------------------------
+
+def test_evaluate_hand_worked():
+    """One linear layer, logits chosen by hand: accuracy exact, loss closed
+    form, ties to the lowest index."""
+    mlp = O.MLP((2, 3))
+    W = np.array([[1.0, 0.0], [0.0, 1.0], [0.0, 0.0]])
+    b = np.zeros(3)
+    theta = np.concatenate([W.ravel(), b])
+    X = np.array([[2.0, 0.0], [0.0, 3.0], [0.0, 0.0], [1.0, 1.0]])
+    y = np.array([0, 2, 0, 1])
+    loss, acc, pred = O.evaluate(mlp, theta, X, y)
+    # logits: [2,0,0] -> 0; [0,3,0] -> 1; [0,0,0] -> tie -> 0; [1,1,0] -> tie -> 0
+    assert pred.tolist() == [0, 1, 0, 0]
+    assert acc == 0.5
+    e = math.e
+    expect = np.mean([math.log(e ** 2 + 2) - 2, math.log(e ** 3 + 2) - 0.0,
+                      math.log(3.0), math.log(2 * e + 1) - 1])
+    assert math.isclose(loss, expect, rel_tol=1e-14)
+
+
+def test_evaluate_uniform_logits_is_log_classes():
+    mlp = O.MLP((4, 5, 7))
+    theta = np.zeros(mlp.num_params)
+    X = np.random.default_rng(3).normal(size=(9, 4))
+    loss, acc, pred = O.evaluate(mlp, theta, X, np.arange(9) % 7)
+    assert math.isclose(loss, math.log(7), rel_tol=1e-15)
+    assert np.all(pred == 0)
+
+
+def test_temporal_efficiency_closed_forms():
+    t = np.linspace(0.0, 10.0, 11)
+    f = 0.3 + 0.05 * t
+    assert O.temporal_efficiency(t, f, t, f) == 1.0
+    assert math.isclose(O.temporal_efficiency(t, 2 * f, t, f), 2.0, rel_tol=1e-15)
+    # f_a(t) = t, f_b = 1 on [0, 4]: E = (16 / 2) / 4
+    assert math.isclose(O.temporal_efficiency([0, 4], [0, 4], [0, 4], [1, 1]), 2.0, rel_tol=1e-15)
+    # the longer curve is cut at the shorter one's end, inside a segment:
+    # f_a = t on [0, 10] (samples at 0 and 10), f_b = 1 on [0, 3]: E = 4.5 / 3
+    assert math.isclose(O.temporal_efficiency([0, 10], [0, 10], [0, 3], [1, 1]), 1.5,
+                        rel_tol=1e-15)
+    # held at its first value before the first sample: f_a = 2 on [0, 1], then 2 -> 4
+    # on [1, 2] (integral 2 + 3 = 5), f_b = 1: E = 5 / 2
+    assert math.isclose(O.temporal_efficiency([1, 2], [2, 4], [0, 2], [1, 1]), 2.5,
+                        rel_tol=1e-15)
+
+
+def test_temporal_efficiency_is_exact_for_piecewise_linear_curves():
+    rng = np.random.default_rng(13)
+    tb = np.sort(rng.uniform(0, 5, 7))
+    tb[0] = 0.0
+    fb = rng.uniform(0.1, 1, 7)
+    ta = np.array([0.0, 5.0])
+    fa = np.array([1.0, 1.0])
+    # integral of the interpolant of (tb, fb) up to tb[-1], by Fractions
+    from fractions import Fraction as F
+    area = sum((F(fb[i]) + F(fb[i + 1])) / 2 * (F(tb[i + 1]) - F(tb[i])) for i in range(6))
+    e = O.temporal_efficiency(ta, fa, tb, fb)
+    assert math.isclose(e, float(F(tb[-1]) / area), rel_tol=1e-14)
