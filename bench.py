@@ -176,7 +176,7 @@ def run_reference(args, wl):
     def step():
         O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:per_step], tau[:per_step], ds, wl.batch,
                   wl.shard, dtype=dtype, staleness_scaled=args.commit_rule == "dynsgd",
-                  elide_accumulator=args.elide_accumulator)
+                  elide_accumulator=args.elide_accumulator, optimizer=args.optimizer)
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
@@ -254,7 +254,8 @@ def run_agn(args, wl):
                 n_samples=wl.n_samples, input_dist=wl.dist, teacher_dims=wl.teacher_dims,
                 normalize=wl.normalize, gemm=GEMMS[args.gemm], stream=st.cuda_stream,
                 commit_rule=agn.AGN_COMMIT_DYNSGD if args.commit_rule == "dynsgd"
-                else agn.AGN_COMMIT_AGN, elide_accumulator=int(args.elide_accumulator))
+                else agn.AGN_COMMIT_AGN, elide_accumulator=int(args.elide_accumulator),
+                local_optimizer=agn.AGN_OPT_ADAM if args.optimizer == "adam" else agn.AGN_OPT_SGD)
 
     def barrier():
         if ws > 1:
@@ -380,6 +381,7 @@ def run_agn(args, wl):
         "config": {"workload": wl.name, "commits_per_step": per_step,
                    "commit_rule": args.commit_rule,
                    "accumulator": "elided" if args.elide_accumulator else "kept",
+                   "local_optimizer": args.optimizer,
                    "parallelism": "replicas" if ws > 1 else "single GPU",
                    "l2": "inputs larger than L2 (dataset 188 MB + replicas and accumulators "
                          "230 MB vs 129 MB L2)" if args.workload == "mnist" else
@@ -415,6 +417,8 @@ def main():
                     help="AGN's commit (Eq. 1) or the DynSGD-style staleness-scaled commit")
     ap.add_argument("--elide-accumulator", action="store_true",
                     help="keep no gradient accumulator; commit from the pulled parameters")
+    ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adam"],
+                    help="the local optimizer of the workers (Algorithm 1's gradient line)")
     ap.add_argument("--workers", type=int, default=0,
                     help="override n (profiling captures of a smaller case)")
     ap.add_argument("--ref-commits", type=int, default=2)

@@ -60,6 +60,10 @@ extern "C" {
                                   AGN_E_UNSUPPORTED); the d_L-wide output
                                   layer always runs on CUDA cores          */
 
+/* Local optimizers (agn_options.local_optimizer) */
+#define AGN_OPT_SGD 0
+#define AGN_OPT_ADAM 1
+
 /* Commit rules (agn_options.commit_rule) */
 #define AGN_COMMIT_AGN 0       /* Delta = -eta a / lambda (Eq. 1)            */
 #define AGN_COMMIT_DYNSGD 1    /* Delta = -eta a / (tau_c + 1), Section 4     */
@@ -110,6 +114,15 @@ typedef struct agn_options {
      seeded generator, labelled by the same teacher (0 = none; not with
      x_init / y_init). */
   int64_t n_eval;
+  /* Local optimizer (AGN_OPT_*): AGN_OPT_SGD (default), g = -eta grad; or
+     AGN_OPT_ADAM (Algorithm 1 names Adam as an example), g = -eta m^/(sqrt(v^)
+     + eps) with per-worker moments that persist across commits and bias
+     corrections at the worker's step count (never reset).  The accumulator
+     then sums the steps g, and a commit adds a/lambda (a/(tau_c+1), a).
+     adam_beta1, adam_beta2, adam_eps: 0 = 0.9, 0.999, 1e-8.  Not with
+     tc_mask bit 3. */
+  int32_t local_optimizer;
+  float adam_beta1, adam_beta2, adam_eps;
 } agn_options;
 
 void agn_default_options(agn_options* opt);

@@ -208,7 +208,8 @@ class AGNResult:
 
 def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
             normalize=True, snapshot_at=(), keep_locals=(), dtype=np.float64,
-            staleness_scaled=False, elide_accumulator=False):
+            staleness_scaled=False, elide_accumulator=False, optimizer="sgd",
+            adam=(0.9, 0.999, 1e-8)):
     """Run the commits of one schedule through the FIFO parameter server.
 
     model      : object with loss_grad(theta, X, y) -> (loss, grad)
@@ -231,6 +232,12 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
     iterate and the pulled parameters, (theta_lambda - theta_pull) scaled the
     same way.  Equal to the accumulated form in exact arithmetic (the
     accumulated updates telescope).
+
+    optimizer="adam": the local step g of Algorithm 1 comes from Adam (named
+    there as an example): with the minibatch gradient gr at the worker's
+    step count t = 1, 2, ... (never reset), m = b1 m + (1 - b1) gr,
+    v = b2 v + (1 - b2) gr^2, g = -eta (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t))
+    + eps); the moments belong to the worker and persist across its commits.
     """
     worker = np.asarray(worker, dtype=np.int64)
     v = schedule_versions(n, worker, tau)
@@ -245,6 +252,10 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
     if 0 in readers:
         snaps[0] = theta_c.copy()
     step = np.zeros(n, dtype=np.int64)
+    if optimizer not in ("sgd", "adam"):
+        raise ValueError("optimizer must be 'sgd' or 'adam'")
+    b1, b2, eps_a = (dtype(x) for x in adam)
+    mom = {}                                            # worker -> (m, v)
     loss = np.zeros(C)
     dnorm = np.zeros(C)
     tnorm = np.zeros(C)
@@ -266,7 +277,15 @@ def agn_run(model, theta0, n, lam, eta, worker, tau, data, batch, shard,
         for _ in range(lam):
             X, y = data(batch_rows(k, int(step[k]), batch, shard))
             li, grad = model.loss_grad(theta, X.astype(dtype, copy=False), y)
-            g = -eta * grad
+            if optimizer == "adam":
+                m1, m2 = mom.get(k, (np.zeros_like(theta), np.zeros_like(theta)))
+                m1 = b1 * m1 + (1 - b1) * grad
+                m2 = b2 * m2 + (1 - b2) * grad * grad
+                mom[k] = (m1, m2)
+                t = int(step[k]) + 1
+                g = -eta * (m1 / (1 - b1 ** t)) / (np.sqrt(m2 / (1 - b2 ** t)) + eps_a)
+            else:
+                g = -eta * grad
             a = a + g
             theta = theta + g
             step[k] += 1

@@ -14,7 +14,7 @@ import ctypes as C
 import numpy as np
 
 from . import _lib
-from ._lib import (AGN_COMMIT_AGN, AGN_COMMIT_DYNSGD,  # noqa: F401
+from ._lib import (AGN_COMMIT_AGN, AGN_COMMIT_DYNSGD, AGN_OPT_ADAM, AGN_OPT_SGD,  # noqa: F401
                    AGN_DIST_NORMAL, AGN_DIST_UNIFORM, AGN_GEMM_AUTO, AGN_GEMM_SIMT,  # noqa: F401
                    AGN_GEMM_TCGEN05, AGN_PREC_BF16, AGN_PREC_FP32, AGN_OK, AGN_E_INVALID,
                    AGN_E_SCHEDULE, AGN_E_OOM, AGN_E_CUDA, AGN_E_TIMEOUT, AGN_E_NONFINITE,
@@ -255,7 +255,7 @@ class AGN:
                  n_samples=2048, input_dist=AGN_DIST_UNIFORM, teacher_dims=None, normalize=1,
                  gemm=AGN_GEMM_AUTO, tau_lo=0, tau_hi=0, stream=None, x=None, y=None,
                  theta0=None, tc_mask=0, commit_rule=AGN_COMMIT_AGN, elide_accumulator=0,
-                 n_eval=0):
+                 n_eval=0, local_optimizer=AGN_OPT_SGD, adam=(0.0, 0.0, 0.0)):
         o = agn_default_options()
         o.precision, o.batch, o.n_samples = int(precision), int(batch), int(n_samples)
         o.input_dist, o.normalize, o.gemm = int(input_dist), int(normalize), int(gemm)
@@ -264,6 +264,8 @@ class AGN:
         o.commit_rule = int(commit_rule)
         o.elide_accumulator = int(elide_accumulator)
         o.n_eval = int(n_eval)
+        o.local_optimizer = int(local_optimizer)
+        o.adam_beta1, o.adam_beta2, o.adam_eps = (float(x) for x in adam)
         self.n_eval = int(n_eval)
         keep = []
         if teacher_dims is not None:

@@ -25,6 +25,8 @@ AGN_PREC_FP32 = 0
 AGN_PREC_BF16 = 1
 AGN_DIST_UNIFORM = 0
 AGN_DIST_NORMAL = 1
+AGN_OPT_SGD = 0
+AGN_OPT_ADAM = 1
 AGN_COMMIT_AGN = 0
 AGN_COMMIT_DYNSGD = 1
 AGN_GEMM_AUTO = 0
@@ -61,6 +63,10 @@ class agn_options(C.Structure):
         ("commit_rule", C.c_int32),
         ("elide_accumulator", C.c_int32),
         ("n_eval", C.c_int64),
+        ("local_optimizer", C.c_int32),
+        ("adam_beta1", C.c_float),
+        ("adam_beta2", C.c_float),
+        ("adam_eps", C.c_float),
     ]
 
 

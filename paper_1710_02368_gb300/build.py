@@ -21,7 +21,7 @@ LIB_NAME = "libagn_gb300.so"
 LIB_PATH = os.path.join(BUILD, LIB_NAME)
 
 SOURCES = ["agn_api.cu", "commit_pull.cu", "commit_pull_noalloc.cu", "mlp_simt.cu", "mlp_head.cu",
-           "mlp_tc.cu", "mlp_tc_dw.cu", "mlp_eval.cu", "host_inputs.cu"]
+           "mlp_tc.cu", "mlp_tc_dw.cu", "mlp_eval.cu", "optim.cu", "host_inputs.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "--expt-relaxed-constexpr",
               "-Xcompiler", "-fPIC,-ffp-contract=off,-O3", "-I", INCLUDE]

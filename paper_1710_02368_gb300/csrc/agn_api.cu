@@ -62,6 +62,13 @@ struct agn_handle {
   // accumulator elided: `acc` holds each worker's theta at its last pull and
   // a commit adds (theta_k - theta_pull) scaled by 1/lambda (or 1/(tau+1), 1)
   bool elide = false;
+  // Adam as the local optimizer: raw gradients go to grad, the moments m, v
+  // persist per worker, the accumulator (if kept) sums the steps
+  bool adam = false;
+  float beta1 = 0.9f, beta2 = 0.999f, eps = 1e-8f;
+  float* grad = nullptr;      // [n][P_pad]
+  float* mom1 = nullptr;      // [n][P_pad]
+  float* mom2 = nullptr;      // [n][P_pad]
   // held-out evaluation set (rows [N, N + n_eval) of the generator) and the
   // buffers of its forward pass, chunk rows at a time
   int64_t n_eval = 0, eval_chunk = 0;
@@ -270,6 +277,7 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.err = h->flag + 1;
   t.theta = h->rep;
   t.acc = h->elide ? nullptr : h->acc;
+  t.grad_out = h->adam ? h->grad : nullptr;
   t.theta_b = h->rep_b;
   t.ld_param = h->P_pad;
   t.piece_plane = h->piece_plane;
@@ -359,8 +367,11 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   const double es = (double)sizeof(T);
   // bytes per parameter of the local step + accumulation: theta RMW, a RMW, and
   // the low-precision copy (one bf16, or three pieces in the split mode)
-  const double upd = (h->elide ? 8.0 : 16.0) +
-                     (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
+  // (with Adam the dW kernels only store the gradient, 4 bytes; the Adam
+  // kernel's own traffic is counted at its launch)
+  const double upd = h->adam ? 4.0
+                             : (h->elide ? 8.0 : 16.0) +
+                                   (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
   // pieces of dZ_l (split mode, hidden tensor-core layers), planes n m d_l apart
   auto dz_pieces = [&](int l) -> bf16* {
     return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZp[l] : nullptr;
@@ -525,6 +536,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         d.piece_plane = h->piece_plane;
         d.ld_param = h->P_pad; d.woff = h->woff[l - 1]; d.boff = h->boff[l - 1];
         d.K = fi; d.C = fo; d.m = m; d.eta = eta;
+        d.grad_out = h->adam ? h->grad : nullptr;
         AGN_TRY(agn::head_backward_dw<T>(d, s, h->stream));
       } else {
         agn::GemmArgs g{};
@@ -536,6 +548,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         g.ld_param = h->P_pad;
         g.piece_plane = h->piece_plane;
         g.woff = h->woff[l - 1]; g.boff = h->boff[l - 1]; g.eta = eta;
+        g.grad_out = h->adam ? h->grad : nullptr;
         AGN_TRY(agn::simt_backward_dw<T>(g, s, h->stream));
       }
     }
@@ -545,6 +558,18 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       t.K = m; t.eta = eta;
       AGN_TRY(agn::tc_backward_dw(tc_dw.data(), (int)tc_dw.size(), t, s, h->stream, h->split,
                                   h->num_sms));
+    }
+    if (h->adam) {   // the local step: Adam on the gradients the dW kernels stored
+      agn::AdamArgs ad{};
+      ad.grad = h->grad; ad.theta = h->rep; ad.acc = h->elide ? nullptr : h->acc;
+      ad.m = h->mom1; ad.v = h->mom2; ad.theta_b = h->rep_b; ad.piece_plane = h->piece_plane;
+      ad.P = h->P_pad; ad.ld = h->P_pad;
+      ad.slot_worker = sw; ad.slot_t0 = st0; ad.step = i;
+      ad.eta = eta; ad.beta1 = h->beta1; ad.beta2 = h->beta2; ad.eps = h->eps;
+      const double copy_b = h->split ? 6.0 : h->rep_b ? 2.0 : 0.0;
+      Launch k(h, AGN_K_BACKWARD_DW, 0.0,
+               (double)s * h->P * (4.0 + 16.0 + 8.0 + (h->elide ? 0.0 : 8.0) + copy_b), launches);
+      AGN_TRY(agn::adam_step(ad, s, h->num_sms, h->stream));
     }
   }
   return Status::Ok();
@@ -668,8 +693,8 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
       cp.norm_slot[c] = (int)(V0 + i);
       if (h->commit_rule == AGN_COMMIT_DYNSGD) {   // Delta = -eta a / (tau_c + 1)
         cp.per_commit_scale = 1;
-        cp.scale[c] = h->elide ? (float)(1.0 / (double)(tau[i] + 1))
-                               : (float)(-(h->eta / (double)(tau[i] + 1)));
+        cp.scale[c] = (h->elide || h->adam) ? (float)(1.0 / (double)(tau[i] + 1))
+                                            : (float)(-(h->eta / (double)(tau[i] + 1)));
       }
       int pb = cp.pull_begin[c];
       for (int p : pulls_at[i + 1]) cp.pull_worker[pb++] = p;
@@ -731,8 +756,9 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   // commit scale: of the raw gradient sum a (-eta / lambda, or -eta without
   // normalisation), or, with the accumulator elided, of theta_k - theta_pull
   // (which already carries -eta): 1 / lambda, or 1
-  const float scale = h->elide ? (float)(h->normalize ? 1.0 / (double)h->lam : 1.0)
-                               : (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
+  const bool steps = h->elide || h->adam;   // the committed quantity already carries -eta
+  const float scale = steps ? (float)(h->normalize ? 1.0 / (double)h->lam : 1.0)
+                            : (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
   for (const Wave& wv : plan.waves) {
     if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
     else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
@@ -810,6 +836,14 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.n_eval > 0 && (o.x_init || o.y_init))
     return Status::Err(AGN_E_INVALID,
                        "the evaluation set is generated: not with caller-supplied inputs");
+  if (o.local_optimizer != AGN_OPT_SGD && o.local_optimizer != AGN_OPT_ADAM)
+    return Status::Err(AGN_E_INVALID, "unknown local_optimizer");
+  if (o.adam_beta1 < 0.f || o.adam_beta1 >= 1.f || o.adam_beta2 < 0.f || o.adam_beta2 >= 1.f ||
+      o.adam_eps < 0.f)
+    return Status::Err(AGN_E_INVALID, "Adam betas must be in [0, 1) and eps >= 0 (0 = default)");
+  if (o.local_optimizer == AGN_OPT_ADAM && (o.tc_mask & 8))
+    return Status::Err(AGN_E_UNSUPPORTED,
+                       "the one-tile-per-CTA dW kernel (tc_mask bit 3) has no gradient output");
   if (o.elide_accumulator && (o.tc_mask & 8))
     return Status::Err(AGN_E_UNSUPPORTED,
                        "the one-tile-per-CTA dW kernel (tc_mask bit 3) keeps the accumulator");
@@ -827,6 +861,10 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->normalize = o.normalize ? 1 : 0;
   h->commit_rule = o.commit_rule;
   h->elide = o.elide_accumulator != 0;
+  h->adam = o.local_optimizer == AGN_OPT_ADAM;
+  if (o.adam_beta1 > 0.f) h->beta1 = o.adam_beta1;
+  if (o.adam_beta2 > 0.f) h->beta2 = o.adam_beta2;
+  if (o.adam_eps > 0.f) h->eps = o.adam_eps;
   h->gemm = o.gemm;
   h->tau_lo = o.tau_lo;
   h->tau_hi = o.tau_hi;
@@ -918,6 +956,13 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY(dalloc_t(h, &h->rep, (size_t)(n * h->P_pad)));
   AGN_TRY(dalloc_t(h, &h->acc, (size_t)(n * h->P_pad)));
   if (h->prec == AGN_PREC_BF16) AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(n * h->P_pad)));
+  if (h->adam) {   // gradients and the two moments of every worker, zero to start
+    AGN_TRY(dalloc_t(h, &h->grad, (size_t)(n * h->P_pad)));
+    AGN_TRY(dalloc_t(h, &h->mom1, (size_t)(n * h->P_pad)));
+    AGN_TRY(dalloc_t(h, &h->mom2, (size_t)(n * h->P_pad)));
+    for (float* p : {h->grad, h->mom1, h->mom2})
+      AGN_TRY_CUDA(cudaMemset(p, 0, (size_t)(n * h->P_pad) * sizeof(float)));
+  }
   if (h->split) {   // three piece planes of every replica, and of the activations
     h->piece_plane = n * h->P_pad;
     AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));

@@ -41,6 +41,8 @@ struct GemmArgs {
   int64_t ld_param;
   int64_t woff, boff;    // offsets of W_l and b_l in a replica
   float eta;
+  float* grad_out;       // dW: store the raw gradient here ([n][ld_param]) instead of
+                         // taking the local step; null = fused local step
 };
 
 template <typename T>
@@ -96,12 +98,32 @@ struct HeadDwArgs {
   int64_t ld_param, woff, boff;
   int K, C, m;
   float eta;
+  float* grad_out;         // store the raw gradient here instead of updating; null = update
 };
 template <typename T>
 Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st);
 // The fused head takes this output layer (classes and shared-memory staging fit).
 template <typename T>
 bool head_fits(int K, int C);
+
+// Adam as the local optimizer (optim.cu): from the raw gradients grad of the
+// wave's slots, the moments m, v and theta_k (a_k += the step, unless acc is
+// null; the bf16 copy or pieces of theta_k, unless theta_b is null).
+struct AdamArgs {
+  const float* grad;       // [n][ld] raw minibatch gradients of this local step
+  float* theta;            // [n][ld] fp32 replicas
+  float* acc;              // [n][ld] accumulators (of the steps), or null
+  float* m;                // [n][ld] first moments
+  float* v;                // [n][ld] second moments
+  bf16* theta_b;           // bf16 copies / piece 0 of three planes, or null
+  int64_t piece_plane;     // > 0: three pieces, planes this far apart
+  int64_t P, ld;           // elements updated per replica (multiple of 4), row stride
+  const int* slot_worker;
+  const long long* slot_t0;   // the worker's step counter before this wave
+  int step;                   // local step index within the wave
+  float eta, beta1, beta2, eps;
+};
+Status adam_step(const AdamArgs& a, int slots, int num_sms, cudaStream_t st);
 
 // Evaluation (mlp_eval.cu): per-sample loss / correctness / prediction of
 // fp32 logits Z [rows][C] against labels y, and their fixed-order means

@@ -270,6 +270,27 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       }
     }
   };
+  if (a.grad_out) {   // raw gradient out (the optimizer runs after)
+    float* go = a.grad_out + (int64_t)w * a.ld_param;
+    if (k < K) {
+      for (int c = warp; c < C; c += kDwGroups) {
+        float v = 0.f;
+#pragma unroll
+        for (int r = 0; r < kDwGroups; ++r) v += red[(r * kMaxC + c) * 32 + lane];
+        go[a.woff + (int64_t)c * K + k] = v;
+      }
+    }
+    if (blockIdx.x == 0 && warp == kDwGroups - 1) {
+      for (int c = 0; c < C; ++c) {
+        float v = 0.f;
+        for (int j = lane; j < m; j += 32) v += cvt(dz[j * C + c]);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if (lane == 0) go[a.boff + c] = v;
+      }
+    }
+    return;
+  }
   if (k < K) {
     constexpr int kPer = (kMaxC + kDwGroups - 1) / kDwGroups;   // classes per warp
     float th[kPer], ac[kPer], gs[kPer];

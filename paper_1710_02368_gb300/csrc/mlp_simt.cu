@@ -141,6 +141,19 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         out[m * g.ldo + n] = from_f<TO>(h > 0.f ? acc[i][j] : 0.f);
       }
     }
+  } else if (g.grad_out) {   // kEpiDW, raw gradient out (the optimizer runs after)
+    float* go = g.grad_out + (int64_t)w * g.ld_param;
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+      const int64_t m = m0 + ty + i * (kBM / kTM);
+      if (m >= g.M) continue;
+#pragma unroll
+      for (int j = 0; j < kTN; ++j) {
+        const int64_t n = n0 + tx + j * (kBN / kTN);
+        if (n < g.N) go[g.woff + m * g.N + n] = acc[i][j];
+      }
+    }
+    if (do_bias && m0 + tid < g.M) go[g.boff + m0 + tid] = bsum;
   } else {   // kEpiDW: theta_k -= eta g, a_k += g (unless elided), bf16 copy refresh
     const bool has_a = g.acc != nullptr;
     float* a = has_a ? g.acc + (int64_t)w * g.ld_param : theta;

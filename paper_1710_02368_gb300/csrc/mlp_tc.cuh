@@ -37,6 +37,10 @@ struct TcArgs {
   int ksplit;
   float* part;
   int* counter;
+  // dW: store the raw gradient at grad_out [n][ld_param] (same layout as the
+  // replicas) instead of taking the local step (the optimizer runs after);
+  // null = fused local step
+  float* grad_out;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N

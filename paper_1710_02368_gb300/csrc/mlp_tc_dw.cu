@@ -62,11 +62,15 @@ constexpr uint64_t kWaitNs = 2000000000ull;    // 2 s
 // kBK samples per stage: one TMA box is 64 MN-elements x kBK samples of bf16
 // (kBK rows of 128 bytes, 128-byte swizzle); A = two boxes (128 inputs),
 // B = BN / 64 boxes.
-// kAcc: theta_k and a_k per chunk (3 slots in flight); without the
-// accumulator (elided, commits from a pull snapshot) theta_k alone (6 slots).
-template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
+// kMode: kDwUpdAcc = the local step and accumulation, theta_k and a_k per
+// chunk (3 slots in flight); kDwUpd = the local step without accumulator
+// (elided: commits from a pull snapshot), theta_k alone (6 slots); kDwGrad =
+// the raw gradient only, stored for a separate optimizer kernel (no chunks).
+enum { kDwUpdAcc = 0, kDwUpd = 1, kDwGrad = 2 };
+template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 struct DwCfg {
-  static constexpr int kArrays = kAcc ? 2 : 1;
+  static constexpr bool kAcc = kMode == kDwUpdAcc;
+  static constexpr int kArrays = kMode == kDwUpdAcc ? 2 : 1;
   static constexpr int kSlotBytes = kArrays * (kChunkBytes + kBiasHalf);
   static constexpr int kRing = kAcc ? 3 : 6;
   static constexpr int kBK = kBKs;
@@ -156,10 +160,11 @@ __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
   }
 }
 
-template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
+template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
-  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kAcc>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kMode>;
+  constexpr bool kAcc = Cfg::kAcc, kGrad = kMode == kDwGrad;
   constexpr int kRing = Cfg::kRing, kSlotBytes = Cfg::kSlotBytes;
   constexpr int kBK = Cfg::kBK, kABytes = Cfg::kABytes, kBox = Cfg::kBox;
   extern __shared__ uint8_t smem_raw[];
@@ -260,6 +265,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           ++ml;
         }
         if (!ok) break;
+        if (kGrad) continue;   // the gradient needs no parameter chunks
         const bool bias_tile = ti.m_tile == L.M / 128;
         const int nch = min(Cfg::kChunks, (L.N - ti.n_tile * BN + kCF - 1) / kCF);
         for (int c = 0; c < nch; ++c) {
@@ -405,6 +411,24 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         }
 #pragma unroll
         for (int i = 0; i < 16; ++i) gS[i * 32 + lane] = __uint_as_float(v[i]);
+        if (kGrad) {   // raw gradient out: grad[w][p] = g, coalesced 16-byte stores
+          __syncwarp();
+          const int fbase = ti.n_tile * BN + c * kCF + 16 * hf;
+          float* gout = args.grad_out + rbase;
+          if (quad_ok) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int i = i0 + 4 * u;
+              if (fbase + i < N)
+                *reinterpret_cast<float4*>(gout + L.woff + (int64_t)(fbase + i) * M + k0 + k4) =
+                    *reinterpret_cast<const float4*>(gS + i * 32 + k4);
+            }
+          }
+          if (kb >= 0 && kb < 32 && lane < 16 && fbase + lane < N)
+            gout[L.boff + fbase + lane] = gS[lane * 32 + kb];
+          __syncwarp();
+          continue;
+        }
         ok = __all_sync(0xffffffffu,
                         tc::wait_or_abort(&cfull[r], (ch / kRing) & 1, abort_flag, kWaitNs));
         if (!ok) break;
@@ -481,13 +505,13 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   if (warp == 1) tc::tmem_dealloc(tmem, Cfg::kTmemCols);
 }
 
-template <int BN, int kSplit, int kStages, int kBKs, bool kAcc>
+template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 Status launch_dw(const DwBatch& batch, const TcArgs& args, int num_sms, cudaStream_t st) {
-  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kAcc>;
+  using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kMode>;
   static_assert(Cfg::kSmem <= 232448, "shared memory");
   static_assert(Cfg::kSmem > 232448 / 2, "one CTA per SM (all 512 TMEM columns)");
   static_assert(Cfg::kTmemCols == 512, "TMEM columns");
-  auto kern = tc_dw_kernel<BN, kSplit, kStages, kBKs, kAcc>;
+  auto kern = tc_dw_kernel<BN, kSplit, kStages, kBKs, kMode>;
   static std::mutex mu;
   static std::set<int> done;
   {
@@ -538,11 +562,18 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
     batch.total_tiles = (int)tiles;
     // split mode: 32 samples per stage, so that two stages fit beside the
     // parameter ring (the next tile's operands land while this one multiplies)
-    const bool acc = args.acc != nullptr;   // null: accumulator elided
-    Status r = split ? (acc ? launch_dw<kTcDwBNSplit, 3, 2, 32, true>(batch, args, num_sms, st)
-                            : launch_dw<kTcDwBNSplit, 3, 2, 32, false>(batch, args, num_sms, st))
-                     : (acc ? launch_dw<kTcDwBN, 1, 2, 64, true>(batch, args, num_sms, st)
-                            : launch_dw<kTcDwBN, 1, 2, 64, false>(batch, args, num_sms, st));
+    // grad_out: gradient only; else acc null: accumulator elided
+    const int mode = args.grad_out ? kDwGrad : args.acc ? kDwUpdAcc : kDwUpd;
+    Status r = Status::Ok();
+    if (split) {
+      r = mode == kDwGrad ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwGrad>(batch, args, num_sms, st)
+          : mode == kDwUpd ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpd>(batch, args, num_sms, st)
+                           : launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpdAcc>(batch, args, num_sms, st);
+    } else {
+      r = mode == kDwGrad ? launch_dw<kTcDwBN, 1, 2, 64, kDwGrad>(batch, args, num_sms, st)
+          : mode == kDwUpd ? launch_dw<kTcDwBN, 1, 2, 64, kDwUpd>(batch, args, num_sms, st)
+                           : launch_dw<kTcDwBN, 1, 2, 64, kDwUpdAcc>(batch, args, num_sms, st);
+    }
     if (!r.ok()) return r;
   }
   return Status::Ok();

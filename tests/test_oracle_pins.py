@@ -539,3 +539,54 @@ def test_temporal_efficiency_is_exact_for_piecewise_linear_curves():
     area = sum((F(fb[i]) + F(fb[i + 1])) / 2 * (F(tb[i + 1]) - F(tb[i])) for i in range(6))
     e = O.temporal_efficiency(ta, fa, tb, fb)
     assert math.isclose(e, float(F(tb[-1]) / area), rel_tol=1e-14)
+
+
+# ----------------------------------------------------------------------------
+# Adam as the local optimizer (Algorithm 1's gradient line)
+# ----------------------------------------------------------------------------
+
+def test_adam_first_step_is_eta_times_the_gradient_sign():
+    """At t = 1 the bias corrections give m^ = gr and v^ = gr^2, so the step
+    is -eta gr / (|gr| + eps)."""
+    mlp, theta, X, y = _tiny_problem(seed=4)
+    eta, eps = 0.01, 1e-8
+    _, gr = mlp.loss_grad(theta, X, y)
+    d = _ListData(X, y)
+    r = O.agn_run(mlp, theta, 1, 1, eta, [0], [0], d, len(y), len(y), optimizer="adam",
+                  adam=(0.9, 0.999, eps))
+    assert np.allclose(r.theta - theta, -eta * gr / (np.abs(gr) + eps), rtol=0, atol=1e-15)
+
+
+def test_adam_moments_persist_across_commits():
+    """An independent loop: moments per worker, bias corrections at the
+    worker's step count, staleness as scheduled."""
+    rng = np.random.default_rng(14)
+    dims, m, S, lam, eta, n = (4, 3, 3), 2, 5, 3, 0.05, 2
+    b1, b2, eps = 0.8, 0.99, 1e-6
+    mlp = O.MLP(dims)
+    X, y = rng.uniform(size=(n * S, dims[0])), rng.integers(0, dims[-1], n * S)
+    th0 = rng.normal(0, 0.5, mlp.num_params)
+    worker = [0, 1, 0, 1, 1, 0]
+    tau = [0, 1, 1, 1, 0, 2]
+    r = O.agn_run(mlp, th0, n, lam, eta, worker, tau, _ListData(X, y), m, S,
+                  snapshot_at=range(len(worker)), optimizer="adam", adam=(b1, b2, eps))
+    V = [th0]
+    steps = [0] * n
+    mom = [(np.zeros_like(th0), np.zeros_like(th0)) for _ in range(n)]
+    for c, (w, t) in enumerate(zip(worker, tau)):
+        theta = V[c - t].copy()
+        a = np.zeros_like(theta)
+        m1, m2 = mom[w]
+        for i in range(lam):
+            rows = w * S + ((steps[w] + i) * m + np.arange(m)) % S
+            _, gr = mlp.loss_grad(theta, X[rows], y[rows])
+            m1 = b1 * m1 + (1 - b1) * gr
+            m2 = b2 * m2 + (1 - b2) * gr ** 2
+            k = steps[w] + i + 1
+            g = -eta * (m1 / (1 - b1 ** k)) / (np.sqrt(m2 / (1 - b2 ** k)) + eps)
+            a += g
+            theta += g
+        mom[w] = (m1, m2)
+        steps[w] += lam
+        V.append(V[-1] + a / lam)
+        assert np.allclose(r.snapshots[c], V[-1], rtol=0, atol=1e-14)
