@@ -51,6 +51,23 @@ def _peaks():
     return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+def max_over_ranks(values, device):
+    """Each value's maximum over the ranks of the default process group (every
+    rank receives it): the slowest rank's time is the job's time."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def whole_job_value(world_size, steps, commits_per_step, lam, batch, ms):
+    """Worker-samples per second of the whole job: every rank runs its own
+    replica of the workload (weak scaling), so the units add up over ranks,
+    divided by the slowest rank's time."""
+    return world_size * steps * commits_per_step * lam * batch / (ms / 1e3)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -322,12 +339,9 @@ def run_agn(args, wl):
     e2e_ms = max(e2.elapsed_time(e3), 1e3 * (time.perf_counter() - t0))
     h2d = 2 * 4 * (per_step + wl.n)           # the schedule window of each step
     if ws > 1:
-        t = torch.tensor([ms, e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
-    units = ws * args.steps * per_step * wl.lam * wl.batch
-    value = units / (ms / 1e3)
-    e2e_value = units / (e2e_ms / 1e3)
+        ms, e2e_ms = max_over_ranks([ms, e2e_ms], dev)
+    value = whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch, ms)
+    e2e_value = whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch, e2e_ms)
 
     hbm, bf16, bf16_sus, peak_src = _peaks()
     dom = max(("forward", "backward_dx", "backward_dw", "commit", "softmax", "gather"),
