@@ -72,6 +72,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
                    float* __restrict__ acc, float* __restrict__ replicas,
                    bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, float s, int zero_acc,
                    double* __restrict__ partials, int64_t plane) {
+  pdl_begin();
   const int nc = plan.n_commits;
   double sq[kMaxCommitsPerLaunch];
 #pragma unroll
@@ -208,6 +209,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
 __global__ void __launch_bounds__(kThreads)
 reduce_norms_kernel(const double* __restrict__ partials, int grid, const __grid_constant__ CommitPlan plan,
                     float* __restrict__ norms, int* __restrict__ flag) {
+  pdl_begin();
   const int c = blockIdx.x;
   const int slot = plan.norm_slot[c];
   const double* row = partials + (int64_t)c * grid;
@@ -250,19 +252,20 @@ Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, fl
   if (plan.n_commits <= 0) return Status::Ok();
   const int z = zero_acc ? 1 : 0;
   auto go = [&](auto kern, bf16* rb, int64_t plane) {
-    kern<<<grid, kThreads, 0, stream>>>(plan, theta_c, acc, replicas, rb, P, ld, scale, z,
-                                        partials, plane);
+    return launch_pdl(kern, grid, kThreads, 0, stream, plan, theta_c, acc, replicas, rb, P, ld,
+                      scale, z, partials, plane);
   };
+  cudaError_t e;
   if (replicas_bf16 && piece_plane > 0)
-    elide ? go(commit_pull_kernel<3, true>, replicas_bf16, piece_plane)
-          : go(commit_pull_kernel<3, false>, replicas_bf16, piece_plane);
+    e = elide ? go(commit_pull_kernel<3, true>, replicas_bf16, piece_plane)
+              : go(commit_pull_kernel<3, false>, replicas_bf16, piece_plane);
   else if (replicas_bf16)
-    elide ? go(commit_pull_kernel<1, true>, replicas_bf16, 0)
-          : go(commit_pull_kernel<1, false>, replicas_bf16, 0);
+    e = elide ? go(commit_pull_kernel<1, true>, replicas_bf16, 0)
+              : go(commit_pull_kernel<1, false>, replicas_bf16, 0);
   else
-    elide ? go(commit_pull_kernel<0, true>, nullptr, 0)
-          : go(commit_pull_kernel<0, false>, nullptr, 0);
-  AGN_TRY_CUDA(cudaGetLastError());
+    e = elide ? go(commit_pull_kernel<0, true>, nullptr, 0)
+              : go(commit_pull_kernel<0, false>, nullptr, 0);
+  AGN_TRY_CUDA(e);
   if (norms && partials && (delta_norm || flag))
     return launch_commit_norms(plan, partials, grid, delta_norm, flag, stream);
   return Status::Ok();
@@ -271,8 +274,11 @@ Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, fl
 Status launch_commit_norms(const CommitPlan& plan, const double* partials, int grid,
                            float* delta_norm, int* flag, cudaStream_t stream) {
   if (plan.n_commits <= 0) return Status::Ok();
-  reduce_norms_kernel<<<plan.n_commits, kThreads, 0, stream>>>(partials, grid, plan, delta_norm,
-                                                               flag);
+  {
+    auto kf = reduce_norms_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, plan.n_commits, kThreads, 0, stream, partials,
+                            grid, plan, delta_norm, flag));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -287,6 +293,7 @@ __global__ void __launch_bounds__(kThreads)
 pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
             bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers,
             int64_t plane, float* __restrict__ snapshot) {
+  pdl_begin();
   const int k = workers[blockIdx.y];
   float* dst = replicas + (int64_t)k * ld;
   float* snap = snapshot ? snapshot + (int64_t)k * ld : nullptr;
@@ -312,6 +319,7 @@ pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
 
 __global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda, int count,
                                      float* __restrict__ loss) {
+  pdl_begin();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= count) return;
   float s = 0.f;
@@ -326,15 +334,22 @@ Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16,
                      int64_t piece_plane, float* snapshot) {
   if (count <= 0) return Status::Ok();
   dim3 grid((unsigned)std::max(1, commit_grid(P) / std::max(1, count) + 1), (unsigned)count);
-  pull_kernel<<<grid, kThreads, 0, st>>>(theta_c, replicas, replicas_bf16, P, ld, workers,
-                                         piece_plane, snapshot);
+  {
+    auto kf = pull_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, 0, st, theta_c,
+                            replicas, replicas_bf16, P, ld, workers, piece_plane, snapshot));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
 
 Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st) {
   if (count <= 0) return Status::Ok();
-  reduce_losses_kernel<<<(unsigned)ceil_div(count, 128), 128, 0, st>>>(parts, lambda, count, loss);
+  {
+    auto kf = reduce_losses_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, (unsigned)ceil_div(count, 128), 128, 0, st, parts,
+                            lambda, count, loss));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -379,6 +394,7 @@ __device__ __forceinline__ float normal_f32(uint64_t k, uint64_t i) {
 __global__ void fill_commit_inputs_kernel(float* __restrict__ theta_c, float* __restrict__ acc,
                                           float* __restrict__ replicas, int64_t P, int64_t ld,
                                           int n, uint64_t key_theta, uint64_t key_acc) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < P; i += stride) {
     const float t = normal_f32(key_theta, (uint64_t)i);
@@ -395,9 +411,12 @@ __global__ void fill_commit_inputs_kernel(float* __restrict__ theta_c, float* __
 Status fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,
                           int n, uint64_t seed, cudaStream_t stream) {
   const int grid = commit_grid(P) * 2;
-  fill_commit_inputs_kernel<<<grid, kThreads, 0, stream>>>(
-      theta_c, acc, replicas, P, ld, n, gen::key(seed, gen::kCommitTheta),
-      gen::key(seed, gen::kCommitAcc));
+  {
+    auto kf = fill_commit_inputs_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, 0, stream, theta_c,
+                            acc, replicas, P, ld, n, gen::key(seed, gen::kCommitTheta),
+                            gen::key(seed, gen::kCommitAcc)));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

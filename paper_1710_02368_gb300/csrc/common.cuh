@@ -8,10 +8,38 @@
 #include <cstdint>
 #include <cstdio>
 #include <string>
+#include <utility>
 
 #include "../../include/agn.h"
 
 namespace agn {
+
+// Programmatic dependent launch: every kernel of the library is launched with
+// programmatic stream serialisation and starts with pdl_begin(), which waits
+// for the preceding kernel of the stream to complete (and its memory to be
+// visible) before touching global memory, then lets the next kernel launch.
+// The next kernel's launch and CTA dispatch thereby overlap this kernel's run;
+// the order of memory accesses is that of plain stream order.
+__device__ __forceinline__ void pdl_begin() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 using bf16 = __nv_bfloat16;
 

@@ -18,6 +18,7 @@ constexpr int kEvalThreads = 256;
 __global__ void __launch_bounds__(kEvalThreads)
 eval_logits_kernel(const float* __restrict__ Z, const int* __restrict__ y, int rows, int C,
                    float* __restrict__ loss, int* __restrict__ correct, int* __restrict__ pred) {
+  pdl_begin();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= rows) return;
   const float* z = Z + (int64_t)i * C;
@@ -42,6 +43,7 @@ eval_logits_kernel(const float* __restrict__ Z, const int* __restrict__ y, int r
 __global__ void __launch_bounds__(kEvalThreads)
 eval_reduce_kernel(const float* __restrict__ loss, const int* __restrict__ correct, int64_t E,
                    float* __restrict__ out) {
+  pdl_begin();
   __shared__ double ws[kEvalThreads / 32][2];
   double l = 0.0, c = 0.0;
   for (int64_t i = threadIdx.x; i < E; i += blockDim.x) {
@@ -75,8 +77,11 @@ eval_reduce_kernel(const float* __restrict__ loss, const int* __restrict__ corre
 Status eval_logits(const float* Z, const int* y, int rows, int C, float* loss, int* correct,
                    int* pred, cudaStream_t st) {
   if (rows <= 0) return Status::Ok();
-  eval_logits_kernel<<<(unsigned)ceil_div(rows, kEvalThreads), kEvalThreads, 0, st>>>(
-      Z, y, rows, C, loss, correct, pred);
+  {
+    auto kf = eval_logits_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, (unsigned)ceil_div(rows, kEvalThreads), kEvalThreads, 0, st, Z,
+                            y, rows, C, loss, correct, pred));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -84,7 +89,10 @@ Status eval_logits(const float* Z, const int* y, int rows, int C, float* loss, i
 Status eval_reduce(const float* loss, const int* correct, int64_t E, float* out,
                    cudaStream_t st) {
   if (E <= 0) return Status::Err(AGN_E_INVALID, "empty evaluation set");
-  eval_reduce_kernel<<<1, kEvalThreads, 0, st>>>(loss, correct, E, out);
+  {
+    auto kf = eval_reduce_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, 1, kEvalThreads, 0, st, loss, correct, E, out));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -64,6 +64,7 @@ __device__ __forceinline__ void stage_wait() {
 
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
+  pdl_begin();
   extern __shared__ __align__(16) uint8_t head_smem[];
   __shared__ float red[kHeadSamples][kHeadSplit][kMaxC];
   __shared__ float ce_s[kHeadSamples];
@@ -210,6 +211,7 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
 constexpr int kDwGroups = 8;
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArgs a) {
+  pdl_begin();
   extern __shared__ __align__(16) uint8_t dw_smem[];
   float* red = reinterpret_cast<float*>(dw_smem);                      // [kDwGroups][kMaxC][32]
   T* dz = reinterpret_cast<T*>(red + kDwGroups * kMaxC * 32);           // [m][C]
@@ -361,7 +363,10 @@ Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st) {
   auto kern = a.C == 10 ? head_kernel<T, 10> : head_kernel<T, kHeadMaxClasses>;
   AGN_TRY(allow_smem(reinterpret_cast<const void*>(kern)));
   dim3 grid((unsigned)ceil_div(a.m, kHeadSamples), (unsigned)slots);
-  kern<<<grid, kHeadThreads, smem, st>>>(a);
+  {
+    auto kf = kern;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kHeadThreads, smem, st, a));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -376,7 +381,10 @@ Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st) {
   auto kern = a.C == 10 ? head_dw_kernel<T, 10> : head_dw_kernel<T, kHeadMaxClasses>;
   AGN_TRY(allow_smem(reinterpret_cast<const void*>(kern)));
   dim3 grid((unsigned)ceil_div(a.K, 32), (unsigned)slots);
-  kern<<<grid, 32 * kDwGroups, smem, st>>>(a);
+  {
+    auto kf = kern;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, 32 * kDwGroups, smem, st, a));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -49,6 +49,7 @@ __device__ __forceinline__ void write_copy(bf16* tb, int64_t plane, int64_t p, f
 // C[M x N] (+)= sum_k A(m, k) B(k, n) for one slot; see GemmArgs for layouts.
 template <typename T, typename TO, bool kAKMajor, bool kBKMajor, int kEpi>
 __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
+  pdl_begin();
   __shared__ float As[kBK][kBM + 1];
   __shared__ float Bs[kBK][kBN + 1];
   const int z = blockIdx.z;
@@ -210,6 +211,7 @@ __global__ void __launch_bounds__(128) softmax_xent_kernel(const float* __restri
                                                            int m, int C, float* loss_parts,
                                                            const int* slot_commit, int lam,
                                                            int step, int* flag) {
+  pdl_begin();
   const int z = blockIdx.x;
   const float* Zs = Z + (int64_t)z * m * C;
   T* dZs = dZ + (int64_t)z * m * C;
@@ -253,6 +255,7 @@ template <typename T>
 __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y, T* Xb, int* yb,
                               int d0, int m, int64_t S, const int* slot_worker,
                               const long long* slot_t0, int step, bf16* pieces, int64_t plane) {
+  pdl_begin();
   const int z = blockIdx.y, j = blockIdx.x;
   const int w = slot_worker[z];
   const long long t = slot_t0[z] + step;
@@ -284,6 +287,7 @@ __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
                                                       const int* slot_worker,
                                                       const long long* slot_t0, int step,
                                                       bf16* pieces, int64_t plane) {
+  pdl_begin();
   struct alignas(4 * sizeof(T)) Vec { T v[4]; };
   struct alignas(8) Piece4 { bf16 v[4]; };
   const int r = blockIdx.x;                 // slot * m + j
@@ -312,7 +316,10 @@ __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
 template <typename T, typename TO, bool kAK, bool kBK, int kEpi>
 Status launch_gemm(const GemmArgs& g, int slots, cudaStream_t st) {
   dim3 grid((unsigned)ceil_div(g.N, kBN), (unsigned)ceil_div(g.M, kBM), (unsigned)slots);
-  gemm_simt_kernel<T, TO, kAK, kBK, kEpi><<<grid, kThreads, 0, st>>>(g);
+  {
+    auto kf = gemm_simt_kernel<T, TO, kAK, kBK, kEpi>;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, 0, st, g));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -336,8 +343,11 @@ template <typename T>
 Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* loss_parts,
                     const int* slot_commit, int lam, int step, int* flag, int slots,
                     cudaStream_t st) {
-  softmax_xent_kernel<T><<<slots, 128, 0, st>>>(Z, yb, dZ, m, C, loss_parts, slot_commit, lam,
-                                                step, flag);
+  {
+    auto kf = softmax_xent_kernel<T>;
+    AGN_TRY_CUDA(launch_pdl(kf, slots, 128, 0, st, Z,
+                            yb, dZ, m, C, loss_parts, slot_commit, lam, step, flag));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -351,12 +361,18 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
   if (slots <= 0 || m <= 0) return Status::Ok();
   if (vec) {
     const int threads = (int)std::min<int64_t>(256, round_up((int64_t)d0 / 4, 32));
-    gather4_kernel<T><<<slots * m, threads, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker,
-                                                     slot_t0, step, pieces, plane);
+    {
+      auto kf = gather4_kernel<T>;
+      AGN_TRY_CUDA(launch_pdl(kf, slots * m, threads, 0, st, X,
+                              y, Xb, yb, d0, m, S, slot_worker, slot_t0, step, pieces, plane));
+    }
   } else {
     dim3 grid((unsigned)m, (unsigned)slots);
-    gather_kernel<T><<<grid, 128, 0, st>>>(X, y, Xb, yb, d0, m, S, slot_worker, slot_t0, step,
-                                           pieces, plane);
+    {
+      auto kf = gather_kernel<T>;
+      AGN_TRY_CUDA(launch_pdl(kf, grid, 128, 0, st, X,
+                              y, Xb, yb, d0, m, S, slot_worker, slot_t0, step, pieces, plane));
+    }
   }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();

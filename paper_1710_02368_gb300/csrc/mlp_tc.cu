@@ -111,6 +111,7 @@ template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 __global__ void __launch_bounds__(kThreads, kEpi == kEpiDW ? 2 : 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const TcArgs args) {
+  pdl_begin();
   using Cfg = TileCfg<BN, kSplit>;
   using TAct = typename std::conditional<kSplit == 1, bf16, float>::type;
   extern __shared__ uint8_t smem_raw[];
@@ -488,6 +489,7 @@ bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
                    const int* __restrict__ slot_worker, float* theta, float* acc,
                    bf16* theta_b, int64_t ld_param, int64_t boff, float eta,
                    int64_t piece_plane) {
+  pdl_begin();
   __shared__ float red[kBiasGroups][32];
   const int fx = threadIdx.x & 31, gy = threadIdx.x >> 5;
   const int f = blockIdx.x * 32 + fx;
@@ -520,6 +522,7 @@ bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
 // out[p * plane + i] = piece p of x[i] (x = piece 0 + piece 1 + piece 2 exactly).
 __global__ void split_pieces_kernel(const float* __restrict__ x, bf16* __restrict__ out,
                                     int64_t count, int64_t plane) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += stride) {
     bf16 q0, q1, q2;
@@ -568,7 +571,10 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
             (unsigned)(slots * ks));
   TcArgs a2 = args;
   a2.ksplit = ks;
-  kern<<<grid, kThreads, smem, st>>>(a, b, a2);
+  {
+    auto kf = kern;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, smem, st, a, b, a2));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -680,15 +686,19 @@ Status bias_update(const void* dz, int m, int d, int64_t dz_bstride, const int* 
   dim3 grid((unsigned)ceil_div(d, 32), (unsigned)slots);
   const int threads = 32 * kBiasGroups;
   if (split)
-    bias_update_kernel<float, 3><<<grid, threads, 0, st>>>(static_cast<const float*>(dz), m, d,
-                                                           dz_bstride, slot_worker, theta, acc,
-                                                           theta_b, ld_param, boff, eta,
-                                                           piece_plane);
+    {
+      auto kf = bias_update_kernel<float, 3>;
+      AGN_TRY_CUDA(launch_pdl(kf, grid, threads, 0, st, static_cast<const float*>(dz),
+                              m, d, dz_bstride, slot_worker, theta, acc, theta_b, ld_param, boff,
+                              eta, piece_plane));
+    }
   else
-    bias_update_kernel<bf16, 1><<<grid, threads, 0, st>>>(static_cast<const bf16*>(dz), m, d,
-                                                          dz_bstride, slot_worker, theta, acc,
-                                                          theta_b, ld_param, boff, eta,
-                                                          piece_plane);
+    {
+      auto kf = bias_update_kernel<bf16, 1>;
+      AGN_TRY_CUDA(launch_pdl(kf, grid, threads, 0, st, static_cast<const bf16*>(dz),
+                              m, d, dz_bstride, slot_worker, theta, acc, theta_b, ld_param, boff,
+                              eta, piece_plane));
+    }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
@@ -696,7 +706,10 @@ Status bias_update(const void* dz, int m, int d, int64_t dz_bstride, const int* 
 Status split_pieces(const float* x, bf16* out, int64_t count, int64_t plane, cudaStream_t st) {
   if (count <= 0) return Status::Ok();
   const int grid = (int)std::min<int64_t>(ceil_div(count, 256), 152 * 8);
-  split_pieces_kernel<<<grid, 256, 0, st>>>(x, out, count, plane);
+  {
+    auto kf = split_pieces_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, 256, 0, st, x, out, count, plane));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -163,6 +163,7 @@ __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
 template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
+  pdl_begin();
   using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kMode>;
   constexpr bool kAcc = Cfg::kAcc, kGrad = kMode == kDwGrad;
   constexpr int kRing = Cfg::kRing, kSlotBytes = Cfg::kSlotBytes;
@@ -526,7 +527,10 @@ Status launch_dw(const DwBatch& batch, const TcArgs& args, int num_sms, cudaStre
   }
   if (batch.total_tiles <= 0) return Status::Ok();
   const int grid = std::min(batch.total_tiles, num_sms);
-  kern<<<grid, kThreads, Cfg::kSmem, st>>>(batch, args);
+  {
+    auto kf = kern;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, Cfg::kSmem, st, batch, args));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }

@@ -37,6 +37,7 @@ __device__ __forceinline__ void write_copy4(bf16* tb, int64_t plane, int64_t p, 
 }
 
 __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
+  pdl_begin();
   const int z = blockIdx.y;
   const int w = a.slot_worker[z];
   __shared__ float s_c1, s_c2;
@@ -88,7 +89,10 @@ Status adam_step(const AdamArgs& a, int slots, int num_sms, cudaStream_t st) {
   const int per_slot = (int)std::max<int64_t>(
       1, std::min<int64_t>(ceil_div(n4, kOptThreads), ceil_div((int64_t)num_sms * 8, slots)));
   dim3 grid((unsigned)per_slot, (unsigned)slots);
-  adam_kernel<<<grid, kOptThreads, 0, st>>>(a);
+  {
+    auto kf = adam_kernel;
+    AGN_TRY_CUDA(launch_pdl(kf, grid, kOptThreads, 0, st, a));
+  }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
