@@ -1360,9 +1360,15 @@ int agn_export_inputs(agn_handle* h, float* x, int32_t* y, float* theta0) {
 
 int agn_profile(agn_handle* h, int32_t mode) {
   if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
-  if (mode == 0) h->prof = false;
-  else if (mode == 1) h->prof = true;
-  else if (mode == 2) std::memset(h->kstats, 0, sizeof(h->kstats));
+  if (mode == 0) {
+    if (h->prof) --agn::g_pdl_off;
+    h->prof = false;
+  } else if (mode == 1) {
+    if (!h->prof) ++agn::g_pdl_off;   // no launch overlap while events time each kernel
+    h->prof = true;
+  } else if (mode == 2) {
+    std::memset(h->kstats, 0, sizeof(h->kstats));
+  }
   else return fail(h, AGN_E_INVALID, "mode must be 0, 1 or 2");
   return AGN_OK;
 }
@@ -1378,6 +1384,7 @@ const char* agn_last_error(const agn_handle* h) { return h ? h->err.c_str() : g_
 
 void agn_destroy(agn_handle* h) {
   if (!h) return;
+  if (h->prof) --agn::g_pdl_off;
   DeviceGuard g(h->device);
   if (h->stream) cudaStreamSynchronize(h->stream);
   for (void* p : h->allocs)

@@ -111,7 +111,6 @@ template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 __global__ void __launch_bounds__(kThreads, kEpi == kEpiDW ? 2 : 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const TcArgs args) {
-  pdl_begin();
   using Cfg = TileCfg<BN, kSplit>;
   using TAct = typename std::conditional<kSplit == 1, bf16, float>::type;
   extern __shared__ uint8_t smem_raw[];
@@ -164,8 +163,46 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   tc::tc_fence_after();
   const uint32_t tmem = *tmem_holder;
 
+  // Programmatic dependent launch: the setup above ran while the preceding
+  // kernel finished.  Everything that reads or writes global memory waits
+  // for it (pdl_begin), except the producer's loads of the weights for the
+  // first stages (forward and dX: A = W, last written two or more kernels
+  // back, and the preceding kernel only starts once its own predecessor is
+  // complete).
+  constexpr bool kPrefetchA = kEpi != kEpiDW;
+  const bool producer = warp == 0 && lane == 0;
+  if (!producer) pdl_begin();
   if (warp == 0) {
     if (lane == 0) {
+      // one box of 3D maps (kSplit = 1) or of 4D maps with the piece index
+      auto load = [&](uint8_t* dst, const CUtensorMap* map, int x, int y, int z, int p,
+                      uint64_t* bar) {
+        if (kSplit == 1) tc::tma_load_3d(dst, map, bar, x, y, z);
+        else tc::tma_load_4d(dst, map, bar, x, y, z, p);
+      };
+      auto load_a = [&](int kt, int s) {
+        uint8_t* sa0 = smem + s * Cfg::kStageBytes;
+        const int kc = (kt0 + kt) * kBK;
+#pragma unroll
+        for (int p = 0; p < kSplit; ++p) {
+          uint8_t* sa = sa0 + p * kABytes;
+          if (!kAMN) {
+            load(sa, &tmA, kc, m_tile * 128, a_z, p, &full[s]);
+          } else {
+            load(sa, &tmA, m_tile * 128, kc, a_z, p, &full[s]);
+            load(sa + 8192, &tmA, m_tile * 128 + 64, kc, a_z, p, &full[s]);
+          }
+        }
+      };
+      // prefetched stages count the A bytes now and arrive with the B bytes
+      // below, so no phase can complete before its B boxes are requested
+      constexpr uint32_t kABytesAll = kSplit * kABytes;
+      const int npre = kPrefetchA ? min(KT, kStages) : 0;
+      for (int kt = 0; kt < npre; ++kt) {
+        tc::mbar_expect_tx(&full[kt], kABytesAll);
+        load_a(kt, kt);
+      }
+      pdl_begin();
       int kt = 0;
       for (; kt < KT; ++kt) {
         const int s = kt % kStages;
@@ -176,34 +213,30 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (*abort_flag) break;
         uint8_t* sa0 = smem + s * Cfg::kStageBytes;
         uint8_t* sb0 = sa0 + kSplit * kABytes;
-        tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes);
-        // one box of 3D maps (kSplit = 1) or of 4D maps with the piece index
-        auto load = [&](uint8_t* dst, const CUtensorMap* map, int x, int y, int z, int p) {
-          if (kSplit == 1) tc::tma_load_3d(dst, map, &full[s], x, y, z);
-          else tc::tma_load_4d(dst, map, &full[s], x, y, z, p);
-        };
+        if (kt >= npre) {
+          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes);
+          load_a(kt, s);
+        } else {
+          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes - kABytesAll);
+        }
 #pragma unroll
         for (int p = 0; p < kSplit; ++p) {
-          uint8_t* sa = sa0 + p * kABytes;
           uint8_t* sb = sb0 + p * Cfg::kBBytes;
           const int kc = (kt0 + kt) * kBK;
-          if (!kAMN) {
-            load(sa, &tmA, kc, m_tile * 128, a_z, p);
-          } else {
-            load(sa, &tmA, m_tile * 128, kc, a_z, p);
-            load(sa + 8192, &tmA, m_tile * 128 + 64, kc, a_z, p);
-          }
           if (!kBMN) {
-            load(sb, &tmB, kc, n_tile * BN, b_z, p);
+            load(sb, &tmB, kc, n_tile * BN, b_z, p, &full[s]);
           } else {
 #pragma unroll
             for (int c = 0; c < BN / 64; ++c)
-              load(sb + c * 8192, &tmB, n_tile * BN + c * 64, kc, b_z, p);
+              load(sb + c * 8192, &tmB, n_tile * BN + c * 64, kc, b_z, p, &full[s]);
           }
         }
       }
       if (*abort_flag) {
-        // drain: wait (bounded) for the copies of the last stages we armed
+        // drain: wait (bounded) for the copies of the last stages we armed;
+        // prefetched stages not reached yet get their arrival first
+        for (int j = kt; j < npre; ++j) tc::mbar_arrive(&full[j]);
+        for (int j = kt; j < npre; ++j) tc::mbar_wait_bounded(&full[j], 0, kWaitNs);
         for (int j = kt - 1; j >= 0 && j >= kt - kStages; --j)
           tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
       }

@@ -163,7 +163,6 @@ __device__ __forceinline__ void write_ones_row(uint8_t* sa, int r) {
 template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
-  pdl_begin();
   using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kMode>;
   constexpr bool kAcc = Cfg::kAcc, kGrad = kMode == kDwGrad;
   constexpr int kRing = Cfg::kRing, kSlotBytes = Cfg::kSlotBytes;
@@ -221,6 +220,9 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  // programmatic dependent launch: the setup above overlapped the preceding
+  // kernel; global memory is touched only after it has completed
+  pdl_begin();
 
   if (warp == 0) {
     if (lane == 0) {

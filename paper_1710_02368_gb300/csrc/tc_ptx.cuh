@@ -43,6 +43,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Add `bytes` to the transaction count of the current phase without arriving
+// (the phase cannot complete before the pending arrival).
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
 // Plain arrive (count 1), release semantics at CTA scope: the caller's earlier
 // shared-memory reads are ordered before a producer that waits on `bar`.
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
