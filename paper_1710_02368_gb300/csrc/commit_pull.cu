@@ -2,7 +2,7 @@
 //
 // For a run of consecutive commits (FIFO order, Eq. 2) the kernel streams the
 // parameter vector once: each thread keeps its slice of theta~ in registers,
-// and for every commit c of the launch reads the committing worker's
+// and for every commit c of the launch takes the committing worker's
 // accumulator, forms Delta = fp32(a * s) with s = fp32(-eta/lambda) (Eq. 1;
 // the normalisation step of Algorithm 1; or a per-commit s = fp32(-eta /
 // (tau_c + 1)) for the DynSGD rule), adds it to theta~ with a plain
@@ -24,7 +24,12 @@ namespace agn {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 2;   // float4 per thread per iteration (memory-level parallelism)
+// Two shapes of the same loop.  Long vectors (many float4 per thread): two
+// float4 per thread and commit by commit, registers kept low for occupancy.
+// Short vectors (a few float4 per thread, the MLP workloads' commits): one
+// float4 per thread and the accumulator loads of eight commits in flight.
+constexpr int kLongUnroll = 2, kLongGroup = 1;
+constexpr int kShortUnroll = 1, kShortGroup = 8;
 
 __device__ __forceinline__ float4 ld_stream(const float4* p) { return __ldcs(p); }
 __device__ __forceinline__ void st_stream(float4* p, float4 v) { __stcs(p, v); }
@@ -66,7 +71,7 @@ __device__ __forceinline__ void pack_pieces_x4(float4 v, uint2& p0, uint2& p1, u
 // of its last pull, the committed quantity is fp32(theta_k - theta_pull) (the
 // sum of the local updates) with s = fp32(1/lambda) (or fp32(1/(tau_c + 1)),
 // or 1), and every pull also refreshes the snapshot.
-template <int kCopy, bool kElide>
+template <int kCopy, bool kElide, int kUnroll, int kGroup>
 __global__ void __launch_bounds__(kThreads)
 commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ theta_c,
                    float* __restrict__ acc, float* __restrict__ replicas,
@@ -92,50 +97,61 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
       live[u] = idx[u] < n4;
       if (live[u]) th[u] = th4[idx[u]];
     }
+    // commits in groups of kGroup: every accumulator load of a group is in
+    // flight before the group's dependent chain of adds (theta~ must see the
+    // commits in FIFO order, the loads need not wait for each other)
 #pragma unroll
-    for (int c = 0; c < kMaxCommitsPerLaunch; ++c) {
-      if (c < nc) {
-        float4* arow = reinterpret_cast<float4*>(acc + (int64_t)plan.worker[c] * ld);
-        float4 a[kUnroll];
-        if (kElide) {
-          const float4* krow =
-              reinterpret_cast<const float4*>(replicas + (int64_t)plan.worker[c] * ld);
+    for (int c0 = 0; c0 < kMaxCommitsPerLaunch; c0 += kGroup) {
+      if (c0 >= nc) break;
+      float4 a[kGroup][kUnroll];
 #pragma unroll
-          for (int u = 0; u < kUnroll; ++u) {
-            if (!live[u]) continue;
-            const float4 tk = ld_stream(krow + idx[u]), tp = ld_stream(arow + idx[u]);
-            a[u] = make_float4(__fsub_rn(tk.x, tp.x), __fsub_rn(tk.y, tp.y),
-                               __fsub_rn(tk.z, tp.z), __fsub_rn(tk.w, tp.w));
+      for (int j = 0; j < kGroup; ++j) {
+        const int c = c0 + j;
+        if (c >= nc) break;
+        const int64_t row = (int64_t)plan.worker[c] * ld;
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          if (!live[u]) continue;
+          if (kElide) {   // theta_k - theta_pull, the sum of the local updates
+            const float4 tk = ld_stream(reinterpret_cast<const float4*>(replicas + row) + idx[u]);
+            const float4 tp = ld_stream(reinterpret_cast<const float4*>(acc + row) + idx[u]);
+            a[j][u] = make_float4(__fsub_rn(tk.x, tp.x), __fsub_rn(tk.y, tp.y),
+                                  __fsub_rn(tk.z, tp.z), __fsub_rn(tk.w, tp.w));
+          } else {
+            a[j][u] = ld_stream(reinterpret_cast<const float4*>(acc + row) + idx[u]);
           }
-        } else {
-#pragma unroll
-          for (int u = 0; u < kUnroll; ++u)
-            if (live[u]) a[u] = ld_stream(arow + idx[u]);
         }
+      }
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        const int c = c0 + j;
+        if (c >= nc) break;
         const float sc = plan.per_commit_scale ? plan.scale[c] : s;
+        const int64_t arow = (int64_t)plan.worker[c] * ld;
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) {
           if (!live[u]) continue;
           float4 d;
-          d.x = __fmul_rn(a[u].x, sc);
-          d.y = __fmul_rn(a[u].y, sc);
-          d.z = __fmul_rn(a[u].z, sc);
-          d.w = __fmul_rn(a[u].w, sc);
+          d.x = __fmul_rn(a[j][u].x, sc);
+          d.y = __fmul_rn(a[j][u].y, sc);
+          d.z = __fmul_rn(a[j][u].z, sc);
+          d.w = __fmul_rn(a[j][u].w, sc);
           th[u].x = __fadd_rn(th[u].x, d.x);
           th[u].y = __fadd_rn(th[u].y, d.y);
           th[u].z = __fadd_rn(th[u].z, d.z);
           th[u].w = __fadd_rn(th[u].w, d.w);
-          float q = d.x * d.x + d.y * d.y + d.z * d.z + d.w * d.w;
+          const float q = d.x * d.x + d.y * d.y + d.z * d.z + d.w * d.w;
           sq[c] += (double)q;
-          if (!kElide && zero_acc) st_stream(arow + idx[u], make_float4(0.f, 0.f, 0.f, 0.f));
+          if (!kElide && zero_acc)
+            st_stream(reinterpret_cast<float4*>(acc + arow) + idx[u],
+                      make_float4(0.f, 0.f, 0.f, 0.f));
         }
         for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
           const int64_t row = (int64_t)plan.pull_worker[p] * ld;
-          float4* rrow = reinterpret_cast<float4*>(replicas + row);
 #pragma unroll
           for (int u = 0; u < kUnroll; ++u) {
             if (!live[u]) continue;
-            rrow[idx[u]] = th[u];
+            reinterpret_cast<float4*>(replicas + row)[idx[u]] = th[u];
             if (kElide) reinterpret_cast<float4*>(acc + row)[idx[u]] = th[u];
             if (kCopy == 1) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
             if (kCopy == 3) {
@@ -240,7 +256,7 @@ int commit_grid(int64_t P) {
     cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
     if (g_num_sms <= 0) g_num_sms = 148;
   }
-  const int64_t need = ceil_div(std::max<int64_t>(P / 4, 1), (int64_t)kThreads * kUnroll);
+  const int64_t need = ceil_div(std::max<int64_t>(P / 4, 1), (int64_t)kThreads * kLongUnroll);
   const int64_t cap = (int64_t)g_num_sms * 4;
   return (int)std::max<int64_t>(1, std::min(need, cap));
 }
@@ -255,16 +271,20 @@ Status launch_commit_pull(const CommitPlan& plan, float* theta_c, float* acc, fl
     return launch_pdl(kern, grid, kThreads, 0, stream, plan, theta_c, acc, replicas, rb, P, ld,
                       scale, z, partials, plane);
   };
+  // short vectors: at most 8 float4 per thread over the grid
+  const bool shrt = P / 4 <= (int64_t)grid * kThreads * 8;
   cudaError_t e;
+#define AGN_COMMIT_GO(C, E, RB, PL)                                                            \
+  (shrt ? go(commit_pull_kernel<C, E, kShortUnroll, kShortGroup>, RB, PL)                       \
+        : go(commit_pull_kernel<C, E, kLongUnroll, kLongGroup>, RB, PL))
   if (replicas_bf16 && piece_plane > 0)
-    e = elide ? go(commit_pull_kernel<3, true>, replicas_bf16, piece_plane)
-              : go(commit_pull_kernel<3, false>, replicas_bf16, piece_plane);
+    e = elide ? AGN_COMMIT_GO(3, true, replicas_bf16, piece_plane)
+              : AGN_COMMIT_GO(3, false, replicas_bf16, piece_plane);
   else if (replicas_bf16)
-    e = elide ? go(commit_pull_kernel<1, true>, replicas_bf16, 0)
-              : go(commit_pull_kernel<1, false>, replicas_bf16, 0);
+    e = elide ? AGN_COMMIT_GO(1, true, replicas_bf16, 0) : AGN_COMMIT_GO(1, false, replicas_bf16, 0);
   else
-    e = elide ? go(commit_pull_kernel<0, true>, nullptr, 0)
-              : go(commit_pull_kernel<0, false>, nullptr, 0);
+    e = elide ? AGN_COMMIT_GO(0, true, nullptr, 0) : AGN_COMMIT_GO(0, false, nullptr, 0);
+#undef AGN_COMMIT_GO
   AGN_TRY_CUDA(e);
   if (norms && partials && (delta_norm || flag))
     return launch_commit_norms(plan, partials, grid, delta_norm, flag, stream);
