@@ -537,6 +537,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         d.ld_param = h->P_pad; d.woff = h->woff[l - 1]; d.boff = h->boff[l - 1];
         d.K = fi; d.C = fo; d.m = m; d.eta = eta;
         d.grad_out = h->adam ? h->grad : nullptr;
+        d.dz_early = L > 2 ? 1 : 0;   // a dX launch ran between the head and this one
         AGN_TRY(agn::head_backward_dw<T>(d, s, h->stream));
       } else {
         agn::GemmArgs g{};

@@ -99,6 +99,8 @@ struct HeadDwArgs {
   int K, C, m;
   float eta;
   float* grad_out;         // store the raw gradient here instead of updating; null = update
+  int dz_early;            // 1: dZ_L was written two or more launches back (may be read
+                           // before the preceding launch completes)
 };
 template <typename T>
 Status head_backward_dw(const HeadDwArgs& a, int slots, cudaStream_t st);

@@ -64,7 +64,6 @@ __device__ __forceinline__ void stage_wait() {
 
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
-  pdl_begin();
   extern __shared__ __align__(16) uint8_t head_smem[];
   __shared__ float red[kHeadSamples][kHeadSplit][kMaxC];
   __shared__ float ce_s[kHeadSamples];
@@ -80,7 +79,12 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   T* Hs = Ws + (int64_t)C * Kp;                             // [kHeadSamples][Kp]
   const T* Wg = static_cast<const T*>(a.W) + (int64_t)w * a.ld_param + a.woff;
   const T* Hg = static_cast<const T*>(a.H) + ((int64_t)z * m + j0) * K;
+  // W_L was last written two or more launches back (this slot's output-layer
+  // update of the previous local step, or a pull), so its copy starts before
+  // waiting for the preceding kernel (programmatic dependent launch); the
+  // input rows come from the preceding forward and wait for it
   for (int c = 0; c < C; ++c) stage(Ws + c * Kp, Wg + (int64_t)c * K, K);
+  pdl_begin();
   for (int r = 0; r < nj; ++r) stage(Hs + r * Kp, Hg + (int64_t)r * K, K);
   stage_wait();
   __syncthreads();
@@ -150,10 +154,13 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
     T* dh = a.dH ? static_cast<T*>(a.dH) + ((int64_t)z * m + j) * K : nullptr;
     bf16* dp = a.dH_pieces ? a.dH_pieces + ((int64_t)z * m + j) * K : nullptr;
     for (int k = 32 * q + lane; dh && k < K; k += kStride) {
-      float v = 0.f;
+      float v0 = 0.f, v1 = 0.f;   // two chains: even and odd classes
 #pragma unroll
-      for (int c = 0; c < kMaxC; ++c)
-        if (c < C) v = fmaf(g[c], cvt(Ws[(int64_t)c * Kp + k]), v);
+      for (int c = 0; c < kMaxC; c += 2) {
+        if (c < C) v0 = fmaf(g[c], cvt(Ws[(int64_t)c * Kp + k]), v0);
+        if (c + 1 < C && c + 1 < kMaxC) v1 = fmaf(g[c + 1], cvt(Ws[(int64_t)(c + 1) * Kp + k]), v1);
+      }
+      const float v = v0 + v1;
       const T out = st_f<T>(cvt(h[k]) > 0.f ? v : 0.f);
       dh[k] = out;
       if (dp) {
@@ -211,14 +218,17 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
 constexpr int kDwGroups = 8;
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArgs a) {
-  pdl_begin();
   extern __shared__ __align__(16) uint8_t dw_smem[];
   float* red = reinterpret_cast<float*>(dw_smem);                      // [kDwGroups][kMaxC][32]
   T* dz = reinterpret_cast<T*>(red + kDwGroups * kMaxC * 32);           // [m][C]
   const int z = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, C = a.C, m = a.m;
-  stage(dz, static_cast<const T*>(a.dZL) + (int64_t)z * m * C, (int64_t)m * C);
+  // dZ_L comes from the output head; when another launch ran in between
+  // (a.dz_early), its copy starts before waiting for the preceding kernel
+  if (a.dz_early) stage(dz, static_cast<const T*>(a.dZL) + (int64_t)z * m * C, (int64_t)m * C);
+  pdl_begin();
+  if (!a.dz_early) stage(dz, static_cast<const T*>(a.dZL) + (int64_t)z * m * C, (int64_t)m * C);
   stage_wait();
   __syncthreads();
   const int w = a.slot_worker[z];

@@ -221,13 +221,49 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   tc::tc_fence_after();
   const uint32_t tmem = *tmem_holder;
   // programmatic dependent launch: the setup above overlapped the preceding
-  // kernel; global memory is touched only after it has completed
-  pdl_begin();
+  // kernel; global memory is touched only after it has completed, except the
+  // producer's first parameter chunks (below)
 
+  if (!(warp == 0 && lane == 0)) pdl_begin();
   if (warp == 0) {
     if (lane == 0) {
       uint32_t ml = 0, ch = 0;   // stage fills and chunk fills issued
       bool ok = true;
+      // theta_k / a_k chunk c of tile ti into ring slot r
+      auto issue_chunk = [&](const TileIdx& ti, int worker, int c, int r) {
+        const DwLayer& L = B.layer[ti.layer];
+        const bool bias_tile = ti.m_tile == L.M / 128;
+        uint8_t* dst = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
+        const int f0 = ti.n_tile * BN + c * kCF;
+        constexpr int kA = Cfg::kArrays;
+        tc::mbar_arrive_expect_tx(&cfull[r], kA * (kChunkBytes + (bias_tile ? kBiasHalf : 0)));
+        tc::tma_load_3d(dst, &B.th[ti.layer], &cfull[r], ti.m_tile * 128, f0, worker);
+        if (kAcc)
+          tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
+                          worker);
+        if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
+          const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
+          tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
+          if (kAcc)
+            tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
+                          &cfull[r]);
+        }
+      };
+      // theta_k and a_k were last written by this kernel's previous launch or
+      // a pull, two or more launches back: the first tile's first chunks are
+      // requested before waiting for the preceding kernel
+      int npre = 0;
+      if (!kGrad && (int)blockIdx.x < T) {
+        const TileIdx t0 = decode(B, blockIdx.x);
+        const DwLayer& L0 = B.layer[t0.layer];
+        npre = min(kRing, min(Cfg::kChunks, (L0.N - t0.n_tile * BN + kCF - 1) / kCF));
+        const int w0 = args.slot_worker[t0.slot];
+        for (int c = 0; c < npre; ++c) {
+          issue_chunk(t0, w0, c, (int)ch);
+          ++ch;
+        }
+      }
+      pdl_begin();
       for (int t = blockIdx.x; ok && t < T; t += gridDim.x) {
         const TileIdx ti = decode(B, t);
         const DwLayer& L = B.layer[ti.layer];
@@ -269,30 +305,15 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         }
         if (!ok) break;
         if (kGrad) continue;   // the gradient needs no parameter chunks
-        const bool bias_tile = ti.m_tile == L.M / 128;
         const int nch = min(Cfg::kChunks, (L.N - ti.n_tile * BN + kCF - 1) / kCF);
-        for (int c = 0; c < nch; ++c) {
+        for (int c = t == (int)blockIdx.x ? npre : 0; c < nch; ++c) {
           const int r = ch % kRing;
           if (ch >= kRing &&
               !tc::wait_or_abort(&cempty[r], ((ch / kRing) - 1) & 1, abort_flag, kWaitNs)) {
             ok = false;
             break;
           }
-          uint8_t* dst = smem + Cfg::kRingOff + (size_t)r * kSlotBytes;
-          const int f0 = ti.n_tile * BN + c * kCF;
-          constexpr int kA = Cfg::kArrays;
-          tc::mbar_arrive_expect_tx(&cfull[r], kA * (kChunkBytes + (bias_tile ? kBiasHalf : 0)));
-          tc::tma_load_3d(dst, &B.th[ti.layer], &cfull[r], ti.m_tile * 128, f0, worker);
-          if (kAcc)
-            tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
-                            worker);
-          if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
-            const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
-            tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
-            if (kAcc)
-              tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
-                            &cfull[r]);
-          }
+          issue_chunk(ti, worker, c, r);
           ++ch;
         }
       }
