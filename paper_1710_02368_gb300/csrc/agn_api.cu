@@ -116,9 +116,12 @@ struct agn_handle {
     CUtensorMap h_mn32, dz_mn32; // split mode: 32-sample boxes for the dW kernel
   };
   int num_sms = 148;
+  // maps of the output layer's dW when it runs in the tensor-core dW launch
+  // (theta, acc, h_mn / h_mn32 over H_{L-1}, dz_mn / dz_mn32 over dZ_L)
   float* tc_part = nullptr;     // split-K partial sums: [SMs][BN <= 256][128]
   int* tc_counter = nullptr;    // split-K arrival count per output tile: [SMs]
   std::vector<LayerMaps> tmaps;
+  LayerMaps out_maps;
   // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
   bool split = false;
   int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
@@ -126,6 +129,11 @@ struct agn_handle {
   std::vector<bf16*> dZp;         // pieces of dZ_l, l = 1..L-1: [3][n][m][d_l]
   // output layer fused into one kernel (forward + softmax-CE + dX) when narrow
   bool use_head = false;
+  // the output layer's dW runs as tiles of the persistent tensor-core dW
+  // launch: dZ_L padded to ldz_out columns (zero beyond d_L) with its pieces,
+  // and H_{L-1}'s pieces kept
+  bool fuse_out_dw = false;
+  int ldz_out = 0;
   float* ce_partial = nullptr;    // [n][ceil(m / kHeadSamples)]
   int* head_counter = nullptr;    // [n]
   int grid = 0;
@@ -323,6 +331,24 @@ Status build_tc_maps(agn_handle* h) {
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
   }
+  if (h->fuse_out_dw) {   // the output layer's dW tiles: M = d_{L-1} inputs, N = d_L
+    const uint64_t fi = h->dims[L - 1], fo = h->dims[L], lz = (uint64_t)h->ldz_out;
+    auto& mp = h->out_maps;
+    AGN_TRY(agn::make_tmap_f32_3d(&mp.theta, h->rep + h->woff[L - 1], fi, fo, n, fi, h->P_pad,
+                                  128, 32));
+    AGN_TRY(agn::make_tmap_f32_3d(&mp.acc, h->acc + h->woff[L - 1], fi, fo, n, fi, h->P_pad,
+                                  128, 32));
+    if (h->split) {
+      const bf16* Hp = h->Hs[L - 1];
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, Hp, fi, m, n, fi, (uint64_t)m * fi,
+                                     (uint64_t)n * m * fi, 64, 32));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn32, h->dZp[L], lz, m, n, lz, (uint64_t)m * lz,
+                                     (uint64_t)n * m * lz, 64, 32));
+    } else {
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_mn, h->H[L - 1], fi, m, n, fi, (uint64_t)m * fi, 64, 64));
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, h->dZ[L], lz, m, n, lz, (uint64_t)m * lz, 64, 64));
+    }
+  }
   return Status::Ok();
 }
 
@@ -398,7 +424,10 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         a.woff = h->woff[L - 1]; a.boff = h->boff[L - 1];
         a.K = fi; a.C = C; a.m = m;
         a.slot_worker = sw; a.yb = h->yb;
-        a.dZL = h->dZ[L]; a.dH = L > 1 ? h->dZ[L - 1] : nullptr;
+        a.dZL = h->dZ[L]; a.ldz = h->ldz_out;
+        a.dZL_pieces = (h->fuse_out_dw && h->split) ? h->dZp[L] : nullptr;
+        a.dZL_plane = (int64_t)n * m * h->ldz_out;
+        a.dH = L > 1 ? h->dZ[L - 1] : nullptr;
         a.dH_pieces = L > 1 ? dz_pieces(L - 1) : nullptr;
         a.dH_plane = L > 1 ? dz_plane(L - 1) : 0;
         a.ce_partial = h->ce_partial; a.counter = h->head_counter;
@@ -423,7 +452,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       const double oes = l == L ? 4.0 : es;
       // pieces of a hidden activation that the next tensor-core GEMMs read
       // (the forward of layer l + 1 and the dW of layer l + 1)
-      bf16* h_pieces = (h->split && l + 1 < L) ? h->Hs[l] : nullptr;
+      bf16* h_pieces =
+          (h->split && (l + 1 < L || (h->fuse_out_dw && l + 1 == L))) ? h->Hs[l] : nullptr;
       bool pieces_done = false;
       {
         Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
@@ -526,6 +556,15 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           tc_flops += flops;
           tc_bytes += bytes;
         }
+        continue;
+      }
+      if (l == L && h->fuse_out_dw) {   // as tiles of the tensor-core dW launch
+        const auto& mp = h->out_maps;
+        tc_dw.insert(tc_dw.begin(), {h->split ? &mp.h_mn32 : &mp.h_mn,
+                                     h->split ? &mp.dz_mn32 : &mp.dz_mn, &mp.theta, &mp.acc, fi,
+                                     fo, h->woff[l - 1], h->boff[l - 1]});
+        tc_flops += flops;
+        tc_bytes += bytes;
         continue;
       }
       Launch k(h, AGN_K_BACKWARD_DW, flops, bytes, launches);
@@ -964,14 +1003,22 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
     for (float* p : {h->grad, h->mom1, h->mom2})
       AGN_TRY_CUDA(cudaMemset(p, 0, (size_t)(n * h->P_pad) * sizeof(float)));
   }
+  h->use_head = h->prec == AGN_PREC_BF16 ? agn::head_fits<bf16>(dims[h->L - 1], dims[h->L])
+                                         : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
+  h->fuse_out_dw = h->use_tc && h->use_head && h->L >= 2 && (h->tc_mask & 4) && !(h->tc_mask & 8);
+  h->ldz_out = h->fuse_out_dw ? (int)round_up(dims[h->L], 8) : dims[h->L];
   if (h->split) {   // three piece planes of every replica, and of the activations
     h->piece_plane = n * h->P_pad;
     AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));
-    h->Hs.assign(h->L - 1, nullptr);
-    for (int l = 0; l + 1 < h->L; ++l)
+    h->Hs.assign(h->L, nullptr);
+    for (int l = 0; l + 1 < h->L + (h->fuse_out_dw ? 1 : 0); ++l)
       AGN_TRY(dalloc_t(h, &h->Hs[l], (size_t)(3 * n * m * dims[l])));
-    h->dZp.assign(h->L, nullptr);
+    h->dZp.assign(h->L + 1, nullptr);
     for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc_t(h, &h->dZp[l], (size_t)(3 * n * m * dims[l])));
+    if (h->fuse_out_dw) {
+      AGN_TRY(dalloc_t(h, &h->dZp[h->L], (size_t)(3 * n * m * h->ldz_out)));
+      AGN_TRY_CUDA(cudaMemset(h->dZp[h->L], 0, (size_t)(3 * n * m * h->ldz_out) * sizeof(bf16)));
+    }
   }
   AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
   AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));
@@ -981,10 +1028,10 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->H[l], (size_t)(n * m * dims[l]) * es));
   AGN_TRY(dalloc_t(h, &h->Z, (size_t)(n * m * dims[h->L])));
   h->dZ.assign(h->L + 1, nullptr);
-  for (int l = 1; l <= h->L; ++l) AGN_TRY(dalloc(h, &h->dZ[l], (size_t)(n * m * dims[l]) * es));
+  for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->dZ[l], (size_t)(n * m * dims[l]) * es));
+  AGN_TRY(dalloc(h, &h->dZ[h->L], (size_t)(n * m * h->ldz_out) * es));
+  AGN_TRY_CUDA(cudaMemset(h->dZ[h->L], 0, (size_t)(n * m * h->ldz_out) * es));
   AGN_TRY(dalloc_t(h, &h->flag, 2));
-  h->use_head = h->prec == AGN_PREC_BF16 ? agn::head_fits<bf16>(dims[h->L - 1], dims[h->L])
-                                         : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
   AGN_TRY(dalloc_t(h, &h->ce_partial, (size_t)(n * ceil_div(m, agn::kHeadSamples))));
   AGN_TRY(dalloc_t(h, &h->head_counter, (size_t)n));
   if (h->n_eval > 0) {

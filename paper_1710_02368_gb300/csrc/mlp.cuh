@@ -73,7 +73,10 @@ struct HeadArgs {
   int K, C, m;
   const int* slot_worker;
   const int* yb;           // labels [slots][m]
-  void* dZL;               // out: dZ_L [slots][m][C] (T)
+  void* dZL;               // out: dZ_L [slots][m][ldz] (T), ldz >= C
+  int ldz;                 // row stride of dZ_L (columns C .. ldz - 1 are left alone)
+  bf16* dZL_pieces;        // fp32 T only: also dZ_L's three exact bf16 pieces (planes
+  int64_t dZL_plane;       // dZL_plane apart, same layout) for the tensor-core dW; null = no
   void* dH;                // out: dZ_{L-1} [slots][m][K] (T)
   bf16* dH_pieces;         // fp32 T only: also its three exact bf16 pieces (planes
   int64_t dH_plane;        // dH_plane apart) for tensor-core GEMMs; null = no

@@ -144,10 +144,21 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
       g[c] = p * inv_m;
     }
     if (q == 0) {
-      T* dzl = static_cast<T*>(a.dZL) + ((int64_t)z * m + j) * C;
+      T* dzl = static_cast<T*>(a.dZL) + ((int64_t)z * m + j) * a.ldz;
+      bf16* dzp = a.dZL_pieces ? a.dZL_pieces + ((int64_t)z * m + j) * a.ldz : nullptr;
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
-        if (c < C && lane == c) dzl[c] = st_f<T>(g[c]);
+        if (c < C && lane == c) {
+          const T gv = st_f<T>(g[c]);
+          dzl[c] = gv;
+          if (dzp) {
+            bf16 q0, q1, q2;
+            split3(cvt(gv), q0, q1, q2);
+            dzp[c] = q0;
+            dzp[a.dZL_plane + c] = q1;
+            dzp[2 * a.dZL_plane + c] = q2;
+          }
+        }
     }
     // dZ_{L-1}[j][k] = sum_c dZ_L[j][c] W_L[c][k], masked by h > 0 (W before its
     // update); skipped when the output layer is the only layer (dH null)
