@@ -36,7 +36,7 @@ constexpr int kThreads = 256;
 constexpr int kBK = 64;                       // K per stage: 64 bf16 = one 128-byte row
 constexpr int kABytes = 128 * 128;            // 128 rows x 128 bytes
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s
-constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles (end of ring)
+constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles
 
 // A stage holds kSplit A pieces then kSplit B pieces (kSplit = 3 in the fp32
 // mode, where every fp32 operand is the exact sum of three bf16 pieces).
@@ -48,6 +48,17 @@ struct TileCfg {
   // piece products a0 b0, columns [BN, 2 BN) the five smaller pairs, so the
   // rounding of the tensor core's running sums is relative to each part
   static constexpr uint32_t kTmemCols = (kSplit == 1 ? 1 : 2) * BN;   // power of two >= 32
+};
+
+// The forward / dX epilogue's transpose tiles sit after the barriers when the
+// CTA's shared memory has room for them (then the whole stage ring can hold
+// split-K partial sums), else at the end of the ring.
+template <int BN, int kSplit, int kStages>
+struct EpiT {
+  static constexpr size_t kRing = (size_t)kStages * TileCfg<BN, kSplit>::kStageBytes;
+  static constexpr bool kSeparate = kRing + 1280 + kEpiTBytes <= 232448;
+  static constexpr size_t kOff = kSeparate ? kRing + 256 : kRing - kEpiTBytes;
+  static constexpr size_t kRingFree = kSeparate ? kRing : kRing - kEpiTBytes;
 };
 
 // Piece pairs (i, j) with i + j <= 2 of the split product: the dropped pairs
@@ -373,7 +384,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // handles four consecutive rows (features, contiguous in memory) of
     // eight columns: 16-byte bias / mask loads, 16-byte stores of the output
     // and 8-byte stores of each bf16 piece.
-    float* tT = reinterpret_cast<float*>(smem + (size_t)kStages * Cfg::kStageBytes - kEpiTBytes) +
+    float* tT = reinterpret_cast<float*>(smem + EpiT<BN, kSplit, kStages>::kOff) +
                 warp * (32 * 32);
     const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
     const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
@@ -570,7 +581,8 @@ template <int BN, int kSplit, int kStages>
 size_t smem_bytes() {
   // Shared memory requested per CTA also caps the CTAs per SM so that their
   // TMEM columns never exceed the 512 an SM has.
-  const size_t ring = (size_t)kStages * TileCfg<BN, kSplit>::kStageBytes + 1024 + 256;
+  const size_t ring = (size_t)kStages * TileCfg<BN, kSplit>::kStageBytes + 1024 + 256 +
+                      (EpiT<BN, kSplit, kStages>::kSeparate ? kEpiTBytes : 0);
   const size_t floor_for_tmem =
       (size_t)(233472 / (512 / TileCfg<BN, kSplit>::kTmemCols + 1)) + 1024;
   return std::max(ring, floor_for_tmem);
@@ -592,7 +604,7 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
   // holds, every rank with a non-empty range of k steps
   int ks = kEpi == kEpiDW ? 1 : std::max(1, args.ksplit);
   if (ks > 1) {
-    const int ring = kStages * TileCfg<BN, kSplit>::kStageBytes - kEpiTBytes;
+    const int ring = (int)EpiT<BN, kSplit, kStages>::kRingFree;
     ks = std::min(ks, 1 + ring / (128 * BN * 4));
     const int kt = (args.K + kBK - 1) / kBK;
     ks = std::min(ks, kt);
