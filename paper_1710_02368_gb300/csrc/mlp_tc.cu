@@ -317,68 +317,22 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       tc::tmem_ld_wait();
     };
-    bool last = true;
+    // Split K (forward / dX): chunk j of the tile (columns 32 j .. 32 j + 31)
+    // is finished by rank j % ks.  Every rank stores its partial sums of the
+    // chunks it does not finish ([column][row], rows contiguous) and counts
+    // itself in (low half of the tile's counter).  A rank that finishes
+    // chunks waits until all ks ranks are in (the CTAs of a launch with
+    // ks > 1 are resident together: at most one per SM, no more than the
+    // SMs), copies the other ranks' partial sums of its chunks into its stage
+    // ring and adds them in rank order, its own from TMEM.  Every rank then
+    // counts itself out (high half); the last one out resets the counter for
+    // the next launch.
+    constexpr int kNch = BN / 32;
+    constexpr uint32_t kChunkBytes = 128u * 32u * 4u;
+    const bool split_k = kEpi != kEpiDW && ks > 1;
+    const int own_rank = split_k ? sk : 0, kstride = split_k ? ks : 1;
+    const int n_own = (kNch - own_rank + kstride - 1) / kstride;   // chunks own_rank + o ks
     const float* red_smem = reinterpret_cast<const float*>(smem);   // the free stage ring
-    if (kEpi != kEpiDW && ks > 1) {
-      // every CTA of the tile stores its partial sums ([column][row], rows
-      // contiguous); the last to finish copies the others' into its stage
-      // ring (TMA bulk copies, all in flight at once) and adds them in rank
-      // order, its own from TMEM
-      float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
-#pragma unroll 1
-      for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
-        uint32_t r[32];
-        tmem_vals(c0, r);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) __stcg(mine + (int64_t)(c0 + i) * 128 + trow, __uint_as_float(r[i]));
-      }
-      // the CTA's stores, ordered by the barrier, are released by one
-      // acquire-release arrival; the last arrival acquires the others'
-      __shared__ int s_last;
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        const int prev = tc::atomic_add_acq_rel_gpu(args.counter + tile_id, 1);
-        s_last = prev == ks - 1;
-        if (s_last) {
-          args.counter[tile_id] = 0;   // ready for the next launch
-          tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
-          constexpr uint32_t kPart = 128u * BN * 4u;
-          tc::mbar_arrive_expect_tx(red, kPart * (uint32_t)(ks - 1));
-          for (int q = 0, d = 0; q < ks; ++q) {
-            if (q == sk) continue;
-            tc::bulk_load(smem + (size_t)d * kPart,
-                          args.part + (tile_id * ks + q) * (int64_t)(128 * BN), kPart, red);
-            ++d;
-          }
-        }
-      }
-      __syncthreads();
-      last = s_last != 0;
-      if (last && !__syncthreads_and(wait_or_abort(red, 0, abort_flag))) {
-        last = false;   // gave up: report, skip the epilogue
-        if (threadIdx.x == 0) atomicExch(args.err, 1);
-      }
-    }
-    auto vals = [&](int c0, uint32_t (&r)[32]) {
-      tmem_vals(c0, r);
-      if (kEpi == kEpiDW || ks == 1) return;
-      float v[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = 0.f;
-      for (int q = 0, d = 0; q < ks; ++q) {
-        if (q == sk) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
-        } else {
-          const float* pq = red_smem + (size_t)d * (128 * BN) + (size_t)c0 * 128 + trow;
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] += pq[i * 128];
-          ++d;
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(v[i]);
-    };
     // Forward and dX epilogues: the warp's 32 rows x 32 columns go through a
     // warp-private shared-memory tile (column-major) so that each lane then
     // handles four consecutive rows (features, contiguous in memory) of
@@ -389,32 +343,115 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
     const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
     const bool row4_ok = row4 < args.M;                      // M % 4 == 0: all four or none
-    if (!last) {
-      // another CTA of this tile finishes it
+    const TAct* mask = kEpi == kEpiDX
+                           ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
+                           : nullptr;
+    // the mask of the warp's first chunk (and the bias) are loaded before
+    // the split-K exchange: they do not depend on it
+    float4 hm[8];
+    auto load_mask = [&](int c0) {
+      if (kEpi == kEpiDX && row4_ok) {   // all mask loads in flight before any store
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int j = n_tile * BN + c0 + jl + 4 * u;
+          hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+    };
+    float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (kEpi == kEpiFwd && row4_ok && half < n_own)
+      bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
+    if (half < n_own) load_mask(32 * (own_rank + half * kstride));
+    bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
+    if (split_k) {
+      float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
+      int c = 0;   // the chunks this rank does not finish, alternately to the two halves
+#pragma unroll
+      for (int j = 0; j < kNch; ++j) {
+        if (j % ks == sk) continue;
+        if ((c++ & 1) != half) continue;
+        uint32_t r[32];
+        tmem_vals(32 * j, r);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          __stcg(mine + (int64_t)(32 * j + i) * 128 + trow, __uint_as_float(r[i]));
+      }
+      // the CTA's stores, ordered by the barrier, are released by one
+      // acquire-release arrival; the wait acquires the other ranks'
+      __shared__ int s_have;
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        int* ctr = args.counter + tile_id;
+        tc::atomic_add_acq_rel_gpu(ctr, 1);
+        bool got = true;
+        if (n_own > 0) {
+          got = tc::wait_count_low(ctr, ks, abort_flag, kWaitNs);
+          if (got) {
+            tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
+            tc::mbar_arrive_expect_tx(red, kChunkBytes * (uint32_t)(n_own * (ks - 1)));
+            for (int o = 0, d = 0; o < n_own; ++o) {
+              const int j = sk + o * ks;
+              for (int q = 0; q < ks; ++q) {
+                if (q == sk) continue;
+                tc::bulk_load(smem + (size_t)d * kChunkBytes,
+                              args.part + (tile_id * ks + q) * (int64_t)(128 * BN) +
+                                  (int64_t)j * (32 * 128),
+                              kChunkBytes, red);
+                ++d;
+              }
+            }
+          }
+        }
+        s_have = got;
+      }
+      __syncthreads();
+      have = s_have != 0;
+      if (have && n_own > 0) have = __syncthreads_and(wait_or_abort(red, 0, abort_flag)) != 0;
+      if (threadIdx.x == 0) {
+        if (have) {
+          const int prev = tc::atomic_add_acq_rel_gpu(args.counter + tile_id, 1 << 16);
+          if ((prev >> 16) == ks - 1) args.counter[tile_id] = 0;   // ready for the next launch
+        } else {
+          atomicExch(args.err, 1);   // gave up: report, skip the epilogue
+        }
+      }
+    }
+    // the accumulated values of this thread's row for chunk j = own_rank + o ks
+    auto vals = [&](int o, int j, uint32_t (&r)[32]) {
+      tmem_vals(32 * j, r);
+      if (!split_k) return;
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = 0.f;
+      for (int q = 0, d = 0; q < ks; ++q) {
+        if (q == sk) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
+        } else {
+          const float* pq = red_smem + (size_t)(o * (ks - 1) + d) * (32 * 128) + trow;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += pq[i * 128];
+          ++d;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(v[i]);
+    };
+    if (!have) {
+      // reported above
     } else if (kEpi == kEpiFwd || kEpi == kEpiDX) {
       TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
-      const TAct* mask = kEpi == kEpiDX
-                             ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
-                             : nullptr;
-      float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (kEpi == kEpiFwd && row4_ok) bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
 #pragma unroll 1
-      for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+      for (int o = half; o < n_own; o += 2) {
+        const int j0 = own_rank + o * kstride, c0 = 32 * j0;
+        if (o > half) load_mask(c0);
         uint32_t r[32];
-        vals(c0, r);
+        vals(o, j0, r);
 #pragma unroll
         for (int i = 0; i < 32; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
         __syncwarp();
         if (row4_ok) {
-          float4 hm[8];
-          if (kEpi == kEpiDX) {   // all mask loads in flight before any store
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              const int j = n_tile * BN + c0 + jl + 4 * u;
-              hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-          }
 #pragma unroll
           for (int u = 0; u < 8; ++u) {
             const int jc = jl + 4 * u;
@@ -433,12 +470,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
                 for (int e = 0; e < 4; ++e) v[e] = hv[e] > 0.f ? v[e] : 0.f;
               }
-              const int64_t o = (int64_t)j * args.ldo + row4;
-              store4(out + o, v);
+              const int64_t o4 = (int64_t)j * args.ldo + row4;
+              store4(out + o4, v);
               if (kSplit == 3 && args.out_pieces) {
                 uint2 q0, q1, q2;
                 split3_x4(v, q0, q1, q2);
-                bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o;
+                bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o4;
                 *reinterpret_cast<uint2*>(pp) = q0;
                 *reinterpret_cast<uint2*>(pp + args.out_plane) = q1;
                 *reinterpret_cast<uint2*>(pp + 2 * args.out_plane) = q2;
@@ -609,6 +646,12 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
     const int kt = (args.K + kBK - 1) / kBK;
     ks = std::min(ks, kt);
     if (ks > 1) ks = (kt + (kt + ks - 1) / ks - 1) / ((kt + ks - 1) / ks);
+  }
+  if (ks > 1) {   // the exchange needs every CTA of the launch resident at once
+    int dev = 0, sms = 0;
+    AGN_TRY_CUDA(cudaGetDevice(&dev));
+    AGN_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    if ((int64_t)ceil_div(args.M, 128) * ceil_div(args.N, BN) * slots * ks > sms) ks = 1;
   }
   if (ks > 1 && (!args.part || !args.counter))
     return Status::Err(AGN_E_INVALID, "split-K GEMM without workspace");

@@ -112,6 +112,26 @@ __device__ __forceinline__ int atomic_add_acq_rel_gpu(int* p, int v) {
   asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
 }
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Bounded wait until the low 16 bits of *p reach `target` (acquire): false
+// after limit_ns, or once another role of the CTA has set *abort_flag.
+__device__ __forceinline__ bool wait_count_low(const int* p, int target, volatile int* abort_flag,
+                                               uint64_t limit_ns) {
+  if ((ld_acquire_gpu(p) & 0xffff) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0;; ++it) {
+    __nanosleep(32);
+    if ((ld_acquire_gpu(p) & 0xffff) >= target) return true;
+    if ((it & 15) == 15) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > limit_ns) return false;
+    }
+  }
+}
 // Order generic-proxy global-memory accesses visible to this thread before
 // its later async-proxy (bulk copy) accesses.
 __device__ __forceinline__ void fence_proxy_async_global() {
