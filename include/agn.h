@@ -93,9 +93,10 @@ typedef struct agn_options {
   const int32_t* y_init;
   const float* theta_init;
   /* Diagnostic: which hidden-layer GEMMs use the tcgen05 kernels when they
-     are on (bit 0 forward, bit 1 dX, bit 2 dW; 0 = bits 0-2).  Bit 3 runs the
+     are on (bit 0 forward, bit 1 dX, bit 2 dW; none of bits 0-2 = all three).  Bit 3 runs the
      dW GEMMs on the earlier non-persistent tcgen05 kernel (one tile per CTA)
-     instead of the persistent one, for comparison. */
+     instead of the persistent one, for comparison.  Bit 4 runs the forward
+     and dX GEMMs without split K (one CTA per output tile). */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);

@@ -109,7 +109,7 @@ struct agn_handle {
   double* partials = nullptr;
   // tcgen05 path (bf16 mode): tensor maps per layer l = 1..L-1 (index l-1)
   bool use_tc = false;
-  int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW
+  int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW, 3 tiled dW, 4 no split K
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
     CUtensorMap theta, acc;      // fp32 W_l of every replica / accumulator, box {128, 32}
@@ -357,6 +357,7 @@ Status build_tc_maps(agn_handle* h) {
 // (small waves); then ks CTAs share each tile, with ks <= SMs / tiles and
 // every CTA's range of 64-deep k steps non-empty.
 int pick_ksplit(const agn_handle* h, int M, int K, int s) {
+  if (h->tc_mask & 16) return 1;
   const int64_t tiles = ceil_div(M, 128) * ceil_div(h->m, agn::tc_bn(h->m)) * (int64_t)s;
   if (tiles >= h->num_sms) return 1;
   const int kt = (int)ceil_div(K, 64);
@@ -868,7 +869,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 15) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 15]");
+  if (o.tc_mask < 0 || o.tc_mask > 31) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 31]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)
@@ -945,7 +946,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
                        "and d_0 .. d_{L-1} multiples of 8");
   h->use_tc = tc_ok && o.gemm != AGN_GEMM_SIMT;
   h->split = h->use_tc && h->prec == AGN_PREC_FP32;
-  h->tc_mask = o.tc_mask == 0 ? 7 : o.tc_mask;
+  h->tc_mask = (o.tc_mask & 7) == 0 ? (o.tc_mask | 7) : o.tc_mask;
   h->prev.assign(h->n, -1);
   h->pulled_v.assign(h->n, 0);
   h->steps.assign(h->n, 0);

@@ -300,19 +300,19 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const bool row_ok = row < args.M;
     const uint32_t lane_base = (uint32_t)(32 * g) << 16;
     float* theta = args.theta + (int64_t)worker * args.ld_param;
-    // Accumulated values of this thread's row for columns c0 .. c0 + 31: from
+    // Accumulated values of this thread's row for columns c0 .. c0 + 15: from
     // TMEM (the sum of the two accumulators in the split mode), or, with
     // split K, the partial sums of all ks CTAs of the tile in rank order.
     const int64_t tile_id = ((int64_t)slot * gridDim.y + n_tile) * gridDim.x + m_tile;
     const int trow = 32 * g + lane;
-    auto tmem_vals = [&](int c0, uint32_t (&r)[32]) {
-      tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)c0, r);
+    auto tmem_vals = [&](int c0, uint32_t (&r)[16]) {
+      tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)c0, r);
       if (kSplit == 3) {
-        uint32_t r2[32];
-        tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(BN + c0), r2);
+        uint32_t r2[16];
+        tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(BN + c0), r2);
         tc::tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
+        for (int i = 0; i < 16; ++i)
           r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
       }
       tc::tmem_ld_wait();
@@ -326,18 +326,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // SMs), copies the other ranks' partial sums of its chunks into its stage
     // ring and adds them in rank order, its own from TMEM.  Every rank then
     // counts itself out (high half); the last one out resets the counter for
-    // the next launch.
+    // the next launch.  Warps 0-3 take columns 0-15 of every chunk, warps
+    // 4-7 columns 16-31.
     constexpr int kNch = BN / 32;
     constexpr uint32_t kChunkBytes = 128u * 32u * 4u;
     const bool split_k = kEpi != kEpiDW && ks > 1;
     const int own_rank = split_k ? sk : 0, kstride = split_k ? ks : 1;
     const int n_own = (kNch - own_rank + kstride - 1) / kstride;   // chunks own_rank + o ks
+    const int co = 16 * half;                                       // this warp's columns of a chunk
     const float* red_smem = reinterpret_cast<const float*>(smem);   // the free stage ring
-    // Forward and dX epilogues: the warp's 32 rows x 32 columns go through a
+    // Forward and dX epilogues: the warp's 32 rows x 16 columns go through a
     // warp-private shared-memory tile (column-major) so that each lane then
-    // handles four consecutive rows (features, contiguous in memory) of
-    // eight columns: 16-byte bias / mask loads, 16-byte stores of the output
-    // and 8-byte stores of each bf16 piece.
+    // handles four consecutive rows (features, contiguous in memory) of four
+    // columns: 16-byte bias / mask loads, 16-byte stores of the output and
+    // 8-byte stores of each bf16 piece.
     float* tT = reinterpret_cast<float*>(smem + EpiT<BN, kSplit, kStages>::kOff) +
                 warp * (32 * 32);
     const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
@@ -346,13 +348,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const TAct* mask = kEpi == kEpiDX
                            ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
                            : nullptr;
-    // the mask of the warp's first chunk (and the bias) are loaded before
+    // the mask of the warp's first columns (and the bias) are loaded before
     // the split-K exchange: they do not depend on it
-    float4 hm[8];
+    float4 hm[4];
     auto load_mask = [&](int c0) {
       if (kEpi == kEpiDX && row4_ok) {   // all mask loads in flight before any store
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < 4; ++u) {
           const int j = n_tile * BN + c0 + jl + 4 * u;
           hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
                              : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -360,22 +362,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     };
     float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (kEpi == kEpiFwd && row4_ok && half < n_own)
+    if (kEpi == kEpiFwd && row4_ok && n_own > 0)
       bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
-    if (half < n_own) load_mask(32 * (own_rank + half * kstride));
+    if (n_own > 0) load_mask(32 * own_rank + co);
     bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
     if (split_k) {
       float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
-      int c = 0;   // the chunks this rank does not finish, alternately to the two halves
 #pragma unroll
       for (int j = 0; j < kNch; ++j) {
         if (j % ks == sk) continue;
-        if ((c++ & 1) != half) continue;
-        uint32_t r[32];
-        tmem_vals(32 * j, r);
+        uint32_t r[16];
+        tmem_vals(32 * j + co, r);
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          __stcg(mine + (int64_t)(32 * j + i) * 128 + trow, __uint_as_float(r[i]));
+        for (int i = 0; i < 16; ++i)
+          __stcg(mine + (int64_t)(32 * j + co + i) * 128 + trow, __uint_as_float(r[i]));
       }
       // the CTA's stores, ordered by the barrier, are released by one
       // acquire-release arrival; the wait acquires the other ranks'
@@ -417,43 +417,44 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
       }
     }
-    // the accumulated values of this thread's row for chunk j = own_rank + o ks
-    auto vals = [&](int o, int j, uint32_t (&r)[32]) {
-      tmem_vals(32 * j, r);
+    // the accumulated values of this thread's row for columns c0 .. c0 + 15
+    // of chunk j = own_rank + o ks (c0 = 32 j + co)
+    auto vals = [&](int o, int c0, uint32_t (&r)[16]) {
+      tmem_vals(c0, r);
       if (!split_k) return;
-      float v[32];
+      float v[16];
 #pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = 0.f;
+      for (int i = 0; i < 16; ++i) v[i] = 0.f;
       for (int q = 0, d = 0; q < ks; ++q) {
         if (q == sk) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
+          for (int i = 0; i < 16; ++i) v[i] += __uint_as_float(r[i]);
         } else {
-          const float* pq = red_smem + (size_t)(o * (ks - 1) + d) * (32 * 128) + trow;
+          const float* pq = red_smem + (size_t)(o * (ks - 1) + d) * (32 * 128) + co * 128 + trow;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] += pq[i * 128];
+          for (int i = 0; i < 16; ++i) v[i] += pq[i * 128];
           ++d;
         }
       }
 #pragma unroll
-      for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(v[i]);
+      for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(v[i]);
     };
     if (!have) {
       // reported above
     } else if (kEpi == kEpiFwd || kEpi == kEpiDX) {
       TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
 #pragma unroll 1
-      for (int o = half; o < n_own; o += 2) {
-        const int j0 = own_rank + o * kstride, c0 = 32 * j0;
-        if (o > half) load_mask(c0);
-        uint32_t r[32];
-        vals(o, j0, r);
+      for (int o = 0; o < n_own; ++o) {
+        const int c0 = 32 * (own_rank + o * kstride) + co;
+        if (o > 0) load_mask(c0);
+        uint32_t r[16];
+        vals(o, c0, r);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
+        for (int i = 0; i < 16; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
         __syncwarp();
         if (row4_ok) {
 #pragma unroll
-          for (int u = 0; u < 8; ++u) {
+          for (int u = 0; u < 4; ++u) {
             const int jc = jl + 4 * u;
             const int j = n_tile * BN + c0 + jc;
             if (j < args.N) {
@@ -637,12 +638,14 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   });
   AGN_TRY_CUDA(attr_err);
-  // split K: at most as many other ranks' partial sums as the stage ring
-  // holds, every rank with a non-empty range of k steps
+  // split K: every rank with a non-empty range of k steps
   int ks = kEpi == kEpiDW ? 1 : std::max(1, args.ksplit);
   if (ks > 1) {
+    // a rank that finishes chunks holds the other ranks' partial sums of
+    // them (16 KB per chunk and rank) in its stage ring
     const int ring = (int)EpiT<BN, kSplit, kStages>::kRingFree;
-    ks = std::min(ks, 1 + ring / (128 * BN * 4));
+    auto need = [](int k) { return ((BN / 32 + k - 1) / k) * (k - 1) * (128 * 32 * 4); };
+    while (ks > 1 && need(ks) > ring) --ks;
     const int kt = (args.K + kBK - 1) / kBK;
     ks = std::min(ks, kt);
     if (ks > 1) ks = (kt + (kt + ks - 1) / ks - 1) / ((kt + ks - 1) / ks);
