@@ -7,12 +7,15 @@
 // of fp32 master weight and accumulator traffic per parameter), so the kernel
 // is laid out around the parameter stream, not the MMA:
 //
-//   warp 0     TMA producer.  Per tile, the GEMM operands (H^T and dZ^T
-//              boxes, MN-major, 128-byte swizzle) into a ring of stages, then
-//              the tile's theta_k and a_k rows, 32 output features x 128
-//              inputs per chunk, into a second ring.  Each slot is refilled
-//              as soon as it frees, so DRAM reads of the next chunks (and of
-//              the next tile) are in flight while the current one is updated.
+//   warp 0     operand producer: per tile, the GEMM operands (H^T and dZ^T
+//              boxes, MN-major, 128-byte swizzle) into a ring of stages, as
+//              fast as the MMA frees them, so the next tile's GEMM runs while
+//              the current tile's epilogue drains.
+//   warp 10    parameter producer: each tile's theta_k and a_k rows, 32
+//              output features x 128 inputs per chunk, into a second ring.
+//              Each slot is refilled as soon as it frees, so DRAM reads of
+//              the next chunks (and of the next tile) are in flight while the
+//              current one is updated.
 //   warp 1     MMA issuer (one thread) and TMEM owner.  Two accumulators
 //              (double buffer): the GEMM of the next tile runs while the
 //              epilogue drains this one.
@@ -51,13 +54,14 @@ namespace agn {
 
 namespace {
 
-constexpr int kWarps = 10;
+constexpr int kWarps = 11;
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kCF = 32;                        // output features per parameter chunk
 constexpr int kChunkBytes = kCF * 128 * 4;     // one fp32 chunk: 32 rows x 128 inputs
 constexpr int kBiasHalf = kCF * 4;            // b_l (or its accumulator) for one chunk
 constexpr uint64_t kWaitNs = 2000000000ull;    // 2 s
+constexpr int kThrottleTiles = 8;              // tiles per CTA from which operands wait for chunks
 
 // kBK samples per stage: one TMA box is 64 MN-elements x kBK samples of bf16
 // (kBK rows of 128 bytes, 128-byte swizzle); A = two boxes (128 inputs),
@@ -179,6 +183,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   uint64_t* fin = tempty + 2;            // MMA drain on abort
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(fin + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  volatile int* chunk_tiles = abort_flag + 1;   // tiles whose chunks are all requested
 
   __shared__ int s_skip;
   if (threadIdx.x == 0) s_skip = *reinterpret_cast<volatile int*>(args.err);
@@ -204,6 +209,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
     }
     tc::mbar_init(fin, 1);
     *abort_flag = 0;
+    *chunk_tiles = 0;
     tc::fence_mbar_init();
     for (int i = 0; i < B.n_layers; ++i) {
       tc::tma_prefetch_desc(&B.a[i]);
@@ -224,10 +230,78 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   // kernel; global memory is touched only after it has completed, except the
   // producer's first parameter chunks (below)
 
-  if (!(warp == 0 && lane == 0)) pdl_begin();
-  if (warp == 0) {
-    if (lane == 0) {
-      uint32_t ml = 0, ch = 0;   // stage fills and chunk fills issued
+  if (!((warp == 0 || warp == kWarps - 1) && lane == 0)) pdl_begin();
+  if (warp == 0 || warp == kWarps - 1) {
+    if (warp == 0 && lane == 0) {
+      // operand producer (warp 0): the GEMM operands of every tile into the
+      // stage ring, as fast as the MMA frees stages
+      pdl_begin();
+      uint32_t ml = 0;   // stage fills issued
+      bool ok = true;
+      // On a long stream of tiles (bound by DRAM) the operands of a tile are
+      // requested only once the previous tile's parameter chunks are, so
+      // those stay first in line; on a short one they run ahead.
+      const bool throttle = !kGrad && T >= kThrottleTiles * (int)gridDim.x;
+      int itp = 0;
+      for (int t = blockIdx.x; ok && t < T; t += gridDim.x, ++itp) {
+        const TileIdx ti = decode(B, t);
+        const CUtensorMap* tmA = &B.a[ti.layer];
+        const CUtensorMap* tmB = &B.b[ti.layer];
+        if (throttle && itp > 0 && *chunk_tiles < itp) {
+          const uint64_t t0 = tc::globaltimer_ns();
+          while (*chunk_tiles < itp) {
+            if (*abort_flag || tc::globaltimer_ns() - t0 > kWaitNs) {
+              ok = false;
+              break;
+            }
+            __nanosleep(64);
+          }
+          if (!ok) break;
+        }
+        for (int kt = 0; kt < KT; ++kt) {
+          const int s = ml % kStages;
+          if (ml >= kStages &&
+              !tc::wait_or_abort(&empty[s], ((ml / kStages) - 1) & 1, abort_flag, kWaitNs)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa0 = smem + s * Cfg::kStageBytes;
+          uint8_t* sb0 = sa0 + kSplit * kABytes;
+          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes);
+  #pragma unroll
+          for (int p = 0; p < kSplit; ++p) {
+            uint8_t* sa = sa0 + p * kABytes;
+            uint8_t* sb = sb0 + p * Cfg::kBBytes;
+            if (kSplit == 1) {
+              tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
+              tc::tma_load_3d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
+  #pragma unroll
+              for (int c = 0; c < BN / 64; ++c)
+                tc::tma_load_3d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                                ti.slot);
+            } else {
+              tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
+              tc::tma_load_4d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
+                              p);
+  #pragma unroll
+              for (int c = 0; c < BN / 64; ++c)
+                tc::tma_load_4d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
+                                ti.slot, p);
+            }
+          }
+          ++ml;
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        // drain (bounded) the copies armed but maybe not yet landed
+        for (uint32_t j = ml > (uint32_t)kStages ? ml - kStages : 0; j < ml; ++j)
+          tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
+      }
+    } else if (lane == 0) {
+      // parameter producer (the last warp): each tile's theta_k and a_k rows
+      // into the chunk ring, as fast as the epilogue frees slots
+      uint32_t ch = 0;   // chunk fills issued
       bool ok = true;
       // theta_k / a_k chunk c of tile ti into ring slot r
       auto issue_chunk = [&](const TileIdx& ti, int worker, int c, int r) {
@@ -245,8 +319,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
           tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
           if (kAcc)
-            tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
-                          &cfull[r]);
+            tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf, &cfull[r]);
         }
       };
       // theta_k and a_k were last written by this kernel's previous launch or
@@ -264,47 +337,10 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         }
       }
       pdl_begin();
-      for (int t = blockIdx.x; ok && t < T; t += gridDim.x) {
+      for (int t = blockIdx.x; !kGrad && ok && t < T; t += gridDim.x) {
         const TileIdx ti = decode(B, t);
         const DwLayer& L = B.layer[ti.layer];
-        const CUtensorMap* tmA = &B.a[ti.layer];
-        const CUtensorMap* tmB = &B.b[ti.layer];
         const int worker = args.slot_worker[ti.slot];
-        for (int kt = 0; kt < KT; ++kt) {
-          const int s = ml % kStages;
-          if (ml >= kStages &&
-              !tc::wait_or_abort(&empty[s], ((ml / kStages) - 1) & 1, abort_flag, kWaitNs)) {
-            ok = false;
-            break;
-          }
-          uint8_t* sa0 = smem + s * Cfg::kStageBytes;
-          uint8_t* sb0 = sa0 + kSplit * kABytes;
-          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes);
-#pragma unroll
-          for (int p = 0; p < kSplit; ++p) {
-            uint8_t* sa = sa0 + p * kABytes;
-            uint8_t* sb = sb0 + p * Cfg::kBBytes;
-            if (kSplit == 1) {
-              tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
-              tc::tma_load_3d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
-#pragma unroll
-              for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_3d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
-                                ti.slot);
-            } else {
-              tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
-              tc::tma_load_4d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
-                              p);
-#pragma unroll
-              for (int c = 0; c < BN / 64; ++c)
-                tc::tma_load_4d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
-                                ti.slot, p);
-            }
-          }
-          ++ml;
-        }
-        if (!ok) break;
-        if (kGrad) continue;   // the gradient needs no parameter chunks
         const int nch = min(Cfg::kChunks, (L.N - ti.n_tile * BN + kCF - 1) / kCF);
         for (int c = t == (int)blockIdx.x ? npre : 0; c < nch; ++c) {
           const int r = ch % kRing;
@@ -316,12 +352,10 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           issue_chunk(ti, worker, c, r);
           ++ch;
         }
+        *chunk_tiles = *chunk_tiles + 1;
       }
       if (!ok) {
         *abort_flag = 1;
-        // drain (bounded) the copies armed but maybe not yet landed
-        for (uint32_t j = ml > (uint32_t)kStages ? ml - kStages : 0; j < ml; ++j)
-          tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
         for (uint32_t j = ch > (uint32_t)kRing ? ch - kRing : 0; j < ch; ++j)
           tc::mbar_wait_bounded(&cfull[j % kRing], (j / kRing) & 1, kWaitNs);
       }
