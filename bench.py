@@ -18,6 +18,7 @@ import argparse
 import hashlib
 import json
 import os
+import select
 import statistics
 import subprocess
 import sys
@@ -89,10 +90,17 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+            return self
+        # the sampler's start-up must not eat the timed region: wait (3 s at
+        # most) for its first sample, which is taken before the region and
+        # not counted
+        ready, _, _ = select.select([self.proc.stdout], [], [], 3.0)
+        if ready:
+            self.proc.stdout.readline()
         return self
 
     def __exit__(self, *a):
@@ -421,7 +429,7 @@ def run_agn(args, wl):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=6)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="agn", choices=["agn", "reference"])
     ap.add_argument("--workload", default="mnist", choices=sorted(WORKLOADS))
