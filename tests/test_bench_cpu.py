@@ -1,0 +1,85 @@
+"""Host-side logic of bench.py (no GPU): the clock-record summary that decides
+whether a measurement stands, and the lookup of ncu DRAM traffic keyed by the
+kernel source's digest."""
+
+import hashlib
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def _line(sm, mx, active="0x0", hw="Not Active", hwt="Not Active", swt="Not Active",
+          pcap="Not Active"):
+    return f"0, {sm}, {mx}, 900.5, {active}, {hw}, {hwt}, {swt}, {pcap}"
+
+
+def test_clock_summary_median_and_reasons():
+    c = bench.ClockSampler(0)
+    c.lines = [_line(2070, 2070), _line(1980, 2070, pcap="Active"), _line(2070, 2070),
+               "garbage", _line(2010, 2070)]
+    s = c.summary()
+    assert s["samples"] == 4
+    assert s["sm_mhz"] == pytest.approx(2040.0)          # median of 2070, 1980, 2070, 2010
+    assert s["sm_max_mhz"] == 2070.0
+    assert s["reasons"] == ["sw_power_cap"]
+
+
+def test_clock_summary_reports_thermal_slowdown():
+    c = bench.ClockSampler(0)
+    c.lines = [_line(1500, 2070, hwt="Active"), _line(1400, 2070, swt="Active", hw="Active")]
+    s = c.summary()
+    assert s["reasons"] == ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"]
+
+
+def test_clock_summary_without_samples():
+    c = bench.ClockSampler(0)
+    c.lines = []
+    assert c.summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+
+
+def _fake_root(tmp_path, src_text, digest_text):
+    csrc = tmp_path / "paper_1710_02368_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (csrc / "mlp_tc_dw.cu").write_text(src_text)
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    (prof / "dram_traffic.txt").write_text(
+        "# kernel_class workload bytes digest\n"
+        f"backward_dw wl-a 1234 {digest_text}\n"
+        f"backward_dw wl-b 99 000000000000\n")
+    return str(tmp_path)
+
+
+def test_traffic_lookup_matches_digest(tmp_path, monkeypatch):
+    src = "// kernel source\n"
+    digest = hashlib.sha256(src.encode()).hexdigest()[:12]
+    monkeypatch.setattr(bench, "ROOT", _fake_root(tmp_path, src, digest))
+    assert bench._traffic_for("backward_dw", "wl-a", True) == 1234.0
+    assert bench._traffic_for("backward_dw", "wl-b", True) is None   # stale digest
+    assert bench._traffic_for("backward_dw", "wl-c", True) is None   # no capture
+    assert bench._traffic_for("gather", "wl-a", True) is None        # no source mapped
+
+
+def test_traffic_lookup_ignores_a_changed_kernel(tmp_path, monkeypatch):
+    src = "// kernel source\n"
+    digest = hashlib.sha256(src.encode()).hexdigest()[:12]
+    root = _fake_root(tmp_path, src, digest)
+    (tmp_path / "paper_1710_02368_gb300" / "csrc" / "mlp_tc_dw.cu").write_text(src + "// edit\n")
+    monkeypatch.setattr(bench, "ROOT", root)
+    assert bench._traffic_for("backward_dw", "wl-a", True) is None
+
+
+def test_committed_traffic_entries_are_well_formed():
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    rows = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    assert rows
+    for r in rows:
+        assert len(r) == 4
+        assert r[0] in ("forward", "backward_dx", "backward_dw", "softmax", "commit")
+        assert float(r[2]) > 0
+        assert len(r[3]) == 12 and all(ch in "0123456789abcdef" for ch in r[3])
