@@ -256,6 +256,36 @@ int agn_make_schedule(int32_t n, int32_t n_commits, int32_t tau_lo, int32_t tau_
                       uint64_t seed, int32_t* worker_out, int32_t* tau_out);
 
 /*
+ * The plan agn_run follows for the first n_commits commits of a fresh handle
+ * with n_workers workers and lambda local steps (pure host helper, no
+ * device).  Commit c reads theta~ after v_c = c - staleness[c] commits
+ * (Figure 1's FIFO server; Algorithm 1's Pull before its local steps), so
+ * the local steps of every commit whose version is already applied can run
+ * together: a wave takes, per worker, its next commit if v_c <= V (V = commits
+ * applied so far); then the longest run of computed commits from V on is
+ * applied in order, and the replicas pull the versions their next commits
+ * read as those versions appear.  worker / staleness as for agn_run
+ * (n_schedule >= n_commits entries; entries past n_commits are look-ahead).
+ * Outputs (host, caller-owned):
+ *   n_waves_out            : number of waves;
+ *   wave_slots[w], wave_end[w] (capacity n_commits each): the commits whose
+ *                            local steps wave w runs, and the number of
+ *                            commits applied once it is done;
+ *   slot_commit[s], slot_t0[s] (capacity n_commits): the commits in wave
+ *                            order, and the worker's step counter t (Algorithm
+ *                            1; never reset) when that commit's steps start;
+ *   pull_version[p], pull_worker[p] (capacity pull_cap; *n_pulls_out entries):
+ *                            the pulls, in order: the worker pulls theta~ right
+ *                            after pull_version commits are applied.
+ * Errors: AGN_E_INVALID (bad sizes or a short buffer), AGN_E_SCHEDULE.
+ */
+int agn_plan_waves(int32_t n_workers, int32_t lambda, int32_t n_commits, const int32_t* worker,
+                   const int32_t* staleness, int32_t n_schedule, int32_t* n_waves_out,
+                   int32_t* wave_slots, int32_t* wave_end, int32_t* slot_commit,
+                   int64_t* slot_t0, int64_t pull_cap, int32_t* pull_version,
+                   int32_t* pull_worker, int64_t* n_pulls_out);
+
+/*
  * Standalone commit + pull (the parameter-server step, Eq. 1-2 and the
  * Commit/Pull of Algorithm 1) on caller device buffers.  For c = 0 .. C-1 in
  * order: k = commit_worker[c];

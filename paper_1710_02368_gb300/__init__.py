@@ -24,7 +24,8 @@ __all__ = [
     "AGNError", "AGN", "agn_default_options", "agn_create", "agn_run", "agn_central",
     "agn_replica", "agn_loss", "agn_delta_norm", "agn_num_params", "agn_num_commits",
     "agn_last_run_stats", "agn_profile", "agn_kernel_stats", "agn_generate_inputs", "agn_export_inputs", "agn_last_error",
-    "agn_destroy", "agn_make_schedule", "agn_commit_pull", "agn_commit_pull_noalloc",
+    "agn_destroy", "agn_make_schedule", "agn_plan_waves", "agn_commit_pull",
+    "agn_commit_pull_noalloc",
     "agn_fill_commit_inputs",
     "library_path",
 ]
@@ -216,6 +217,33 @@ def agn_make_schedule(n, n_commits, tau_lo, tau_hi, seed):
     _check(_L().agn_make_schedule(int(n), int(n_commits), int(tau_lo), int(tau_hi), int(seed),
                                   w.ctypes.data_as(_lib._I32P), t.ctypes.data_as(_lib._I32P)))
     return w, t
+
+
+def agn_plan_waves(n, lam, n_commits, worker, staleness):
+    """The wave plan agn_run follows on a fresh handle (host only): returns
+    (wave_slots, wave_end, slot_commit, slot_t0, pulls) with pulls an [n_pulls, 2]
+    array of (version, worker) in order."""
+    w, wp = _i32(worker)
+    t, tp = _i32(staleness)
+    k = int(n_commits)
+    cap = max(1, k)
+    ws = np.empty(cap, dtype=np.int32)
+    we = np.empty(cap, dtype=np.int32)
+    sc = np.empty(cap, dtype=np.int32)
+    st = np.empty(cap, dtype=np.int64)
+    pcap = len(w) + int(n) + 1
+    pv = np.empty(pcap, dtype=np.int32)
+    pw = np.empty(pcap, dtype=np.int32)
+    nw = C.c_int32(0)
+    npl = C.c_int64(0)
+    _check(_L().agn_plan_waves(int(n), int(lam), k, wp, tp, len(w), C.byref(nw),
+                               ws.ctypes.data_as(_lib._I32P), we.ctypes.data_as(_lib._I32P),
+                               sc.ctypes.data_as(_lib._I32P), st.ctypes.data_as(_lib._I64P),
+                               pcap, pv.ctypes.data_as(_lib._I32P),
+                               pw.ctypes.data_as(_lib._I32P), C.byref(npl)))
+    nwv, npv = nw.value, npl.value
+    return (ws[:nwv].copy(), we[:nwv].copy(), sc[:k].copy(), st[:k].copy(),
+            np.stack([pv[:npv], pw[:npv]], axis=1))
 
 
 def agn_commit_pull(theta_c, acc, replicas, replicas_bf16, P, ld, n, commit_worker,

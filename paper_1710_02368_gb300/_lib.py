@@ -71,6 +71,7 @@ class agn_options(C.Structure):
 
 
 _I32P = C.POINTER(C.c_int32)
+_I64P = C.POINTER(C.c_int64)
 _F32P = C.POINTER(C.c_float)
 _F64P = C.POINTER(C.c_double)
 
@@ -99,6 +100,9 @@ SIGNATURES = {
     "agn_destroy": (None, [C.c_void_p]),
     "agn_make_schedule": (C.c_int, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_uint64,
                                     _I32P, _I32P]),
+    "agn_plan_waves": (C.c_int, [C.c_int32, C.c_int32, C.c_int32, _I32P, _I32P, C.c_int32,
+                                 _I32P, _I32P, _I32P, _I32P, _I64P, C.c_int64, _I32P, _I32P,
+                                 _I64P]),
     "agn_commit_pull": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64,
                                   C.c_int64, C.c_int32, C.c_int32, _I32P, _I32P, _I32P,
                                   C.c_double, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]),

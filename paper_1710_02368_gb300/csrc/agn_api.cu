@@ -1453,6 +1453,60 @@ int agn_make_schedule(int32_t n, int32_t n_commits, int32_t tau_lo, int32_t tau_
   return AGN_OK;
 }
 
+int agn_plan_waves(int32_t n_workers, int32_t lambda, int32_t n_commits, const int32_t* worker,
+                   const int32_t* staleness, int32_t n_schedule, int32_t* n_waves_out,
+                   int32_t* wave_slots, int32_t* wave_end, int32_t* slot_commit,
+                   int64_t* slot_t0, int64_t pull_cap, int32_t* pull_version,
+                   int32_t* pull_worker, int64_t* n_pulls_out) {
+  if (n_workers < 1 || lambda < 1 || n_commits < 0 || n_schedule < n_commits || pull_cap < 0 ||
+      !n_waves_out || !n_pulls_out ||
+      (n_schedule > 0 && (!worker || !staleness)) ||
+      (n_commits > 0 && (!wave_slots || !wave_end || !slot_commit || !slot_t0)) ||
+      (pull_cap > 0 && (!pull_version || !pull_worker)))
+    return fail(nullptr, AGN_E_INVALID, "bad plan arguments");
+  // the planning state of a fresh handle: no commits, every replica at version 0
+  agn_handle h;
+  h.n = n_workers;
+  h.lam = lambda;
+  h.V = 0;
+  h.prev.assign(n_workers, -1);
+  h.pulled_v.assign(n_workers, 0);
+  h.steps.assign(n_workers, 0);
+  RunPlan plan;
+  Status s = build_plan(&h, n_commits, worker, staleness, n_schedule, &plan);
+  if (!s.ok()) return fail(nullptr, s);
+  int64_t np = 0;
+  auto add_pull = [&](int v, int w) {
+    if (np < pull_cap) {
+      pull_version[np] = v;
+      pull_worker[np] = w;
+    }
+    ++np;
+  };
+  for (int w : plan.start_pulls) add_pull(0, w);
+  int applied = 0;
+  for (size_t i = 0; i < plan.waves.size(); ++i) {
+    const Wave& wv = plan.waves[i];
+    wave_slots[i] = wv.slots;
+    for (const CommitPlan& cp : wv.commits) {
+      for (int c = 0; c < cp.n_commits; ++c) {
+        for (int p = cp.pull_begin[c]; p < cp.pull_begin[c + 1]; ++p)
+          add_pull(cp.norm_slot[c] + 1, cp.pull_worker[p]);
+        ++applied;
+      }
+    }
+    wave_end[i] = applied;
+  }
+  for (size_t s2 = 0; s2 < plan.slot_commit.size(); ++s2) {
+    slot_commit[s2] = plan.slot_commit[s2];
+    slot_t0[s2] = plan.slot_t0[s2];
+  }
+  *n_waves_out = (int32_t)plan.waves.size();
+  *n_pulls_out = np;
+  if (np > pull_cap) return fail(nullptr, AGN_E_INVALID, "pull buffer too short");
+  return AGN_OK;
+}
+
 int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_bf16, int64_t P,
                     int64_t ld, int32_t n, int32_t C, const int32_t* commit_worker,
                     const int32_t* pull_offsets, const int32_t* pull_workers, double eta,
