@@ -216,7 +216,9 @@ def run_reference(args, wl):
         "dtype": "f64" if dtype == np.float64 else "f32", "data": "synthetic",
         "config": {"workload": wl.name, "commits_per_step": per_step,
                    "commit_rule": args.commit_rule,
-                   "sample": f"each step re-runs the first {per_step} commits on the CPU"},
+                   "sample": f"{per_step}-commit {'fp64' if dtype == np.float64 else 'fp32'} "
+                             f"sample: each step re-runs the first {per_step} commits of the "
+                             "workload on the CPU"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
                          "kind": "oracle",
                          "sample": f"{per_step} commits ({per_step * wl.lam} worker-steps) "
@@ -227,7 +229,28 @@ def run_reference(args, wl):
     return 0
 
 
-def commit_kernel_bench(agn, torch, dev, P=1 << 28, reps=3):
+def commit_plan_launches(order, pulls, max_commits=16, max_pulls=256):
+    """Commit launches the library makes for one pass: runs of at most 16
+    consecutive commits, cut early at a repeated worker or when the pulls of
+    the run would exceed 256 (the grouping of agn_commit_pull)."""
+    launches, cur, npulls = 0, set(), 0
+    for k, p in zip(order, pulls):
+        if cur and (len(cur) == max_commits or int(k) in cur or npulls + len(p) > max_pulls):
+            launches += 1
+            cur, npulls = set(), 0
+        cur.add(int(k))
+        npulls += len(p)
+    return launches + (1 if cur else 0)
+
+
+def commit_pass_bytes(P, n_commits, n_pulls, launches):
+    """Bytes one pass of the standalone commit workload must move: theta~ read
+    and written once per launch (8P), each commit's accumulator read and
+    zeroed (8P), each pull's replica written (4P)."""
+    return float(P) * (8.0 * launches + 8.0 * n_commits + 4.0 * n_pulls)
+
+
+def commit_kernel_bench(agn, torch, dev, P, min_ms=200.0):
     """The standalone commit+pull kernel: 64 accumulators, the seeded order,
     4 pulls after each commit (one pass = 64 commits)."""
     wl = WL.COMMIT_PULL
@@ -244,35 +267,133 @@ def commit_kernel_bench(agn, torch, dev, P=1 << 28, reps=3):
     def one():
         agn.agn_commit_pull(theta, acc, reps_t, None, P, P, n, order, offs, flat, wl.eta, wl.lam,
                             stream=st.cuda_stream)
-    one()
+    for _ in range(3):
+        one()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    one()
+    e1.record(st)
+    torch.cuda.synchronize()
+    reps = max(3, int(min_ms / max(e0.elapsed_time(e1), 1e-3)))
     e0.record(st)
     for _ in range(reps):
         one()
     e1.record(st)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / reps
-    bytes_ = P * 4.0 * (2 + 2 * n + n * wl.pulls_per_commit)
+    launches = commit_plan_launches(order, pulls)
+    bytes_ = commit_pass_bytes(P, n, len(flat), launches)
     del theta, acc, reps_t
     torch.cuda.empty_cache()
-    return {"P": P, "commits": n, "pulls_per_commit": wl.pulls_per_commit,
-            "ms_per_pass": ms, "GB/s": bytes_ / ms / 1e6, "launches_per_pass": 2 * ((n + 15) // 16)}
+    return {"P": P, "commits": n, "pulls_per_commit": wl.pulls_per_commit, "passes_timed": reps,
+            "ms_per_pass": ms, "GB/s": bytes_ / ms / 1e6, "bytes_per_pass": bytes_,
+            "launches_per_pass": launches,
+            "inputs": f"{(2 * n + 1) * P * 4 / 1e9:.2f} GB of accumulators, replicas and theta~ "
+                      "(larger than L2)"}
 
 
-def run_agn(args, wl):
-    import torch
-    import paper_1710_02368_gb300 as agn
-    ws, rank, local = _dist()
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
+def method_bytes_per_worker_step(wl, cls):
+    """Bytes the method itself moves per worker-step (one local step of one
+    worker) in a kernel class: each local step reads and writes the fp32
+    replica theta_k and accumulator a_k of every parameter (Algorithm 1: 16 B
+    per parameter; 18 with the bf16 working copy the bf16 mode refreshes),
+    plus the GEMM operands at the mode's element size (fp32 4 B, bf16 2 B).
+    The fp32 mode's tensor-core pieces (6 B per operand element) are this
+    implementation's cost and are left out.  None for classes without a
+    per-step formula."""
+    es = 4.0 if wl.precision == WL.PREC_FP32 else 2.0
+    d, m = wl.dims, wl.batch
+    L = len(d) - 1
+    P = I.num_params(d)
+    if cls == "backward_dw":
+        return P * (16.0 if wl.precision == WL.PREC_FP32 else 18.0) + sum(
+            m * (d[l] + d[l - 1]) * es for l in range(1, L + 1))
+    if cls == "forward":        # the hidden layers (the output layer runs in the head)
+        return sum(d[l] * d[l - 1] * es + 4.0 * d[l] + m * (d[l - 1] + d[l]) * es
+                   for l in range(1, L))
+    if cls == "backward_dx":    # layers L-1 .. 2 (the head writes layer L's dX)
+        return sum(d[l] * d[l - 1] * es + m * d[l] * es + 2.0 * m * d[l - 1] * es
+                   for l in range(2, L))
+    if cls == "softmax":        # output layer: forward, softmax-CE, dX
+        return (d[L] * d[L - 1] * es + 4.0 * d[L] + 2.0 * m * d[L - 1] * es + m * d[L] * es
+                + 4.0 * m)
+    if cls == "gather":
+        return m * (2.0 * d[0] * es + 8.0)
+    return None
+
+
+GEMM_CLASSES = ("forward", "backward_dx", "backward_dw", "softmax")
+
+
+def roofline(wl, kst, worker_steps, on_tc, hbm, bf16, peak_src):
+    """Roofline of the dominant kernel class (by device time) from the CUDA
+    events of the profiled region: achieved = method bytes (or flops) per
+    launch / average launch time."""
+    dom = max(("forward", "backward_dx", "backward_dw", "commit", "softmax", "gather"),
+              key=lambda k: kst[k]["ms"])
+    d = kst[dom]
+    launches = max(d["launches"], 1)
+    sec = d["ms"] / 1e3 / launches
+    impl_bytes = d["bytes"] / launches
+    mb = method_bytes_per_worker_step(wl, dom)
+    method_bytes = mb * worker_steps / launches if mb is not None else impl_bytes
+    flops = d["flops"] / launches
+    # fp32 mode on the tensor cores issues six bf16 piece products per fp32 product
+    mma_per_flop = 6.0 if (wl.precision == WL.PREC_FP32 and on_tc) else 1.0
+    if wl.precision == WL.PREC_FP32 and not on_tc and dom in GEMM_CLASSES:
+        roof = {"bound": "alu", "achieved": flops / sec / 1e12, "peak": FP32_FMA_PEAK_TFLOPS,
+                "unit": "TFLOP/s",
+                "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
+    elif flops * mma_per_flop / max(method_bytes, 1.0) >= bf16 * 1e12 / (hbm * 1e9):
+        roof = {"bound": "tensor", "achieved": flops * mma_per_flop / sec / 1e12, "peak": bf16,
+                "unit": "TFLOP/s", "peak_source": f"{peak_src} bf16 burst"}
+    else:
+        roof = {"bound": "hbm", "achieved": method_bytes / sec / 1e9, "peak": hbm,
+                "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = dom
+    roof["avg_launch_us"] = 1e6 * sec
+    roof["bytes_basis"] = ("method: fp32 theta_k and a_k read-modify-write per parameter and "
+                           "local step (16 B; 18 B with the bf16 copy) plus the GEMM operands at "
+                           "the mode's element size" if dom == "backward_dw" else
+                           "method: the class's weights and activations at the mode's element "
+                           "size" if mb is not None else "implementation bytes")
+    roof["method_bytes_per_launch"] = method_bytes
+    roof["impl_bytes_per_launch"] = impl_bytes
+    roof["impl_frac"] = impl_bytes / sec / 1e9 / hbm
+    roof["flops_per_launch"] = flops
+    if dom in GEMM_CLASSES and on_tc:
+        roof["tensor_pipe_frac_of_bf16_peak"] = mma_per_flop * flops / sec / 1e12 / bf16
+    roof["traffic"] = _traffic_for(dom, wl.name, on_tc)
+    return roof
+
+
+def tensor_summary(wl, kst, ms_step, worker_steps_step, on_tc, bf16):
+    """Tensor-pipe use of the GEMM classes: their method flops over their own
+    device time, and over the whole step, against the bf16 burst peak (issued
+    = six bf16 piece products per fp32 product in the fp32 mode)."""
+    mma = 6.0 if (wl.precision == WL.PREC_FP32 and on_tc) else 1.0
+    fl = sum(kst[k]["flops"] for k in GEMM_CLASSES)
+    t = sum(kst[k]["ms"] for k in GEMM_CLASSES) / 1e3
+    d, m = wl.dims, wl.batch
+    W_f = sum(d[l] * d[l - 1] for l in range(1, len(d)))
+    W_x = sum(d[l] * d[l - 1] for l in range(2, len(d)))
+    step_flops = worker_steps_step * m * (4.0 * W_f + 2.0 * W_x)
+    return {"gemm_method_tflops": fl / max(t, 1e-12) / 1e12,
+            "gemm_issued_frac_of_bf16_peak": mma * fl / max(t, 1e-12) / 1e12 / bf16,
+            "step_method_tflops": step_flops / (ms_step / 1e3) / 1e12,
+            "step_issued_frac_of_bf16_peak": mma * step_flops / (ms_step / 1e3) / 1e12 / bf16}
+
+
+def measure_workload(args, wl, agn, torch, dev, per_step, ws, clock_index=None):
+    """Three timed regions over consecutive steps of one run of the workload:
+    (1) device-resident inputs, no per-kernel events (the value); (2) CUDA
+    events around every launch (per-kernel durations for the roofline and the
+    shares); (3) end to end through the public API with the step's schedule
+    from host memory and its losses read back."""
     st = torch.cuda.current_stream()
     seed = I.DEFAULT_SEED
-    per_step = args.commits_per_step or (
-        COMMITS_PER_STEP[args.workload] if not args.workers else 2 * wl.n)
     total = (args.warmup + 3 * args.steps) * per_step + wl.n
     w, tau = agn.agn_make_schedule(wl.n, total, wl.tau_lo, wl.tau_hi, seed)
     h = agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, seed, precision=wl.precision, batch=wl.batch,
@@ -290,29 +411,25 @@ def run_agn(args, wl):
     def step(i, e2e=False):
         a = i * per_step
         h.run(per_step, w[a:], tau[a:])
-        if e2e:
-            return h.loss()
-        return None
+        return h.loss() if e2e else None
 
     for i in range(args.warmup):
         step(i)
-    # timed region 1: device-resident inputs, no per-kernel events (the
-    # headline value)
     launches = 0
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
-        e0.record(st)
-        for i in range(args.warmup, args.warmup + args.steps):
-            step(i)
-            launches += int(h.last_run_stats()["launches"])
-        e1.record(st)
-        barrier()
+    clk = ClockSampler(clock_index) if clock_index is not None else None
+    if clk is not None:
+        clk.__enter__()
+    e0.record(st)
+    for i in range(args.warmup, args.warmup + args.steps):
+        step(i)
+        launches += int(h.last_run_stats()["launches"])
+    e1.record(st)
+    barrier()
+    if clk is not None:
+        clk.__exit__(None, None, None)
     ms = e0.elapsed_time(e1)
-    # timed region 2: the next steps of the same run with CUDA events around
-    # every kernel launch on the launching stream (per-kernel durations for
-    # the roofline and the shares; the events themselves cost some time, so
-    # this region is not the headline)
     h.profile(2)
     h.profile(1)
     barrier()
@@ -325,97 +442,108 @@ def run_agn(args, wl):
     h.profile(0)
     prof_ms = p0.elapsed_time(p1)
     kst = h.kernel_stats()
-    tc_ok = wl.batch <= 256 and all(d % 8 == 0 for d in wl.dims[:-1])
-    if args.gemm != "simt" and tc_ok:
-        gemm_used = ("tcgen05 bf16" if wl.precision == WL.PREC_BF16 else
-                     "tcgen05 fp32 as three exact bf16 pieces") + \
-                    " (hidden layers); fused output layer on CUDA cores"
-    else:
-        gemm_used = "CUDA-core GEMMs; fused output layer"
-    # timed region 2: end to end through the public API with host buffers
     barrier()
     t0 = time.perf_counter()
-    e2 = torch.cuda.Event(enable_timing=True)
-    e3 = torch.cuda.Event(enable_timing=True)
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2.record(st)
     d2h = 0
     for i in range(args.warmup + 2 * args.steps, args.warmup + 3 * args.steps):
-        losses = step(i, e2e=True)
-        d2h += losses.nbytes
+        d2h += step(i, e2e=True).nbytes
     e3.record(st)
     barrier()
     e2e_ms = max(e2.elapsed_time(e3), 1e3 * (time.perf_counter() - t0))
-    h2d = 2 * 4 * (per_step + wl.n)           # the schedule window of each step
-    if ws > 1:
-        ms, e2e_ms = max_over_ranks([ms, e2e_ms], dev)
-    value = whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch, ms)
-    e2e_value = whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch, e2e_ms)
-
-    hbm, bf16, bf16_sus, peak_src = _peaks()
-    dom = max(("forward", "backward_dx", "backward_dw", "commit", "softmax", "gather"),
-              key=lambda k: kst[k]["ms"])
-    d = kst[dom]
-    on_tc = args.gemm != "simt" and tc_ok
-    if dom in ("forward", "backward_dx", "backward_dw"):
-        if wl.precision == WL.PREC_FP32 and not on_tc:
-            roof = {"bound": "alu", "achieved": d["flops"] / d["ms"] / 1e9,
-                    "peak": FP32_FMA_PEAK_TFLOPS, "unit": "TFLOP/s",
-                    "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
-        else:
-            # bf16 GEMMs: the bound is set by the arithmetic intensity against
-            # the ridge point of the measured peaks (bf16 TFLOP/s / HBM GB/s)
-            ai = d["flops"] / max(d["bytes"], 1.0)
-            if ai >= bf16 * 1e12 / (hbm * 1e9):
-                roof = {"bound": "tensor", "achieved": d["flops"] / d["ms"] / 1e9, "peak": bf16,
-                        "unit": "TFLOP/s", "peak_source": f"{peak_src} bf16 burst"}
-            else:
-                roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
-                        "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
-            # fp32 mode on tensor cores issues six bf16 piece products per fp32 product
-            mma_per_flop = 6.0 if wl.precision == WL.PREC_FP32 else 1.0
-            roof["tensor_pipe_frac_of_bf16_peak"] = mma_per_flop * d["flops"] / d["ms"] / 1e9 / bf16
-            roof["arithmetic_intensity_flop_per_byte"] = ai
-    else:
-        roof = {"bound": "hbm", "achieved": d["bytes"] / d["ms"] / 1e6, "peak": hbm,
-                "unit": "GB/s", "peak_source": f"{peak_src} copy bandwidth"}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    tr = _traffic_for(dom, wl.name, on_tc)
-    roof["traffic"] = tr
-    roof["kernel"] = dom
-    roof["avg_launch_us"] = 1e3 * d["ms"] / max(d["launches"], 1)
-    roof["events_region_ms_per_step"] = prof_ms / args.steps
-    roof["algorithmic_per_launch"] = {"flops": d["flops"] / max(d["launches"], 1),
-                                      "bytes": d["bytes"] / max(d["launches"], 1)}
-    kernels = {k: {"launches": int(v["launches"]), "ms": round(v["ms"], 3),
-                   "share": round(v["ms"] / max(sum(x["ms"] for x in kst.values()), 1e-9), 4)}
-               for k, v in kst.items() if v["launches"]}
     h.close()
+    return {"ms": ms, "prof_ms": prof_ms, "e2e_ms": e2e_ms, "kst": kst, "launches": launches,
+            "clk": clk, "d2h": d2h, "h2d": 2 * 4 * (per_step + wl.n)}
+
+
+def tc_eligible(wl, gemm):
+    return (gemm != "simt" and wl.batch <= 256 and len(wl.dims) >= 3
+            and all(d % 8 == 0 for d in wl.dims[:-1]))
+
+
+def workload_record(args, wl, r, per_step, ws, hbm, bf16, peak_src):
+    on_tc = tc_eligible(wl, args.gemm)
+    ms_step = r["ms"] / args.steps
+    ws_step = per_step * wl.lam
+    value = whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch, r["ms"])
+    rec = {
+        "value": value, "unit": UNIT, "ms_per_step": ms_step,
+        "dtype": "f32" if wl.precision == WL.PREC_FP32 else "bf16",
+        "config": {"workload": wl.name, "commits_per_step": per_step,
+                   "l2": "inputs larger than L2 (replicas and accumulators of all workers: "
+                         f"{2 * wl.n * I.num_params(wl.dims) * 4 / 1e6:.0f} MB vs 129 MB L2)",
+                   "gemm": ("tcgen05 bf16" if wl.precision == WL.PREC_BF16 else
+                            "tcgen05 fp32 as three exact bf16 pieces") +
+                           " (hidden layers); fused output layer on CUDA cores" if on_tc else
+                           "CUDA-core GEMMs; fused output layer"},
+        "roofline": roofline(wl, r["kst"], args.steps * ws_step, on_tc, hbm, bf16, peak_src),
+        "tensor": tensor_summary(wl, r["kst"], r["prof_ms"] / args.steps, ws_step, on_tc, bf16),
+        "events_region_ms_per_step": r["prof_ms"] / args.steps,
+        "kernels": {k: {"launches": int(v["launches"]), "ms": round(v["ms"], 3),
+                        "share": round(v["ms"] / max(sum(x["ms"] for x in r["kst"].values()),
+                                                     1e-9), 4)}
+                    for k, v in r["kst"].items() if v["launches"]},
+        "e2e": {"value": whole_job_value(ws, args.steps, per_step, wl.lam, wl.batch,
+                                         r["e2e_ms"]),
+                "unit": UNIT, "h2d_bytes_per_step": r["h2d"],
+                "d2h_bytes_per_step": r["d2h"] // max(args.steps, 1)},
+        "gpu_launches": r["launches"],
+    }
+    return rec
+
+
+def run_agn(args, wl):
+    import torch
+    import paper_1710_02368_gb300 as agn
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    per_step = args.commits_per_step or (
+        COMMITS_PER_STEP[args.workload] if not args.workers else 2 * wl.n)
+    hbm, bf16, _, peak_src = _peaks()
+    r = measure_workload(args, wl, agn, torch, dev, per_step, ws, clock_index=local)
+    if ws > 1:
+        r["ms"], r["e2e_ms"] = max_over_ranks([r["ms"], r["e2e_ms"]], dev)
+    head = workload_record(args, wl, r, per_step, ws, hbm, bf16, peak_src)
+    # the other MLP workloads of the benchmark, each measured the same way
+    # (sub-records; the headline stays the workload above)
+    subs = {}
+    if rank == 0 and ws == 1 and not args.no_sub_workloads and args.workload == "mnist":
+        for key in ("wide", "large"):
+            swl = WORKLOADS[key]
+            sr = measure_workload(args, swl, agn, torch, dev, COMMITS_PER_STEP[key], 1)
+            subs[swl.name] = workload_record(args, swl, sr, COMMITS_PER_STEP[key], 1, hbm, bf16,
+                                             peak_src)
     commit = None
     if rank == 0 and not args.no_commit_bench:
-        commit = commit_kernel_bench(agn, torch, dev)
-        commit["frac_of_measured_hbm"] = commit["GB/s"] / hbm
+        commit = {}
+        for P in WL.COMMIT_PULL.sizes:
+            cr = commit_kernel_bench(agn, torch, dev, P)
+            cr["frac_of_measured_hbm"] = cr["GB/s"] / hbm
+            commit[str(P)] = cr
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None,
-        "dtype": "f32" if wl.precision == WL.PREC_FP32 else "bf16",
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": head["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": head["dtype"],
         "data": "synthetic (seeded MNIST-shaped teacher-labelled set; MNIST itself unavailable)",
-        "config": {"workload": wl.name, "commits_per_step": per_step,
-                   "commit_rule": args.commit_rule,
-                   "accumulator": "elided" if args.elide_accumulator else "kept",
-                   "local_optimizer": args.optimizer,
-                   "parallelism": "replicas" if ws > 1 else "single GPU",
-                   "l2": "inputs larger than L2 (dataset 188 MB + replicas and accumulators "
-                         "230 MB vs 129 MB L2)" if args.workload == "mnist" else
-                         "inputs larger than L2 (replicas and accumulators of all workers)",
-                   "gemm": gemm_used},
-        "roofline": roof,
-        "kernels": kernels,
+        "config": dict(head["config"], commit_rule=args.commit_rule,
+                       accumulator="elided" if args.elide_accumulator else "kept",
+                       local_optimizer=args.optimizer,
+                       parallelism="replicas" if ws > 1 else "single GPU"),
+        "roofline": head["roofline"],
+        "tensor": head["tensor"],
+        "events_region_ms_per_step": head["events_region_ms_per_step"],
+        "kernels": head["kernels"],
+        "gpu_launches": head["gpu_launches"],
+        "clocks": r["clk"].summary() if r["clk"] is not None else None,
+        "e2e": head["e2e"],
+        "workloads": subs,
         "commit_pull_kernel": commit,
-        "gpu_launches": launches,
-        "clocks": clk.summary(),
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h // max(args.steps, 1)},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
@@ -447,6 +575,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-commit-bench", action="store_true")
+    ap.add_argument("--no-sub-workloads", action="store_true",
+                    help="time only the headline workload (not the two bf16 workloads)")
     args = ap.parse_args()
     wl = WORKLOADS[args.workload]
     if args.workers:

@@ -54,11 +54,15 @@ extern "C" {
 
 #define AGN_GEMM_AUTO 0        /* tcgen05 where eligible, else CUDA cores   */
 #define AGN_GEMM_SIMT 1        /* CUDA-core GEMM kernels only                */
-#define AGN_GEMM_TCGEN05 2     /* tcgen05/TMEM GEMMs for the hidden layers;
-                                  needs bf16 mode, batch <= 256 and d_0 ..
-                                  d_{L-1} multiples of 8 (else
-                                  AGN_E_UNSUPPORTED); the d_L-wide output
-                                  layer always runs on CUDA cores          */
+#define AGN_GEMM_TCGEN05 2     /* tcgen05/TMEM GEMMs for the hidden layers in
+                                  either precision (fp32 mode feeds every fp32
+                                  operand as three exact bf16 pieces, fp32
+                                  accumulation); needs at least one hidden
+                                  layer, batch <= 256 and d_0 .. d_{L-1}
+                                  multiples of 8 (else AGN_E_UNSUPPORTED).
+                                  The d_L-wide output layer's forward,
+                                  softmax-CE and dX run on CUDA cores; its dW
+                                  joins the tensor-core dW launch          */
 
 /* Local optimizers (agn_options.local_optimizer) */
 #define AGN_OPT_SGD 0
@@ -163,13 +167,24 @@ int agn_create(const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t l
 int agn_run(agn_handle* h, int32_t n_commits, const int32_t* worker,
             const int32_t* staleness, int32_t n_schedule);
 
-/* theta~ after the commits run so far, fp32, flat order, into host out[P]. */
+/*
+ * The central variable theta~ after the commits run so far: theta~^0 plus
+ * every commit Delta theta^k added in FIFO order by the parameter server
+ * (Eq. 2; Algorithm 1's Commit).  fp32, flat order, into host out[P]
+ * (cap >= P, else AGN_E_INVALID).  Waits for the handle's queued work.
+ */
 int agn_central(agn_handle* h, float* out, int64_t cap);
 
 /* Replica theta_k (fp32 master), flat order, into host out[P]. */
 int agn_replica(agn_handle* h, int32_t k, float* out, int64_t cap);
 
-/* Per commit so far: the mean of its lambda minibatch losses (host out[C]). */
+/*
+ * Per commit c so far (index order): the mean over the worker's lambda local
+ * steps of the minibatch loss (1/m) sum_j L(theta_i; x_ij, y_ij), the
+ * objective whose gradient Eq. 1 sums, L being softmax cross-entropy.  fp32
+ * into host out[C], C = agn_num_commits (cap >= C, else AGN_E_INVALID).
+ * Waits for the handle's queued work.
+ */
 int agn_loss(agn_handle* h, float* out, int64_t cap);
 
 /*
@@ -257,8 +272,8 @@ int agn_make_schedule(int32_t n, int32_t n_commits, int32_t tau_lo, int32_t tau_
 
 /*
  * The plan agn_run follows for the first n_commits commits of a fresh handle
- * with n_workers workers and lambda local steps (pure host helper, no
- * device).  Commit c reads theta~ after v_c = c - staleness[c] commits
+ * with n_workers workers (1 .. 256, as agn_create) and lambda local steps
+ * (pure host helper, no device).  Commit c reads theta~ after v_c = c - staleness[c] commits
  * (Figure 1's FIFO server; Algorithm 1's Pull before its local steps), so
  * the local steps of every commit whose version is already applied can run
  * together: a wave takes, per worker, its next commit if v_c <= V (V = commits
@@ -320,8 +335,9 @@ int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_
  * outside it, or a latency-bound loop where an allocation, which can
  * synchronise the device or fail under memory pressure, is not allowed.
  * Same arguments, same kernels and bit-identical results as agn_commit_pull
- * (theta~, accumulators, replicas, and the norms, which are reduced in the
- * same fixed order).  It allocates nothing: its scratch (the per-block
+ * (theta~, accumulators and replicas always; the norms too whenever the
+ * commit kernel's grid fits the fixed array, i.e. on every GPU with at most
+ * 256 SMs, GB300 included: they are then reduced in the same fixed order).  It allocates nothing: its scratch (the per-block
  * partial sums of the norms) is a fixed array of 16 x 1024 doubles
  * (128 KiB) in device global memory that every GPU loading the library holds
  * until the process exits.

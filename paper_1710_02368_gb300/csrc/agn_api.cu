@@ -738,6 +738,10 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
                                             : (float)(-(h->eta / (double)(tau[i] + 1)));
       }
       int pb = cp.pull_begin[c];
+      // a run of pulls longer than one launch carries cannot arise while
+      // n <= kMaxPullsPerLaunch (each worker pulls a version at most once)
+      if (pb + np > agn::kMaxPullsPerLaunch)
+        return Status::Err(AGN_E_INVALID, "internal: more pulls at one version than workers");
       for (int p : pulls_at[i + 1]) cp.pull_worker[pb++] = p;
       cp.pull_begin[c + 1] = pb;
       cp.n_commits = c + 1;
@@ -1179,13 +1183,15 @@ Status commit_pull(float* theta_c, float* acc, float* reps, void* reps_b, int64_
     return Status::Err(AGN_E_INVALID, "device buffers must be 16-byte aligned");
   if (C == 0) return Status::Ok();
   if (po[0] != 0) return Status::Err(AGN_E_INVALID, "pull_offsets[0] must be 0");
+  // offsets first (they bound every later read), then the pointers the pulls need
+  for (int c = 0; c < C; ++c)
+    if (po[c + 1] < po[c]) return Status::Err(AGN_E_INVALID, "pull_offsets must not decrease");
+  if (po[C] > 0 && (!reps || !pw)) return Status::Err(AGN_E_INVALID, "pulls need replicas");
   for (int c = 0; c < C; ++c) {
     if (cw[c] < 0 || cw[c] >= n) return Status::Err(AGN_E_INVALID, "commit worker out of range");
-    if (po[c + 1] < po[c]) return Status::Err(AGN_E_INVALID, "pull_offsets must not decrease");
     for (int p = po[c]; p < po[c + 1]; ++p)
       if (pw[p] < 0 || pw[p] >= n) return Status::Err(AGN_E_INVALID, "pull worker out of range");
   }
-  if (po[C] > 0 && (!reps || !pw)) return Status::Err(AGN_E_INVALID, "pulls need replicas");
   const float scale = (float)(normalize ? -(eta / (double)lambda) : -eta);
   const int grid = agn::commit_grid(P);
   double* partials = nullptr;
@@ -1458,7 +1464,8 @@ int agn_plan_waves(int32_t n_workers, int32_t lambda, int32_t n_commits, const i
                    int32_t* wave_slots, int32_t* wave_end, int32_t* slot_commit,
                    int64_t* slot_t0, int64_t pull_cap, int32_t* pull_version,
                    int32_t* pull_worker, int64_t* n_pulls_out) {
-  if (n_workers < 1 || lambda < 1 || n_commits < 0 || n_schedule < n_commits || pull_cap < 0 ||
+  if (n_workers < 1 || n_workers > agn::kMaxPullsPerLaunch || lambda < 1 || n_commits < 0 ||
+      n_schedule < n_commits || pull_cap < 0 ||
       !n_waves_out || !n_pulls_out ||
       (n_schedule > 0 && (!worker || !staleness)) ||
       (n_commits > 0 && (!wave_slots || !wave_end || !slot_commit || !slot_t0)) ||

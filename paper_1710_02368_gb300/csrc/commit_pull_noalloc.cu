@@ -69,9 +69,12 @@ agn::Status commit_pull_noalloc(float* theta_c, float* acc, float* reps, void* r
     return Status::Err(AGN_E_INVALID, "device buffers must be 16-byte aligned");
   if (C == 0) return Status::Ok();
   if (po[0] != 0) return Status::Err(AGN_E_INVALID, "pull_offsets[0] must be 0");
+  // offsets first (they bound every later read), then the pointers the pulls need
+  for (int c = 0; c < C; ++c)
+    if (po[c + 1] < po[c]) return Status::Err(AGN_E_INVALID, "pull_offsets must not decrease");
+  if (po[C] > 0 && (!reps || !pw)) return Status::Err(AGN_E_INVALID, "pulls need replicas");
   for (int c = 0; c < C; ++c) {
     if (cw[c] < 0 || cw[c] >= n) return Status::Err(AGN_E_INVALID, "commit worker out of range");
-    if (po[c + 1] < po[c]) return Status::Err(AGN_E_INVALID, "pull_offsets must not decrease");
     if (po[c + 1] - po[c] > agn::kMaxPullsPerLaunch)
       return Status::Err(AGN_E_INVALID,
                          "commit " + std::to_string(c) + " has " + std::to_string(po[c + 1] - po[c]) +
@@ -80,7 +83,6 @@ agn::Status commit_pull_noalloc(float* theta_c, float* acc, float* reps, void* r
     for (int p = po[c]; p < po[c + 1]; ++p)
       if (pw[p] < 0 || pw[p] >= n) return Status::Err(AGN_E_INVALID, "pull worker out of range");
   }
-  if (po[C] > 0 && (!reps || !pw)) return Status::Err(AGN_E_INVALID, "pulls need replicas");
   double* scratch = nullptr;
   AGN_TRY(scratch_on_current_device(&scratch));
   const float scale = (float)(normalize ? -(eta / (double)lambda) : -eta);

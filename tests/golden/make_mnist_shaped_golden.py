@@ -10,7 +10,10 @@ trajectory; the GPU parity test uses that drift as its envelope.
 Stored: per commit the float64 loss (mean of the lambda minibatch losses)
 and ||Delta_c||; at checkpoints c = 0, 100, .., 1900, 1999 the float64
 ||theta~||, the float32 run's relative L2 deviation, and theta~ (float64) at
-256 seeded parameter indices.  Takes about 30 minutes on 8 cores.
+256 seeded parameter indices; and, in mnist_shaped_2000_full.npz, the whole
+theta~ after the last commit from both runs (float64 values rounded to
+float32, a relative change of at most 2^-24 per element).  Takes about 30
+minutes on 8 cores.
 
 Usage: python tests/golden/make_mnist_shaped_golden.py
 """
@@ -28,6 +31,7 @@ import oracle as O  # noqa: E402
 from agn_inputs import workloads as WL  # noqa: E402
 
 OUT = os.path.join(os.path.dirname(os.path.abspath(__file__)), "mnist_shaped_2000.txt")
+FULL_OUT = os.path.join(os.path.dirname(os.path.abspath(__file__)), "mnist_shaped_2000_full.npz")
 N_SAMPLED = 256
 
 
@@ -66,7 +70,11 @@ def main():
             dev = np.linalg.norm(r32.snapshots[c].astype(np.float64) - a) / np.linalg.norm(a)
             f.write(f"checkpoint {c} {np.linalg.norm(a):.17g} {dev:.17g} "
                     + " ".join(f"{v:.17g}" for v in a[idx]) + "\n")
-    print("wrote", OUT)
+    last = cps[-1]
+    np.savez_compressed(FULL_OUT, commit=np.int64(last),
+                        theta64=r64.snapshots[last].astype(np.float32),
+                        theta32=r32.snapshots[last].astype(np.float32))
+    print("wrote", OUT, FULL_OUT)
 
 
 def load():
@@ -85,6 +93,13 @@ def load():
             elif p[0] == "checkpoint":
                 cps[int(p[1])] = (float(p[2]), float(p[3]), np.array([float(v) for v in p[4:]]))
     return idx, np.array(loss), np.array(dn), cps
+
+
+def load_full():
+    """(commit index, float64 oracle's theta~, float32 oracle's theta~) after
+    the last commit, both as float32 arrays of P values in flat order."""
+    z = np.load(FULL_OUT)
+    return int(z["commit"]), z["theta64"], z["theta32"]
 
 
 if __name__ == "__main__":

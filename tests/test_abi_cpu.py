@@ -129,3 +129,22 @@ def test_temporal_efficiency_through_the_abi(agn):
         with pytest.raises(agn.AGNError) as e:
             agn.agn_temporal_efficiency(*bad)
         assert e.value.code == agn.AGN_E_INVALID
+
+
+@pytest.mark.parametrize("entry", ["agn_commit_pull", "agn_commit_pull_noalloc"])
+def test_commit_pull_rejects_pulls_without_buffers_before_reading_them(agn, entry):
+    """Pull offsets that promise pulls with a null pull list (or no replicas)
+    are rejected with AGN_E_INVALID before any pull index is read (no device
+    is touched: validation comes first)."""
+    import ctypes as C
+    from paper_1710_02368_gb300 import _lib
+    lib = _lib.load()
+    fake = C.c_void_p(1 << 20)            # aligned, never dereferenced on the host
+    cw = (C.c_int32 * 1)(0)
+    po = (C.c_int32 * 2)(0, 2)
+    pw = (C.c_int32 * 2)(0, 1)
+    fn = getattr(lib, entry)
+    rc = fn(fake, fake, fake, None, 64, 64, 2, 1, cw, po, None, 0.01, 10, 1, None, None)
+    assert rc == agn.AGN_E_INVALID and "pulls need replicas" in agn.agn_last_error()
+    rc = fn(fake, fake, None, None, 64, 64, 2, 1, cw, po, pw, 0.01, 10, 1, None, None)
+    assert rc == agn.AGN_E_INVALID and "pulls need replicas" in agn.agn_last_error()

@@ -83,3 +83,27 @@ def test_committed_traffic_entries_are_well_formed():
         assert r[0] in ("forward", "backward_dx", "backward_dw", "softmax", "commit")
         assert float(r[2]) > 0
         assert len(r[3]) == 12 and all(ch in "0123456789abcdef" for ch in r[3])
+
+
+def test_commit_launch_grouping_and_bytes():
+    """The standalone commit workload's launches (runs of <= 16 commits, cut at
+    a repeated worker or past 256 pulls) and the bytes a pass must move:
+    theta~ 8P per launch, 8P per commit, 4P per pull."""
+    order, pulls = list(range(64)), [[1, 2, 3, 4]] * 64
+    assert bench.commit_plan_launches(order, pulls) == 4
+    assert bench.commit_plan_launches([0, 1, 0, 2], [[]] * 4) == 2
+    assert bench.commit_plan_launches(list(range(8)), [list(range(100))] * 8) == 4
+    P = 1 << 20
+    assert bench.commit_pass_bytes(P, 64, 256, 4) == P * (8 * 4 + 8 * 64 + 4 * 256)
+
+
+def test_method_bytes_of_the_dw_class_by_hand():
+    """784-1000-1000-10 fp32, m = 128: theta_k and a_k read-modify-write,
+    16 B per parameter (P = 1,796,010), plus the operands of the three layers'
+    weight gradients (dZ_l and H_{l-1}, 4 B each)."""
+    from agn_inputs import workloads as WL
+    wl = WL.MNIST_SHAPED
+    got = bench.method_bytes_per_worker_step(wl, "backward_dw")
+    assert got == 16 * 1796010 + 128 * 4 * ((1000 + 784) + (1000 + 1000) + (10 + 1000))
+    bf = bench.method_bytes_per_worker_step(WL.LARGE_BF16, "backward_dw")
+    assert bf == 18 * 20037642 + 64 * 2 * ((4096 + 784) + (4096 + 4096) + (10 + 4096))

@@ -1,0 +1,103 @@
+"""fp32 parity at the shapes the benchmark times: the default GEMM path (tcgen05
+with fp32 operands as three exact bf16 pieces) with multi-worker waves, i.e.
+several commits per agn_run call, so that every wave batches the local steps
+of several workers (Algorithm 1) and the forward / dX GEMMs take the tile and
+split-K choices of those wave sizes, against the float64 oracle (Eq. 1-2).
+
+Tolerance.  theta~ within 1e-5 relative L2 of the float64 oracle after each
+checked commit, except where float32 arithmetic itself has left 1e-5 of the
+float64 trajectory: the oracle is also run in float32 (NumPy single
+precision, the same algorithm), and the bound is max(1e-5, 3 x that run's
+own deviation from float64) at the checked commit.  Per-commit losses and
+||Delta_c|| likewise: 1e-5 relative, or 3x the float32 run's largest
+deviation so far.
+"""
+
+import numpy as np
+import pytest
+
+import agn_inputs as I
+import oracle as O
+from agn_inputs import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+REL_STEP = 1e-5
+
+
+@pytest.fixture(scope="module")
+def agn():
+    import __graft_entry__ as g
+    g.build()
+    import paper_1710_02368_gb300 as agn
+    return agn
+
+
+def _rel(a, b):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+
+def _oracles(wl, C, snaps):
+    seed = I.DEFAULT_SEED
+    w, tau = I.make_schedule(wl.n, C + wl.n, wl.tau_lo, wl.tau_hi, seed)
+    ds = I.workload_dataset(wl, seed)
+    th0 = I.init_params(seed, wl.dims)
+    r64 = O.agn_run(O.MLP(wl.dims), th0, wl.n, wl.lam, wl.eta, w[:C], tau[:C], ds, wl.batch,
+                    wl.shard, snapshot_at=snaps)
+    r32 = O.agn_run(O.MLP(wl.dims, np.float32), th0, wl.n, wl.lam, wl.eta, w[:C], tau[:C], ds,
+                    wl.batch, wl.shard, snapshot_at=snaps, dtype=np.float32)
+    return w, tau, r64, r32
+
+
+def _envelope(got, ref64, ref32):
+    """Per commit: max(1e-5 |ref64|, 3 x the float32 run's largest deviation so far)."""
+    dev = np.maximum.accumulate(np.abs(np.asarray(ref32, dtype=np.float64) - ref64))
+    bound = np.maximum(REL_STEP * np.abs(ref64), 3.0 * dev)
+    return np.abs(np.asarray(got, dtype=np.float64) - ref64), bound
+
+
+def _check(wl, bounds, h, w, tau, r64, r32):
+    waves = 0
+    for a, b in zip(bounds[:-1], bounds[1:]):
+        h.run(b - a, w[a:], tau[a:])
+        waves += int(h.last_run_stats()["waves"])
+        c = b - 1
+        th = h.central()
+        err = _rel(th, r64.snapshots[c])
+        dev32 = _rel(r32.snapshots[c], r64.snapshots[c])
+        assert err <= max(REL_STEP, 3.0 * dev32), (c, err, dev32)
+    C = bounds[-1]
+    d, bnd = _envelope(h.loss(), r64.loss, r32.loss)
+    assert np.all(d <= bnd), (int(np.argmax(d - bnd)), float(np.max(d)))
+    d, bnd = _envelope(h.delta_norm(), r64.delta_norm, r32.delta_norm)
+    assert np.all(d <= bnd), (int(np.argmax(d - bnd)), float(np.max(d)))
+    return C / waves
+
+
+def test_small_workload_in_one_call(agn):
+    """784-128-10, n=4, lambda=5, m=32, tau in {0,1,2}: all 50 commits in one
+    agn_run call (waves of up to four workers), theta~ at the end."""
+    wl = WL.SMALL
+    C = wl.commits
+    w, tau, r64, r32 = _oracles(wl, C, [C - 1])
+    with agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, I.DEFAULT_SEED, batch=wl.batch,
+                 n_samples=wl.n_samples, gemm=agn.AGN_GEMM_AUTO) as h:
+        mean_wave = _check(wl, [0, C], h, w, tau, r64, r32)
+    assert mean_wave > 1.5, mean_wave
+
+
+def test_mnist_shaped_in_benchmark_calls(agn):
+    """784-1000-1000-10, n=16, lambda=15, m=128, tau in {0..15}, at full size:
+    three calls of 16 commits, then one call of 100 commits (the benchmark's
+    step), theta~ compared in full after each call."""
+    wl = WL.MNIST_SHAPED
+    bounds = [0, 16, 32, 48, 148]
+    C = bounds[-1]
+    w, tau, r64, r32 = _oracles(wl, C, [b - 1 for b in bounds[1:]])
+    with agn.AGN(wl.dims, wl.n, wl.lam, wl.eta, I.DEFAULT_SEED, batch=wl.batch,
+                 n_samples=wl.n_samples, gemm=agn.AGN_GEMM_AUTO) as h:
+        mean_wave = _check(wl, bounds, h, w, tau, r64, r32)
+    # the benchmark's waves average about 4.5 workers on this schedule
+    assert mean_wave > 3.0, mean_wave

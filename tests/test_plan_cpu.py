@@ -116,3 +116,16 @@ def test_plan_rejects_infeasible_schedules(agn):
     with pytest.raises(agn.AGNError) as e:
         agn.agn_plan_waves(2, 1, 3, [0, 1], [0, 0])         # fewer entries than commits
     assert e.value.code == agn.AGN_E_INVALID
+
+
+def test_plan_rejects_more_workers_than_create_accepts(agn):
+    """agn_create takes 1 .. 256 workers; the planner rejects n = 257 alike
+    (a version pulled by more workers than one commit launch carries)."""
+    n = 257
+    w = np.arange(n, dtype=np.int32)
+    tau = np.zeros(n, dtype=np.int32)
+    tau[1:] = np.arange(n - 1)            # commits 1 .. n-1 all read version 1
+    with pytest.raises(agn.AGNError) as e:
+        agn.agn_plan_waves(n, 1, n, w, tau)
+    assert e.value.code == agn.AGN_E_INVALID
+    check_plan(agn, 256, 1, w[:256], tau[:256], 256)
