@@ -100,7 +100,9 @@ typedef struct agn_options {
      are on (bit 0 forward, bit 1 dX, bit 2 dW; none of bits 0-2 = all three).  Bit 3 runs the
      dW GEMMs on the earlier non-persistent tcgen05 kernel (one tile per CTA)
      instead of the persistent one, for comparison.  Bit 4 runs the forward
-     and dX GEMMs without split K (one CTA per output tile). */
+     and dX GEMMs without split K (one CTA per output tile).  Bit 5 runs the
+     output layer (forward, softmax-CE, dX) as a kernel of its own instead of
+     in the epilogue of the last hidden layer's forward GEMM. */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);
@@ -218,7 +220,9 @@ int64_t agn_num_commits(const agn_handle* h);  /* commits applied so far */
 
 /*
  * Statistics of the last agn_run: [0] waves, [1] kernel launches, [2] GPU
- * milliseconds (CUDA events around the queued work), [3] worker-steps.
+ * milliseconds (CUDA events around the queued work), [3] worker-steps, and,
+ * when cap >= 5, [4] host milliseconds from the call's start until all of its
+ * work was queued (planning and launches, before the final wait).
  */
 int agn_last_run_stats(const agn_handle* h, double* out, int64_t cap);
 

@@ -11,6 +11,7 @@
 // most kMaxCommitsPerLaunch commits); each pull happens right after the commit
 // that creates the version it reads.  This gives the same theta~ as applying
 // the commits one at a time in schedule order.
+#include <chrono>
 #include <cmath>
 #include <cstdint>
 #include <new>
@@ -109,7 +110,8 @@ struct agn_handle {
   double* partials = nullptr;
   // tcgen05 path (bf16 mode): tensor maps per layer l = 1..L-1 (index l-1)
   bool use_tc = false;
-  int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW, 3 tiled dW, 4 no split K
+  int tc_mask = 7;            // bit 0 forward, bit 1 dX, bit 2 dW, 3 tiled dW, 4 no split K,
+                              // 5 output layer as its own kernel
   struct LayerMaps {
     CUtensorMap w_k, w_mn, h_k, h_mn, dz_k, dz_mn;
     CUtensorMap theta, acc;      // fp32 W_l of every replica / accumulator, box {128, 32}
@@ -136,6 +138,15 @@ struct agn_handle {
   int ldz_out = 0;
   float* ce_partial = nullptr;    // [n][ceil(m / kHeadSamples)]
   int* head_counter = nullptr;    // [n]
+  // the output layer fused into the last hidden layer's tensor-core forward
+  // (when the launch's CTAs fit the SMs at once): partial logits, counters
+  bool fuse_head = false;
+  float* fh_part = nullptr;       // [n][ceil(m / 32)][ceil(d_{L-1} / 128)][32][16]
+  int* fh_counter = nullptr;      // [n][ceil(m / 32)]
+  // loss_parts holds loss_q values per local step of a commit: the fused
+  // output layer writes one per 32-sample chunk, the other paths the step's
+  // loss in the first and zeros after it
+  int loss_q = 1;
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
   float* dnorm = nullptr;     // [cap_commits]
@@ -153,7 +164,7 @@ struct agn_handle {
   int64_t V = 0;                                  // commits applied
   std::vector<int64_t> prev, pulled_v, steps;     // per worker
   std::string err;
-  double stats[4] = {0, 0, 0, 0};
+  double stats[5] = {0, 0, 0, 0, 0};
   // per-kernel profiling (agn_profile)
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
@@ -415,8 +426,15 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
                                    (int64_t)n * m * h->dims[0]));
     }
     bool dz_ready = false;   // pieces of the next layer's dZ already written by its producer
+    // the output layer rides in the last hidden layer's forward when that
+    // launch's CTAs fit the SMs at once
+    const bool fuse_head_now =
+        h->fuse_head && tc_layer(h, L - 1) &&
+        ceil_div(h->dims[L - 1], 128) * (int64_t)s <= (int64_t)h->num_sms;
+    bool head_done = false;
     // forward, l = 1..L
     for (int l = 1; l <= L; ++l) {
+      if (l == L && head_done) continue;
       if (l == L && h->use_head) {   // output layer: forward + softmax-CE + dX, one kernel
         agn::HeadArgs a{};
         const int fi = h->dims[L - 1], C = h->dims[L];
@@ -432,7 +450,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         a.dH_pieces = L > 1 ? dz_pieces(L - 1) : nullptr;
         a.dH_plane = L > 1 ? dz_plane(L - 1) : 0;
         a.ce_partial = h->ce_partial; a.counter = h->head_counter;
-        a.loss_parts = h->loss_parts; a.slot_commit = sc; a.lam = h->lam; a.step = i;
+        a.loss_parts = h->loss_parts; a.loss_q = h->loss_q; a.slot_commit = sc; a.lam = h->lam; a.step = i;
         a.flag = h->flag;
         Launch k(h, AGN_K_SOFTMAX, 4.0 * s * m * fi * C,
                  (double)s * ((double)C * fi * es + 2.0 * m * fi * es + (double)m * C * es), launches);
@@ -456,12 +474,46 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       bf16* h_pieces =
           (h->split && (l + 1 < L || (h->fuse_out_dw && l + 1 == L))) ? h->Hs[l] : nullptr;
       bool pieces_done = false;
+      const bool fuse = fuse_head_now && l == L - 1;
       {
-        Launch k(h, AGN_K_FORWARD, 2.0 * s * m * fo * fi,
+        // with the output layer fused: its forward and dX flops, W_L, dZ_L
+        // and dZ_{L-1} (with pieces) bytes too
+        const int C = h->dims[L];
+        Launch k(h, AGN_K_FORWARD,
+                 2.0 * s * m * fo * fi + (fuse ? 4.0 * s * m * fo * C : 0.0),
                  (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es +
-                              (double)m * fo * (oes + (h_pieces ? 6.0 : 0.0))),
+                              (double)m * fo * (oes + (h_pieces ? 6.0 : 0.0))) +
+                     (fuse ? (double)s * (4.0 * C * (fo + 1) +
+                                          (double)m * C * (es + (h->split ? 6.0 : 0.0)) +
+                                          (double)m * fo * (2.0 * es + (h->split ? 6.0 : 0.0)))
+                           : 0.0),
                  launches);
-        if (tc_layer(h, l) && (h->tc_mask & 1)) {
+        if (fuse) {
+          agn::TcArgs t = tc_args(h, sw);
+          t.M = fo; t.N = m; t.K = fi;
+          t.a_by_worker = 1;
+          t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
+          t.relu = 1; t.boff = h->boff[l - 1];
+          t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
+          t.head_woff = h->woff[L - 1]; t.head_boff = h->boff[L - 1]; t.head_C = C;
+          t.yb = h->yb;
+          t.dzl = h->dZ[L]; t.ldz = h->ldz_out;
+          t.dzl_pieces = (h->fuse_out_dw && h->split) ? h->dZp[L] : nullptr;
+          t.dzl_plane = (int64_t)n * m * h->ldz_out;
+          t.dh = h->dZ[L - 1]; t.dh_pieces = dz_pieces(L - 1); t.dh_plane = dz_plane(L - 1);
+          t.head_part = h->fh_part; t.head_counter = h->fh_counter;
+          t.loss_parts = h->loss_parts; t.slot_commit = sc; t.lam = h->lam; t.step = i;
+          t.nonfinite = h->flag;
+          const auto& mp = h->tmaps[l - 1];
+          t.ksplit = pick_ksplit(h, fo, fi, s);
+          bool launched = false;
+          AGN_TRY(agn::tc_forward_head(mp.w_k, mp.h_k, t, s, h->stream, h->split,
+                                       agn::tc_bn(m), h->num_sms, &launched));
+          if (!launched) return Status::Err(AGN_E_CUDA, "internal: fused output layer not resident");
+          pieces_done = true;
+          head_done = true;
+          dz_ready = t.dh_pieces != nullptr;
+        } else if (tc_layer(h, l) && (h->tc_mask & 1)) {
           agn::TcArgs t = tc_args(h, sw);
           t.M = fo; t.N = m; t.K = fi;
           t.a_by_worker = 1;
@@ -760,6 +812,7 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
 }
 
 Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, int ns) {
+  const auto t_host0 = std::chrono::steady_clock::now();
   RunPlan plan;
   AGN_TRY(build_plan(h, k, worker, tau, ns, &plan));
   const int64_t V0 = h->V;
@@ -770,7 +823,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     AGN_TRY(grow(h, &h->dnorm, &c2, V0 + k, V0));
     h->cap_commits = c1;
   }
-  AGN_TRY(grow(h, &h->loss_parts, &h->cap_parts, (int64_t)k * h->lam, 0));
+  AGN_TRY(grow(h, &h->loss_parts, &h->cap_parts, (int64_t)k * h->lam * h->loss_q, 0));
   if (total_slots > h->cap_plan) {  // the three plan arrays share one capacity
     int64_t c1 = h->cap_plan, c2 = h->cap_plan, c3 = h->cap_plan;
     AGN_TRY(grow(h, &h->plan_worker, &c1, total_slots, 0));
@@ -826,11 +879,13 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   }
   {
     Launch kl(h, AGN_K_OTHER, 0.0, 4.0 * k * (h->lam + 1), &launches);
-    AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, k, h->loss + V0, h->stream));
+    AGN_TRY(agn::reduce_losses(h->loss_parts, h->lam, h->loss_q, k, h->loss + V0, h->stream));
   }
   AGN_TRY_CUDA(cudaEventRecord(h->ev1, h->stream));
   int flags[2] = {0, 0};
   AGN_TRY_CUDA(cudaMemcpyAsync(flags, h->flag, 2 * sizeof(int), cudaMemcpyDeviceToHost, h->stream));
+  const double host_ms =
+      std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t_host0).count();
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
   float ms = 0.f;
   cudaEventElapsedTime(&ms, h->ev0, h->ev1);
@@ -839,6 +894,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   h->stats[1] = (double)launches;
   h->stats[2] = ms;
   h->stats[3] = (double)k * h->lam;
+  h->stats[4] = host_ms;
   h->V = V0 + k;
   h->prev = plan.prev;
   h->pulled_v = plan.pulled_v;
@@ -847,6 +903,10 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
     if (flags[1] && h->tc_counter)   // CTAs that gave up may have left tiles unfinished
       AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)h->num_sms * sizeof(int), h->stream));
+    if (flags[1] && h->fuse_head) {
+      AGN_TRY_CUDA(cudaMemsetAsync(h->fh_counter, 0,
+                                   (size_t)(h->n * ceil_div(h->m, 32)) * sizeof(int), h->stream));
+    }
     AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
     if (flags[1])
       return Status::Err(AGN_E_TIMEOUT, "a tensor-core GEMM gave up on a bounded wait");
@@ -873,7 +933,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 31) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 31]");
+  if (o.tc_mask < 0 || o.tc_mask > 63) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 63]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)
@@ -1012,6 +1072,8 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
                                          : agn::head_fits<float>(dims[h->L - 1], dims[h->L]);
   h->fuse_out_dw = h->use_tc && h->use_head && h->L >= 2 && (h->tc_mask & 4) && !(h->tc_mask & 8);
   h->ldz_out = h->fuse_out_dw ? (int)round_up(dims[h->L], 8) : dims[h->L];
+  h->fuse_head = h->use_tc && h->use_head && h->L >= 2 && (h->tc_mask & 1) &&
+                 !(h->tc_mask & 32) && dims[h->L] <= agn::kHeadMaxClasses;
   if (h->split) {   // three piece planes of every replica, and of the activations
     h->piece_plane = n * h->P_pad;
     AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));
@@ -1059,6 +1121,13 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
     AGN_TRY_CUDA(cudaMemset(h->e_sw, 0, sizeof(int)));
   }
   AGN_TRY_CUDA(cudaMemsetAsync(h->head_counter, 0, (size_t)n * sizeof(int), h->stream));
+  if (h->fuse_head) {
+    const int64_t nchk = ceil_div(m, 32), mt = ceil_div(dims[h->L - 1], 128);
+    AGN_TRY(dalloc_t(h, &h->fh_part, (size_t)(n * nchk * mt * 32 * agn::kHeadMaxClasses)));
+    AGN_TRY(dalloc_t(h, &h->fh_counter, (size_t)(n * nchk)));
+    AGN_TRY_CUDA(cudaMemsetAsync(h->fh_counter, 0, (size_t)(n * nchk) * sizeof(int), h->stream));
+    h->loss_q = (int)nchk;
+  }
   h->grid = agn::commit_grid(h->P_pad);
   AGN_TRY(dalloc_t(h, &h->partials, (size_t)agn::kMaxCommitsPerLaunch * h->grid));
   AGN_TRY(dalloc_t(h, &h->pull_list, (size_t)n));
@@ -1369,7 +1438,7 @@ int64_t agn_num_commits(const agn_handle* h) { return h ? h->V : -1; }
 
 int agn_last_run_stats(const agn_handle* h, double* out, int64_t cap) {
   if (!h || !out || cap < 4) return fail(const_cast<agn_handle*>(h), AGN_E_INVALID, "need 4 slots");
-  for (int i = 0; i < 4; ++i) out[i] = h->stats[i];
+  for (int i = 0; i < (int)std::min<int64_t>(cap, 5); ++i) out[i] = h->stats[i];
   return AGN_OK;
 }
 

@@ -337,13 +337,18 @@ pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
   }
 }
 
-__global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda, int count,
-                                     float* __restrict__ loss) {
+__global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda, int q_per,
+                                     int count, float* __restrict__ loss) {
   pdl_begin();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= count) return;
   float s = 0.f;
-  for (int i = 0; i < lambda; ++i) s += parts[(int64_t)c * lambda + i];
+  for (int i = 0; i < lambda; ++i) {
+    const float* p = parts + ((int64_t)c * lambda + i) * q_per;
+    float st = p[0];
+    for (int q = 1; q < q_per; ++q) st += p[q];
+    s += st;
+  }
   loss[c] = s / (float)lambda;
 }
 
@@ -363,12 +368,13 @@ Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16,
   return Status::Ok();
 }
 
-Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st) {
+Status reduce_losses(const float* parts, int lambda, int q_per, int count, float* loss,
+                     cudaStream_t st) {
   if (count <= 0) return Status::Ok();
   {
     auto kf = reduce_losses_kernel;
     AGN_TRY_CUDA(launch_pdl(kf, (unsigned)ceil_div(count, 128), 128, 0, st, parts,
-                            lambda, count, loss));
+                            lambda, q_per, count, loss));
   }
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();

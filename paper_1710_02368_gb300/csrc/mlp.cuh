@@ -6,7 +6,7 @@
 
 namespace agn {
 
-enum { kEpiFwd = 0, kEpiDX = 1, kEpiDW = 2 };
+enum { kEpiFwd = 0, kEpiDX = 1, kEpiDW = 2, kEpiFwdHead = 3 };
 
 // One batched GEMM over the slots of a wave: C[M x N] = sum_k A(m,k) B(k,n).
 // Slot z reads operand X at X + (X_by_worker ? slot_worker[z] : z) * X_bstride.
@@ -82,7 +82,8 @@ struct HeadArgs {
   int64_t dH_plane;        // dH_plane apart) for tensor-core GEMMs; null = no
   float* ce_partial;       // [slots][ceil(m / kHeadSamples)] scratch
   int* counter;            // [slots], zero between launches
-  float* loss_parts;
+  float* loss_parts;       // [commit][lam][loss_q]: the step's loss in slot 0, zeros after
+  int loss_q;
   const int* slot_commit;
   int lam, step;
   int* flag;
@@ -148,7 +149,9 @@ Status pull_replicas(const float* theta_c, float* replicas, bf16* replicas_bf16,
                      int64_t ld, const int* workers, int count, cudaStream_t st,
                      int64_t piece_plane = 0, float* snapshot = nullptr);
 // loss[c] = mean_i parts[c * lambda + i] for c < count.
-Status reduce_losses(const float* parts, int lambda, int count, float* loss, cudaStream_t st);
+// loss[c] = (1/lambda) sum_i sum_q parts[(c lambda + i) q_per + q] (fixed order).
+Status reduce_losses(const float* parts, int lambda, int q_per, int count, float* loss,
+                     cudaStream_t st);
 // Device-side standalone-commit input generator.
 Status fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,
                           int n, uint64_t seed, cudaStream_t stream);

@@ -211,7 +211,9 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
     float tot = 0.f;
     for (int q = 0; q < kHeadThreads / 32; ++q) tot += warp_sum[q];
     const float loss = tot / (float)m;
-    a.loss_parts[(int64_t)a.slot_commit[z] * a.lam + a.step] = loss;
+    float* lp = a.loss_parts + ((int64_t)a.slot_commit[z] * a.lam + a.step) * a.loss_q;
+    lp[0] = loss;
+    for (int q = 1; q < a.loss_q; ++q) lp[q] = 0.f;
     if (!isfinite(loss)) atomicExch(a.flag, 1);
     a.counter[z] = 0;
   }

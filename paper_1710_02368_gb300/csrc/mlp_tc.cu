@@ -37,6 +37,11 @@ constexpr int kBK = 64;                       // K per stage: 64 bf16 = one 128-
 constexpr int kABytes = 128 * 128;            // 128 rows x 128 bytes
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s
 constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles
+// Fused output layer (kEpiFwdHead): at most kHC classes; shared scratch of
+// W_L's 128 x kHC slice, the warps' partial logits [8][16][kHC] and the
+// chunk's logits / dZ_L [32][kHC].
+constexpr int kHC = kHeadMaxClasses;
+constexpr int kHeadScratch = (kHC * 128 + 8 * 16 * kHC + 32 * kHC) * 4 + 8 * 256 * 2;
 
 // A stage holds kSplit A pieces then kSplit B pieces (kSplit = 3 in the fp32
 // mode, where every fp32 operand is the exact sum of three bf16 pieces).
@@ -59,6 +64,9 @@ struct EpiT {
   static constexpr bool kSeparate = kRing + 1280 + kEpiTBytes <= 232448;
   static constexpr size_t kOff = kSeparate ? kRing + 256 : kRing - kEpiTBytes;
   static constexpr size_t kRingFree = kSeparate ? kRing : kRing - kEpiTBytes;
+  // the fused output layer's scratch, at the end of the free ring (below the
+  // split-K partial sums' reach, which the host bounds accordingly)
+  static constexpr size_t kHeadOff = kRingFree - kHeadScratch;
 };
 
 // Piece pairs (i, j) with i + j <= 2 of the split product: the dropped pairs
@@ -361,10 +369,24 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
       }
     };
+    constexpr bool kFwd = kEpi == kEpiFwd || kEpi == kEpiFwdHead;
     float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (kEpi == kEpiFwd && row4_ok && n_own > 0)
+    if (kFwd && row4_ok && n_own > 0)
       bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
     if (n_own > 0) load_mask(32 * own_rank + co);
+    // fused output layer: this tile's 128 columns of W_L (kHC x 128, zero past
+    // C and M), loads in flight across the split-K exchange
+    constexpr int kW3Per = kHC * 128 / kThreads;
+    float w3v_reg[kEpi == kEpiFwdHead ? kW3Per : 1];
+    if (kEpi == kEpiFwdHead) {
+      const float* w3g = theta + args.head_woff;
+#pragma unroll
+      for (int k = 0; k < kW3Per; ++k) {
+        const int i = threadIdx.x + k * kThreads;
+        const int c = i >> 7, rr = 128 * m_tile + (i & 127);
+        w3v_reg[k] = (c < args.head_C && rr < args.M) ? w3g[(int64_t)c * args.M + rr] : 0.f;
+      }
+    }
     bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
     if (split_k) {
       float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
@@ -439,9 +461,21 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
       for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(v[i]);
     };
+    // fused output layer: W_L's rows for this tile's 128 features, the number
+    // of 32-sample chunks with samples, and the scratch
+    float* sW3 = reinterpret_cast<float*>(smem + EpiT<BN, kSplit, kStages>::kHeadOff);
+    float* sPart = sW3 + kHC * 128;
+    float* sG = sPart + 8 * 16 * kHC;
+    uint16_t* sMask = reinterpret_cast<uint16_t*>(sG + 32 * kHC);   // [owned chunk][thread]
+    const int nchk = (args.N + 31) / 32;
+    if (kEpi == kEpiFwdHead && have) {
+#pragma unroll
+      for (int k = 0; k < kW3Per; ++k) sW3[threadIdx.x + k * kThreads] = w3v_reg[k];
+      __syncthreads();
+    }
     if (!have) {
       // reported above
-    } else if (kEpi == kEpiFwd || kEpi == kEpiDX) {
+    } else if (kEpi == kEpiFwd || kEpi == kEpiDX || kEpi == kEpiFwdHead) {
       TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
 #pragma unroll 1
       for (int o = 0; o < n_own; ++o) {
@@ -452,6 +486,91 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
         for (int i = 0; i < 16; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
         __syncwarp();
+        if (kEpi == kEpiFwdHead && (c0 - co) / 32 < nchk) {
+          // Pass 1 of the fused output layer, before this chunk's stores (so
+          // that the release below orders only the partials): this CTA's
+          // share of the chunk's logits, sum over its 128 features of
+          // H_{L-1}[j][f] W_L[c][f].  A lane sums its four features; the eight
+          // lanes of a column fold by a fixed shuffle tree; the four row
+          // quadrants of a column half are added in order below.  The ReLU
+          // mask of the lane's 4 x 4 values goes to shared memory for pass 2.
+          const int C = args.head_C;
+          uint32_t mbits = 0;
+          float hq[4][4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int j = n_tile * BN + c0 + jl + 4 * u;
+            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (row4_ok && j < args.N) {
+              a = *reinterpret_cast<const float4*>(tT + (jl + 4 * u) * 32 + r4);
+              a.x = fmaxf(a.x + bias4.x, 0.f);
+              a.y = fmaxf(a.y + bias4.y, 0.f);
+              a.z = fmaxf(a.z + bias4.z, 0.f);
+              a.w = fmaxf(a.w + bias4.w, 0.f);
+            }
+            hq[u][0] = a.x; hq[u][1] = a.y; hq[u][2] = a.z; hq[u][3] = a.w;
+#pragma unroll
+            for (int e = 0; e < 4; ++e)   // the mask of the value as stored
+              mbits |= (static_cast<float>(static_cast<TAct>(hq[u][e])) > 0.f ? 1u : 0u)
+                       << (4 * u + e);
+          }
+          // W_L rows past C are zero in shared memory: all kHC classes are
+          // summed unguarded, as independent chains
+          const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            float zp[kHC];
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) {
+              const float4 w = w3v[c * 32];
+              float t = hq[u][0] * w.x;
+              t = fmaf(hq[u][1], w.y, t);
+              t = fmaf(hq[u][2], w.z, t);
+              zp[c] = fmaf(hq[u][3], w.w, t);
+            }
+            // fold the eight lanes of the column (lane bits 0-2) by a fixed
+            // reduce-scatter: each round a lane keeps half of its classes and
+            // adds its partner's share of them; afterwards the lane holds the
+            // column's sums of classes kb and kb + 1, kb = 8 b2 + 4 b1 + 2 b0
+            static_assert(kHC == 16, "the reduce-scatter folds 16 classes");
+            const int b2 = (lane >> 2) & 1, b1 = (lane >> 1) & 1, b0 = lane & 1;
+            float k8[8], k4[4], k2[2];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const float keep = b2 ? zp[k + 8] : zp[k], send = b2 ? zp[k] : zp[k + 8];
+              k8[k] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float keep = b1 ? k8[k + 4] : k8[k], send = b1 ? k8[k] : k8[k + 4];
+              k4[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+            }
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+              const float keep = b0 ? k4[k + 2] : k4[k], send = b0 ? k4[k] : k4[k + 2];
+              k2[k] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+            }
+            *reinterpret_cast<float2*>(sPart + (warp * 16 + jl + 4 * u) * kHC + 8 * b2 + 4 * b1 +
+                                       2 * b0) = make_float2(k2[0], k2[1]);
+          }
+          sMask[o * kThreads + threadIdx.x] = (uint16_t)mbits;
+          __syncthreads();
+          const int chunk = (c0 - co) / 32;
+          float* gp = args.head_part +
+                      (((int64_t)slot * nchk + chunk) * gridDim.x + m_tile) * (32 * kHC);
+          for (int i = threadIdx.x; i < 32 * kHC; i += kThreads) {
+            const int cc = i / kHC, c = i % kHC, hf = cc >> 4, jcl = cc & 15;
+            float sum = 0.f;
+            if (c < C)
+              for (int gq = 0; gq < 4; ++gq) sum += sPart[((gq + 4 * hf) * 16 + jcl) * kHC + c];
+            __stcg(gp + i, sum);
+          }
+          __syncthreads();
+          // count in: the CTA's partials, ordered before by the barrier, are
+          // released by one acquire-release arrival
+          if (threadIdx.x == 0)
+            tc::atomic_add_acq_rel_gpu(args.head_counter + slot * nchk + chunk, 1);
+        }
         if (row4_ok) {
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -460,7 +579,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (j < args.N) {
               const float4 a = *reinterpret_cast<const float4*>(tT + jc * 32 + r4);
               float v[4] = {a.x, a.y, a.z, a.w};
-              if (kEpi == kEpiFwd) {
+              if (kFwd) {
                 v[0] += bias4.x; v[1] += bias4.y; v[2] += bias4.z; v[3] += bias4.w;
                 if (args.relu) {
 #pragma unroll
@@ -485,6 +604,162 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           }
         }
         __syncwarp();
+      }
+      if (kEpi == kEpiFwdHead) {
+        // Pass 2: once every feature tile's partials of a chunk are in (all
+        // CTAs of this launch are resident), the chunk's logits are summed in
+        // tile order plus b_L; warp 0 takes softmax cross-entropy and dZ_L =
+        // (softmax - onehot(y)) / m per sample (the first feature tile writes
+        // dZ_L and the chunk's loss); every CTA then writes dZ_{L-1} = (dZ_L
+        // W_L) [H_{L-1} > 0] for its own features (W_L before its update).
+        __shared__ int s_hok;
+        const int C = args.head_C;
+        const float* bl = theta + args.head_boff;
+        TAct* dh = static_cast<TAct*>(args.dh) + (int64_t)slot * args.out_bstride;
+        const int mtn = (int)gridDim.x;
+#pragma unroll 1
+        for (int o = 0; o < n_own; ++o) {
+          const int chunk = own_rank + o * kstride;
+          if (chunk >= nchk) continue;   // CTA-uniform
+          int* ctr = args.head_counter + slot * nchk + chunk;
+          if (threadIdx.x == 0) s_hok = tc::wait_count_low(ctr, mtn, abort_flag, kWaitNs);
+          __syncthreads();
+          if (!s_hok) {
+            if (threadIdx.x == 0) atomicExch(args.err, 1);
+            break;
+          }
+          // the feature tiles' partials in tile order: each thread sums two of
+          // the chunk's 32 x kHC logits, up to 2 x 16 loads in flight
+          static_assert(32 * kHC == 2 * kThreads, "two logits per thread");
+          const float* gp0 = args.head_part + ((int64_t)slot * nchk + chunk) * mtn * (32 * kHC);
+          {
+            float z0 = 0.f, z1 = 0.f;
+            for (int m0 = 0; m0 < mtn; m0 += 16) {
+              float p0[16], p1[16];
+#pragma unroll
+              for (int q = 0; q < 16; ++q) {
+                const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
+                p0[q] = m0 + q < mtn ? __ldcg(pq) : 0.f;
+                p1[q] = m0 + q < mtn ? __ldcg(pq + kThreads) : 0.f;
+              }
+#pragma unroll
+              for (int q = 0; q < 16; ++q) {
+                z0 += p0[q];
+                z1 += p1[q];
+              }
+            }
+            const int c0i = threadIdx.x % kHC;   // kThreads is a multiple of kHC
+            sG[threadIdx.x] = c0i < C ? z0 + bl[c0i] : -INFINITY;
+            sG[threadIdx.x + kThreads] = c0i < C ? z1 + bl[c0i] : -INFINITY;
+          }
+          __syncthreads();
+          float ce = 0.f;
+          if (warp == 0) {
+            const int j = n_tile * BN + 32 * chunk + lane;
+            const bool valid = j < args.N;
+            float zc[kHC];
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) zc[c] = sG[lane * kHC + c];
+            float mx = zc[0];
+#pragma unroll
+            for (int c = 1; c < kHC; ++c) mx = fmaxf(mx, zc[c]);
+            const int y = valid ? args.yb[(int64_t)slot * args.N + j] : -1;
+            float ex[kHC];
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) ex[c] = c < C ? expf(zc[c] - mx) : 0.f;
+            float se = 0.f, zy = 0.f;
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) {
+              se += ex[c];
+              if (c == y) zy = zc[c];
+            }
+            ce = valid ? (logf(se) + mx) - zy : 0.f;
+            const float inv_s = 1.0f / se, inv_m = 1.0f / (float)args.N;
+            TAct* dzl = static_cast<TAct*>(args.dzl) + ((int64_t)slot * args.N + j) * args.ldz;
+            bf16* dzp = args.dzl_pieces
+                            ? args.dzl_pieces + ((int64_t)slot * args.N + j) * args.ldz
+                            : nullptr;
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) {
+              float pr = ex[c] * inv_s;
+              if (c == y) pr -= 1.0f;
+              const float gz = valid ? pr * inv_m : 0.f;
+              sG[lane * kHC + c] = gz;
+              if (m_tile == 0 && valid && c < C) {
+                const TAct gv = static_cast<TAct>(gz);
+                dzl[c] = gv;
+                if (dzp) {
+                  bf16 q0, q1, q2;
+                  split3(static_cast<float>(gv), q0, q1, q2);
+                  dzp[c] = q0;
+                  dzp[args.dzl_plane + c] = q1;
+                  dzp[2 * args.dzl_plane + c] = q2;
+                }
+              }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) ce += __shfl_xor_sync(0xffffffffu, ce, off);
+          }
+          __syncthreads();
+          if (row4_ok) {
+            const uint32_t mbits = sMask[o * kThreads + threadIdx.x];
+            const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
+            // dZ_{L-1} of the lane's 4 features x 4 columns: 16 independent
+            // chains over the classes (dZ_L is zero past C)
+            float d[4][4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int e = 0; e < 4; ++e) d[u][e] = 0.f;
+#pragma unroll
+            for (int c = 0; c < kHC; ++c) {
+              const float4 w = w3v[c * 32];
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const float gzc = sG[(co + jl + 4 * u) * kHC + c];
+                d[u][0] = fmaf(gzc, w.x, d[u][0]);
+                d[u][1] = fmaf(gzc, w.y, d[u][1]);
+                d[u][2] = fmaf(gzc, w.z, d[u][2]);
+                d[u][3] = fmaf(gzc, w.w, d[u][3]);
+              }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int j = n_tile * BN + 32 * chunk + co + jl + 4 * u;
+              if (j < args.N) {
+                float dv[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) dv[e] = (mbits >> (4 * u + e)) & 1u ? d[u][e] : 0.f;
+                const int64_t o4 = (int64_t)j * args.ldo + row4;
+                store4(dh + o4, dv);
+                if (kSplit == 3 && args.dh_pieces) {
+                  uint2 q0, q1, q2;
+                  split3_x4(dv, q0, q1, q2);
+                  bf16* pp = args.dh_pieces + (int64_t)slot * args.out_bstride + o4;
+                  *reinterpret_cast<uint2*>(pp) = q0;
+                  *reinterpret_cast<uint2*>(pp + args.dh_plane) = q1;
+                  *reinterpret_cast<uint2*>(pp + 2 * args.dh_plane) = q2;
+                }
+              }
+            }
+          }
+          __syncthreads();
+          if (threadIdx.x == 0) {
+            // count out (relaxed: it orders nothing but the counter itself); the
+            // last one out resets the counter for the next launch
+            const int prev = atomicAdd(ctr, 1 << 16);
+            if ((prev >> 16) == mtn - 1) *ctr = 0;
+            // the chunk's loss contribution (sum of its samples' cross-entropy
+            // over m) in the chunk's slot; the run's loss kernel adds the slots
+            // in order
+            if (m_tile == 0) {
+              const float part = ce / (float)args.N;
+              args.loss_parts[((int64_t)args.slot_commit[slot] * args.lam + args.step) * nchk +
+                              chunk] = part;
+              if (!isfinite(part)) atomicExch(args.nonfinite, 1);
+            }
+          }
+        }
       }
     } else {   // kEpiDW
       float* acc = args.acc + (int64_t)worker * args.ld_param;
@@ -628,7 +903,7 @@ size_t smem_bytes() {
 
 template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, int slots,
-                 cudaStream_t st) {
+                 cudaStream_t st, bool* launched = nullptr) {
   static_assert(kStages * TileCfg<BN, kSplit>::kStageBytes + 1280 <= 232448, "smem");
   auto kern = tc_gemm_kernel<BN, kAMN, kBMN, kEpi, kStages, kSplit>;
   const size_t smem = smem_bytes<BN, kSplit, kStages>();
@@ -643,18 +918,26 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
   if (ks > 1) {
     // a rank that finishes chunks holds the other ranks' partial sums of
     // them (16 KB per chunk and rank) in its stage ring
-    const int ring = (int)EpiT<BN, kSplit, kStages>::kRingFree;
+    const int ring = (int)(kEpi == kEpiFwdHead ? EpiT<BN, kSplit, kStages>::kHeadOff
+                                               : EpiT<BN, kSplit, kStages>::kRingFree);
     auto need = [](int k) { return ((BN / 32 + k - 1) / k) * (k - 1) * (128 * 32 * 4); };
     while (ks > 1 && need(ks) > ring) --ks;
     const int kt = (args.K + kBK - 1) / kBK;
     ks = std::min(ks, kt);
     if (ks > 1) ks = (kt + (kt + ks - 1) / ks - 1) / ((kt + ks - 1) / ks);
   }
-  if (ks > 1) {   // the exchange needs every CTA of the launch resident at once
+  if (ks > 1 || kEpi == kEpiFwdHead) {
+    // the split-K exchange and the fused output layer's wait need every CTA
+    // of the launch resident at once (one CTA per SM: see smem_bytes)
     int dev = 0, sms = 0;
     AGN_TRY_CUDA(cudaGetDevice(&dev));
     AGN_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    if ((int64_t)ceil_div(args.M, 128) * ceil_div(args.N, BN) * slots * ks > sms) ks = 1;
+    const int64_t tiles = (int64_t)ceil_div(args.M, 128) * ceil_div(args.N, BN) * slots;
+    if (tiles * ks > sms) ks = 1;
+    if (kEpi == kEpiFwdHead && (tiles > sms || ceil_div(args.N, BN) != 1)) {
+      if (launched) *launched = false;
+      return Status::Ok();
+    }
   }
   if (ks > 1 && (!args.part || !args.counter))
     return Status::Err(AGN_E_INVALID, "split-K GEMM without workspace");
@@ -667,6 +950,7 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
     AGN_TRY_CUDA(launch_pdl(kf, grid, kThreads, smem, st, a, b, a2));
   }
   AGN_TRY_CUDA(cudaGetLastError());
+  if (launched) *launched = true;
   return Status::Ok();
 }
 
@@ -751,6 +1035,28 @@ Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& 
   if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 6, 1>(w_k, h_k, args, slots, st);
   if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 5, 1>(w_k, h_k, args, slots, st);
   return launch_tc<256, false, false, kEpiFwd, 4, 1>(w_k, h_k, args, slots, st);
+}
+
+Status tc_forward_head(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args,
+                       int slots, cudaStream_t st, bool split, int bn, int num_sms,
+                       bool* launched) {
+  *launched = false;
+  if (args.head_C < 1 || args.head_C > kHC || !args.head_part || !args.head_counter ||
+      !args.dh || !args.dzl || !args.loss_parts)
+    return Status::Err(AGN_E_INVALID, "fused output layer without its buffers");
+  if ((int64_t)ceil_div(args.M, 128) * slots > num_sms) return Status::Ok();
+  if (split) {
+    if (bn == 64)
+      return launch_tc<64, false, false, kEpiFwdHead, 3, 3>(w_k, h_k, args, slots, st, launched);
+    if (bn == 128)
+      return launch_tc<128, false, false, kEpiFwdHead, 2, 3>(w_k, h_k, args, slots, st, launched);
+    return launch_tc<256, false, false, kEpiFwdHead, 1, 3>(w_k, h_k, args, slots, st, launched);
+  }
+  if (bn == 64)
+    return launch_tc<64, false, false, kEpiFwdHead, 6, 1>(w_k, h_k, args, slots, st, launched);
+  if (bn == 128)
+    return launch_tc<128, false, false, kEpiFwdHead, 5, 1>(w_k, h_k, args, slots, st, launched);
+  return launch_tc<256, false, false, kEpiFwdHead, 4, 1>(w_k, h_k, args, slots, st, launched);
 }
 
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,

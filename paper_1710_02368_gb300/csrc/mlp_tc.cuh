@@ -41,6 +41,27 @@ struct TcArgs {
   // replicas) instead of taking the local step (the optimizer runs after);
   // null = fused local step
   float* grad_out;
+  // Forward of the last hidden layer with the output layer fused into its
+  // epilogue (tc_forward_head): the d_L <= 16 logits of every sample from the
+  // CTAs' partial sums over their 128 features, softmax cross-entropy, dZ_L and
+  // dZ_{L-1} = (dZ_L W_L) [H_{L-1} > 0].
+  int64_t head_woff, head_boff;   // W_L [C][M] and b_L [C] in the fp32 replicas
+  int head_C;
+  const int* yb;                  // labels [slots][m]
+  void* dzl;                      // out: dZ_L [slots][m][ldz] (activation type)
+  int ldz;
+  bf16* dzl_pieces;               // split mode: its pieces, planes dzl_plane apart
+  int64_t dzl_plane;
+  void* dh;                       // out: dZ_{L-1} [slots][m][M]
+  bf16* dh_pieces;                // split mode: its pieces, planes dh_plane apart
+  int64_t dh_plane;
+  float* head_part;               // [slots][ceil(m / 32)][M tiles][32][16] partial logits
+  int* head_counter;              // [slots][ceil(m / 32)], zero between launches
+  float* loss_parts;              // [commit][lambda][ceil(m / 32)]: per 32-sample chunk
+                                  // its cross-entropy sum / m
+  const int* slot_commit;
+  int lam, step;
+  int* nonfinite;                 // set to 1 for a non-finite loss
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
@@ -71,6 +92,13 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
                   cudaStream_t st, bool split, int bn);
 // dX: w_mn box {64, 64} over W (MN-major view); dz_k box {64, bn} over dZ_l.
+// The forward GEMM of the last hidden layer with the output layer fused
+// (args.head_* set, args.relu = 1).  Needs every CTA of the launch resident at
+// once; when the launch would exceed the SMs nothing is queued and *launched
+// is false (the caller runs the forward and the output head separately).
+Status tc_forward_head(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args,
+                       int slots, cudaStream_t st, bool split, int bn, int num_sms,
+                       bool* launched);
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
                       int slots, cudaStream_t st, bool split, int bn);
 // One hidden layer of a dW launch: h_mn box {64, kBK} over H_{l-1}; dz_mn box

@@ -8,9 +8,15 @@ Tolerance.  theta~ within 1e-5 relative L2 of the float64 oracle after each
 checked commit, except where float32 arithmetic itself has left 1e-5 of the
 float64 trajectory: the oracle is also run in float32 (NumPy single
 precision, the same algorithm), and the bound is max(1e-5, 3 x that run's
-own deviation from float64) at the checked commit.  Per-commit losses and
-||Delta_c|| likewise: 1e-5 relative, or 3x the float32 run's largest
-deviation so far.
+own deviation from float64) at the checked commit.  Per-commit losses
+likewise: 1e-5 relative, or 3x the float32 run's largest deviation so far.
+||Delta_c|| within 2e-3 relative (or 3x the float32 run's largest
+deviation so far, where that is larger): a ReLU decision at a pre-activation
+within float32 rounding of zero can flip (differently in every float32
+summation order, the CUDA-core kernels and the float32 oracle included),
+which changes one sample's term of the minibatch gradient; measured on the
+16-worker workload, such flips move ||Delta_c|| of single commits by up to
+9e-4 relative on every GEMM path while theta~ stays within 5e-6.
 """
 
 import numpy as np
@@ -23,6 +29,7 @@ from agn_inputs import workloads as WL
 pytestmark = pytest.mark.gpu
 
 REL_STEP = 1e-5
+REL_DELTA_NORM = 2e-3
 
 
 @pytest.fixture(scope="module")
@@ -72,7 +79,8 @@ def _check(wl, bounds, h, w, tau, r64, r32):
     d, bnd = _envelope(h.loss(), r64.loss, r32.loss)
     assert np.all(d <= bnd), (int(np.argmax(d - bnd)), float(np.max(d)))
     d, bnd = _envelope(h.delta_norm(), r64.delta_norm, r32.delta_norm)
-    assert np.all(d <= bnd), (int(np.argmax(d - bnd)), float(np.max(d)))
+    bnd = np.maximum(bnd, REL_DELTA_NORM * r64.delta_norm)
+    assert np.all(d <= bnd), (int(np.argmax(d / bnd)), float(np.max(d / r64.delta_norm)))
     return C / waves
 
 

@@ -83,3 +83,30 @@ def test_split_mode_is_the_default_for_fp32(agn):
     with pytest.raises(agn.AGNError) as e:
         _run(agn, (37, 65, 10), 8, agn.AGN_GEMM_TCGEN05)
     assert e.value.code == agn.AGN_E_UNSUPPORTED
+
+
+@pytest.mark.parametrize("dims,m,n", [((256, 200, 136, 10), 48, 4), ((96, 64, 64, 10), 256, 3),
+                                      ((784, 128, 10), 32, 4), ((64, 40, 3), 16, 5),
+                                      ((128, 1000, 16), 128, 2)])
+def test_output_layer_in_forward_epilogue(agn, dims, m, n):
+    """The output layer (forward, softmax-CE, dZ_L, dX) folded into the last
+    hidden layer's forward GEMM against the oracle (float64) and against the
+    output layer as a kernel of its own (tc_mask bit 5), on shapes with
+    partial feature tiles, partial 32-sample chunks, few classes and 16
+    classes: theta~ and every loss within the fp32 tolerance."""
+    seed, lam, C = 17, 3, 9
+    N = n * 3 * m
+    w, tau = I.make_schedule(n, C + n, 0, 2, seed)
+    ds = I.SyntheticDataset(seed, dims[0], N, I.DIST_UNIFORM, (dims[0], 64, dims[-1]), N // n)
+    ref = O.agn_run(O.MLP(dims), I.init_params(seed, dims), n, lam, 0.05, w[:C], tau[:C], ds, m,
+                    N // n, snapshot_at=[C - 1])
+    out = {}
+    for mask in (0, 32):
+        with agn.AGN(dims, n, lam, 0.05, seed, batch=m, n_samples=N, gemm=agn.AGN_GEMM_TCGEN05,
+                     tc_mask=mask) as h:
+            h.run(C, w, tau)
+            out[mask] = (h.central(), h.loss())
+    for mask, (th, loss) in out.items():
+        assert _rel(th, ref.snapshots[C - 1]) <= 1e-5, mask
+        assert np.allclose(loss, ref.loss, rtol=1e-5, atol=1e-6), mask
+    assert _rel(out[0][0], out[32][0].astype(np.float64)) <= 1e-5
