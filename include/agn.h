@@ -363,6 +363,20 @@ int agn_commit_pull_noalloc(float* theta_c, float* acc, float* replicas, void* r
                             int32_t normalize, float* delta_norm, void* stream);
 
 /*
+ * Test hook of the failure path of the bounded device waits (the paper has no
+ * counterpart).  The tensor-core GEMMs' split-K exchange and the fused output
+ * layer wait, on the device, for the other CTAs of their launch; every such
+ * wait gives up after a time limit, the kernel then returns without its
+ * results and agn_run reports AGN_E_TIMEOUT.  wait_ns > 0 sets that limit for
+ * this handle's later runs (0 = the default, 2 s); withhold_rank >= 0 makes
+ * split-K rank withhold_rank of every split-K launch skip its arrival on the
+ * tile counter, so that the ranks waiting for it give up after wait_ns
+ * (-1 = none).  After a run that timed out, the handle's results are not
+ * valid: destroy it.  Errors: AGN_E_INVALID.
+ */
+int agn_debug_waits(agn_handle* h, int64_t wait_ns, int32_t withhold_rank);
+
+/*
  * Fill the inputs of the standalone commit workload on the device with the
  * seeded generator: theta_c[i] = fp32(N(0,1) number i of the commit-theta
  * stream); acc[k][i] = fp32(0.1 * N(0,1) number k*P + i of the commit-acc

@@ -26,7 +26,7 @@ __all__ = [
     "agn_last_run_stats", "agn_profile", "agn_kernel_stats", "agn_generate_inputs", "agn_export_inputs", "agn_last_error",
     "agn_destroy", "agn_make_schedule", "agn_plan_waves", "agn_commit_pull",
     "agn_commit_pull_noalloc",
-    "agn_fill_commit_inputs",
+    "agn_fill_commit_inputs", "agn_debug_waits",
     "library_path",
 ]
 
@@ -158,9 +158,10 @@ def agn_num_commits(h) -> int:
 
 
 def agn_last_run_stats(h) -> dict:
-    out = (C.c_double * 4)()
-    _check(_L().agn_last_run_stats(h, out, 4), h)
-    return {"waves": out[0], "launches": out[1], "gpu_ms": out[2], "worker_steps": out[3]}
+    out = (C.c_double * 5)()
+    _check(_L().agn_last_run_stats(h, out, 5), h)
+    return {"waves": out[0], "launches": out[1], "gpu_ms": out[2], "worker_steps": out[3],
+            "host_ms": out[4]}
 
 
 def agn_profile(h, mode):
@@ -269,6 +270,12 @@ def agn_commit_pull_noalloc(theta_c, acc, replicas, replicas_bf16, P, ld, n, com
         _ptr(theta_c), _ptr(acc), _ptr(replicas), _ptr(replicas_bf16), int(P), int(ld), int(n),
         len(cw), cwp, pop, pwp, float(eta), int(lam), int(normalize), _ptr(delta_norm),
         _ptr(stream)))
+
+
+def agn_debug_waits(h, wait_ns, withhold_rank=-1):
+    """Test hook: bound the device waits of later runs by wait_ns (0 = 2 s) and
+    make one split-K rank withhold its arrival (-1 = none)."""
+    _check(_L().agn_debug_waits(h, int(wait_ns), int(withhold_rank)), h)
 
 
 def agn_fill_commit_inputs(theta_c, acc, replicas, P, ld, n, seed, stream=None):

@@ -110,6 +110,7 @@ SIGNATURES = {
                                           C.c_int64, C.c_int64, C.c_int32, C.c_int32, _I32P,
                                           _I32P, _I32P, C.c_double, C.c_int32, C.c_int32,
                                           C.c_void_p, C.c_void_p]),
+    "agn_debug_waits": (C.c_int, [C.c_void_p, C.c_int64, C.c_int32]),
     "agn_fill_commit_inputs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64,
                                          C.c_int64, C.c_int32, C.c_uint64, C.c_void_p]),
 }

@@ -19,6 +19,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "host_inputs.h"
 #include "mlp.cuh"
 #include "mlp_tc.cuh"
@@ -42,6 +44,12 @@ struct DeviceGuard {
     int cur = -1;
     if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
   }
+};
+
+// NVTX range for the duration of a scope (a no-op without a tool attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
 };
 
 struct Wave {
@@ -147,6 +155,9 @@ struct agn_handle {
   // output layer writes one per 32-sample chunk, the other paths the step's
   // loss in the first and zeros after it
   int loss_q = 1;
+  // test hook of the bounded waits (agn_debug_waits)
+  uint64_t dbg_wait_ns = 0;
+  int dbg_withhold = 0;
   int grid = 0;
   float* loss = nullptr;      // [cap_commits]
   float* dnorm = nullptr;     // [cap_commits]
@@ -300,6 +311,8 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.theta_b = h->rep_b;
   t.ld_param = h->P_pad;
   t.piece_plane = h->piece_plane;
+  t.wait_ns = h->dbg_wait_ns;
+  t.withhold_rank = h->dbg_withhold;
   return t;
 }
 
@@ -813,8 +826,12 @@ Status build_plan(const agn_handle* h, int k, const int32_t* worker, const int32
 
 Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, int ns) {
   const auto t_host0 = std::chrono::steady_clock::now();
+  NvtxRange run_range("agn_run");
   RunPlan plan;
-  AGN_TRY(build_plan(h, k, worker, tau, ns, &plan));
+  {
+    NvtxRange r("plan waves");
+    AGN_TRY(build_plan(h, k, worker, tau, ns, &plan));
+  }
   const int64_t V0 = h->V;
   const int64_t total_slots = (int64_t)plan.slot_worker.size();
   if (V0 + k > h->cap_commits) {   // loss and dnorm share one capacity
@@ -858,8 +875,13 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   const float scale = steps ? (float)(h->normalize ? 1.0 / (double)h->lam : 1.0)
                             : (float)(h->normalize ? -(h->eta / (double)h->lam) : -h->eta);
   for (const Wave& wv : plan.waves) {
-    if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
-    else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
+    NvtxRange wave_range("wave");
+    {
+      NvtxRange r("local steps");
+      if (h->prec == AGN_PREC_BF16) AGN_TRY(run_wave_steps<bf16>(h, wv, &launches));
+      else AGN_TRY(run_wave_steps<float>(h, wv, &launches));
+    }
+    NvtxRange commit_range("commit + pull");
     for (const CommitPlan& cp : wv.commits) {
       const double pulls = cp.pull_begin[cp.n_commits];
       {
@@ -1591,6 +1613,15 @@ int agn_commit_pull(float* theta_c, float* acc, float* replicas, void* replicas_
                          pull_offsets, pull_workers, eta, lambda, normalize, delta_norm,
                          static_cast<cudaStream_t>(stream));
   return s.ok() ? AGN_OK : fail(nullptr, s);
+}
+
+int agn_debug_waits(agn_handle* h, int64_t wait_ns, int32_t withhold_rank) {
+  if (!h) return fail(nullptr, AGN_E_INVALID, "null handle");
+  if (wait_ns < 0 || wait_ns > 2000000000ll || withhold_rank < -1 || withhold_rank > 65534)
+    return fail(h, AGN_E_INVALID, "wait_ns must be in [0, 2e9], withhold_rank >= -1");
+  h->dbg_wait_ns = (uint64_t)wait_ns;
+  h->dbg_withhold = withhold_rank + 1;
+  return AGN_OK;
 }
 
 int agn_fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P, int64_t ld,

@@ -405,10 +405,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       __syncthreads();
       if (threadIdx.x == 0) {
         int* ctr = args.counter + tile_id;
-        tc::atomic_add_acq_rel_gpu(ctr, 1);
+        if (sk + 1 != args.withhold_rank) tc::atomic_add_acq_rel_gpu(ctr, 1);
         bool got = true;
         if (n_own > 0) {
-          got = tc::wait_count_low(ctr, ks, abort_flag, kWaitNs);
+          got = tc::wait_count_low(ctr, ks, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
           if (got) {
             tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
             tc::mbar_arrive_expect_tx(red, kChunkBytes * (uint32_t)(n_own * (ks - 1)));
@@ -622,7 +622,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           const int chunk = own_rank + o * kstride;
           if (chunk >= nchk) continue;   // CTA-uniform
           int* ctr = args.head_counter + slot * nchk + chunk;
-          if (threadIdx.x == 0) s_hok = tc::wait_count_low(ctr, mtn, abort_flag, kWaitNs);
+          if (threadIdx.x == 0)
+            s_hok = tc::wait_count_low(ctr, mtn, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
           __syncthreads();
           if (!s_hok) {
             if (threadIdx.x == 0) atomicExch(args.err, 1);

@@ -62,6 +62,12 @@ struct TcArgs {
   const int* slot_commit;
   int lam, step;
   int* nonfinite;                 // set to 1 for a non-finite loss
+  // Test hook of the bounded waits (agn_debug_waits): wait_ns > 0 bounds the
+  // split-K and output-layer waits by that many nanoseconds instead of 2 s;
+  // withhold_rank = r + 1 makes split-K rank r withhold its arrival on the
+  // tile counter (0 = none), so that the ranks waiting for it give up.
+  uint64_t wait_ns;
+  int withhold_rank;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N

@@ -148,3 +148,12 @@ def test_commit_pull_rejects_pulls_without_buffers_before_reading_them(agn, entr
     assert rc == agn.AGN_E_INVALID and "pulls need replicas" in agn.agn_last_error()
     rc = fn(fake, fake, None, None, 64, 64, 2, 1, cw, po, pw, 0.01, 10, 1, None, None)
     assert rc == agn.AGN_E_INVALID and "pulls need replicas" in agn.agn_last_error()
+
+
+def test_debug_waits_validates_its_arguments(agn):
+    """The bounded-wait test hook rejects a null handle and out-of-range values
+    before touching anything."""
+    import ctypes as C
+    from paper_1710_02368_gb300 import _lib
+    lib = _lib.load()
+    assert lib.agn_debug_waits(None, 1000, 0) == agn.AGN_E_INVALID
