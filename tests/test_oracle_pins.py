@@ -557,6 +557,36 @@ def test_adam_first_step_is_eta_times_the_gradient_sign():
     assert np.allclose(r.theta - theta, -eta * gr / (np.abs(gr) + eps), rtol=0, atol=1e-15)
 
 
+def _adam_golden_rows():
+    rows = []
+    with open(os.path.join(GOLDEN, "adam_scalar_examples.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                lam, nc, val = line.split()
+                rows.append((int(lam), int(nc), Fraction(val)))
+    return rows
+
+
+@pytest.mark.parametrize("lam,n_commits,expect", _adam_golden_rows())
+def test_adam_hand_worked_two_steps(lam, n_commits, expect):
+    """Two Adam steps worked by hand in exact rationals (the bias corrections
+    at t = 1 and t = 2, moments kept across a commit): the oracle within a few
+    roundings of the exact value."""
+    lsq = O.LeastSquares(1, 1)
+    data = _ListData(np.array([[1.0]]), np.array([[0.0]]))
+
+    class WOnly:
+        num_params = 1
+
+        def loss_grad(self, theta, X, Y):
+            loss, g = lsq.loss_grad(np.array([theta[0], 0.0]), X, Y)
+            return loss, g[:1]
+    r = O.agn_run(WOnly(), np.array([1.0]), 1, lam, 0.5, [0] * n_commits, [0] * n_commits,
+                  data, 1, 1, optimizer="adam", adam=(0.5, 11 / 64, 0.0))
+    assert abs(Fraction(float(r.theta[0])) - expect) <= Fraction(1, 2 ** 48)
+
+
 def test_adam_moments_persist_across_commits():
     """An independent loop: moments per worker, bias corrections at the
     worker's step count, staleness as scheduled."""
