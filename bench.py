@@ -493,6 +493,29 @@ def workload_record(args, wl, r, per_step, ws, hbm, bf16, peak_src):
     return rec
 
 
+def commit_sizes(args):
+    """P values of the standalone commit workload (all four by default)."""
+    if args.commit_log2p:
+        return [1 << int(v) for v in args.commit_log2p.split(",")]
+    return list(WL.COMMIT_PULL.sizes)
+
+
+def run_commit_only(args):
+    """Only the standalone commit+pull kernel (profiler captures of small P)."""
+    import torch
+    import paper_1710_02368_gb300 as agn
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    hbm, _, _, _ = _peaks()
+    out = {}
+    for P in commit_sizes(args):
+        cr = commit_kernel_bench(agn, torch, dev, P)
+        cr["frac_of_measured_hbm"] = cr["GB/s"] / hbm
+        out[str(P)] = cr
+    print(json.dumps({"commit_pull_kernel": out}), flush=True)
+    return 0
+
+
 def run_agn(args, wl):
     import torch
     import paper_1710_02368_gb300 as agn
@@ -521,7 +544,7 @@ def run_agn(args, wl):
     commit = None
     if rank == 0 and not args.no_commit_bench:
         commit = {}
-        for P in WL.COMMIT_PULL.sizes:
+        for P in commit_sizes(args):
             cr = commit_kernel_bench(agn, torch, dev, P)
             cr["frac_of_measured_hbm"] = cr["GB/s"] / hbm
             commit[str(P)] = cr
@@ -575,6 +598,10 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-commit-bench", action="store_true")
+    ap.add_argument("--commit-log2p", default="",
+                    help="comma-separated log2 P of the commit kernel runs (default: 20,24,26,28)")
+    ap.add_argument("--commit-only", action="store_true",
+                    help="time only the standalone commit+pull kernel")
     ap.add_argument("--no-sub-workloads", action="store_true",
                     help="time only the headline workload (not the two bf16 workloads)")
     args = ap.parse_args()
@@ -589,6 +616,8 @@ def main():
                                  tau_hi=min(wl.tau_hi, args.workers - 1))
     if args.impl == "reference":
         return run_reference(args, wl)
+    if args.commit_only:
+        return run_commit_only(args)
     return run_agn(args, wl)
 
 
