@@ -132,6 +132,7 @@ struct agn_handle {
   int* tc_counter = nullptr;    // split-K arrival count per output tile: [SMs]
   std::vector<LayerMaps> tmaps;
   LayerMaps out_maps;
+  LayerMaps l1_alt;               // layer 1's maps over the alternate operand buffer
   // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
   bool split = false;
   int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
@@ -155,6 +156,13 @@ struct agn_handle {
   // output layer writes one per 32-sample chunk, the other paths the step's
   // loss in the first and zeros after it
   int loss_q = 1;
+  // the gather copies a local step's minibatch before waiting for the
+  // preceding kernel: the layer-1 operand the tensor-core kernels read
+  // alternates between two buffers by local step (gparity)
+  bool early_gather = false;
+  int gparity = 0;
+  void* Xb_alt = nullptr;         // bf16 mode: [n][m][d0]
+  bf16* Hs0_alt = nullptr;        // fp32 mode: pieces [3][n][m][d0]
   // test hook of the bounded waits (agn_debug_waits)
   uint64_t dbg_wait_ns = 0;
   int dbg_withhold = 0;
@@ -355,6 +363,23 @@ Status build_tc_maps(agn_handle* h) {
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
   }
+  if (h->early_gather) {   // layer 1's operand maps over the alternate buffer
+    const uint64_t fi = h->dims[0];
+    h->l1_alt = h->tmaps[0];
+    auto& mp = h->l1_alt;
+    if (h->split) {
+      const uint64_t hp = (uint64_t)n * m * fi;
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp, 64,
+                                     bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp, 64,
+                                     64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp,
+                                     64, 32));
+    } else {
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k, h->Xb_alt, fi, m, n, fi, (uint64_t)m * fi, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_mn, h->Xb_alt, fi, m, n, fi, (uint64_t)m * fi, 64, 64));
+    }
+  }
   if (h->fuse_out_dw) {   // the output layer's dW tiles: M = d_{L-1} inputs, N = d_L
     const uint64_t fi = h->dims[L - 1], fo = h->dims[L], lz = (uint64_t)h->ldz_out;
     auto& mp = h->out_maps;
@@ -429,15 +454,25 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   };
   auto dz_plane = [&](int l) -> int64_t { return (int64_t)n * m * h->dims[l]; };
   for (int i = 0; i < h->lam; ++i) {
+    // this local step's buffer of layer 1's tensor-core operand
+    const bool alt = h->early_gather && h->gparity;
+    const agn_handle::LayerMaps& l1 = alt ? h->l1_alt : h->tmaps.empty() ? h->l1_alt : h->tmaps[0];
+    auto maps_of = [&](int l) -> const agn_handle::LayerMaps& { return l == 1 ? l1 : h->tmaps[l - 1]; };
     {
+      // fp32 mode with the early gather: the fp32 rows are not read by the
+      // tensor-core kernels, only their pieces
+      T* xb = h->early_gather ? (h->split ? nullptr : static_cast<T*>(alt ? h->Xb_alt : h->Xb))
+                              : static_cast<T*>(h->Xb);
       Launch k(h, AGN_K_GATHER, 0.0,
-               (double)s * m * (2.0 * h->dims[0] * es + 8.0 + (h->split ? 6.0 * h->dims[0] : 0.0)),
+               (double)s * m * ((xb ? 2.0 : 1.0) * h->dims[0] * es + 8.0 +
+                                (h->split ? 6.0 * h->dims[0] : 0.0)),
                launches);
-      AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, static_cast<T*>(h->Xb),
-                                   h->yb, h->dims[0], m, h->S, sw, st0, i, s, h->stream,
-                                   h->split ? h->Hs[0] : nullptr,
-                                   (int64_t)n * m * h->dims[0]));
+      AGN_TRY(agn::gather_batch<T>(static_cast<const T*>(h->X), h->y, xb, h->yb, h->dims[0], m,
+                                   h->S, sw, st0, i, s, h->stream,
+                                   h->split ? (alt ? h->Hs0_alt : h->Hs[0]) : nullptr,
+                                   (int64_t)n * m * h->dims[0], h->early_gather ? 1 : 0));
     }
+    if (h->early_gather) h->gparity ^= 1;
     bool dz_ready = false;   // pieces of the next layer's dZ already written by its producer
     // the output layer rides in the last hidden layer's forward when that
     // launch's CTAs fit the SMs at once
@@ -517,7 +552,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.head_part = h->fh_part; t.head_counter = h->fh_counter;
           t.loss_parts = h->loss_parts; t.slot_commit = sc; t.lam = h->lam; t.step = i;
           t.nonfinite = h->flag;
-          const auto& mp = h->tmaps[l - 1];
+          const auto& mp = maps_of(l);
           t.ksplit = pick_ksplit(h, fo, fi, s);
           bool launched = false;
           AGN_TRY(agn::tc_forward_head(mp.w_k, mp.h_k, t, s, h->stream, h->split,
@@ -533,7 +568,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
           t.relu = 1; t.boff = h->boff[l - 1];
           t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
-          const auto& mp = h->tmaps[l - 1];
+          const auto& mp = maps_of(l);
           t.ksplit = pick_ksplit(h, fo, fi, s);
           AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split, agn::tc_bn(m)));
           pieces_done = true;
@@ -616,7 +651,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
                                    h->rep_b, h->P_pad, h->boff[l - 1], eta, s, h->stream,
                                    h->split, h->piece_plane));
         } else {
-          const auto& mp = h->tmaps[l - 1];
+          const auto& mp = maps_of(l);
           tc_dw.push_back({h->split ? &mp.h_mn32 : &mp.h_mn, h->split ? &mp.dz_mn32 : &mp.dz_mn,
                            &mp.theta, &mp.acc, fi, fo, h->woff[l - 1], h->boff[l - 1]});
           tc_flops += flops;
@@ -1112,6 +1147,14 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY(dalloc(h, &h->X, (size_t)h->N * d0 * es));
   AGN_TRY(dalloc_t(h, &h->y, (size_t)h->N));
   AGN_TRY(dalloc(h, &h->Xb, (size_t)(n * m * d0) * es));
+  // the gather may run ahead of the preceding kernel when every reader of
+  // layer 1's operand is a tensor-core kernel (forward and dW)
+  h->early_gather = h->use_tc && (h->tc_mask & 1) && (h->tc_mask & 4) && !(h->tc_mask & 8) &&
+                    h->L >= 2 && d0 % 4 == 0;
+  if (h->early_gather) {
+    if (h->split) AGN_TRY(dalloc_t(h, &h->Hs0_alt, (size_t)(3 * n * m * d0)));
+    else AGN_TRY(dalloc(h, &h->Xb_alt, (size_t)(n * m * d0) * es));
+  }
   AGN_TRY(dalloc_t(h, &h->yb, (size_t)(n * m)));
   h->H.assign(h->L, nullptr);
   for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->H[l], (size_t)(n * m * dims[l]) * es));

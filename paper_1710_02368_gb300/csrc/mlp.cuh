@@ -59,7 +59,8 @@ Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* l
 template <typename T>
 Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
-                    cudaStream_t st, bf16* pieces = nullptr, int64_t plane = 0);
+                    cudaStream_t st, bf16* pieces = nullptr, int64_t plane = 0,
+                    int early = 0);
 
 // Output layer fused (mlp_head.cu): forward, softmax cross-entropy and dX of
 // layer L for d_L <= kHeadMaxClasses; kHeadSamples samples per block.

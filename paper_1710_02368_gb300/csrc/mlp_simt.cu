@@ -280,14 +280,21 @@ __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y
 // The same gather, four consecutive elements per thread (d_0 a multiple of
 // 4): a block per minibatch row, one 16-byte (fp32) or 8-byte (bf16) load and
 // store per thread and group, and 8-byte piece stores.
+//
+// early = 1: the destination buffers are not read by the preceding kernel
+// (the tensor-core operand alternates between two buffers by local step, and
+// the labels' last reader finished before this launch could start), so the
+// rows are copied before waiting for the preceding kernel; the wait at the
+// end keeps this launch's completion ordered after it for the next kernel.
 template <typename T>
 __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
                                                       const int* __restrict__ y, T* Xb, int* yb,
                                                       int d0, int m, int64_t S,
                                                       const int* slot_worker,
                                                       const long long* slot_t0, int step,
-                                                      bf16* pieces, int64_t plane) {
-  pdl_begin();
+                                                      bf16* pieces, int64_t plane, int early) {
+  if (early) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  else pdl_begin();
   struct alignas(4 * sizeof(T)) Vec { T v[4]; };
   struct alignas(8) Piece4 { bf16 v[4]; };
   const int r = blockIdx.x;                 // slot * m + j
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
   const int64_t o = (int64_t)r * d0;
   for (int c = threadIdx.x * 4; c < d0; c += blockDim.x * 4) {
     const Vec v = *reinterpret_cast<const Vec*>(src + c);
-    *reinterpret_cast<Vec*>(Xb + o + c) = v;
+    if (Xb) *reinterpret_cast<Vec*>(Xb + o + c) = v;
     if (pieces) {
       Piece4 p0, p1, p2;
 #pragma unroll
@@ -311,6 +318,7 @@ __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
     }
   }
   if (threadIdx.x == 0) yb[r] = y[row];
+  if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 template <typename T, typename TO, bool kAK, bool kBK, int kEpi>
@@ -354,7 +362,7 @@ Status softmax_xent(const float* Z, const int* yb, T* dZ, int m, int C, float* l
 template <typename T>
 Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int64_t S,
                     const int* slot_worker, const long long* slot_t0, int step, int slots,
-                    cudaStream_t st, bf16* pieces, int64_t plane) {
+                    cudaStream_t st, bf16* pieces, int64_t plane, int early) {
   const bool vec = d0 % 4 == 0 && plane % 4 == 0 &&
                    ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(Xb) |
                      reinterpret_cast<uintptr_t>(pieces)) & 15) == 0;
@@ -364,9 +372,11 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
     {
       auto kf = gather4_kernel<T>;
       AGN_TRY_CUDA(launch_pdl(kf, slots * m, threads, 0, st, X,
-                              y, Xb, yb, d0, m, S, slot_worker, slot_t0, step, pieces, plane));
+                              y, Xb, yb, d0, m, S, slot_worker, slot_t0, step, pieces, plane,
+                              early));
     }
   } else {
+    if (early) return Status::Err(AGN_E_INVALID, "internal: early gather needs d_0 % 4 == 0");
     dim3 grid((unsigned)m, (unsigned)slots);
     {
       auto kf = gather_kernel<T>;
@@ -386,7 +396,7 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
                                   int, int, int*, int, cudaStream_t);                        \
   template Status gather_batch<T>(const T*, const int*, T*, int*, int, int, int64_t,          \
                                   const int*, const long long*, int, int, cudaStream_t,       \
-                                  bf16*, int64_t);
+                                  bf16*, int64_t, int);
 AGN_INST(float)
 AGN_INST(bf16)
 #undef AGN_INST
