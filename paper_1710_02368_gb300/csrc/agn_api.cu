@@ -129,7 +129,8 @@ struct agn_handle {
   // maps of the output layer's dW when it runs in the tensor-core dW launch
   // (theta, acc, h_mn / h_mn32 over H_{L-1}, dz_mn / dz_mn32 over dZ_L)
   float* tc_part = nullptr;     // split-K partial sums: [SMs][BN <= 256][128]
-  int* tc_counter = nullptr;    // split-K arrival count per output tile: [SMs]
+  int* tc_counter = nullptr;    // split-K arrival counts per output tile: [2][SMs]
+  int ctr_parity = 0;           // which half the next split-K launch counts in
   std::vector<LayerMaps> tmaps;
   LayerMaps out_maps;
   LayerMaps l1_alt;               // layer 1's maps over the alternate operand buffer
@@ -151,7 +152,8 @@ struct agn_handle {
   // (when the launch's CTAs fit the SMs at once): partial logits, counters
   bool fuse_head = false;
   float* fh_part = nullptr;       // [n][ceil(m / 32)][ceil(d_{L-1} / 128)][32][16]
-  int* fh_counter = nullptr;      // [n][ceil(m / 32)]
+  int* fh_counter = nullptr;      // [2][n][ceil(m / 32)]
+  int fh_parity = 0;
   // loss_parts holds loss_q values per local step of a commit: the fused
   // output layer writes one per 32-sample chunk, the other paths the step's
   // loss in the first and zeros after it
@@ -311,7 +313,7 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.slot_worker = sw;
   t.ksplit = 1;
   t.part = h->tc_part;
-  t.counter = h->tc_counter;
+  t.counter = nullptr;            // set per forward / dX launch (next_counters)
   t.err = h->flag + 1;
   t.theta = h->rep;
   t.acc = h->elide ? nullptr : h->acc;
@@ -322,6 +324,15 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw) {
   t.wait_ns = h->dbg_wait_ns;
   t.withhold_rank = h->dbg_withhold;
   return t;
+}
+
+// The split-K arrival counters of the next forward / dX launch: one half of
+// tc_counter, the other half (the previous launch's) cleared by its CTA 0.
+void next_counters(agn_handle* h, agn::TcArgs* t) {
+  t->counter = h->tc_counter + h->ctr_parity * h->num_sms;
+  t->counter_clear = h->tc_counter + (1 - h->ctr_parity) * h->num_sms;
+  t->counter_clear_n = h->num_sms;
+  h->ctr_parity ^= 1;
 }
 
 // Tensor maps of the tcgen05 path (addresses are fixed for the handle's life).
@@ -549,11 +560,19 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.dzl_pieces = (h->fuse_out_dw && h->split) ? h->dZp[L] : nullptr;
           t.dzl_plane = (int64_t)n * m * h->ldz_out;
           t.dh = h->dZ[L - 1]; t.dh_pieces = dz_pieces(L - 1); t.dh_plane = dz_plane(L - 1);
-          t.head_part = h->fh_part; t.head_counter = h->fh_counter;
+          t.head_part = h->fh_part;
+          {   // the fused output layer's counters alternate like the split-K ones
+            const int hn = n * (int)ceil_div(m, 32);
+            t.head_counter = h->fh_counter + h->fh_parity * hn;
+            t.head_counter_clear = h->fh_counter + (1 - h->fh_parity) * hn;
+            t.head_counter_clear_n = hn;
+            h->fh_parity ^= 1;
+          }
           t.loss_parts = h->loss_parts; t.slot_commit = sc; t.lam = h->lam; t.step = i;
           t.nonfinite = h->flag;
           const auto& mp = maps_of(l);
           t.ksplit = pick_ksplit(h, fo, fi, s);
+          next_counters(h, &t);
           bool launched = false;
           AGN_TRY(agn::tc_forward_head(mp.w_k, mp.h_k, t, s, h->stream, h->split,
                                        agn::tc_bn(m), h->num_sms, &launched));
@@ -570,6 +589,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
           const auto& mp = maps_of(l);
           t.ksplit = pick_ksplit(h, fo, fi, s);
+          next_counters(h, &t);
           AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split, agn::tc_bn(m)));
           pieces_done = true;
         } else {
@@ -613,6 +633,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         t.out_pieces = next_pieces; t.out_plane = dz_plane(l - 1);
         const auto& mp = h->tmaps[l - 1];
         t.ksplit = pick_ksplit(h, fi, fo, s);
+        next_counters(h, &t);
         AGN_TRY(agn::tc_backward_dx(mp.w_mn, mp.dz_k, t, s, h->stream, h->split,
                                     agn::tc_bn(m)));
         have_pieces[l - 1] = next_pieces != nullptr;
@@ -959,10 +980,12 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   if (flags[0] || flags[1]) {
     AGN_TRY_CUDA(cudaMemsetAsync(h->flag, 0, 2 * sizeof(int), h->stream));
     if (flags[1] && h->tc_counter)   // CTAs that gave up may have left tiles unfinished
-      AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)h->num_sms * sizeof(int), h->stream));
+      AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)(2 * h->num_sms) * sizeof(int),
+                                   h->stream));
     if (flags[1] && h->fuse_head) {
       AGN_TRY_CUDA(cudaMemsetAsync(h->fh_counter, 0,
-                                   (size_t)(h->n * ceil_div(h->m, 32)) * sizeof(int), h->stream));
+                                   (size_t)(2 * h->n * ceil_div(h->m, 32)) * sizeof(int),
+                                   h->stream));
     }
     AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
     if (flags[1])
@@ -1189,8 +1212,9 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (h->fuse_head) {
     const int64_t nchk = ceil_div(m, 32), mt = ceil_div(dims[h->L - 1], 128);
     AGN_TRY(dalloc_t(h, &h->fh_part, (size_t)(n * nchk * mt * 32 * agn::kHeadMaxClasses)));
-    AGN_TRY(dalloc_t(h, &h->fh_counter, (size_t)(n * nchk)));
-    AGN_TRY_CUDA(cudaMemsetAsync(h->fh_counter, 0, (size_t)(n * nchk) * sizeof(int), h->stream));
+    AGN_TRY(dalloc_t(h, &h->fh_counter, (size_t)(2 * n * nchk)));
+    AGN_TRY_CUDA(cudaMemsetAsync(h->fh_counter, 0, (size_t)(2 * n * nchk) * sizeof(int),
+                                 h->stream));
     h->loss_q = (int)nchk;
   }
   h->grid = agn::commit_grid(h->P_pad);
@@ -1224,8 +1248,9 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (h->use_tc) {
     AGN_TRY(build_tc_maps(h));
     AGN_TRY(dalloc_t(h, &h->tc_part, (size_t)h->num_sms * 256 * 128));
-    AGN_TRY(dalloc_t(h, &h->tc_counter, (size_t)h->num_sms));
-    AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)h->num_sms * sizeof(int), h->stream));
+    AGN_TRY(dalloc_t(h, &h->tc_counter, (size_t)(2 * h->num_sms)));
+    AGN_TRY_CUDA(cudaMemsetAsync(h->tc_counter, 0, (size_t)(2 * h->num_sms) * sizeof(int),
+                                 h->stream));
   }
   std::vector<int> all(n);
   for (int w = 0; w < n; ++w) all[w] = w;

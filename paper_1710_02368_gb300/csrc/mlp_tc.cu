@@ -296,6 +296,16 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   }
   __syncwarp();
 
+  // CTA 0 clears the counter arrays the previous launch used (every thread
+  // has passed its dependency wait by now; this launch's own arrays were
+  // cleared by the launch before it)
+  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) {
+    if (args.counter_clear)
+      for (int i = threadIdx.x; i < args.counter_clear_n; i += kThreads) args.counter_clear[i] = 0;
+    if (kEpi == kEpiFwdHead && args.head_counter_clear)
+      for (int i = threadIdx.x; i < args.head_counter_clear_n; i += kThreads)
+        args.head_counter_clear[i] = 0;
+  }
   // block-uniform, so that the epilogue's barriers and warp-wide TMEM loads
   // are reached by every thread or by none
   const bool ok = __syncthreads_and(wait_or_abort(done, 0, abort_flag) && !*abort_flag) != 0;
@@ -328,14 +338,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // Split K (forward / dX): chunk j of the tile (columns 32 j .. 32 j + 31)
     // is finished by rank j % ks.  Every rank stores its partial sums of the
     // chunks it does not finish ([column][row], rows contiguous) and counts
-    // itself in (low half of the tile's counter).  A rank that finishes
-    // chunks waits until all ks ranks are in (the CTAs of a launch with
-    // ks > 1 are resident together: at most one per SM, no more than the
-    // SMs), copies the other ranks' partial sums of its chunks into its stage
-    // ring and adds them in rank order, its own from TMEM.  Every rank then
-    // counts itself out (high half); the last one out resets the counter for
-    // the next launch.  Warps 0-3 take columns 0-15 of every chunk, warps
-    // 4-7 columns 16-31.
+    // itself in on the tile's counter (an array the previous launch cleared).
+    // A rank that finishes chunks waits until all ks ranks are in (the CTAs
+    // of a launch with ks > 1 are resident together: at most one per SM, no
+    // more than the SMs), copies the other ranks' partial sums of its chunks
+    // into its stage ring and adds them in rank order, its own from TMEM.
+    // Warps 0-3 take columns 0-15 of every chunk, warps 4-7 columns 16-31.
     constexpr int kNch = BN / 32;
     constexpr uint32_t kChunkBytes = 128u * 32u * 4u;
     const bool split_k = kEpi != kEpiDW && ks > 1;
@@ -430,14 +438,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       __syncthreads();
       have = s_have != 0;
       if (have && n_own > 0) have = __syncthreads_and(wait_or_abort(red, 0, abort_flag)) != 0;
-      if (threadIdx.x == 0) {
-        if (have) {
-          const int prev = tc::atomic_add_acq_rel_gpu(args.counter + tile_id, 1 << 16);
-          if ((prev >> 16) == ks - 1) args.counter[tile_id] = 0;   // ready for the next launch
-        } else {
-          atomicExch(args.err, 1);   // gave up: report, skip the epilogue
-        }
-      }
+      if (threadIdx.x == 0 && !have) atomicExch(args.err, 1);   // gave up: report, skip the epilogue
     }
     // the accumulated values of this thread's row for columns c0 .. c0 + 15
     // of chunk j = own_rank + o ks (c0 = 32 j + co)
@@ -744,12 +745,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               }
             }
           }
-          __syncthreads();
           if (threadIdx.x == 0) {
-            // count out (relaxed: it orders nothing but the counter itself); the
-            // last one out resets the counter for the next launch
-            const int prev = atomicAdd(ctr, 1 << 16);
-            if ((prev >> 16) == mtn - 1) *ctr = 0;
             // the chunk's loss contribution (sum of its samples' cross-entropy
             // over m) in the chunk's slot; the run's loss kernel adds the slots
             // in order

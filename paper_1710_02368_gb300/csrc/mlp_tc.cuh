@@ -37,6 +37,12 @@ struct TcArgs {
   int ksplit;
   float* part;
   int* counter;
+  // The per-tile arrival counters (and the fused output layer's) alternate
+  // between two arrays by launch: CTA 0 of a launch clears, after its
+  // dependency wait, the array the previous launch used (null = none), so no
+  // launch has to count its CTAs out to reset its own.
+  int* counter_clear;
+  int counter_clear_n;
   // dW: store the raw gradient at grad_out [n][ld_param] (same layout as the
   // replicas) instead of taking the local step (the optimizer runs after);
   // null = fused local step
@@ -56,7 +62,9 @@ struct TcArgs {
   bf16* dh_pieces;                // split mode: its pieces, planes dh_plane apart
   int64_t dh_plane;
   float* head_part;               // [slots][ceil(m / 32)][M tiles][32][16] partial logits
-  int* head_counter;              // [slots][ceil(m / 32)], zero between launches
+  int* head_counter;              // [slots][ceil(m / 32)], zero at launch
+  int* head_counter_clear;        // the other array, cleared by CTA 0 (null = none)
+  int head_counter_clear_n;
   float* loss_parts;              // [commit][lambda][ceil(m / 32)]: per 32-sample chunk
                                   // its cross-entropy sum / m
   const int* slot_commit;
