@@ -140,8 +140,9 @@ def _traffic_for(kernel_class, workload, on_tc):
     if not os.path.exists(path):
         return None
     if on_tc:
-        src = {"forward": "mlp_tc.cu", "backward_dx": "mlp_tc.cu", "backward_dw": "mlp_tc_dw.cu",
-               "softmax": "mlp_head.cu", "commit": "commit_pull.cu"}.get(kernel_class)
+        src = {"forward": "mlp_tc.cu", "forward_head": "mlp_tc.cu", "backward_dx": "mlp_tc.cu",
+               "backward_dw": "mlp_tc_dw.cu", "softmax": "mlp_head.cu",
+               "commit": "commit_pull.cu"}.get(kernel_class)
     else:
         src = {"forward": "mlp_simt.cu", "backward_dx": "mlp_simt.cu",
                "backward_dw": "mlp_simt.cu", "commit": "commit_pull.cu"}.get(kernel_class)
@@ -293,7 +294,7 @@ def commit_kernel_bench(agn, torch, dev, P, min_ms=200.0):
                       "(larger than L2)"}
 
 
-def method_bytes_per_worker_step(wl, cls):
+def method_bytes_per_worker_step(wl, cls, fused_head=False):
     """Bytes the method itself moves per worker-step (one local step of one
     worker) in a kernel class: each local step reads and writes the fp32
     replica theta_k and accumulator a_k of every parameter (Algorithm 1: 16 B
@@ -309,12 +310,16 @@ def method_bytes_per_worker_step(wl, cls):
     if cls == "backward_dw":
         return P * (16.0 if wl.precision == WL.PREC_FP32 else 18.0) + sum(
             m * (d[l] + d[l - 1]) * es for l in range(1, L + 1))
-    if cls == "forward":        # the hidden layers (the output layer runs in the head)
+    if cls == "forward":        # the hidden layers (the last one not, when the output
+        # layer rides in its epilogue: that launch is the forward_head class)
         return sum(d[l] * d[l - 1] * es + 4.0 * d[l] + m * (d[l - 1] + d[l]) * es
-                   for l in range(1, L))
+                   for l in range(1, L - 1 if fused_head else L))
     if cls == "backward_dx":    # layers L-1 .. 2 (the head writes layer L's dX)
         return sum(d[l] * d[l - 1] * es + m * d[l] * es + 2.0 * m * d[l - 1] * es
                    for l in range(2, L))
+    if cls == "forward_head":   # the last hidden layer's forward and the output layer
+        return (d[L - 1] * d[L - 2] * es + 4.0 * d[L - 1] + m * (d[L - 2] + 2.0 * d[L - 1]) * es
+                + d[L] * d[L - 1] * es + 4.0 * d[L] + m * d[L] * es + 4.0 * m)
     if cls == "softmax":        # output layer: forward, softmax-CE, dX
         return (d[L] * d[L - 1] * es + 4.0 * d[L] + 2.0 * m * d[L - 1] * es + m * d[L] * es
                 + 4.0 * m)
@@ -323,20 +328,20 @@ def method_bytes_per_worker_step(wl, cls):
     return None
 
 
-GEMM_CLASSES = ("forward", "backward_dx", "backward_dw", "softmax")
+GEMM_CLASSES = ("forward", "forward_head", "backward_dx", "backward_dw", "softmax")
 
 
 def roofline(wl, kst, worker_steps, on_tc, hbm, bf16, peak_src):
     """Roofline of the dominant kernel class (by device time) from the CUDA
     events of the profiled region: achieved = method bytes (or flops) per
     launch / average launch time."""
-    dom = max(("forward", "backward_dx", "backward_dw", "commit", "softmax", "gather"),
-              key=lambda k: kst[k]["ms"])
+    dom = max(("forward", "forward_head", "backward_dx", "backward_dw", "commit", "softmax",
+               "gather"), key=lambda k: kst[k]["ms"])
     d = kst[dom]
     launches = max(d["launches"], 1)
     sec = d["ms"] / 1e3 / launches
     impl_bytes = d["bytes"] / launches
-    mb = method_bytes_per_worker_step(wl, dom)
+    mb = method_bytes_per_worker_step(wl, dom, fused_head=kst["forward_head"]["launches"] > 0)
     method_bytes = mb * worker_steps / launches if mb is not None else impl_bytes
     flops = d["flops"] / launches
     # fp32 mode on the tensor cores issues six bf16 piece products per fp32 product

@@ -254,7 +254,10 @@ int agn_generate_inputs(const int32_t* dims, int32_t n_dims, int32_t input_dist,
 #define AGN_K_COMMIT 5       /* fused commit + pull                              */
 #define AGN_K_NORMS 6        /* per-commit norm reduction                        */
 #define AGN_K_OTHER 7        /* pulls outside commits, loss means                */
-#define AGN_KERNEL_CLASSES 8
+#define AGN_K_FORWARD_HEAD 8 /* the last hidden layer's forward GEMM with the
+                                output layer in its epilogue (forward,
+                                softmax-CE, dX of the last hidden layer)         */
+#define AGN_KERNEL_CLASSES 9
 int agn_profile(agn_handle* h, int32_t mode);
 int agn_kernel_stats(const agn_handle* h, double* out, int64_t cap);
 

@@ -34,7 +34,7 @@ AGN_GEMM_SIMT = 1
 AGN_GEMM_TCGEN05 = 2
 
 KERNEL_CLASSES = ["gather", "forward", "softmax", "backward_dx", "backward_dw", "commit",
-                  "norms", "other"]
+                  "norms", "other", "forward_head"]
 
 ERROR_NAMES = {
     AGN_E_INVALID: "AGN_E_INVALID", AGN_E_SCHEDULE: "AGN_E_SCHEDULE", AGN_E_OOM: "AGN_E_OOM",

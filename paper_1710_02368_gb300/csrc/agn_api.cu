@@ -136,7 +136,7 @@ struct agn_handle {
   LayerMaps l1_alt;               // layer 1's maps over the alternate operand buffer
   // fp32 mode on the tensor cores: every operand is three exact bf16 pieces
   bool split = false;
-  int64_t piece_plane = 0;        // between weight piece planes of rep_b ([3][n][P_pad])
+  int64_t piece_plane = 0;        // 0: no replica keeps weight pieces (fp32 mode splits in the GEMMs)
   std::vector<bf16*> Hs;          // pieces of H_l, l = 0..L-2: [3][n][m][d_l]
   std::vector<bf16*> dZp;         // pieces of dZ_l, l = 1..L-1: [3][n][m][d_l]
   // output layer fused into one kernel (forward + softmax-CE + dX) when narrow
@@ -347,11 +347,13 @@ Status build_tc_maps(agn_handle* h) {
                                   128, 32));
     AGN_TRY(agn::make_tmap_f32_3d(&mp.acc, h->acc + h->woff[l - 1], fi, fo, n, fi, h->P_pad,
                                   128, 32));
-    if (h->split) {   // 4D maps over the three piece planes
-      const bf16* W = h->rep_b + h->woff[l - 1];
-      const uint64_t wp = (uint64_t)h->piece_plane;
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, wp, 64, 128));
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, wp, 64, 64));
+    if (h->split) {
+      // the fp32 weights themselves (the GEMMs split them into pieces in
+      // shared memory): a 64-deep k step of 128 features (forward, K-major)
+      // or 128 inputs of 64 features (dX); activations as 4D piece maps
+      const float* W = h->rep + h->woff[l - 1];
+      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, 64, 128));
+      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 128, 64));
       const bf16* Hp = h->Hs[l - 1];
       const uint64_t hp = (uint64_t)n * m * fi;
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, bn));
@@ -457,8 +459,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
   // (with Adam the dW kernels only store the gradient, 4 bytes; the Adam
   // kernel's own traffic is counted at its launch)
   const double upd = h->adam ? 4.0
-                             : (h->elide ? 8.0 : 16.0) +
-                                   (h->split ? 6.0 : h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
+                             : (h->elide ? 8.0 : 16.0) + (h->prec == AGN_PREC_BF16 ? 2.0 : 0.0);
   // pieces of dZ_l (split mode, hidden tensor-core layers), planes n m d_l apart
   auto dz_pieces = [&](int l) -> bf16* {
     return (h->split && l >= 1 && tc_layer(h, l)) ? h->dZp[l] : nullptr;
@@ -538,7 +539,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         // with the output layer fused: its forward and dX flops, W_L, dZ_L
         // and dZ_{L-1} (with pieces) bytes too
         const int C = h->dims[L];
-        Launch k(h, AGN_K_FORWARD,
+        Launch k(h, fuse ? AGN_K_FORWARD_HEAD : AGN_K_FORWARD,
                  2.0 * s * m * fo * fi + (fuse ? 4.0 * s * m * fo * C : 0.0),
                  (double)s * ((double)fo * fi * es + 4.0 * fo + (double)m * fi * es +
                               (double)m * fo * (oes + (h_pieces ? 6.0 : 0.0))) +
@@ -728,7 +729,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
       ad.P = h->P_pad; ad.ld = h->P_pad;
       ad.slot_worker = sw; ad.slot_t0 = st0; ad.step = i;
       ad.eta = eta; ad.beta1 = h->beta1; ad.beta2 = h->beta2; ad.eps = h->eps;
-      const double copy_b = h->split ? 6.0 : h->rep_b ? 2.0 : 0.0;
+      const double copy_b = h->rep_b ? 2.0 : 0.0;
       Launch k(h, AGN_K_BACKWARD_DW, 0.0,
                (double)s * h->P * (4.0 + 16.0 + 8.0 + (h->elide ? 0.0 : 8.0) + copy_b), launches);
       AGN_TRY(agn::adam_step(ad, s, h->num_sms, h->stream));
@@ -941,7 +942,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     for (const CommitPlan& cp : wv.commits) {
       const double pulls = cp.pull_begin[cp.n_commits];
       {
-        const double copy_b = h->split ? 6.0 : h->rep_b ? 2.0 : 0.0;
+        const double copy_b = h->rep_b ? 2.0 : 0.0;
         Launch kc(h, AGN_K_COMMIT, 2.0 * cp.n_commits * h->P,
                   (double)h->P * (8.0 + 8.0 * cp.n_commits +
                                   pulls * (4.0 + copy_b + (h->elide ? 4.0 : 0.0))),
@@ -1154,9 +1155,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   h->ldz_out = h->fuse_out_dw ? (int)round_up(dims[h->L], 8) : dims[h->L];
   h->fuse_head = h->use_tc && h->use_head && h->L >= 2 && (h->tc_mask & 1) &&
                  !(h->tc_mask & 32) && dims[h->L] <= agn::kHeadMaxClasses;
-  if (h->split) {   // three piece planes of every replica, and of the activations
-    h->piece_plane = n * h->P_pad;
-    AGN_TRY(dalloc_t(h, &h->rep_b, (size_t)(3 * h->piece_plane)));
+  if (h->split) {   // three piece planes of the activations (the weights stay fp32)
     h->Hs.assign(h->L, nullptr);
     for (int l = 0; l + 1 < h->L + (h->fuse_out_dw ? 1 : 0); ++l)
       AGN_TRY(dalloc_t(h, &h->Hs[l], (size_t)(3 * n * m * dims[l])));

@@ -37,6 +37,10 @@ constexpr int kBK = 64;                       // K per stage: 64 bf16 = one 128-
 constexpr int kABytes = 128 * 128;            // 128 rows x 128 bytes
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s
 constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles
+// fp32 mode: one k step of fp32 weights (128 x 64), converted in place into
+// its bf16 pieces by kConvWarps warps
+constexpr uint32_t kA32Bytes = 128 * 64 * 4;
+constexpr int kConvWarps = 6;
 // Fused output layer (kEpiFwdHead): at most kHC classes; shared scratch of
 // W_L's 128 x kHC slice, the warps' partial logits [8][16][kHC] and the
 // chunk's logits / dZ_L [32][kHC].
@@ -132,6 +136,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                const TcArgs args) {
   using Cfg = TileCfg<BN, kSplit>;
   using TAct = typename std::conditional<kSplit == 1, bf16, float>::type;
+  // fp32 mode, forward and dX: A = W arrives as fp32 (TMA, 128 x 64 floats
+  // into the first 32 KB of the stage's 48 KB of A pieces) and warps 2-7
+  // replace it, in place, by its three bf16 pieces in the swizzled layout the
+  // MMA reads; the replicas hold no weight pieces.
+  constexpr bool kWConv = kSplit == 3 && kEpi != kEpiDW;
+  static_assert(!kWConv || kA32Bytes <= 3 * kABytes, "fp32 tile within the A slots");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -139,7 +149,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* empty = full + kStages;
   uint64_t* done = empty + kStages;
   uint64_t* red = done + 1;              // split K: the other ranks' partial sums landed
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(red + 1);
+  uint64_t* conv = red + 1;              // fp32 weights: stage s's A pieces written
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(conv + kStages);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   // A CTA that gave up earlier in this launch (or run) makes the rest return
@@ -168,6 +179,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     tc::mbar_init(done, 1);
     tc::mbar_init(red, 1);
+    for (int s = 0; s < kStages; ++s) tc::mbar_init(&conv[s], kConvWarps);
     *abort_flag = 0;
     tc::fence_mbar_init();
     tc::tma_prefetch_desc(&tmA);
@@ -213,13 +225,22 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           }
         }
       };
+      // fp32 weights of k step kt into stage s's A slots (completing on full[s])
+      auto load_a32 = [&](int kt, int s) {
+        uint8_t* dst = smem + s * Cfg::kStageBytes;
+        const int kc = (kt0 + kt) * kBK;
+        if (!kAMN) tc::tma_load_3d(dst, &tmA, &full[s], kc, m_tile * 128, a_z);
+        else tc::tma_load_3d(dst, &tmA, &full[s], m_tile * 128, kc, a_z);
+      };
       // prefetched stages count the A bytes now and arrive with the B bytes
       // below, so no phase can complete before its B boxes are requested
-      constexpr uint32_t kABytesAll = kSplit * kABytes;
+      constexpr uint32_t kABytesAll = kWConv ? kA32Bytes : kSplit * kABytes;
+      constexpr uint32_t kBBytesAll = kSplit * Cfg::kBBytes;
       const int npre = kPrefetchA ? min(KT, kStages) : 0;
       for (int kt = 0; kt < npre; ++kt) {
         tc::mbar_expect_tx(&full[kt], kABytesAll);
-        load_a(kt, kt);
+        if (kWConv) load_a32(kt, kt);
+        else load_a(kt, kt);
       }
       pdl_begin();
       int kt = 0;
@@ -233,10 +254,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         uint8_t* sa0 = smem + s * Cfg::kStageBytes;
         uint8_t* sb0 = sa0 + kSplit * kABytes;
         if (kt >= npre) {
-          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes);
-          load_a(kt, s);
+          tc::mbar_arrive_expect_tx(&full[s], kABytesAll + kBBytesAll);
+          if (kWConv) load_a32(kt, s);
+          else load_a(kt, s);
         } else {
-          tc::mbar_arrive_expect_tx(&full[s], Cfg::kStageBytes - kABytesAll);
+          tc::mbar_arrive_expect_tx(&full[s], kBBytesAll);
         }
 #pragma unroll
         for (int p = 0; p < kSplit; ++p) {
@@ -260,12 +282,70 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
       }
     }
+  } else if (kWConv && warp >= 2) {
+    // Converters: the fp32 weight tile of each k step into its three bf16
+    // pieces (x0 = bf16(x), x1 = bf16(x - x0), x2 = bf16(x - x0 - x1)), in
+    // place: every converter thread first loads its elements (four
+    // consecutive floats per item, 16-byte shared loads), the six warps meet
+    // at a named barrier, then each writes its items' pieces (three 8-byte
+    // stores at the 128-byte-swizzled positions the TMA would have used).
+    // The barrier also ANDs the warps' waits, so that they give up together.
+    const int ct = threadIdx.x - 64;
+    constexpr int kItems = 2048, kPer = (kItems + kConvWarps * 32 - 1) / (kConvWarps * 32);
+    for (int kt = 0; kt < KT; ++kt) {
+      const int s = kt % kStages;
+      const bool got = __all_sync(0xffffffffu,
+                                  wait_or_abort(&full[s], (kt / kStages) & 1, abort_flag));
+      int all_ok;
+      asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+                   "bar.red.and.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+                   : "=r"(all_ok) : "r"((unsigned)got), "n"(kConvWarps * 32) : "memory");
+      if (!all_ok) {
+        if (lane == 0) *abort_flag = 1;
+        break;
+      }
+      uint8_t* sa0 = smem + s * Cfg::kStageBytes;
+      const float* a32 = reinterpret_cast<const float*>(sa0);
+      float4 x[kPer];
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        const int it = ct + j * kConvWarps * 32;
+        if (it < kItems) {
+          if (!kAMN) x[j] = *reinterpret_cast<const float4*>(a32 + (it >> 4) * 64 + 4 * (it & 15));
+          else x[j] = *reinterpret_cast<const float4*>(a32 + (it >> 5) * 128 + 4 * (it & 31));
+        }
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(kConvWarps * 32) : "memory");
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        const int it = ct + j * kConvWarps * 32;
+        if (it < kItems) {
+          int off;                        // byte offset in a piece tile
+          if (!kAMN) {                    // K-major: 128 rows (features) x 64 k
+            const int r = it >> 4, q = it & 15;
+            off = r * 128 + ((((q >> 1) ^ (r & 7))) << 4) + (q & 1) * 8;
+          } else {                        // MN-major: 64 k rows x 128 inputs, two 64-wide boxes
+            const int f = it >> 5, q = it & 31, mh = q >> 4, qm = q & 15;
+            off = mh * 8192 + f * 128 + ((((qm >> 1) ^ (f & 7))) << 4) + (qm & 1) * 8;
+          }
+          const float xv[4] = {x[j].x, x[j].y, x[j].z, x[j].w};
+          uint2 q0, q1, q2;
+          split3_x4(xv, q0, q1, q2);
+          *reinterpret_cast<uint2*>(sa0 + off) = q0;
+          *reinterpret_cast<uint2*>(sa0 + kABytes + off) = q1;
+          *reinterpret_cast<uint2*>(sa0 + 2 * kABytes + off) = q2;
+        }
+      }
+      tc::fence_proxy_async_smem();       // before the MMAs (async proxy) read them
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&conv[s]);
+    }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, BN, kAMN, kBMN);
       for (int kt = 0; kt < KT; ++kt) {
         const int s = kt % kStages;
-        if (!wait_or_abort(&full[s], (kt / kStages) & 1, abort_flag)) {
+        if (!wait_or_abort(kWConv ? &conv[s] : &full[s], (kt / kStages) & 1, abort_flag)) {
           *abort_flag = 1;
           break;
         }
@@ -813,15 +893,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const float t = fmaf(-eta, gr, th[i]);
             theta[p] = t;
             acc[p] = ac[i] + gr;
-            if (kSplit == 1) {
-              tb[p] = __float2bfloat16_rn(t);
-            } else {
-              bf16 q0, q1, q2;
-              split3(t, q0, q1, q2);
-              tb[p] = q0;
-              tb[args.piece_plane + p] = q1;
-              tb[2 * args.piece_plane + p] = q2;
-            }
+            if (kSplit == 1) tb[p] = __float2bfloat16_rn(t);   // fp32 mode keeps no weight pieces
           }
         }
       }
@@ -862,15 +934,7 @@ bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
   const float t = fmaf(-eta, s, theta[p]);
   theta[p] = t;
   acc[p] += s;
-  if (kSplit == 1) {
-    theta_b[p] = __float2bfloat16_rn(t);
-  } else {
-    bf16 q0, q1, q2;
-    split3(t, q0, q1, q2);
-    theta_b[p] = q0;
-    theta_b[piece_plane + p] = q1;
-    theta_b[2 * piece_plane + p] = q2;
-  }
+  if (kSplit == 1 && theta_b) theta_b[p] = __float2bfloat16_rn(t);   // fp32 mode: no pieces
 }
 
 // out[p * plane + i] = piece p of x[i] (x = piece 0 + piece 1 + piece 2 exactly).

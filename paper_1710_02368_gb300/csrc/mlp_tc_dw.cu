@@ -99,24 +99,6 @@ __device__ __forceinline__ uint2 bf16x4(const float (&x)[4]) {
   const __nv_bfloat162 hi = __floats2bfloat162_rn(x[2], x[3]);
   return make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
 }
-// The three exact bf16 pieces of four floats (split3 of each), packed.
-__device__ __forceinline__ void split3_x4(const float (&x)[4], uint2& q0, uint2& q1, uint2& q2) {
-  float r[4];
-  q0 = bf16x4(x);
-  const __nv_bfloat162* p0 = reinterpret_cast<const __nv_bfloat162*>(&q0);
-  r[0] = __fsub_rn(x[0], __low2float(p0[0]));
-  r[1] = __fsub_rn(x[1], __high2float(p0[0]));
-  r[2] = __fsub_rn(x[2], __low2float(p0[1]));
-  r[3] = __fsub_rn(x[3], __high2float(p0[1]));
-  q1 = bf16x4(r);
-  const __nv_bfloat162* p1 = reinterpret_cast<const __nv_bfloat162*>(&q1);
-  r[0] = __fsub_rn(r[0], __low2float(p1[0]));
-  r[1] = __fsub_rn(r[1], __high2float(p1[0]));
-  r[2] = __fsub_rn(r[2], __low2float(p1[1]));
-  r[3] = __fsub_rn(r[3], __high2float(p1[1]));
-  q2 = bf16x4(r);
-}
-
 // Piece pairs (i, j), i + j <= 2, of the split product (pair 0 = a0 b0).
 __device__ __forceinline__ int pair_a(int q) { return q == 2 || q == 4 ? 1 : q == 5 ? 2 : 0; }
 __device__ __forceinline__ int pair_b(int q) { return q == 1 || q == 4 ? 1 : q == 3 ? 2 : 0; }
@@ -451,7 +433,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
       const int64_t rbase = (int64_t)worker * args.ld_param;
       float* theta = args.theta + rbase;
       float* acc = kAcc ? args.acc + rbase : nullptr;
-      bf16* tb = args.theta_b + rbase;
+      bf16* tb = args.theta_b ? args.theta_b + rbase : nullptr;   // bf16 mode only
       const int nch = min(Cfg::kChunks, (N - ti.n_tile * BN + kCF - 1) / kCF);
       for (int c = 0; c < nch; ++c) {
         const int r = ch % kRing;
@@ -515,15 +497,9 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
                 *reinterpret_cast<float4*>(acc + p) =
                     make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w);
               }
-              if (kSplit == 1) {
-                *reinterpret_cast<uint2*>(tb + p) = bf16x4(tn);
-              } else {
-                uint2 q0, q1, q2;
-                split3_x4(tn, q0, q1, q2);
-                *reinterpret_cast<uint2*>(tb + p) = q0;
-                *reinterpret_cast<uint2*>(tb + args.piece_plane + p) = q1;
-                *reinterpret_cast<uint2*>(tb + 2 * args.piece_plane + p) = q2;
-              }
+              // the bf16 copy (bf16 mode); the fp32 mode's GEMMs split the
+              // fp32 weights themselves
+              if (kSplit == 1) *reinterpret_cast<uint2*>(tb + p) = bf16x4(tn);
             }
           }
         }
@@ -535,15 +511,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
           theta[pb] = tn;
           if (kAcc) acc[pb] = sTb[kCF + 16 * hf + lane] + gb;
-          if (kSplit == 1) {
-            tb[pb] = __float2bfloat16_rn(tn);
-          } else {
-            bf16 q0, q1, q2;
-            split3(tn, q0, q1, q2);
-            tb[pb] = q0;
-            tb[args.piece_plane + pb] = q1;
-            tb[2 * args.piece_plane + pb] = q2;
-          }
+          if (kSplit == 1) tb[pb] = __float2bfloat16_rn(tn);
         }
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&cempty[r]);

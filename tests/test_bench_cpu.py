@@ -80,7 +80,8 @@ def test_committed_traffic_entries_are_well_formed():
     assert rows
     for r in rows:
         assert len(r) == 4
-        assert r[0] in ("forward", "backward_dx", "backward_dw", "softmax", "commit")
+        assert r[0] in ("forward", "forward_head", "backward_dx", "backward_dw", "softmax",
+                        "commit")
         assert float(r[2]) > 0
         assert len(r[3]) == 12 and all(ch in "0123456789abcdef" for ch in r[3])
 
@@ -107,3 +108,17 @@ def test_method_bytes_of_the_dw_class_by_hand():
     assert got == 16 * 1796010 + 128 * 4 * ((1000 + 784) + (1000 + 1000) + (10 + 1000))
     bf = bench.method_bytes_per_worker_step(WL.LARGE_BF16, "backward_dw")
     assert bf == 18 * 20037642 + 64 * 2 * ((4096 + 784) + (4096 + 4096) + (10 + 4096))
+
+
+def test_method_bytes_of_the_forward_classes_split_at_the_fused_launch():
+    """With the output layer in the last hidden layer's forward, the forward
+    class covers the other hidden layers and forward_head that layer plus the
+    output layer; together they count each layer once."""
+    from agn_inputs import workloads as WL
+    wl = WL.MNIST_SHAPED
+    plain = bench.method_bytes_per_worker_step(wl, "forward")
+    first = bench.method_bytes_per_worker_step(wl, "forward", fused_head=True)
+    head = bench.method_bytes_per_worker_step(wl, "forward_head")
+    out = bench.method_bytes_per_worker_step(wl, "softmax")
+    assert first == 1000 * 784 * 4 + 4 * 1000 + 128 * (784 + 1000) * 4
+    assert abs((first + head) - (plain + out)) <= 4 * 128 * 1000 + 1e-6
