@@ -150,7 +150,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* done = empty + kStages;
   uint64_t* red = done + 1;              // split K: the other ranks' partial sums landed
   uint64_t* conv = red + 1;              // fp32 weights: stage s's A pieces written
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(conv + kStages);
+  uint64_t* afull = conv + kStages;      // fp32 weights: stage s's fp32 tile landed
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(afull + kStages);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   // A CTA that gave up earlier in this launch (or run) makes the rest return
@@ -179,7 +180,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     tc::mbar_init(done, 1);
     tc::mbar_init(red, 1);
-    for (int s = 0; s < kStages; ++s) tc::mbar_init(&conv[s], kConvWarps);
+    for (int s = 0; s < kStages; ++s) {
+      tc::mbar_init(&conv[s], kConvWarps);
+      tc::mbar_init(&afull[s], 1);
+    }
     *abort_flag = 0;
     tc::fence_mbar_init();
     tc::tma_prefetch_desc(&tmA);
@@ -225,22 +229,28 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           }
         }
       };
-      // fp32 weights of k step kt into stage s's A slots (completing on full[s])
+      // fp32 weights of k step kt into stage s's A slots, on their own barrier
+      // (afull[s]) so that the converters can start before the activations
+      // land, for prefetched stages before the preceding kernel completes
       auto load_a32 = [&](int kt, int s) {
         uint8_t* dst = smem + s * Cfg::kStageBytes;
         const int kc = (kt0 + kt) * kBK;
-        if (!kAMN) tc::tma_load_3d(dst, &tmA, &full[s], kc, m_tile * 128, a_z);
-        else tc::tma_load_3d(dst, &tmA, &full[s], m_tile * 128, kc, a_z);
+        tc::mbar_arrive_expect_tx(&afull[s], kA32Bytes);
+        if (!kAMN) tc::tma_load_3d(dst, &tmA, &afull[s], kc, m_tile * 128, a_z);
+        else tc::tma_load_3d(dst, &tmA, &afull[s], m_tile * 128, kc, a_z);
       };
       // prefetched stages count the A bytes now and arrive with the B bytes
       // below, so no phase can complete before its B boxes are requested
-      constexpr uint32_t kABytesAll = kWConv ? kA32Bytes : kSplit * kABytes;
+      constexpr uint32_t kABytesAll = kWConv ? 0u : kSplit * kABytes;   // A bytes on full[s]
       constexpr uint32_t kBBytesAll = kSplit * Cfg::kBBytes;
       const int npre = kPrefetchA ? min(KT, kStages) : 0;
       for (int kt = 0; kt < npre; ++kt) {
-        tc::mbar_expect_tx(&full[kt], kABytesAll);
-        if (kWConv) load_a32(kt, kt);
-        else load_a(kt, kt);
+        if (kWConv) {
+          load_a32(kt, kt);
+        } else {
+          tc::mbar_expect_tx(&full[kt], kABytesAll);
+          load_a(kt, kt);
+        }
       }
       pdl_begin();
       int kt = 0;
@@ -280,6 +290,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int j = kt; j < npre; ++j) tc::mbar_wait_bounded(&full[j], 0, kWaitNs);
         for (int j = kt - 1; j >= 0 && j >= kt - kStages; --j)
           tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
+        if (kWConv)   // the fp32 weight tiles armed (prefetched or in the loop)
+          for (int j = max(kt, npre) - 1; j >= 0 && j >= max(kt, npre) - kStages; --j)
+            tc::mbar_wait_bounded(&afull[j % kStages], (j / kStages) & 1, kWaitNs);
       }
     }
   } else if (kWConv && warp >= 2) {
@@ -295,7 +308,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     for (int kt = 0; kt < KT; ++kt) {
       const int s = kt % kStages;
       const bool got = __all_sync(0xffffffffu,
-                                  wait_or_abort(&full[s], (kt / kStages) & 1, abort_flag));
+                                  wait_or_abort(&afull[s], (kt / kStages) & 1, abort_flag));
       int all_ok;
       asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
                    "bar.red.and.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
@@ -345,7 +358,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, BN, kAMN, kBMN);
       for (int kt = 0; kt < KT; ++kt) {
         const int s = kt % kStages;
-        if (!wait_or_abort(kWConv ? &conv[s] : &full[s], (kt / kStages) & 1, abort_flag)) {
+        if (!wait_or_abort(&full[s], (kt / kStages) & 1, abort_flag) ||
+            (kWConv && !wait_or_abort(&conv[s], (kt / kStages) & 1, abort_flag))) {
           *abort_flag = 1;
           break;
         }
