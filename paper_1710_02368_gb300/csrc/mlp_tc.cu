@@ -492,7 +492,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
     if (split_k) {
       float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
-#pragma unroll
+#pragma unroll 1
       for (int j = 0; j < kNch; ++j) {
         if (j % ks == sk) continue;
         uint32_t r[16];
@@ -589,10 +589,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           // lanes of a column fold by a fixed shuffle tree; the four row
           // quadrants of a column half are added in order below.  The ReLU
           // mask of the lane's 4 x 4 values goes to shared memory for pass 2.
+          // This code runs once per chunk and launch, from a cold instruction
+          // cache: it loops over the lane's four columns (u) rather than
+          // unrolling them, which keeps it a quarter of the size.
           const int C = args.head_C;
           uint32_t mbits = 0;
-          float hq[4][4];
-#pragma unroll
+          // W_L rows past C are zero in shared memory: all kHC classes are
+          // summed unguarded, as independent chains
+          const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
+#pragma unroll 1
           for (int u = 0; u < 4; ++u) {
             const int j = n_tile * BN + c0 + jl + 4 * u;
             float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -603,25 +608,19 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               a.z = fmaxf(a.z + bias4.z, 0.f);
               a.w = fmaxf(a.w + bias4.w, 0.f);
             }
-            hq[u][0] = a.x; hq[u][1] = a.y; hq[u][2] = a.z; hq[u][3] = a.w;
+            const float hq[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e)   // the mask of the value as stored
-              mbits |= (static_cast<float>(static_cast<TAct>(hq[u][e])) > 0.f ? 1u : 0u)
+              mbits |= (static_cast<float>(static_cast<TAct>(hq[e])) > 0.f ? 1u : 0u)
                        << (4 * u + e);
-          }
-          // W_L rows past C are zero in shared memory: all kHC classes are
-          // summed unguarded, as independent chains
-          const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
             float zp[kHC];
 #pragma unroll
             for (int c = 0; c < kHC; ++c) {
               const float4 w = w3v[c * 32];
-              float t = hq[u][0] * w.x;
-              t = fmaf(hq[u][1], w.y, t);
-              t = fmaf(hq[u][2], w.z, t);
-              zp[c] = fmaf(hq[u][3], w.w, t);
+              float t = hq[0] * w.x;
+              t = fmaf(hq[1], w.y, t);
+              t = fmaf(hq[2], w.z, t);
+              zp[c] = fmaf(hq[3], w.w, t);
             }
             // fold the eight lanes of the column (lane bits 0-2) by a fixed
             // reduce-scatter: each round a lane keeps half of its classes and
@@ -703,10 +702,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (kEpi == kEpiFwdHead) {
         // Pass 2: once every feature tile's partials of a chunk are in (all
         // CTAs of this launch are resident), the chunk's logits are summed in
-        // tile order plus b_L; warp 0 takes softmax cross-entropy and dZ_L =
-        // (softmax - onehot(y)) / m per sample (the first feature tile writes
-        // dZ_L and the chunk's loss); every CTA then writes dZ_{L-1} = (dZ_L
-        // W_L) [H_{L-1} > 0] for its own features (W_L before its update).
+        // tile order plus b_L; every half-warp takes softmax cross-entropy and
+        // dZ_L = (softmax - onehot(y)) / m of a sample (the first feature tile
+        // writes dZ_L and the chunk's loss); every CTA then writes dZ_{L-1} =
+        // (dZ_L W_L) [H_{L-1} > 0] for its own features (W_L before its
+        // update).
         __shared__ int s_hok;
         const int C = args.head_C;
         const float* bl = theta + args.head_boff;
@@ -725,78 +725,79 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             break;
           }
           // the feature tiles' partials in tile order: each thread sums two of
-          // the chunk's 32 x kHC logits, up to 2 x 16 loads in flight
+          // the chunk's 32 x kHC logits, up to 2 x 16 loads in flight; thread
+          // t holds class t % kHC of samples t / kHC and 16 + t / kHC, so the
+          // 16 lanes of a half-warp hold one sample's logits
           static_assert(32 * kHC == 2 * kThreads, "two logits per thread");
+          static_assert(kHC == 16, "one sample per half-warp");
           const float* gp0 = args.head_part + ((int64_t)slot * nchk + chunk) * mtn * (32 * kHC);
-          {
-            float z0 = 0.f, z1 = 0.f;
-            for (int m0 = 0; m0 < mtn; m0 += 16) {
-              float p0[16], p1[16];
+          float zz[2] = {0.f, 0.f};
+          for (int m0 = 0; m0 < mtn; m0 += 16) {
+            float p0[16], p1[16];
 #pragma unroll
-              for (int q = 0; q < 16; ++q) {
-                const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
-                p0[q] = m0 + q < mtn ? __ldcg(pq) : 0.f;
-                p1[q] = m0 + q < mtn ? __ldcg(pq + kThreads) : 0.f;
-              }
-#pragma unroll
-              for (int q = 0; q < 16; ++q) {
-                z0 += p0[q];
-                z1 += p1[q];
-              }
+            for (int q = 0; q < 16; ++q) {
+              const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
+              p0[q] = m0 + q < mtn ? __ldcg(pq) : 0.f;
+              p1[q] = m0 + q < mtn ? __ldcg(pq + kThreads) : 0.f;
             }
-            const int c0i = threadIdx.x % kHC;   // kThreads is a multiple of kHC
-            sG[threadIdx.x] = c0i < C ? z0 + bl[c0i] : -INFINITY;
-            sG[threadIdx.x + kThreads] = c0i < C ? z1 + bl[c0i] : -INFINITY;
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              zz[0] += p0[q];
+              zz[1] += p1[q];
+            }
+          }
+          // softmax cross-entropy and dZ_L = (softmax - onehot(y)) / m of the
+          // thread's two (sample, class) entries: max and sum over the
+          // sample's classes by a fixed shuffle tree within the half-warp;
+          // the first feature tile writes dZ_L
+          float* sCE = sPart;   // [32] per-sample cross-entropy (pass 1 is done with sPart)
+          {
+            const int cl = threadIdx.x % kHC;
+            const bool cv = cl < C;
+            const float inv_m = 1.0f / (float)args.N;
+            const float bc = cv ? bl[cl] : 0.f;
+#pragma unroll 1
+            for (int hh = 0; hh < 2; ++hh) {
+              const int sl = 16 * hh + (threadIdx.x >> 4);   // sample within the chunk
+              const int j = n_tile * BN + 32 * chunk + sl;
+              const bool valid = j < args.N;
+              const float z = cv ? (hh ? zz[1] : zz[0]) + bc : -INFINITY;
+              float mx = z;
+#pragma unroll
+              for (int off = 8; off > 0; off >>= 1)
+                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+              const float ex = cv ? expf(z - mx) : 0.f;
+              float se = ex;
+#pragma unroll
+              for (int off = 8; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
+              const int y = valid ? args.yb[(int64_t)slot * args.N + j] : -1;
+              const float zy = __shfl_sync(0xffffffffu, z, (lane & 16) + (y > 0 ? y : 0));
+              float pr = ex * (1.0f / se);
+              if (cl == y) pr -= 1.0f;
+              const float gz = valid ? pr * inv_m : 0.f;
+              sG[sl * kHC + cl] = gz;
+              if (m_tile == 0 && valid && cv) {
+                const TAct gv = static_cast<TAct>(gz);
+                const int64_t zi = ((int64_t)slot * args.N + j) * args.ldz + cl;
+                static_cast<TAct*>(args.dzl)[zi] = gv;
+                if (args.dzl_pieces) {
+                  bf16 q0, q1, q2;
+                  split3(static_cast<float>(gv), q0, q1, q2);
+                  args.dzl_pieces[zi] = q0;
+                  args.dzl_pieces[args.dzl_plane + zi] = q1;
+                  args.dzl_pieces[2 * args.dzl_plane + zi] = q2;
+                }
+              }
+              if (cl == 0) sCE[sl] = valid ? (logf(se) + mx) - zy : 0.f;
+            }
           }
           __syncthreads();
           float ce = 0.f;
-          if (warp == 0) {
-            const int j = n_tile * BN + 32 * chunk + lane;
-            const bool valid = j < args.N;
-            float zc[kHC];
-#pragma unroll
-            for (int c = 0; c < kHC; ++c) zc[c] = sG[lane * kHC + c];
-            float mx = zc[0];
-#pragma unroll
-            for (int c = 1; c < kHC; ++c) mx = fmaxf(mx, zc[c]);
-            const int y = valid ? args.yb[(int64_t)slot * args.N + j] : -1;
-            float ex[kHC];
-#pragma unroll
-            for (int c = 0; c < kHC; ++c) ex[c] = c < C ? expf(zc[c] - mx) : 0.f;
-            float se = 0.f, zy = 0.f;
-#pragma unroll
-            for (int c = 0; c < kHC; ++c) {
-              se += ex[c];
-              if (c == y) zy = zc[c];
-            }
-            ce = valid ? (logf(se) + mx) - zy : 0.f;
-            const float inv_s = 1.0f / se, inv_m = 1.0f / (float)args.N;
-            TAct* dzl = static_cast<TAct*>(args.dzl) + ((int64_t)slot * args.N + j) * args.ldz;
-            bf16* dzp = args.dzl_pieces
-                            ? args.dzl_pieces + ((int64_t)slot * args.N + j) * args.ldz
-                            : nullptr;
-#pragma unroll
-            for (int c = 0; c < kHC; ++c) {
-              float pr = ex[c] * inv_s;
-              if (c == y) pr -= 1.0f;
-              const float gz = valid ? pr * inv_m : 0.f;
-              sG[lane * kHC + c] = gz;
-              if (m_tile == 0 && valid && c < C) {
-                const TAct gv = static_cast<TAct>(gz);
-                dzl[c] = gv;
-                if (dzp) {
-                  bf16 q0, q1, q2;
-                  split3(static_cast<float>(gv), q0, q1, q2);
-                  dzp[c] = q0;
-                  dzp[args.dzl_plane + c] = q1;
-                  dzp[2 * args.dzl_plane + c] = q2;
-                }
-              }
-            }
+          if (warp == 0) {   // the chunk's cross-entropy sum, fixed tree over its samples
+            ce = sCE[lane];
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) ce += __shfl_xor_sync(0xffffffffu, ce, off);
           }
-          __syncthreads();
           if (row4_ok) {
             const uint32_t mbits = sMask[o * kThreads + threadIdx.x];
             const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
@@ -807,7 +808,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             for (int u = 0; u < 4; ++u)
 #pragma unroll
               for (int e = 0; e < 4; ++e) d[u][e] = 0.f;
-#pragma unroll
+#pragma unroll 2
             for (int c = 0; c < kHC; ++c) {
               const float4 w = w3v[c * 32];
 #pragma unroll
