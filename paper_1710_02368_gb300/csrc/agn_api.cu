@@ -349,18 +349,20 @@ Status build_tc_maps(agn_handle* h) {
                                   128, 32));
     if (h->split) {
       // the fp32 weights themselves (the GEMMs split them into pieces in
-      // shared memory): a 64-deep k step of 128 features (forward, K-major)
-      // or 128 inputs of 64 features (dX); activations as 4D piece maps
+      // shared memory): a kTcSplitBK-deep k step of 128 features (forward,
+      // K-major) or 128 inputs of kTcSplitBK features (dX); activations as 4D
+      // piece maps, kTcSplitBK-deep k steps for the forward and dX
+      constexpr uint32_t bk = agn::kTcSplitBK;
       const float* W = h->rep + h->woff[l - 1];
-      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, 64, 128));
-      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 128, 64));
+      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, bk, 128));
+      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 128, bk));
       const bf16* Hp = h->Hs[l - 1];
       const uint64_t hp = (uint64_t)n * m * fi;
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, bk, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 64));
       const uint64_t dp = (uint64_t)n * m * fo;
       const bf16* dZp = h->dZp[l];
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_k, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, bk, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 64));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, Hp, fi, m, n, fi, (uint64_t)m * fi, hp, 64, 32));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.dz_mn32, dZp, fo, m, n, fo, (uint64_t)m * fo, dp, 64, 32));
@@ -382,8 +384,8 @@ Status build_tc_maps(agn_handle* h) {
     auto& mp = h->l1_alt;
     if (h->split) {
       const uint64_t hp = (uint64_t)n * m * fi;
-      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp, 64,
-                                     bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp,
+                                     agn::kTcSplitBK, bn));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp, 64,
                                      64));
       AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, h->Hs0_alt, fi, m, n, fi, (uint64_t)m * fi, hp,

@@ -33,14 +33,17 @@ namespace agn {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kBK = 64;                       // K per stage: 64 bf16 = one 128-byte row
-constexpr int kABytes = 128 * 128;            // 128 rows x 128 bytes
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s
 constexpr int kEpiTBytes = 8 * 32 * 32 * 4;   // forward / dX epilogue transpose tiles
-// fp32 mode: one k step of fp32 weights (128 x 64), converted in place into
-// its bf16 pieces by kConvWarps warps
-constexpr uint32_t kA32Bytes = 128 * 64 * 4;
+// fp32 mode: each k step's fp32 weights (128 x K per stage) are converted in
+// place into their bf16 pieces by kConvWarps warps
 constexpr int kConvWarps = 6;
+
+// K per stage: 64 bf16, one 128-byte row (128-byte swizzle); 32 bf16, one
+// 64-byte row (64-byte swizzle), for the fp32 mode's forward and dX GEMMs,
+// whose stages hold three pieces of each operand: half the bytes per stage,
+// so twice the stages in flight to hide the load and conversion latency.
+constexpr int stage_k(int split, int epi) { return split == 3 && epi != kEpiDW ? kTcSplitBK : 64; }
 // Fused output layer (kEpiFwdHead): at most kHC classes; shared scratch of
 // W_L's 128 x kHC slice, the warps' partial logits [8][16][kHC] and the
 // chunk's logits / dZ_L [32][kHC].
@@ -48,11 +51,16 @@ constexpr int kHC = kHeadMaxClasses;
 constexpr int kHeadScratch = (kHC * 128 + 8 * 16 * kHC + 32 * kHC) * 4 + 8 * 256 * 2;
 
 // A stage holds kSplit A pieces then kSplit B pieces (kSplit = 3 in the fp32
-// mode, where every fp32 operand is the exact sum of three bf16 pieces).
-template <int BN, int kSplit>
+// mode, where every fp32 operand is the exact sum of three bf16 pieces), of
+// kBK k each (rows of 2 kBK bytes).
+template <int BN, int kSplit, int kBKs = 64>
 struct TileCfg {
-  static constexpr int kBBytes = BN * 128;
+  static constexpr int kBK = kBKs;
+  static constexpr int kRowBytes = 2 * kBK;
+  static constexpr int kABytes = 128 * kRowBytes;
+  static constexpr int kBBytes = BN * kRowBytes;
   static constexpr int kStageBytes = kSplit * (kABytes + kBBytes);
+  static constexpr uint32_t kA32Bytes = 128 * kBK * 4;   // an fp32 weight tile
   // split mode keeps two accumulators: columns [0, BN) take the leading
   // piece products a0 b0, columns [BN, 2 BN) the five smaller pairs, so the
   // rounding of the tensor core's running sums is relative to each part
@@ -62,9 +70,9 @@ struct TileCfg {
 // The forward / dX epilogue's transpose tiles sit after the barriers when the
 // CTA's shared memory has room for them (then the whole stage ring can hold
 // split-K partial sums), else at the end of the ring.
-template <int BN, int kSplit, int kStages>
+template <int BN, int kSplit, int kStages, int kBKs>
 struct EpiT {
-  static constexpr size_t kRing = (size_t)kStages * TileCfg<BN, kSplit>::kStageBytes;
+  static constexpr size_t kRing = (size_t)kStages * TileCfg<BN, kSplit, kBKs>::kStageBytes;
   static constexpr bool kSeparate = kRing + 1280 + kEpiTBytes <= 232448;
   static constexpr size_t kOff = kSeparate ? kRing + 256 : kRing - kEpiTBytes;
   static constexpr size_t kRingFree = kSeparate ? kRing : kRing - kEpiTBytes;
@@ -134,10 +142,15 @@ template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 __global__ void __launch_bounds__(kThreads, kEpi == kEpiDW ? 2 : 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const TcArgs args) {
-  using Cfg = TileCfg<BN, kSplit>;
+  constexpr int kBK = stage_k(kSplit, kEpi);
+  using Cfg = TileCfg<BN, kSplit, kBK>;
+  using Epi = EpiT<BN, kSplit, kStages, kBK>;
+  constexpr int kABytes = Cfg::kABytes;
+  constexpr uint32_t kA32Bytes = Cfg::kA32Bytes;
+  constexpr int kBox = kBK * 128;   // one 64-wide MN box of kBK rows (MN-major operands)
   using TAct = typename std::conditional<kSplit == 1, bf16, float>::type;
-  // fp32 mode, forward and dX: A = W arrives as fp32 (TMA, 128 x 64 floats
-  // into the first 32 KB of the stage's 48 KB of A pieces) and warps 2-7
+  // fp32 mode, forward and dX: A = W arrives as fp32 (TMA, 128 x kBK floats
+  // into the first 16 KB of the stage's 24 KB of A pieces) and warps 2-7
   // replace it, in place, by its three bf16 pieces in the swizzled layout the
   // MMA reads; the replicas hold no weight pieces.
   constexpr bool kWConv = kSplit == 3 && kEpi != kEpiDW;
@@ -225,7 +238,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             load(sa, &tmA, kc, m_tile * 128, a_z, p, &full[s]);
           } else {
             load(sa, &tmA, m_tile * 128, kc, a_z, p, &full[s]);
-            load(sa + 8192, &tmA, m_tile * 128 + 64, kc, a_z, p, &full[s]);
+            load(sa + kBox, &tmA, m_tile * 128 + 64, kc, a_z, p, &full[s]);
           }
         }
       };
@@ -279,7 +292,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           } else {
 #pragma unroll
             for (int c = 0; c < BN / 64; ++c)
-              load(sb + c * 8192, &tmB, n_tile * BN + c * 64, kc, b_z, p, &full[s]);
+              load(sb + c * kBox, &tmB, n_tile * BN + c * 64, kc, b_z, p, &full[s]);
           }
         }
       }
@@ -304,7 +317,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // stores at the 128-byte-swizzled positions the TMA would have used).
     // The barrier also ANDs the warps' waits, so that they give up together.
     const int ct = threadIdx.x - 64;
-    constexpr int kItems = 2048, kPer = (kItems + kConvWarps * 32 - 1) / (kConvWarps * 32);
+    constexpr int kItems = 128 * kBK / 4, kPer = (kItems + kConvWarps * 32 - 1) / (kConvWarps * 32);
+    constexpr int kQ = kBK / 4;   // 4-float items per K-major row
     for (int kt = 0; kt < KT; ++kt) {
       const int s = kt % kStages;
       const bool got = __all_sync(0xffffffffu,
@@ -324,7 +338,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       for (int j = 0; j < kPer; ++j) {
         const int it = ct + j * kConvWarps * 32;
         if (it < kItems) {
-          if (!kAMN) x[j] = *reinterpret_cast<const float4*>(a32 + (it >> 4) * 64 + 4 * (it & 15));
+          if (!kAMN) x[j] = *reinterpret_cast<const float4*>(a32 + (it / kQ) * kBK + 4 * (it % kQ));
           else x[j] = *reinterpret_cast<const float4*>(a32 + (it >> 5) * 128 + 4 * (it & 31));
         }
       }
@@ -334,12 +348,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int it = ct + j * kConvWarps * 32;
         if (it < kItems) {
           int off;                        // byte offset in a piece tile
-          if (!kAMN) {                    // K-major: 128 rows (features) x 64 k
-            const int r = it >> 4, q = it & 15;
-            off = r * 128 + ((((q >> 1) ^ (r & 7))) << 4) + (q & 1) * 8;
-          } else {                        // MN-major: 64 k rows x 128 inputs, two 64-wide boxes
+          if (!kAMN) {                    // K-major: 128 rows (features) x kBK k
+            // 16-byte chunk c of row r sits at chunk c ^ (r mod 8) (128-byte
+            // swizzle) or c ^ ((r / 2) mod 4) (64-byte swizzle)
+            const int r = it / kQ, q = it % kQ;
+            const int sw = kBK == 64 ? (r & 7) : ((r >> 1) & 3);
+            off = r * (2 * kBK) + ((((q >> 1) ^ sw)) << 4) + (q & 1) * 8;
+          } else {                        // MN-major: kBK k rows x 128 inputs, two 64-wide boxes
             const int f = it >> 5, q = it & 31, mh = q >> 4, qm = q & 15;
-            off = mh * 8192 + f * 128 + ((((qm >> 1) ^ (f & 7))) << 4) + (qm & 1) * 8;
+            off = mh * kBox + f * 128 + ((((qm >> 1) ^ (f & 7))) << 4) + (qm & 1) * 8;
           }
           const float xv[4] = {x[j].x, x[j].y, x[j].z, x[j].w};
           uint2 q0, q1, q2;
@@ -373,10 +390,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           for (int q = 0; q < kPairs; ++q) {
             const uint32_t sa = sa0 + (kSplit == 1 ? 0 : kPairA[q]) * kABytes;
             const uint32_t sb = sb0 + (kSplit == 1 ? 0 : kPairB[q]) * Cfg::kBBytes;
-            const uint64_t ad = kAMN ? tc::smem_desc_sw128(sa + kk * 2048, 8192, 1024)
-                                     : tc::smem_desc_sw128(sa + kk * 32, 16, 1024);
-            const uint64_t bd = kBMN ? tc::smem_desc_sw128(sb + kk * 2048, 8192, 1024)
-                                     : tc::smem_desc_sw128(sb + kk * 32, 16, 1024);
+            // MN-major: 16 k rows of 128 bytes per k16 step, the two 64-wide
+            // boxes kBox apart; K-major: 32 bytes along the row per k16 step,
+            // 8-row groups 8 rows apart
+            const uint64_t ad = kAMN ? tc::smem_desc_sw128(sa + kk * 2048, kBox, 1024)
+                                : kBK == 64 ? tc::smem_desc_sw128(sa + kk * 32, 16, 1024)
+                                            : tc::smem_desc_sw64(sa + kk * 32, 16, 512);
+            const uint64_t bd = kBMN ? tc::smem_desc_sw128(sb + kk * 2048, kBox, 1024)
+                                : kBK == 64 ? tc::smem_desc_sw128(sb + kk * 32, 16, 1024)
+                                            : tc::smem_desc_sw64(sb + kk * 32, 16, 512);
             const uint32_t dcol = (kSplit == 3 && q > 0) ? (uint32_t)BN : 0u;
             const bool acc_on = kSplit == 1 ? (kt | kk | q) != 0
                                             : (q == 0 ? (kt | kk) != 0 : ((kt | kk) != 0 || q > 1));
@@ -450,7 +472,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // handles four consecutive rows (features, contiguous in memory) of four
     // columns: 16-byte bias / mask loads, 16-byte stores of the output and
     // 8-byte stores of each bf16 piece.
-    float* tT = reinterpret_cast<float*>(smem + EpiT<BN, kSplit, kStages>::kOff) +
+    float* tT = reinterpret_cast<float*>(smem + Epi::kOff) +
                 warp * (32 * 32);
     const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
     const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
@@ -558,7 +580,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     };
     // fused output layer: W_L's rows for this tile's 128 features, the number
     // of 32-sample chunks with samples, and the scratch
-    float* sW3 = reinterpret_cast<float*>(smem + EpiT<BN, kSplit, kStages>::kHeadOff);
+    float* sW3 = reinterpret_cast<float*>(smem + Epi::kHeadOff);
     float* sPart = sW3 + kHC * 128;
     float* sG = sPart + 8 * 16 * kHC;
     uint16_t* sMask = reinterpret_cast<uint16_t*>(sG + 32 * kHC);   // [owned chunk][thread]
@@ -966,23 +988,25 @@ __global__ void split_pieces_kernel(const float* __restrict__ x, bf16* __restric
   }
 }
 
-template <int BN, int kSplit, int kStages>
+template <int BN, int kSplit, int kStages, int kBK>
 size_t smem_bytes() {
   // Shared memory requested per CTA also caps the CTAs per SM so that their
   // TMEM columns never exceed the 512 an SM has.
-  const size_t ring = (size_t)kStages * TileCfg<BN, kSplit>::kStageBytes + 1024 + 256 +
-                      (EpiT<BN, kSplit, kStages>::kSeparate ? kEpiTBytes : 0);
+  const size_t ring = (size_t)kStages * TileCfg<BN, kSplit, kBK>::kStageBytes + 1024 + 256 +
+                      (EpiT<BN, kSplit, kStages, kBK>::kSeparate ? kEpiTBytes : 0);
   const size_t floor_for_tmem =
-      (size_t)(233472 / (512 / TileCfg<BN, kSplit>::kTmemCols + 1)) + 1024;
+      (size_t)(233472 / (512 / TileCfg<BN, kSplit, kBK>::kTmemCols + 1)) + 1024;
   return std::max(ring, floor_for_tmem);
 }
 
 template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, int slots,
                  cudaStream_t st, bool* launched = nullptr) {
-  static_assert(kStages * TileCfg<BN, kSplit>::kStageBytes + 1280 <= 232448, "smem");
+  constexpr int kBK = stage_k(kSplit, kEpi);
+  using Epi = EpiT<BN, kSplit, kStages, kBK>;
+  static_assert(kStages * TileCfg<BN, kSplit, kBK>::kStageBytes + 1280 <= 232448, "smem");
   auto kern = tc_gemm_kernel<BN, kAMN, kBMN, kEpi, kStages, kSplit>;
-  const size_t smem = smem_bytes<BN, kSplit, kStages>();
+  const size_t smem = smem_bytes<BN, kSplit, kStages, kBK>();
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -994,8 +1018,7 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
   if (ks > 1) {
     // a rank that finishes chunks holds the other ranks' partial sums of
     // them (16 KB per chunk and rank) in its stage ring
-    const int ring = (int)(kEpi == kEpiFwdHead ? EpiT<BN, kSplit, kStages>::kHeadOff
-                                               : EpiT<BN, kSplit, kStages>::kRingFree);
+    const int ring = (int)(kEpi == kEpiFwdHead ? Epi::kHeadOff : Epi::kRingFree);
     auto need = [](int k) { return ((BN / 32 + k - 1) / k) * (k - 1) * (128 * 32 * 4); };
     while (ks > 1 && need(ks) > ring) --ks;
     const int kt = (args.K + kBK - 1) / kBK;
@@ -1088,7 +1111,9 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
   cuuint64_t dims[4] = {inner, rows, batch, 3};
   cuuint64_t strides[3] = {row_stride_elems * 2, batch_stride_elems * 2, piece_stride_elems * 2};
   cuuint32_t box[4] = {box_inner, box_rows, 1, 1};
-  return encode(map, 4, base, dims, strides, box);
+  // rows of 64 bytes take the 64-byte swizzle, rows of 128 bytes the 128-byte one
+  return encode(map, 4, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                box_inner * 2 == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
@@ -1104,9 +1129,9 @@ Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
                   cudaStream_t st, bool split, int bn) {
   if (split) {
-    if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 3, 3>(w_k, h_k, args, slots, st);
-    if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 2, 3>(w_k, h_k, args, slots, st);
-    return launch_tc<256, false, false, kEpiFwd, 1, 3>(w_k, h_k, args, slots, st);
+    if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 6, 3>(w_k, h_k, args, slots, st);
+    if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 4, 3>(w_k, h_k, args, slots, st);
+    return launch_tc<256, false, false, kEpiFwd, 3, 3>(w_k, h_k, args, slots, st);
   }
   if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 6, 1>(w_k, h_k, args, slots, st);
   if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 5, 1>(w_k, h_k, args, slots, st);
@@ -1123,10 +1148,10 @@ Status tc_forward_head(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcA
   if ((int64_t)ceil_div(args.M, 128) * slots > num_sms) return Status::Ok();
   if (split) {
     if (bn == 64)
-      return launch_tc<64, false, false, kEpiFwdHead, 3, 3>(w_k, h_k, args, slots, st, launched);
+      return launch_tc<64, false, false, kEpiFwdHead, 6, 3>(w_k, h_k, args, slots, st, launched);
     if (bn == 128)
-      return launch_tc<128, false, false, kEpiFwdHead, 2, 3>(w_k, h_k, args, slots, st, launched);
-    return launch_tc<256, false, false, kEpiFwdHead, 1, 3>(w_k, h_k, args, slots, st, launched);
+      return launch_tc<128, false, false, kEpiFwdHead, 4, 3>(w_k, h_k, args, slots, st, launched);
+    return launch_tc<256, false, false, kEpiFwdHead, 3, 3>(w_k, h_k, args, slots, st, launched);
   }
   if (bn == 64)
     return launch_tc<64, false, false, kEpiFwdHead, 6, 1>(w_k, h_k, args, slots, st, launched);
@@ -1138,9 +1163,9 @@ Status tc_forward_head(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcA
 Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const TcArgs& args,
                       int slots, cudaStream_t st, bool split, int bn) {
   if (split) {
-    if (bn == 64) return launch_tc<64, true, false, kEpiDX, 3, 3>(w_mn, dz_k, args, slots, st);
-    if (bn == 128) return launch_tc<128, true, false, kEpiDX, 2, 3>(w_mn, dz_k, args, slots, st);
-    return launch_tc<256, true, false, kEpiDX, 1, 3>(w_mn, dz_k, args, slots, st);
+    if (bn == 64) return launch_tc<64, true, false, kEpiDX, 6, 3>(w_mn, dz_k, args, slots, st);
+    if (bn == 128) return launch_tc<128, true, false, kEpiDX, 4, 3>(w_mn, dz_k, args, slots, st);
+    return launch_tc<256, true, false, kEpiDX, 3, 3>(w_mn, dz_k, args, slots, st);
   }
   if (bn == 64) return launch_tc<64, true, false, kEpiDX, 6, 1>(w_mn, dz_k, args, slots, st);
   if (bn == 128) return launch_tc<128, true, false, kEpiDX, 5, 1>(w_mn, dz_k, args, slots, st);

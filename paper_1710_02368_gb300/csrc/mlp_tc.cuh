@@ -81,6 +81,7 @@ struct TcArgs {
 // Column tile used for an N: the tensor map of the operand that spans N
 // must have this many rows (K-major) or 64-element chunks summing to it.
 inline int tc_bn(int N) { return N <= 64 ? 64 : N <= 128 ? 128 : 256; }
+constexpr int kTcSplitBK = 32;      // forward / dX k per stage, split (fp32) mode
 constexpr int kTcDwBN = 256;        // dW column tile, bf16 mode
 constexpr int kTcDwBNSplit = 128;   // dW column tile, split (fp32) mode
 

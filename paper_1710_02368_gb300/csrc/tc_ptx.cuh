@@ -233,6 +233,19 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
   return d;
 }
 
+// The same for a 64-byte swizzle (layout type 4): K-major tiles of 64-byte
+// rows, 8-row groups 512 bytes apart.
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr, uint32_t lbo_bytes,
+                                                   uint32_t sbo_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)4 << 61;
+  return d;
+}
+
 // Instruction descriptor of kind::f16 with bf16 A and B, f32 D, dense:
 // D format (1 = f32) bits 4-5, A format (1 = bf16) bits 7-9, B format bits
 // 10-12, A major (1 = MN-major) bit 15, B major bit 16, N >> 3 in 17-22,
