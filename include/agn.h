@@ -44,6 +44,9 @@ extern "C" {
 #define AGN_E_NONFINITE (-6)   /* a loss or a commit was not finite; the run
                                   still completed and theta~ is readable     */
 #define AGN_E_UNSUPPORTED (-7) /* valid request this build cannot serve      */
+#define AGN_E_BOUNDS (-8)      /* bounds-checked build only: a kernel access
+                                  outside every known device buffer was
+                                  refused (not performed); see agn_last_error */
 
 #define AGN_PREC_FP32 0        /* fp32 parameters, activations and GEMMs    */
 #define AGN_PREC_BF16 1        /* bf16 GEMM operands, fp32 accumulation, fp32

@@ -18,7 +18,7 @@ from ._lib import (AGN_COMMIT_AGN, AGN_COMMIT_DYNSGD, AGN_OPT_ADAM, AGN_OPT_SGD,
                    AGN_DIST_NORMAL, AGN_DIST_UNIFORM, AGN_GEMM_AUTO, AGN_GEMM_SIMT,  # noqa: F401
                    AGN_GEMM_TCGEN05, AGN_PREC_BF16, AGN_PREC_FP32, AGN_OK, AGN_E_INVALID,
                    AGN_E_SCHEDULE, AGN_E_OOM, AGN_E_CUDA, AGN_E_TIMEOUT, AGN_E_NONFINITE,
-                   AGN_E_UNSUPPORTED, agn_options)
+                   AGN_E_UNSUPPORTED, AGN_E_BOUNDS, agn_options)
 
 __all__ = [
     "AGNError", "AGN", "agn_default_options", "agn_create", "agn_run", "agn_central",
@@ -39,7 +39,7 @@ class AGNError(RuntimeError):
 
 
 def library_path() -> str:
-    return _lib.LIB_PATH
+    return _lib.library_file()
 
 
 def _L():

@@ -1,7 +1,9 @@
 """ctypes view of the AGN C ABI (include/agn.h): library loading and signatures.
 
 The library is built in-tree (`_build/libagn_gb300.so`, see build.py).  There
-is no fallback: if it is missing, loading raises.
+is no fallback: if it is missing, loading raises.  With AGN_LIB_VARIANT=check
+in the environment the bounds-checked build (`_build_check/
+libagn_gb300_check.so`) is loaded instead.
 """
 
 from __future__ import annotations
@@ -11,6 +13,7 @@ import os
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_build", "libagn_gb300.so")
+LIB_CHECK_PATH = os.path.join(HERE, "_build_check", "libagn_gb300_check.so")
 
 AGN_OK = 0
 AGN_E_INVALID = -1
@@ -20,6 +23,7 @@ AGN_E_CUDA = -4
 AGN_E_TIMEOUT = -5
 AGN_E_NONFINITE = -6
 AGN_E_UNSUPPORTED = -7
+AGN_E_BOUNDS = -8
 
 AGN_PREC_FP32 = 0
 AGN_PREC_BF16 = 1
@@ -40,6 +44,7 @@ ERROR_NAMES = {
     AGN_E_INVALID: "AGN_E_INVALID", AGN_E_SCHEDULE: "AGN_E_SCHEDULE", AGN_E_OOM: "AGN_E_OOM",
     AGN_E_CUDA: "AGN_E_CUDA", AGN_E_TIMEOUT: "AGN_E_TIMEOUT",
     AGN_E_NONFINITE: "AGN_E_NONFINITE", AGN_E_UNSUPPORTED: "AGN_E_UNSUPPORTED",
+    AGN_E_BOUNDS: "AGN_E_BOUNDS",
 }
 
 
@@ -118,15 +123,22 @@ SIGNATURES = {
 _LIB = None
 
 
+def library_file() -> str:
+    """The library this process loads: the bounds-checked build when
+    AGN_LIB_VARIANT=check, else the normal one."""
+    return LIB_CHECK_PATH if os.environ.get("AGN_LIB_VARIANT") == "check" else LIB_PATH
+
+
 def load():
     """Load the library (once) and declare every signature; raise if missing."""
     global _LIB
     if _LIB is None:
-        if not os.path.exists(LIB_PATH):
+        path = library_file()
+        if not os.path.exists(path):
             raise RuntimeError(
-                f"AGN CUDA library not found at {LIB_PATH}; build it first "
+                f"AGN CUDA library not found at {path}; build it first "
                 "(python -c 'import __graft_entry__ as g; g.build()')")
-        lib = C.CDLL(LIB_PATH)
+        lib = C.CDLL(path)
         for name, (res, args) in SIGNATURES.items():
             fn = getattr(lib, name)
             fn.restype = res

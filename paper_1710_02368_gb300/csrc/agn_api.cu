@@ -12,6 +12,8 @@
 // that creates the version it reads.  This gives the same theta~ as applying
 // the commits one at a time in schedule order.
 #include <chrono>
+#include <cstdlib>
+#include <mutex>
 #include <cmath>
 #include <cstdint>
 #include <new>
@@ -59,6 +61,99 @@ struct Wave {
 };
 
 }  // namespace
+
+#ifdef AGN_BOUNDS_CHECK
+namespace agn {
+// Each kernel translation unit's copy of the table (AGN_BOUNDS_UNIT).
+#define AGN_BOUNDS_DECL(unit)                                                           \
+  cudaError_t bounds_set_##unit(const BoundsTable& t, cudaStream_t st);                  \
+  cudaError_t bounds_get_##unit(unsigned long long* first, unsigned int* count, cudaStream_t st);
+AGN_BOUNDS_DECL(commit)
+AGN_BOUNDS_DECL(eval)
+AGN_BOUNDS_DECL(head)
+AGN_BOUNDS_DECL(simt)
+AGN_BOUNDS_DECL(tc)
+AGN_BOUNDS_DECL(dw)
+AGN_BOUNDS_DECL(optim)
+#undef AGN_BOUNDS_DECL
+
+namespace {
+std::mutex g_bounds_mu;
+std::vector<std::pair<unsigned long long, unsigned long long>> g_bounds_ranges;
+}  // namespace
+
+void bounds_add(const void* p, size_t bytes) {
+  if (!p || bytes == 0) return;
+  // self-test of the checker (tests/bounds_cases.py, case detect): every
+  // buffer registered this many bytes short of its end, so that accesses near
+  // the end, inside the real allocation, are refused
+  static const long long shrink =
+      std::getenv("AGN_BOUNDS_TEST_SHRINK") ? std::atoll(std::getenv("AGN_BOUNDS_TEST_SHRINK")) : 0;
+  if (shrink > 0) bytes = bytes > (size_t)shrink ? bytes - (size_t)shrink : 0;
+  std::lock_guard<std::mutex> lock(g_bounds_mu);
+  const unsigned long long a = reinterpret_cast<unsigned long long>(p);
+  g_bounds_ranges.push_back({a, a + bytes});
+}
+
+void bounds_remove(const void* p) {
+  std::lock_guard<std::mutex> lock(g_bounds_mu);
+  const unsigned long long a = reinterpret_cast<unsigned long long>(p);
+  for (size_t i = 0; i < g_bounds_ranges.size(); ++i)
+    if (g_bounds_ranges[i].first == a) {
+      g_bounds_ranges.erase(g_bounds_ranges.begin() + (std::ptrdiff_t)i);
+      return;
+    }
+}
+
+bool bounds_host_ok(const void* p, size_t bytes) {
+  std::lock_guard<std::mutex> lock(g_bounds_mu);
+  const unsigned long long a = reinterpret_cast<unsigned long long>(p);
+  for (const auto& r : g_bounds_ranges)
+    if (a >= r.first && a + bytes <= r.second) return true;
+  return false;
+}
+
+Status bounds_upload(cudaStream_t st) {
+  BoundsTable t{};
+  {
+    std::lock_guard<std::mutex> lock(g_bounds_mu);
+    if ((int)g_bounds_ranges.size() > kBoundsMax)
+      return Status::Err(AGN_E_UNSUPPORTED, "bounds-checked build: more than " +
+                                                std::to_string(kBoundsMax) + " live buffers");
+    t.n = (int)g_bounds_ranges.size();
+    for (int i = 0; i < t.n; ++i) {
+      t.lo[i] = g_bounds_ranges[i].first;
+      t.hi[i] = g_bounds_ranges[i].second;
+    }
+  }
+  using SetFn = cudaError_t (*)(const BoundsTable&, cudaStream_t);
+  for (SetFn f : {bounds_set_commit, bounds_set_eval, bounds_set_head, bounds_set_simt,
+                  bounds_set_tc, bounds_set_dw, bounds_set_optim})
+    AGN_TRY_CUDA(f(t, st));
+  return Status::Ok();
+}
+
+Status bounds_collect(cudaStream_t st) {
+  using GetFn = cudaError_t (*)(unsigned long long*, unsigned int*, cudaStream_t);
+  unsigned long long first = 0;
+  unsigned long long total = 0;
+  for (GetFn f : {bounds_get_commit, bounds_get_eval, bounds_get_head, bounds_get_simt,
+                  bounds_get_tc, bounds_get_dw, bounds_get_optim}) {
+    unsigned long long a = 0;
+    unsigned int c = 0;
+    AGN_TRY_CUDA(f(&a, &c, st));
+    total += c;
+    if (!first) first = a;
+  }
+  if (total == 0) return Status::Ok();
+  char buf[32];
+  std::snprintf(buf, sizeof(buf), "%llx", first);
+  return Status::Err(AGN_E_BOUNDS, "bounds-checked build: " + std::to_string(total) +
+                                       " kernel accesses outside every known device buffer "
+                                       "were refused, the first at 0x" + buf);
+}
+}  // namespace agn
+#endif
 
 struct agn_handle {
   // problem
@@ -217,6 +312,7 @@ Status dalloc(agn_handle* h, void** p, size_t bytes) {
                                       cudaGetErrorString(e));
   }
   h->allocs.push_back(*p);
+  agn::bounds_add(*p, bytes);
   return Status::Ok();
 }
 
@@ -224,6 +320,7 @@ void dfree(agn_handle* h, void* p) {
   if (!p) return;
   for (auto& a : h->allocs)
     if (a == p) a = nullptr;
+  agn::bounds_remove(p);
   cudaFree(p);
 }
 
@@ -907,6 +1004,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
     AGN_TRY(grow(h, &h->plan_t0, &c3, total_slots, 0));
     h->cap_plan = c1;
   }
+  AGN_TRY(agn::bounds_upload(h->stream));   // bounds-checked build: buffers as grown
   if (total_slots > 0) {
     AGN_TRY_CUDA(cudaMemcpyAsync(h->plan_worker, plan.slot_worker.data(), total_slots * sizeof(int),
                                  cudaMemcpyHostToDevice, h->stream));
@@ -968,6 +1066,7 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
   const double host_ms =
       std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t_host0).count();
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  const Status bounds = agn::bounds_collect(h->stream);   // bounds-checked build only
   float ms = 0.f;
   cudaEventElapsedTime(&ms, h->ev0, h->ev1);
   if (h->prof) collect_profile(h);
@@ -991,11 +1090,12 @@ Status do_run(agn_handle* h, int k, const int32_t* worker, const int32_t* tau, i
                                    h->stream));
     }
     AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+    if (!bounds.ok()) return bounds;
     if (flags[1])
       return Status::Err(AGN_E_TIMEOUT, "a tensor-core GEMM gave up on a bounded wait");
     return Status::Err(AGN_E_NONFINITE, "a loss or a commit was not finite");
   }
-  return Status::Ok();
+  return bounds;
 }
 
 Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_workers, int32_t lambda,
@@ -1257,10 +1357,12 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   for (int w = 0; w < n; ++w) all[w] = w;
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,
                                h->stream));
+  AGN_TRY(agn::bounds_upload(h->stream));   // bounds-checked build: the handle's buffers
   AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
                              (int)n, h->stream, h->piece_plane,
                              h->elide ? h->acc : nullptr));   // every worker pulls version 0
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  AGN_TRY(agn::bounds_collect(h->stream));
   return Status::Ok();
 }
 
@@ -1272,6 +1374,7 @@ Status evaluate(agn_handle* h, float* loss, float* accuracy, int32_t* pred, int6
     return Status::Err(AGN_E_INVALID, "the handle has no evaluation set (agn_options.n_eval)");
   if (pred && cap < h->n_eval) return Status::Err(AGN_E_INVALID, "pred shorter than n_eval");
   const int L = h->L, C = h->dims[L];
+  AGN_TRY(agn::bounds_upload(h->stream));   // bounds-checked build only
   for (int64_t r0 = 0; r0 < h->n_eval; r0 += h->eval_chunk) {
     const int rows = (int)std::min<int64_t>(h->eval_chunk, h->n_eval - r0);
     const float* in = h->Xe + r0 * h->dims[0];
@@ -1299,6 +1402,7 @@ Status evaluate(agn_handle* h, float* loss, float* accuracy, int32_t* pred, int6
     AGN_TRY_CUDA(cudaMemcpyAsync(pred, h->e_pred, (size_t)h->n_eval * sizeof(int32_t),
                                  cudaMemcpyDeviceToHost, h->stream));
   AGN_TRY_CUDA(cudaStreamSynchronize(h->stream));
+  AGN_TRY(agn::bounds_collect(h->stream));
   if (loss) *loss = o2[0];
   if (accuracy) *accuracy = o2[1];
   return Status::Ok();
@@ -1357,10 +1461,37 @@ Status commit_pull(float* theta_c, float* acc, float* reps, void* reps_b, int64_
   double* partials = nullptr;
   if (dnorm) AGN_TRY_CUDA(cudaMallocAsync((void**)&partials,
                                           sizeof(double) * agn::kMaxCommitsPerLaunch * grid, st));
+  int* extra_dev = nullptr;
+  // bounds-checked build: the caller's buffers are known for this call
+  // (the extents this entry point's arguments give them)
+  struct CallBuffers {
+    std::vector<const void*> added;
+    void add(const void* p, size_t b) {
+      if (p) {
+        agn::bounds_add(p, b);
+        added.push_back(p);
+      }
+    }
+    ~CallBuffers() {
+      for (const void* p : added) agn::bounds_remove(p);
+    }
+  } call;
+  call.add(theta_c, (size_t)P * sizeof(float));
+  call.add(acc, (size_t)n * ld * sizeof(float));
+  call.add(reps, (size_t)n * ld * sizeof(float));
+  call.add(reps_b, (size_t)n * ld * sizeof(bf16));
+  call.add(dnorm, (size_t)C * sizeof(float));
+  call.add(partials, sizeof(double) * agn::kMaxCommitsPerLaunch * grid);
+#ifdef AGN_BOUNDS_CHECK
+  if (po[C] > 0) {   // the list of pulls beyond one launch's capacity, known up front
+    AGN_TRY_CUDA(cudaMallocAsync((void**)&extra_dev, sizeof(int) * n, st));
+    call.add(extra_dev, sizeof(int) * n);
+  }
+#endif
+  AGN_TRY(agn::bounds_upload(st));
   Status result = Status::Ok();
   CommitPlan cp{};
   std::vector<int> extra;            // pulls that did not fit into the launch
-  int* extra_dev = nullptr;
   auto flush = [&]() -> Status {
     if (cp.n_commits > 0)
       AGN_TRY(agn::launch_commit_pull(cp, theta_c, acc, reps, static_cast<bf16*>(reps_b), P, ld,
@@ -1404,6 +1535,7 @@ Status commit_pull(float* theta_c, float* acc, float* reps, void* reps_b, int64_
     }
   }
   if (result.ok()) result = flush();
+  if (result.ok()) result = agn::bounds_collect(st);   // bounds-checked build only
   if (partials) cudaFreeAsync(partials, st);
   if (extra_dev) cudaFreeAsync(extra_dev, st);
   return result;
@@ -1603,7 +1735,10 @@ void agn_destroy(agn_handle* h) {
   DeviceGuard g(h->device);
   if (h->stream) cudaStreamSynchronize(h->stream);
   for (void* p : h->allocs)
-    if (p) cudaFree(p);
+    if (p) {
+      agn::bounds_remove(p);
+      cudaFree(p);
+    }
   for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
   if (h->ev0) cudaEventDestroy(h->ev0);
   if (h->ev1) cudaEventDestroy(h->ev1);

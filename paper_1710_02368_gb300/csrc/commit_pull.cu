@@ -31,8 +31,8 @@ constexpr int kThreads = 256;
 constexpr int kLongUnroll = 2, kLongGroup = 1;
 constexpr int kShortUnroll = 1, kShortGroup = 8;
 
-__device__ __forceinline__ float4 ld_stream(const float4* p) { return __ldcs(p); }
-__device__ __forceinline__ void st_stream(float4* p, float4 v) { __stcs(p, v); }
+__device__ __forceinline__ float4 ld_stream(const float4* p) { return AGN_LDCS(p); }
+__device__ __forceinline__ void st_stream(float4* p, float4 v) { AGN_STCS(p, v); }
 
 __device__ __forceinline__ uint2 pack_bf16x4(float4 v) {
   __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y);
@@ -95,7 +95,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
     for (int u = 0; u < kUnroll; ++u) {
       idx[u] = base + (int64_t)u * kThreads;
       live[u] = idx[u] < n4;
-      if (live[u]) th[u] = th4[idx[u]];
+      if (live[u]) th[u] = AGN_LD(th4 + idx[u]);
     }
     // commits in groups of kGroup: every accumulator load of a group is in
     // flight before the group's dependent chain of adds (theta~ must see the
@@ -151,15 +151,16 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
 #pragma unroll
           for (int u = 0; u < kUnroll; ++u) {
             if (!live[u]) continue;
-            reinterpret_cast<float4*>(replicas + row)[idx[u]] = th[u];
-            if (kElide) reinterpret_cast<float4*>(acc + row)[idx[u]] = th[u];
-            if (kCopy == 1) reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = pack_bf16x4(th[u]);
+            AGN_ST(reinterpret_cast<float4*>(replicas + row) + idx[u], th[u]);
+            if (kElide) AGN_ST(reinterpret_cast<float4*>(acc + row) + idx[u], th[u]);
+            if (kCopy == 1)
+              AGN_ST(reinterpret_cast<uint2*>(rep_bf16 + row) + idx[u], pack_bf16x4(th[u]));
             if (kCopy == 3) {
               uint2 q0, q1, q2;
               pack_pieces_x4(th[u], q0, q1, q2);
-              reinterpret_cast<uint2*>(rep_bf16 + row)[idx[u]] = q0;
-              reinterpret_cast<uint2*>(rep_bf16 + plane + row)[idx[u]] = q1;
-              reinterpret_cast<uint2*>(rep_bf16 + 2 * plane + row)[idx[u]] = q2;
+              AGN_ST(reinterpret_cast<uint2*>(rep_bf16 + row) + idx[u], q0);
+              AGN_ST(reinterpret_cast<uint2*>(rep_bf16 + plane + row) + idx[u], q1);
+              AGN_ST(reinterpret_cast<uint2*>(rep_bf16 + 2 * plane + row) + idx[u], q2);
             }
           }
         }
@@ -167,38 +168,41 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u)
-      if (live[u]) th4[idx[u]] = th[u];
+      if (live[u]) AGN_ST(th4 + idx[u], th[u]);
   }
 
   // Tail of P % 4 elements: block 0, one element per thread.
   if (blockIdx.x == 0 && threadIdx.x < (int)(P - n4 * 4)) {
     const int64_t i = n4 * 4 + threadIdx.x;
-    float t = theta_c[i];
+    float t = AGN_LD(theta_c + i);
     for (int c = 0; c < nc; ++c) {
       float* ap = acc + (int64_t)plan.worker[c] * ld + i;
-      const float av = kElide ? __fsub_rn(replicas[(int64_t)plan.worker[c] * ld + i], *ap) : *ap;
+      const float av = kElide ? __fsub_rn(AGN_LD(replicas + (int64_t)plan.worker[c] * ld + i),
+                                          AGN_LD(ap))
+                              : AGN_LD(ap);
       float d = __fmul_rn(av, plan.per_commit_scale ? plan.scale[c] : s);
       t = __fadd_rn(t, d);
 #pragma unroll
       for (int cc = 0; cc < kMaxCommitsPerLaunch; ++cc)
         if (cc == c) sq[cc] += (double)(d * d);
-      if (!kElide && zero_acc) *ap = 0.f;
+      if (!kElide && zero_acc) AGN_ST(ap, 0.f);
       for (int p = plan.pull_begin[c]; p < plan.pull_begin[c + 1]; ++p) {
         const int64_t row = (int64_t)plan.pull_worker[p] * ld;
-        replicas[row + i] = t;
-        if (kElide) acc[row + i] = t;
-        if (kCopy == 1) rep_bf16[row + i] = __float2bfloat16_rn(t);
+        AGN_ST(replicas + row + i, t);
+        if (kElide) AGN_ST(acc + row + i, t);
+        if (kCopy == 1) AGN_ST(rep_bf16 + row + i, __float2bfloat16_rn(t));
         if (kCopy == 3) {
           const bf16 q0 = __float2bfloat16_rn(t);
           const float r1 = __fsub_rn(t, __bfloat162float(q0));
           const bf16 q1 = __float2bfloat16_rn(r1);
-          rep_bf16[row + i] = q0;
-          rep_bf16[plane + row + i] = q1;
-          rep_bf16[2 * plane + row + i] = __float2bfloat16_rn(__fsub_rn(r1, __bfloat162float(q1)));
+          AGN_ST(rep_bf16 + row + i, q0);
+          AGN_ST(rep_bf16 + plane + row + i, q1);
+          AGN_ST(rep_bf16 + 2 * plane + row + i,
+                 __float2bfloat16_rn(__fsub_rn(r1, __bfloat162float(q1))));
         }
       }
     }
-    theta_c[i] = t;
+    AGN_ST(theta_c + i, t);
   }
 
   if (partials == nullptr) return;
@@ -217,7 +221,7 @@ commit_pull_kernel(const __grid_constant__ CommitPlan plan, float* __restrict__ 
   if (threadIdx.x < nc) {
     double v = 0.0;
     for (int w = 0; w < kThreads / 32; ++w) v += red[w][threadIdx.x];
-    partials[(int64_t)threadIdx.x * gridDim.x + blockIdx.x] = v;
+    AGN_ST(partials + (int64_t)threadIdx.x * gridDim.x + blockIdx.x, v);
   }
 }
 
@@ -230,7 +234,7 @@ reduce_norms_kernel(const double* __restrict__ partials, int grid, const __grid_
   const int slot = plan.norm_slot[c];
   const double* row = partials + (int64_t)c * grid;
   double v = 0.0;
-  for (int b = threadIdx.x; b < grid; b += kThreads) v += row[b];
+  for (int b = threadIdx.x; b < grid; b += kThreads) v += AGN_LD(row + b);
   __shared__ double red[kThreads];
   red[threadIdx.x] = v;
   __syncthreads();
@@ -240,7 +244,7 @@ reduce_norms_kernel(const double* __restrict__ partials, int grid, const __grid_
   }
   if (threadIdx.x == 0) {
     float nrm = (float)sqrt(red[0]);
-    if (norms) norms[slot] = nrm;
+    if (norms) AGN_ST(norms + slot, nrm);
     if (flag && !isfinite(nrm)) atomicExch(flag, 1);
   }
 }
@@ -314,24 +318,24 @@ pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
             bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers,
             int64_t plane, float* __restrict__ snapshot) {
   pdl_begin();
-  const int k = workers[blockIdx.y];
+  const int k = AGN_LD(workers + blockIdx.y);
   float* dst = replicas + (int64_t)k * ld;
   float* snap = snapshot ? snapshot + (int64_t)k * ld : nullptr;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < P; i += stride) {
-    const float t = theta_c[i];
-    dst[i] = t;
-    if (snap) snap[i] = t;
+    const float t = AGN_LD(theta_c + i);
+    AGN_ST(dst + i, t);
+    if (snap) AGN_ST(snap + i, t);
     if (rep_bf16) {
       const int64_t o = (int64_t)k * ld + i;
       if (plane > 0) {
         bf16 q0, q1, q2;
         split3(t, q0, q1, q2);
-        rep_bf16[o] = q0;
-        rep_bf16[plane + o] = q1;
-        rep_bf16[2 * plane + o] = q2;
+        AGN_ST(rep_bf16 + o, q0);
+        AGN_ST(rep_bf16 + plane + o, q1);
+        AGN_ST(rep_bf16 + 2 * plane + o, q2);
       } else {
-        rep_bf16[o] = __float2bfloat16_rn(t);
+        AGN_ST(rep_bf16 + o, __float2bfloat16_rn(t));
       }
     }
   }
@@ -345,11 +349,11 @@ __global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda
   float s = 0.f;
   for (int i = 0; i < lambda; ++i) {
     const float* p = parts + ((int64_t)c * lambda + i) * q_per;
-    float st = p[0];
-    for (int q = 1; q < q_per; ++q) st += p[q];
+    float st = AGN_LD(p);
+    for (int q = 1; q < q_per; ++q) st += AGN_LD(p + q);
     s += st;
   }
-  loss[c] = s / (float)lambda;
+  AGN_ST(loss + c, s / (float)lambda);
 }
 
 }  // namespace
@@ -446,5 +450,7 @@ Status fill_commit_inputs(float* theta_c, float* acc, float* replicas, int64_t P
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
+
+AGN_BOUNDS_UNIT(commit)
 
 }  // namespace agn

@@ -87,6 +87,28 @@ agn::Status commit_pull_noalloc(float* theta_c, float* acc, float* reps, void* r
   AGN_TRY(scratch_on_current_device(&scratch));
   const float scale = (float)(normalize ? -(eta / (double)lambda) : -eta);
   const int grid = std::min(agn::commit_grid(P), kNoAllocMaxGrid);
+  // bounds-checked build: the caller's buffers and the scratch array are known
+  // for this call (nothing is allocated; in the normal build this is empty)
+  struct CallBuffers {
+    const void* p[6] = {};
+    int k = 0;
+    void add(const void* q, size_t b) {
+      if (q) {
+        agn::bounds_add(q, b);
+        p[k++] = q;
+      }
+    }
+    ~CallBuffers() {
+      for (int i = 0; i < k; ++i) agn::bounds_remove(p[i]);
+    }
+  } call;
+  call.add(theta_c, (size_t)P * sizeof(float));
+  call.add(acc, (size_t)n * ld * sizeof(float));
+  call.add(reps, (size_t)n * ld * sizeof(float));
+  call.add(reps_b, (size_t)n * ld * sizeof(agn::bf16));
+  call.add(dnorm, (size_t)C * sizeof(float));
+  call.add(scratch, kScratchDoubles * sizeof(double));
+  AGN_TRY(agn::bounds_upload(st));
   agn::CommitPlan cp{};
   auto flush = [&]() -> Status {
     if (cp.n_commits > 0)
@@ -111,7 +133,8 @@ agn::Status commit_pull_noalloc(float* theta_c, float* acc, float* reps, void* r
     cp.pull_begin[i + 1] = pb;
     cp.n_commits = i + 1;
   }
-  return flush();
+  AGN_TRY(flush());
+  return agn::bounds_collect(st);   // bounds-checked build only
 }
 
 }  // namespace

@@ -12,6 +12,7 @@
 #include <utility>
 
 #include "../../include/agn.h"
+#include "bounds.cuh"
 
 namespace agn {
 
@@ -74,6 +75,25 @@ inline Status cuda_status(cudaError_t e, const char* what) {
     ::agn::Status s__ = (expr);   \
     if (!s__.ok()) return s__;    \
   } while (0)
+
+// The host's table of device buffers for the bounds-checked build
+// (bounds.cuh): buffers are added when allocated (or, for a standalone call,
+// for its duration), the table is uploaded to every kernel translation unit
+// before kernels run and the units' refusal counts are collected after.  In
+// the normal build these do nothing.
+#ifdef AGN_BOUNDS_CHECK
+void bounds_add(const void* p, size_t bytes);
+void bounds_remove(const void* p);
+bool bounds_host_ok(const void* p, size_t bytes);
+Status bounds_upload(cudaStream_t st);
+Status bounds_collect(cudaStream_t st);
+#else
+inline void bounds_add(const void*, size_t) {}
+inline void bounds_remove(const void*) {}
+inline bool bounds_host_ok(const void*, size_t) { return true; }
+inline Status bounds_upload(cudaStream_t) { return Status::Ok(); }
+inline Status bounds_collect(cudaStream_t) { return Status::Ok(); }
+#endif
 
 constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }

@@ -22,20 +22,21 @@ eval_logits_kernel(const float* __restrict__ Z, const int* __restrict__ y, int r
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= rows) return;
   const float* z = Z + (int64_t)i * C;
-  float mx = z[0];
+  float mx = AGN_LD(z);
   int am = 0;
   for (int c = 1; c < C; ++c) {
-    if (z[c] > mx) {   // strict: the lowest index wins ties
-      mx = z[c];
+    const float zc = AGN_LD(z + c);
+    if (zc > mx) {   // strict: the lowest index wins ties
+      mx = zc;
       am = c;
     }
   }
   float s = 0.f;
-  for (int c = 0; c < C; ++c) s += expf(z[c] - mx);
-  const int yi = y[i];
-  loss[i] = (logf(s) + mx) - z[yi];
-  correct[i] = am == yi ? 1 : 0;
-  if (pred) pred[i] = am;
+  for (int c = 0; c < C; ++c) s += expf(AGN_LD(z + c) - mx);
+  const int yi = AGN_LD(y + i);
+  AGN_ST(loss + i, (logf(s) + mx) - AGN_LD(z + yi));
+  AGN_ST(correct + i, am == yi ? 1 : 0);
+  if (pred) AGN_ST(pred + i, am);
 }
 
 // out[0] = mean loss, out[1] = accuracy over E samples: thread t sums samples
@@ -47,8 +48,8 @@ eval_reduce_kernel(const float* __restrict__ loss, const int* __restrict__ corre
   __shared__ double ws[kEvalThreads / 32][2];
   double l = 0.0, c = 0.0;
   for (int64_t i = threadIdx.x; i < E; i += blockDim.x) {
-    l += (double)loss[i];
-    c += (double)correct[i];
+    l += (double)AGN_LD(loss + i);
+    c += (double)AGN_LD(correct + i);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -67,8 +68,8 @@ eval_reduce_kernel(const float* __restrict__ loss, const int* __restrict__ corre
       L += ws[w][0];
       Cc += ws[w][1];
     }
-    out[0] = (float)(L / (double)E);
-    out[1] = (float)(Cc / (double)E);
+    AGN_ST(out, (float)(L / (double)E));
+    AGN_ST(out + 1, (float)(Cc / (double)E));
   }
 }
 
@@ -135,5 +136,7 @@ Status temporal_efficiency(const double* ta, const double* fa, int64_t na, const
   *out = integral_to(ta, fa, na, m) / ib;
   return Status::Ok();
 }
+
+AGN_BOUNDS_UNIT(eval)
 
 }  // namespace agn

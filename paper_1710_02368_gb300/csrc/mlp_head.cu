@@ -42,6 +42,11 @@ __device__ __forceinline__ bf16 st_f<bf16>(float v) { return __float2bfloat16_rn
 // elsewhere.  The caller waits with cp.async.wait_all before its barrier.
 template <typename T>
 __device__ __forceinline__ void stage(T* dst, const T* src, int64_t count) {
+  // bounds-checked build: a source row outside every known buffer is not copied
+  if (!AGN_BOUNDS_OK(src, (unsigned int)(count * sizeof(T)))) {
+    if (threadIdx.x == 0) AGN_BOUNDS_FAIL(src);
+    return;
+  }
   constexpr int kVec = 16 / sizeof(T);
   const bool aligned = ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0;
   if (aligned) {
@@ -73,7 +78,7 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   const int j0 = blockIdx.x * kHeadSamples;
   const int K = a.K, C = a.C, m = a.m;
   const int nj = min(kHeadSamples, m - j0);
-  const int w = a.slot_worker[z];
+  const int w = AGN_LD(a.slot_worker + z);
   const int64_t Kp = (K + 7) / 8 * 8;   // padded row length in shared memory
   T* Ws = reinterpret_cast<T*>(head_smem);                  // [C][Kp]
   T* Hs = Ws + (int64_t)C * Kp;                             // [kHeadSamples][Kp]
@@ -122,9 +127,9 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
       float v = 0.f;
 #pragma unroll
       for (int r = 0; r < kHeadSplit; ++r) v += red[sj][r][c < C ? c : 0];
-      zc[c] = c < C ? v + bias[c] : -INFINITY;
+      zc[c] = c < C ? v + AGN_LD(bias + c) : -INFINITY;
     }
-    const int y = a.yb[(int64_t)z * m + j];
+    const int y = AGN_LD(a.yb + (int64_t)z * m + j);
     float mx = zc[0];
 #pragma unroll
     for (int c = 1; c < kMaxC; ++c) mx = fmaxf(mx, zc[c]);
@@ -150,13 +155,13 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
       for (int c = 0; c < kMaxC; ++c)
         if (c < C && lane == c) {
           const T gv = st_f<T>(g[c]);
-          dzl[c] = gv;
+          AGN_ST(dzl + c, gv);
           if (dzp) {
             bf16 q0, q1, q2;
             split3(cvt(gv), q0, q1, q2);
-            dzp[c] = q0;
-            dzp[a.dZL_plane + c] = q1;
-            dzp[2 * a.dZL_plane + c] = q2;
+            AGN_ST(dzp + c, q0);
+            AGN_ST(dzp + a.dZL_plane + c, q1);
+            AGN_ST(dzp + 2 * a.dZL_plane + c, q2);
           }
         }
     }
@@ -173,13 +178,13 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
       }
       const float v = v0 + v1;
       const T out = st_f<T>(cvt(h[k]) > 0.f ? v : 0.f);
-      dh[k] = out;
+      AGN_ST(dh + k, out);
       if (dp) {
         bf16 q0, q1, q2;
         split3(cvt(out), q0, q1, q2);
-        dp[k] = q0;
-        dp[a.dH_plane + k] = q1;
-        dp[2 * a.dH_plane + k] = q2;
+        AGN_ST(dp + k, q0);
+        AGN_ST(dp + a.dH_plane + k, q1);
+        AGN_ST(dp + 2 * a.dH_plane + k, q2);
       }
     }
   }
@@ -194,15 +199,21 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   if (threadIdx.x == 0) {
     float part = 0.f;
     for (int r = 0; r < kHeadSamples; ++r) part += ce_s[r];
-    a.ce_partial[(int64_t)z * nblk + blockIdx.x] = part;
+    AGN_ST(a.ce_partial + (int64_t)z * nblk + blockIdx.x, part);
     __threadfence();
-    s_last = atomicAdd(a.counter + z, 1) == nblk - 1;
+    if (AGN_BOUNDS_OK(a.counter + z, 4)) {
+      s_last = atomicAdd(a.counter + z, 1) == nblk - 1;
+    } else {
+      AGN_BOUNDS_FAIL(a.counter + z);
+      s_last = 0;
+    }
   }
   __syncthreads();
   if (!s_last) return;   // uniform across the block
   __threadfence();
   float v = 0.f;
-  for (int b = threadIdx.x; b < nblk; b += blockDim.x) v += __ldcg(a.ce_partial + (int64_t)z * nblk + b);
+  for (int b = threadIdx.x; b < nblk; b += blockDim.x)
+    v += AGN_LDCG(a.ce_partial + (int64_t)z * nblk + b);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
   if (lane == 0) warp_sum[warp] = v;
@@ -211,11 +222,11 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
     float tot = 0.f;
     for (int q = 0; q < kHeadThreads / 32; ++q) tot += warp_sum[q];
     const float loss = tot / (float)m;
-    float* lp = a.loss_parts + ((int64_t)a.slot_commit[z] * a.lam + a.step) * a.loss_q;
-    lp[0] = loss;
-    for (int q = 1; q < a.loss_q; ++q) lp[q] = 0.f;
+    float* lp = a.loss_parts + ((int64_t)AGN_LD(a.slot_commit + z) * a.lam + a.step) * a.loss_q;
+    AGN_ST(lp, loss);
+    for (int q = 1; q < a.loss_q; ++q) AGN_ST(lp + q, 0.f);
     if (!isfinite(loss)) atomicExch(a.flag, 1);
-    a.counter[z] = 0;
+    AGN_ST(a.counter + z, 0);
   }
 }
 
@@ -244,7 +255,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
   if (!a.dz_early) stage(dz, static_cast<const T*>(a.dZL) + (int64_t)z * m * C, (int64_t)m * C);
   stage_wait();
   __syncthreads();
-  const int w = a.slot_worker[z];
+  const int w = AGN_LD(a.slot_worker + z);
   const int k = blockIdx.x * 32 + lane;
   const T* hg = static_cast<const T*>(a.H) + (int64_t)z * m * K + k;
   float g[kMaxC];
@@ -256,7 +267,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
     for (; j + (kU - 1) * kDwGroups < m; j += kU * kDwGroups) {
       float hv[kU];
 #pragma unroll
-      for (int u = 0; u < kU; ++u) hv[u] = cvt(hg[(int64_t)(j + u * kDwGroups) * K]);
+      for (int u = 0; u < kU; ++u) hv[u] = cvt(AGN_LD(hg + (int64_t)(j + u * kDwGroups) * K));
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
         const T* dzj = dz + (j + u * kDwGroups) * C;
@@ -266,7 +277,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       }
     }
     for (; j < m; j += kDwGroups) {
-      const float hv = cvt(hg[(int64_t)j * K]);
+      const float hv = cvt(AGN_LD(hg + (int64_t)j * K));
       const T* dzj = dz + j * C;
 #pragma unroll
       for (int c = 0; c < kMaxC; ++c)
@@ -281,17 +292,17 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
   bf16* tb = a.theta_b ? a.theta_b + (int64_t)w * a.ld_param : nullptr;
   auto update = [&](int64_t p, float gr, float th, float ac) {
     const float t = fmaf(-a.eta, gr, th);
-    theta[p] = t;
-    if (acc) acc[p] = ac + gr;
+    AGN_ST(theta + p, t);
+    if (acc) AGN_ST(acc + p, ac + gr);
     if (tb) {
       if (a.piece_plane > 0) {
         bf16 q0, q1, q2;
         split3(t, q0, q1, q2);
-        tb[p] = q0;
-        tb[a.piece_plane + p] = q1;
-        tb[2 * a.piece_plane + p] = q2;
+        AGN_ST(tb + p, q0);
+        AGN_ST(tb + a.piece_plane + p, q1);
+        AGN_ST(tb + 2 * a.piece_plane + p, q2);
       } else {
-        tb[p] = __float2bfloat16_rn(t);
+        AGN_ST(tb + p, __float2bfloat16_rn(t));
       }
     }
   };
@@ -302,7 +313,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
         float v = 0.f;
 #pragma unroll
         for (int r = 0; r < kDwGroups; ++r) v += red[(r * kMaxC + c) * 32 + lane];
-        go[a.woff + (int64_t)c * K + k] = v;
+        AGN_ST(go + a.woff + (int64_t)c * K + k, v);
       }
     }
     if (blockIdx.x == 0 && warp == kDwGroups - 1) {
@@ -311,7 +322,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
         for (int j = lane; j < m; j += 32) v += cvt(dz[j * C + c]);
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) go[a.boff + c] = v;
+        if (lane == 0) AGN_ST(go + a.boff + c, v);
       }
     }
     return;
@@ -324,8 +335,8 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       const int c = warp + e * kDwGroups;
       if (c < C) {
         const int64_t p = a.woff + (int64_t)c * K + k;
-        th[e] = theta[p];
-        ac[e] = acc ? acc[p] : 0.f;
+        th[e] = AGN_LD(theta + p);
+        ac[e] = acc ? AGN_LD(acc + p) : 0.f;
         float v = 0.f;
 #pragma unroll
         for (int r = 0; r < kDwGroups; ++r) v += red[(r * kMaxC + c) * 32 + lane];
@@ -344,7 +355,8 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
       for (int j = lane; j < m; j += 32) v += cvt(dz[j * C + c]);
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (lane == 0) update(a.boff + c, v, theta[a.boff + c], acc ? acc[a.boff + c] : 0.f);
+      if (lane == 0)
+        update(a.boff + c, v, AGN_LD(theta + a.boff + c), acc ? AGN_LD(acc + a.boff + c) : 0.f);
     }
   }
 }
@@ -418,5 +430,7 @@ template Status head_forward_backward<float>(const HeadArgs&, int, cudaStream_t)
 template Status head_forward_backward<bf16>(const HeadArgs&, int, cudaStream_t);
 template Status head_backward_dw<float>(const HeadDwArgs&, int, cudaStream_t);
 template Status head_backward_dw<bf16>(const HeadDwArgs&, int, cudaStream_t);
+
+AGN_BOUNDS_UNIT(head)
 
 }  // namespace agn

@@ -38,11 +38,11 @@ __device__ __forceinline__ void write_copy(bf16* tb, int64_t plane, int64_t p, f
   if (plane > 0) {
     bf16 q0, q1, q2;
     split3(t, q0, q1, q2);
-    tb[p] = q0;
-    tb[plane + p] = q1;
-    tb[2 * plane + p] = q2;
+    AGN_ST(tb + p, q0);
+    AGN_ST(tb + plane + p, q1);
+    AGN_ST(tb + 2 * plane + p, q2);
   } else {
-    tb[p] = __float2bfloat16_rn(t);
+    AGN_ST(tb + p, __float2bfloat16_rn(t));
   }
 }
 
@@ -53,7 +53,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
   __shared__ float As[kBK][kBM + 1];
   __shared__ float Bs[kBK][kBN + 1];
   const int z = blockIdx.z;
-  const int w = g.slot_worker[z];
+  const int w = AGN_LD(g.slot_worker + z);
   const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * kBN;
   const T* A = reinterpret_cast<const T*>(g.a) + (g.a_by_worker ? (int64_t)w : z) * g.a_bstride;
   const T* B = reinterpret_cast<const T*>(g.b) + (g.b_by_worker ? (int64_t)w : z) * g.b_bstride;
@@ -76,7 +76,8 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       if (kAKMajor) { mm = e / kBK; kk = e % kBK; } else { kk = e / kBM; mm = e % kBM; }
       const int64_t gm = m0 + mm, gk = k0 + kk;
       float v = 0.f;
-      if (gm < g.M && gk < g.K) v = to_f(kAKMajor ? A[gm * g.lda + gk] : A[gk * g.lda + gm]);
+      if (gm < g.M && gk < g.K)
+        v = to_f(AGN_LD(kAKMajor ? A + gm * g.lda + gk : A + gk * g.lda + gm));
       As[kk][mm] = v;
     }
 #pragma unroll
@@ -86,7 +87,8 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       if (kBKMajor) { nn = e / kBK; kk = e % kBK; } else { kk = e / kBN; nn = e % kBN; }
       const int64_t gn = n0 + nn, gk = k0 + kk;
       float v = 0.f;
-      if (gn < g.N && gk < g.K) v = to_f(kBKMajor ? B[gn * g.ldb + gk] : B[gk * g.ldb + gn]);
+      if (gn < g.N && gk < g.K)
+        v = to_f(AGN_LD(kBKMajor ? B + gn * g.ldb + gk : B + gk * g.ldb + gn));
       Bs[kk][nn] = v;
     }
     __syncthreads();
@@ -122,9 +124,9 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       for (int j = 0; j < kTN; ++j) {
         const int64_t n = n0 + tx + j * (kBN / kTN);
         if (n >= g.N) continue;
-        float v = acc[i][j] + bias[n];
+        float v = acc[i][j] + AGN_LD(bias + n);
         if (g.relu) v = fmaxf(v, 0.f);
-        out[m * g.ldo + n] = from_f<TO>(v);
+        AGN_ST(out + m * g.ldo + n, from_f<TO>(v));
       }
     }
   } else if (kEpi == kEpiDX) {
@@ -138,8 +140,8 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
       for (int j = 0; j < kTN; ++j) {
         const int64_t n = n0 + tx + j * (kBN / kTN);
         if (n >= g.N) continue;
-        const float h = to_f(mask[m * g.ldo + n]);
-        out[m * g.ldo + n] = from_f<TO>(h > 0.f ? acc[i][j] : 0.f);
+        const float h = to_f(AGN_LD(mask + m * g.ldo + n));
+        AGN_ST(out + m * g.ldo + n, from_f<TO>(h > 0.f ? acc[i][j] : 0.f));
       }
     }
   } else if (g.grad_out) {   // kEpiDW, raw gradient out (the optimizer runs after)
@@ -151,10 +153,10 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
 #pragma unroll
       for (int j = 0; j < kTN; ++j) {
         const int64_t n = n0 + tx + j * (kBN / kTN);
-        if (n < g.N) go[g.woff + m * g.N + n] = acc[i][j];
+        if (n < g.N) AGN_ST(go + g.woff + m * g.N + n, acc[i][j]);
       }
     }
-    if (do_bias && m0 + tid < g.M) go[g.boff + m0 + tid] = bsum;
+    if (do_bias && m0 + tid < g.M) AGN_ST(go + g.boff + m0 + tid, bsum);
   } else {   // kEpiDW: theta_k -= eta g, a_k += g (unless elided), bf16 copy refresh
     const bool has_a = g.acc != nullptr;
     float* a = has_a ? g.acc + (int64_t)w * g.ld_param : theta;
@@ -171,8 +173,8 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         const int64_t n = n0 + tx + j * (kBN / kTN);
         if (m < g.M && n < g.N) {
           const int64_t p = g.woff + m * g.N + n;
-          th[i][j] = __ldcs(th_in + p);
-          av[i][j] = has_a ? __ldcs(a_in + p) : 0.f;
+          th[i][j] = AGN_LDCS(th_in + p);
+          av[i][j] = has_a ? AGN_LDCS(a_in + p) : 0.f;
         }
       }
     }
@@ -187,16 +189,16 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         const int64_t p = g.woff + m * g.N + n;
         const float gr = acc[i][j];
         const float t = fmaf(-g.eta, gr, th[i][j]);
-        theta[p] = t;
-        if (has_a) a[p] = av[i][j] + gr;
+        AGN_ST(theta + p, t);
+        if (has_a) AGN_ST(a + p, av[i][j] + gr);
         if (tb) write_copy(tb, g.piece_plane, p, t);
       }
     }
     if (do_bias && m0 + tid < g.M) {
       const int64_t p = g.boff + m0 + tid;
-      const float t = fmaf(-g.eta, bsum, theta[p]);
-      theta[p] = t;
-      if (has_a) a[p] += bsum;
+      const float t = fmaf(-g.eta, bsum, AGN_LD(theta + p));
+      AGN_ST(theta + p, t);
+      if (has_a) AGN_ST(a + p, AGN_LD(a + p) + bsum);
       if (tb) write_copy(tb, g.piece_plane, p, t);
     }
   }
@@ -220,17 +222,17 @@ __global__ void __launch_bounds__(128) softmax_xent_kernel(const float* __restri
   float part = 0.f;
   for (int j = threadIdx.x; j < m; j += blockDim.x) {
     const float* zr = Zs + (int64_t)j * C;
-    float mx = zr[0];
-    for (int c = 1; c < C; ++c) mx = fmaxf(mx, zr[c]);
+    float mx = AGN_LD(zr);
+    for (int c = 1; c < C; ++c) mx = fmaxf(mx, AGN_LD(zr + c));
     float s = 0.f;
-    for (int c = 0; c < C; ++c) s += expf(zr[c] - mx);
-    const int y = ys[j];
-    part += (logf(s) + mx) - zr[y];
+    for (int c = 0; c < C; ++c) s += expf(AGN_LD(zr + c) - mx);
+    const int y = AGN_LD(ys + j);
+    part += (logf(s) + mx) - AGN_LD(zr + y);
     const float inv_s = 1.0f / s;
     for (int c = 0; c < C; ++c) {
-      float p = expf(zr[c] - mx) * inv_s;
+      float p = expf(AGN_LD(zr + c) - mx) * inv_s;
       if (c == y) p -= 1.0f;
-      dZs[(int64_t)j * C + c] = from_f<T>(p * inv_m);
+      AGN_ST(dZs + (int64_t)j * C + c, from_f<T>(p * inv_m));
     }
   }
   __shared__ float red[128];
@@ -242,7 +244,7 @@ __global__ void __launch_bounds__(128) softmax_xent_kernel(const float* __restri
   }
   if (threadIdx.x == 0) {
     const float loss = red[0] * inv_m;
-    loss_parts[(int64_t)slot_commit[z] * lam + step] = loss;
+    AGN_ST(loss_parts + (int64_t)AGN_LD(slot_commit + z) * lam + step, loss);
     if (!isfinite(loss)) atomicExch(flag, 1);
   }
 }
@@ -257,24 +259,24 @@ __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ y
                               const long long* slot_t0, int step, bf16* pieces, int64_t plane) {
   pdl_begin();
   const int z = blockIdx.y, j = blockIdx.x;
-  const int w = slot_worker[z];
-  const long long t = slot_t0[z] + step;
+  const int w = AGN_LD(slot_worker + z);
+  const long long t = AGN_LD(slot_t0 + z) + step;
   const int64_t row = (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
   const T* src = X + row * d0;
   const int64_t o = ((int64_t)z * m + j) * d0;
   T* dst = Xb + o;
   for (int c = threadIdx.x; c < d0; c += blockDim.x) {
-    const T v = src[c];
-    dst[c] = v;
+    const T v = AGN_LD(src + c);
+    AGN_ST(dst + c, v);
     if (pieces) {
       bf16 q0, q1, q2;
       split3(to_f(v), q0, q1, q2);
-      pieces[o + c] = q0;
-      pieces[plane + o + c] = q1;
-      pieces[2 * plane + o + c] = q2;
+      AGN_ST(pieces + o + c, q0);
+      AGN_ST(pieces + plane + o + c, q1);
+      AGN_ST(pieces + 2 * plane + o + c, q2);
     }
   }
-  if (threadIdx.x == 0) yb[(int64_t)z * m + j] = y[row];
+  if (threadIdx.x == 0) AGN_ST(yb + (int64_t)z * m + j, AGN_LD(y + row));
 }
 
 // The same gather, four consecutive elements per thread (d_0 a multiple of
@@ -299,25 +301,25 @@ __global__ void __launch_bounds__(256) gather4_kernel(const T* __restrict__ X,
   struct alignas(8) Piece4 { bf16 v[4]; };
   const int r = blockIdx.x;                 // slot * m + j
   const int z = r / m, j = r - z * m;
-  const int w = slot_worker[z];
-  const long long t = slot_t0[z] + step;
+  const int w = AGN_LD(slot_worker + z);
+  const long long t = AGN_LD(slot_t0 + z) + step;
   const int64_t row =
       (int64_t)w * S + (int64_t)(((unsigned long long)t * m + j) % (unsigned long long)S);
   const T* src = X + row * d0;
   const int64_t o = (int64_t)r * d0;
   for (int c = threadIdx.x * 4; c < d0; c += blockDim.x * 4) {
-    const Vec v = *reinterpret_cast<const Vec*>(src + c);
-    if (Xb) *reinterpret_cast<Vec*>(Xb + o + c) = v;
+    const Vec v = AGN_LD(reinterpret_cast<const Vec*>(src + c));
+    if (Xb) AGN_ST(reinterpret_cast<Vec*>(Xb + o + c), v);
     if (pieces) {
       Piece4 p0, p1, p2;
 #pragma unroll
       for (int e = 0; e < 4; ++e) split3(to_f(v.v[e]), p0.v[e], p1.v[e], p2.v[e]);
-      *reinterpret_cast<Piece4*>(pieces + o + c) = p0;
-      *reinterpret_cast<Piece4*>(pieces + plane + o + c) = p1;
-      *reinterpret_cast<Piece4*>(pieces + 2 * plane + o + c) = p2;
+      AGN_ST(reinterpret_cast<Piece4*>(pieces + o + c), p0);
+      AGN_ST(reinterpret_cast<Piece4*>(pieces + plane + o + c), p1);
+      AGN_ST(reinterpret_cast<Piece4*>(pieces + 2 * plane + o + c), p2);
     }
   }
-  if (threadIdx.x == 0) yb[r] = y[row];
+  if (threadIdx.x == 0) AGN_ST(yb + r, AGN_LD(y + row));
   if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
@@ -400,5 +402,7 @@ Status gather_batch(const T* X, const int* y, T* Xb, int* yb, int d0, int m, int
 AGN_INST(float)
 AGN_INST(bf16)
 #undef AGN_INST
+
+AGN_BOUNDS_UNIT(simt)
 
 }  // namespace agn

@@ -90,9 +90,11 @@ __device__ __forceinline__ float from_act(bf16 v) { return __bfloat162float(v); 
 __device__ __forceinline__ float from_act(float v) { return v; }
 
 // Four consecutive activations (16-byte aligned fp32, or 8-byte aligned bf16).
-__device__ __forceinline__ float4 load4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 load4(const float* p) {
+  return AGN_LD(reinterpret_cast<const float4*>(p));
+}
 __device__ __forceinline__ float4 load4(const bf16* p) {
-  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const uint2 u = AGN_LD(reinterpret_cast<const uint2*>(p));
   const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
   const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
   return make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
@@ -103,10 +105,10 @@ __device__ __forceinline__ uint2 bf16x4(const float (&x)[4]) {
   return make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
 }
 __device__ __forceinline__ void store4(float* p, const float (&v)[4]) {
-  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  AGN_ST(reinterpret_cast<float4*>(p), make_float4(v[0], v[1], v[2], v[3]));
 }
 __device__ __forceinline__ void store4(bf16* p, const float (&v)[4]) {
-  *reinterpret_cast<uint2*>(p) = bf16x4(v);
+  AGN_ST(reinterpret_cast<uint2*>(p), bf16x4(v));
 }
 // The three exact bf16 pieces of four floats (split3 of each), packed.
 __device__ __forceinline__ void split3_x4(const float (&x)[4], uint2& q0, uint2& q1, uint2& q2) {
@@ -177,7 +179,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int ks = kEpi == kEpiDW ? 1 : args.ksplit;   // CTAs sharing one output tile
   const int m_tile = blockIdx.x, n_tile = blockIdx.y;
   const int slot = blockIdx.z / ks, sk = blockIdx.z % ks;
-  const int worker = args.slot_worker[slot];
+  const int worker = AGN_LD(args.slot_worker + slot);
   // k steps [kt0, kt0 + KT) of this CTA (the host picks ks so that none is empty)
   const int KT_all = (args.K + kBK - 1) / kBK;
   const int kt_per = (KT_all + ks - 1) / ks;
@@ -417,10 +419,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // cleared by the launch before it)
   if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) {
     if (args.counter_clear)
-      for (int i = threadIdx.x; i < args.counter_clear_n; i += kThreads) args.counter_clear[i] = 0;
+      for (int i = threadIdx.x; i < args.counter_clear_n; i += kThreads)
+        AGN_ST(args.counter_clear + i, 0);
     if (kEpi == kEpiFwdHead && args.head_counter_clear)
       for (int i = threadIdx.x; i < args.head_counter_clear_n; i += kThreads)
-        args.head_counter_clear[i] = 0;
+        AGN_ST(args.head_counter_clear + i, 0);
   }
   // block-uniform, so that the epilogue's barriers and warp-wide TMEM loads
   // are reached by every thread or by none
@@ -496,7 +499,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     constexpr bool kFwd = kEpi == kEpiFwd || kEpi == kEpiFwdHead;
     float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
     if (kFwd && row4_ok && n_own > 0)
-      bias4 = *reinterpret_cast<const float4*>(theta + args.boff + row4);
+      bias4 = AGN_LD(reinterpret_cast<const float4*>(theta + args.boff + row4));
     if (n_own > 0) load_mask(32 * own_rank + co);
     // fused output layer: this tile's 128 columns of W_L (kHC x 128, zero past
     // C and M), loads in flight across the split-K exchange
@@ -508,7 +511,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       for (int k = 0; k < kW3Per; ++k) {
         const int i = threadIdx.x + k * kThreads;
         const int c = i >> 7, rr = 128 * m_tile + (i & 127);
-        w3v_reg[k] = (c < args.head_C && rr < args.M) ? w3g[(int64_t)c * args.M + rr] : 0.f;
+        w3v_reg[k] = (c < args.head_C && rr < args.M) ? AGN_LD(w3g + (int64_t)c * args.M + rr) : 0.f;
       }
     }
     bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
@@ -521,7 +524,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         tmem_vals(32 * j + co, r);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          __stcg(mine + (int64_t)(32 * j + co + i) * 128 + trow, __uint_as_float(r[i]));
+          AGN_STCG(mine + (int64_t)(32 * j + co + i) * 128 + trow, __uint_as_float(r[i]));
       }
       // the CTA's stores, ordered by the barrier, are released by one
       // acquire-release arrival; the wait acquires the other ranks'
@@ -529,9 +532,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       __syncthreads();
       if (threadIdx.x == 0) {
         int* ctr = args.counter + tile_id;
-        if (sk + 1 != args.withhold_rank) tc::atomic_add_acq_rel_gpu(ctr, 1);
-        bool got = true;
-        if (n_own > 0) {
+        bool got = AGN_BOUNDS_OK(ctr, 4);
+        if (!got) AGN_BOUNDS_FAIL(ctr);   // bounds-checked build: no wait on a stray counter
+        if (got && sk + 1 != args.withhold_rank) tc::atomic_add_acq_rel_gpu(ctr, 1);
+        if (got && n_own > 0) {
           got = tc::wait_count_low(ctr, ks, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
           if (got) {
             tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
@@ -540,10 +544,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               const int j = sk + o * ks;
               for (int q = 0; q < ks; ++q) {
                 if (q == sk) continue;
-                tc::bulk_load(smem + (size_t)d * kChunkBytes,
-                              args.part + (tile_id * ks + q) * (int64_t)(128 * BN) +
-                                  (int64_t)j * (32 * 128),
-                              kChunkBytes, red);
+                const float* src = args.part + (tile_id * ks + q) * (int64_t)(128 * BN) +
+                                   (int64_t)j * (32 * 128);
+                if (AGN_BOUNDS_OK(src, kChunkBytes)) {
+                  tc::bulk_load(smem + (size_t)d * kChunkBytes, src, kChunkBytes, red);
+                } else {   // bounds-checked build: account for the bytes, skip the copy
+                  AGN_BOUNDS_FAIL(src);
+                  tc::mbar_complete_tx(red, kChunkBytes);
+                }
                 ++d;
               }
             }
@@ -679,13 +687,16 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             float sum = 0.f;
             if (c < C)
               for (int gq = 0; gq < 4; ++gq) sum += sPart[((gq + 4 * hf) * 16 + jcl) * kHC + c];
-            __stcg(gp + i, sum);
+            AGN_STCG(gp + i, sum);
           }
           __syncthreads();
           // count in: the CTA's partials, ordered before by the barrier, are
           // released by one acquire-release arrival
-          if (threadIdx.x == 0)
-            tc::atomic_add_acq_rel_gpu(args.head_counter + slot * nchk + chunk, 1);
+          if (threadIdx.x == 0) {
+            int* hc = args.head_counter + slot * nchk + chunk;
+            if (AGN_BOUNDS_OK(hc, 4)) tc::atomic_add_acq_rel_gpu(hc, 1);
+            else AGN_BOUNDS_FAIL(hc);
+          }
         }
         if (row4_ok) {
 #pragma unroll
@@ -712,9 +723,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 uint2 q0, q1, q2;
                 split3_x4(v, q0, q1, q2);
                 bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o4;
-                *reinterpret_cast<uint2*>(pp) = q0;
-                *reinterpret_cast<uint2*>(pp + args.out_plane) = q1;
-                *reinterpret_cast<uint2*>(pp + 2 * args.out_plane) = q2;
+                AGN_ST(reinterpret_cast<uint2*>(pp), q0);
+                AGN_ST(reinterpret_cast<uint2*>(pp + args.out_plane), q1);
+                AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.out_plane), q2);
               }
             }
           }
@@ -740,7 +751,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (chunk >= nchk) continue;   // CTA-uniform
           int* ctr = args.head_counter + slot * nchk + chunk;
           if (threadIdx.x == 0)
-            s_hok = tc::wait_count_low(ctr, mtn, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
+            s_hok = AGN_BOUNDS_OK(ctr, 4) &&
+                    tc::wait_count_low(ctr, mtn, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
           __syncthreads();
           if (!s_hok) {
             if (threadIdx.x == 0) atomicExch(args.err, 1);
@@ -759,8 +771,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
             for (int q = 0; q < 16; ++q) {
               const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
-              p0[q] = m0 + q < mtn ? __ldcg(pq) : 0.f;
-              p1[q] = m0 + q < mtn ? __ldcg(pq + kThreads) : 0.f;
+              p0[q] = m0 + q < mtn ? AGN_LDCG(pq) : 0.f;
+              p1[q] = m0 + q < mtn ? AGN_LDCG(pq + kThreads) : 0.f;
             }
 #pragma unroll
             for (int q = 0; q < 16; ++q) {
@@ -777,7 +789,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const int cl = threadIdx.x % kHC;
             const bool cv = cl < C;
             const float inv_m = 1.0f / (float)args.N;
-            const float bc = cv ? bl[cl] : 0.f;
+            const float bc = cv ? AGN_LD(bl + cl) : 0.f;
 #pragma unroll 1
             for (int hh = 0; hh < 2; ++hh) {
               const int sl = 16 * hh + (threadIdx.x >> 4);   // sample within the chunk
@@ -792,7 +804,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               float se = ex;
 #pragma unroll
               for (int off = 8; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
-              const int y = valid ? args.yb[(int64_t)slot * args.N + j] : -1;
+              const int y = valid ? AGN_LD(args.yb + (int64_t)slot * args.N + j) : -1;
               const float zy = __shfl_sync(0xffffffffu, z, (lane & 16) + (y > 0 ? y : 0));
               float pr = ex * (1.0f / se);
               if (cl == y) pr -= 1.0f;
@@ -801,13 +813,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               if (m_tile == 0 && valid && cv) {
                 const TAct gv = static_cast<TAct>(gz);
                 const int64_t zi = ((int64_t)slot * args.N + j) * args.ldz + cl;
-                static_cast<TAct*>(args.dzl)[zi] = gv;
+                AGN_ST(static_cast<TAct*>(args.dzl) + zi, gv);
                 if (args.dzl_pieces) {
                   bf16 q0, q1, q2;
                   split3(static_cast<float>(gv), q0, q1, q2);
-                  args.dzl_pieces[zi] = q0;
-                  args.dzl_pieces[args.dzl_plane + zi] = q1;
-                  args.dzl_pieces[2 * args.dzl_plane + zi] = q2;
+                  AGN_ST(args.dzl_pieces + zi, q0);
+                  AGN_ST(args.dzl_pieces + args.dzl_plane + zi, q1);
+                  AGN_ST(args.dzl_pieces + 2 * args.dzl_plane + zi, q2);
                 }
               }
               if (cl == 0) sCE[sl] = valid ? (logf(se) + mx) - zy : 0.f;
@@ -855,9 +867,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                   uint2 q0, q1, q2;
                   split3_x4(dv, q0, q1, q2);
                   bf16* pp = args.dh_pieces + (int64_t)slot * args.out_bstride + o4;
-                  *reinterpret_cast<uint2*>(pp) = q0;
-                  *reinterpret_cast<uint2*>(pp + args.dh_plane) = q1;
-                  *reinterpret_cast<uint2*>(pp + 2 * args.dh_plane) = q2;
+                  AGN_ST(reinterpret_cast<uint2*>(pp), q0);
+                  AGN_ST(reinterpret_cast<uint2*>(pp + args.dh_plane), q1);
+                  AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.dh_plane), q2);
                 }
               }
             }
@@ -868,8 +880,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             // in order
             if (m_tile == 0) {
               const float part = ce / (float)args.N;
-              args.loss_parts[((int64_t)args.slot_commit[slot] * args.lam + args.step) * nchk +
-                              chunk] = part;
+              AGN_ST(args.loss_parts +
+                         ((int64_t)AGN_LD(args.slot_commit + slot) * args.lam + args.step) * nchk +
+                         chunk,
+                     part);
               if (!isfinite(part)) atomicExch(args.nonfinite, 1);
             }
           }
@@ -895,8 +909,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int i = 0; i < kCh; ++i) {
           if (i < nvalid) {
             const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
-            thn[i] = __ldcs(th_in + p);
-            acn[i] = __ldcs(ac_in + p);
+            thn[i] = AGN_LDCS(th_in + p);
+            acn[i] = AGN_LDCS(ac_in + p);
           }
         }
       };
@@ -928,9 +942,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
             const float gr = __uint_as_float(r[i]);
             const float t = fmaf(-eta, gr, th[i]);
-            theta[p] = t;
-            acc[p] = ac[i] + gr;
-            if (kSplit == 1) tb[p] = __float2bfloat16_rn(t);   // fp32 mode keeps no weight pieces
+            AGN_ST(theta + p, t);
+            AGN_ST(acc + p, ac[i] + gr);
+            if (kSplit == 1) AGN_ST(tb + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces
           }
         }
       }
@@ -960,18 +974,18 @@ bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
   const TD* col = dz + (int64_t)z * dz_bstride + f;
   float part = 0.f;
   if (f < d)
-    for (int j = gy; j < m; j += kBiasGroups) part += from_act(col[(int64_t)j * d]);
+    for (int j = gy; j < m; j += kBiasGroups) part += from_act(AGN_LD(col + (int64_t)j * d));
   red[gy][fx] = part;
   __syncthreads();
   if (gy != 0 || f >= d) return;
   float s = 0.f;
 #pragma unroll
   for (int q = 0; q < kBiasGroups; ++q) s += red[q][fx];
-  const int64_t p = (int64_t)slot_worker[z] * ld_param + boff + f;
-  const float t = fmaf(-eta, s, theta[p]);
-  theta[p] = t;
-  acc[p] += s;
-  if (kSplit == 1 && theta_b) theta_b[p] = __float2bfloat16_rn(t);   // fp32 mode: no pieces
+  const int64_t p = (int64_t)AGN_LD(slot_worker + z) * ld_param + boff + f;
+  const float t = fmaf(-eta, s, AGN_LD(theta + p));
+  AGN_ST(theta + p, t);
+  AGN_ST(acc + p, AGN_LD(acc + p) + s);
+  if (kSplit == 1 && theta_b) AGN_ST(theta_b + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces
 }
 
 // out[p * plane + i] = piece p of x[i] (x = piece 0 + piece 1 + piece 2 exactly).
@@ -981,10 +995,10 @@ __global__ void split_pieces_kernel(const float* __restrict__ x, bf16* __restric
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += stride) {
     bf16 q0, q1, q2;
-    split3(x[i], q0, q1, q2);
-    out[i] = q0;
-    out[plane + i] = q1;
-    out[2 * plane + i] = q2;
+    split3(AGN_LD(x + i), q0, q1, q2);
+    AGN_ST(out + i, q0);
+    AGN_ST(out + plane + i, q1);
+    AGN_ST(out + 2 * plane + i, q2);
   }
 }
 
@@ -1069,6 +1083,15 @@ Status encode(CUtensorMap* map, int rank, const void* base, const cuuint64_t* di
   for (int i = 0; i < rank - 1; ++i)
     if (strides_bytes[i] % 16)
       return Status::Err(AGN_E_UNSUPPORTED, "tensor map stride not a multiple of 16 bytes");
+#ifdef AGN_BOUNDS_CHECK
+  {   // bounds-checked build: the whole span the map addresses lies in one known buffer
+    size_t span = (size_t)dims[0] * esize;
+    for (int i = 1; i < rank; ++i) span += (size_t)(dims[i] - 1) * strides_bytes[i - 1];
+    if (!bounds_host_ok(base, span))
+      return Status::Err(AGN_E_BOUNDS, "bounds-checked build: a tensor map spans " +
+                                           std::to_string(span) + " bytes beyond a known buffer");
+  }
+#endif
   cuuint32_t estr[5] = {1, 1, 1, 1, 1};
   CUresult r = g_encode(map, dtype, rank, const_cast<void*>(base), dims, strides_bytes, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1211,5 +1234,7 @@ Status split_pieces(const float* x, bf16* out, int64_t count, int64_t plane, cud
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
+
+AGN_BOUNDS_UNIT(tc)
 
 }  // namespace agn

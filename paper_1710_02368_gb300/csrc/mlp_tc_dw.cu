@@ -299,9 +299,21 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
                           worker);
         if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
           const int64_t pb = (int64_t)worker * args.ld_param + L.boff + f0;
-          tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
-          if (kAcc)
-            tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf, &cfull[r]);
+          if (AGN_BOUNDS_OK(args.theta + pb, kBiasHalf)) {
+            tc::bulk_load(dst + kA * kChunkBytes, args.theta + pb, kBiasHalf, &cfull[r]);
+          } else {   // bounds-checked build: account for the bytes, skip the copy
+            AGN_BOUNDS_FAIL(args.theta + pb);
+            tc::mbar_complete_tx(&cfull[r], kBiasHalf);
+          }
+          if (kAcc) {
+            if (AGN_BOUNDS_OK(args.acc + pb, kBiasHalf)) {
+              tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
+                            &cfull[r]);
+            } else {
+              AGN_BOUNDS_FAIL(args.acc + pb);
+              tc::mbar_complete_tx(&cfull[r], kBiasHalf);
+            }
+          }
         }
       };
       // theta_k and a_k were last written by this kernel's previous launch or
@@ -312,7 +324,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         const TileIdx t0 = decode(B, blockIdx.x);
         const DwLayer& L0 = B.layer[t0.layer];
         npre = min(kRing, min(Cfg::kChunks, (L0.N - t0.n_tile * BN + kCF - 1) / kCF));
-        const int w0 = args.slot_worker[t0.slot];
+        const int w0 = AGN_LD(args.slot_worker + t0.slot);
         for (int c = 0; c < npre; ++c) {
           issue_chunk(t0, w0, c, (int)ch);
           ++ch;
@@ -322,7 +334,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
       for (int t = blockIdx.x; !kGrad && ok && t < T; t += gridDim.x) {
         const TileIdx ti = decode(B, t);
         const DwLayer& L = B.layer[ti.layer];
-        const int worker = args.slot_worker[ti.slot];
+        const int worker = AGN_LD(args.slot_worker + ti.slot);
         const int nch = min(Cfg::kChunks, (L.N - ti.n_tile * BN + kCF - 1) / kCF);
         for (int c = t == (int)blockIdx.x ? npre : 0; c < nch; ++c) {
           const int r = ch % kRing;
@@ -417,7 +429,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
       const TileIdx ti = decode(B, t);
       const DwLayer& L = B.layer[ti.layer];
       const int M = L.M, N = L.N;
-      const int worker = args.slot_worker[ti.slot];
+      const int worker = AGN_LD(args.slot_worker + ti.slot);
       const int b = it & 1;
       // waits are warp-uniform: a lane that gave up takes its whole warp out
       // before the next .sync.aligned TMEM load
@@ -460,12 +472,12 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
             for (int u = 0; u < 4; ++u) {
               const int i = i0 + 4 * u;
               if (fbase + i < N)
-                *reinterpret_cast<float4*>(gout + L.woff + (int64_t)(fbase + i) * M + k0 + k4) =
-                    *reinterpret_cast<const float4*>(gS + i * 32 + k4);
+                AGN_ST(reinterpret_cast<float4*>(gout + L.woff + (int64_t)(fbase + i) * M + k0 + k4),
+                       *reinterpret_cast<const float4*>(gS + i * 32 + k4));
             }
           }
           if (kb >= 0 && kb < 32 && lane < 16 && fbase + lane < N)
-            gout[L.boff + fbase + lane] = gS[lane * 32 + kb];
+            AGN_ST(gout + L.boff + fbase + lane, gS[lane * 32 + kb]);
           __syncwarp();
           continue;
         }
@@ -490,16 +502,16 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
               tn[2] = fmaf(-eta, gv.z, tv.z);
               tn[3] = fmaf(-eta, gv.w, tv.w);
               const int64_t p = L.woff + (int64_t)(fbase + i) * M + k0 + k4;
-              *reinterpret_cast<float4*>(theta + p) = make_float4(tn[0], tn[1], tn[2], tn[3]);
+              AGN_ST(reinterpret_cast<float4*>(theta + p), make_float4(tn[0], tn[1], tn[2], tn[3]));
               if (kAcc) {
                 const float4 av = *reinterpret_cast<const float4*>(
                     reinterpret_cast<const float*>(slot + kChunkBytes) + so);
-                *reinterpret_cast<float4*>(acc + p) =
-                    make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w);
+                AGN_ST(reinterpret_cast<float4*>(acc + p),
+                       make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w));
               }
               // the bf16 copy (bf16 mode); the fp32 mode's GEMMs split the
               // fp32 weights themselves
-              if (kSplit == 1) *reinterpret_cast<uint2*>(tb + p) = bf16x4(tn);
+              if (kSplit == 1) AGN_ST(reinterpret_cast<uint2*>(tb + p), bf16x4(tn));
             }
           }
         }
@@ -509,9 +521,9 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           const float gb = gS[lane * 32 + kb];
           const int64_t pb = L.boff + fbase + lane;
           const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
-          theta[pb] = tn;
-          if (kAcc) acc[pb] = sTb[kCF + 16 * hf + lane] + gb;
-          if (kSplit == 1) tb[pb] = __float2bfloat16_rn(tn);
+          AGN_ST(theta + pb, tn);
+          if (kAcc) AGN_ST(acc + pb, sTb[kCF + 16 * hf + lane] + gb);
+          if (kSplit == 1) AGN_ST(tb + pb, __float2bfloat16_rn(tn));
         }
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&cempty[r]);
@@ -607,5 +619,7 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
   }
   return Status::Ok();
 }
+
+AGN_BOUNDS_UNIT(dw)
 
 }  // namespace agn

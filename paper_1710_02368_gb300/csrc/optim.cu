@@ -25,24 +25,25 @@ __device__ __forceinline__ void write_copy4(bf16* tb, int64_t plane, int64_t p, 
     for (int k = 0; k < 3; ++k) {
       const __nv_bfloat162 lo = __halves2bfloat162(q[k][0], q[k][1]);
       const __nv_bfloat162 hi = __halves2bfloat162(q[k][2], q[k][3]);
-      *reinterpret_cast<uint2*>(tb + k * plane + p) =
-          make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+      AGN_ST(reinterpret_cast<uint2*>(tb + k * plane + p),
+             make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                        *reinterpret_cast<const uint32_t*>(&hi)));
     }
   } else {
     const __nv_bfloat162 lo = __floats2bfloat162_rn(t[0], t[1]);
     const __nv_bfloat162 hi = __floats2bfloat162_rn(t[2], t[3]);
-    *reinterpret_cast<uint2*>(tb + p) =
-        make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+    AGN_ST(reinterpret_cast<uint2*>(tb + p),
+           make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi)));
   }
 }
 
 __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
   pdl_begin();
   const int z = blockIdx.y;
-  const int w = a.slot_worker[z];
+  const int w = AGN_LD(a.slot_worker + z);
   __shared__ float s_c1, s_c2;
   if (threadIdx.x == 0) {
-    const double t = (double)(a.slot_t0[z] + a.step + 1);
+    const double t = (double)(AGN_LD(a.slot_t0 + z) + a.step + 1);
     s_c1 = (float)(1.0 / (1.0 - pow((double)a.beta1, t)));
     s_c2 = (float)(1.0 / (1.0 - pow((double)a.beta2, t)));
   }
@@ -54,10 +55,10 @@ __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
     const int64_t p = base + 4 * i;
-    const float4 g4 = *reinterpret_cast<const float4*>(a.grad + p);
-    const float4 t4 = *reinterpret_cast<const float4*>(a.theta + p);
-    float4 m4 = *reinterpret_cast<const float4*>(a.m + p);
-    float4 v4 = *reinterpret_cast<const float4*>(a.v + p);
+    const float4 g4 = AGN_LD(reinterpret_cast<const float4*>(a.grad + p));
+    const float4 t4 = AGN_LD(reinterpret_cast<const float4*>(a.theta + p));
+    float4 m4 = AGN_LD(reinterpret_cast<const float4*>(a.m + p));
+    float4 v4 = AGN_LD(reinterpret_cast<const float4*>(a.v + p));
     const float gr[4] = {g4.x, g4.y, g4.z, g4.w};
     float mm[4] = {m4.x, m4.y, m4.z, m4.w}, vv[4] = {v4.x, v4.y, v4.z, v4.w};
     float th[4] = {t4.x, t4.y, t4.z, t4.w}, u[4];
@@ -68,13 +69,13 @@ __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
       u[e] = -a.eta * (mm[e] * c1) / (sqrtf(vv[e] * c2) + a.eps);
       th[e] = th[e] + u[e];
     }
-    *reinterpret_cast<float4*>(a.m + p) = make_float4(mm[0], mm[1], mm[2], mm[3]);
-    *reinterpret_cast<float4*>(a.v + p) = make_float4(vv[0], vv[1], vv[2], vv[3]);
-    *reinterpret_cast<float4*>(a.theta + p) = make_float4(th[0], th[1], th[2], th[3]);
+    AGN_ST(reinterpret_cast<float4*>(a.m + p), make_float4(mm[0], mm[1], mm[2], mm[3]));
+    AGN_ST(reinterpret_cast<float4*>(a.v + p), make_float4(vv[0], vv[1], vv[2], vv[3]));
+    AGN_ST(reinterpret_cast<float4*>(a.theta + p), make_float4(th[0], th[1], th[2], th[3]));
     if (a.acc) {
-      const float4 c4 = *reinterpret_cast<const float4*>(a.acc + p);
-      *reinterpret_cast<float4*>(a.acc + p) =
-          make_float4(c4.x + u[0], c4.y + u[1], c4.z + u[2], c4.w + u[3]);
+      const float4 c4 = AGN_LD(reinterpret_cast<const float4*>(a.acc + p));
+      AGN_ST(reinterpret_cast<float4*>(a.acc + p),
+             make_float4(c4.x + u[0], c4.y + u[1], c4.z + u[2], c4.w + u[3]));
     }
     if (a.theta_b) write_copy4(a.theta_b, a.piece_plane, p, th);
   }
@@ -96,5 +97,7 @@ Status adam_step(const AdamArgs& a, int slots, int num_sms, cudaStream_t st) {
   AGN_TRY_CUDA(cudaGetLastError());
   return Status::Ok();
 }
+
+AGN_BOUNDS_UNIT(optim)
 
 }  // namespace agn

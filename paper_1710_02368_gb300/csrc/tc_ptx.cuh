@@ -98,6 +98,12 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_
 
 // 1D bulk copy global -> shared (both 16-byte aligned, bytes a multiple of 16),
 // completing `bytes` transactions on `bar`.
+// Account for bytes on the barrier without a copy (the bounds-checked build
+// skips a bulk copy from outside every known buffer).
+__device__ __forceinline__ void mbar_complete_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
                                           uint64_t* bar) {
   asm volatile(
