@@ -451,7 +451,9 @@ Status build_tc_maps(agn_handle* h) {
       // piece maps, kTcSplitBK-deep k steps for the forward and dX
       constexpr uint32_t bk = agn::kTcSplitBK;
       const float* W = h->rep + h->woff[l - 1];
-      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, bk, 128));
+      // (with column tiles up to 128 the forward's converters read the tile
+      // row by row into tensor memory: 128-byte swizzle, conflict-free)
+      AGN_TRY(agn::make_tmap_f32_3d(&mp.w_k, W, fi, fo, n, fi, h->P_pad, bk, 128, bn <= 128));
       AGN_TRY(agn::make_tmap_f32_3d(&mp.w_mn, W, fi, fo, n, fi, h->P_pad, 128, bk));
       const bf16* Hp = h->Hs[l - 1];
       const uint64_t hp = (uint64_t)n * m * fi;

@@ -44,6 +44,14 @@ constexpr int kConvWarps = 6;
 // whose stages hold three pieces of each operand: half the bytes per stage,
 // so twice the stages in flight to hide the load and conversion latency.
 constexpr int stage_k(int split, int epi) { return split == 3 && epi != kEpiDW ? kTcSplitBK : 64; }
+// fp32 mode, forward and dX, column tiles up to 128: the converters write the
+// weight pieces (the MMA's A operand) into tensor memory instead of shared
+// memory.  The stages' shared-memory traffic (TMA writes, the converters'
+// reads and writes, the MMAs' operand reads) had bound the mainloop; the MMAs
+// then read only B from shared memory.
+constexpr bool a_in_tmem(int split, int epi, int bn) {
+  return split == 3 && epi != kEpiDW && bn <= 128;
+}
 // Fused output layer (kEpiFwdHead): at most kHC classes; shared scratch of
 // W_L's 128 x kHC slice, the warps' partial logits [8][16][kHC] and the
 // chunk's logits / dZ_L [32][kHC].
@@ -52,27 +60,34 @@ constexpr int kHeadScratch = (kHC * 128 + 8 * 16 * kHC + 32 * kHC) * 4 + 8 * 256
 
 // A stage holds kSplit A pieces then kSplit B pieces (kSplit = 3 in the fp32
 // mode, where every fp32 operand is the exact sum of three bf16 pieces), of
-// kBK k each (rows of 2 kBK bytes).
-template <int BN, int kSplit, int kBKs = 64>
+// kBK k each (rows of 2 kBK bytes).  With A in tensor memory (kATmem) the
+// stage holds the fp32 weight tile the converters read, then the B pieces,
+// and A's pieces take kACols TMEM columns per stage after the accumulators.
+template <int BN, int kSplit, int kBKs = 64, bool kATmemT = false>
 struct TileCfg {
   static constexpr int kBK = kBKs;
+  static constexpr bool kATmem = kATmemT;
   static constexpr int kRowBytes = 2 * kBK;
   static constexpr int kABytes = 128 * kRowBytes;
   static constexpr int kBBytes = BN * kRowBytes;
-  static constexpr int kStageBytes = kSplit * (kABytes + kBBytes);
   static constexpr uint32_t kA32Bytes = 128 * kBK * 4;   // an fp32 weight tile
+  static constexpr int kAArea = kATmem ? (int)kA32Bytes : kSplit * kABytes;
+  static constexpr int kStageBytes = kAArea + kSplit * kBBytes;
   // split mode keeps two accumulators: columns [0, BN) take the leading
   // piece products a0 b0, columns [BN, 2 BN) the five smaller pairs, so the
   // rounding of the tensor core's running sums is relative to each part
-  static constexpr uint32_t kTmemCols = (kSplit == 1 ? 1 : 2) * BN;   // power of two >= 32
+  static constexpr uint32_t kAccCols = (kSplit == 1 ? 1 : 2) * BN;
+  static constexpr uint32_t kACols = kSplit * kBK / 2;   // A pieces of one stage in TMEM
+  static constexpr uint32_t kTmemCols = kATmem ? 512 : kAccCols;   // power of two >= 32
 };
 
 // The forward / dX epilogue's transpose tiles sit after the barriers when the
 // CTA's shared memory has room for them (then the whole stage ring can hold
 // split-K partial sums), else at the end of the ring.
-template <int BN, int kSplit, int kStages, int kBKs>
+template <int BN, int kSplit, int kStages, int kBKs, bool kATmem>
 struct EpiT {
-  static constexpr size_t kRing = (size_t)kStages * TileCfg<BN, kSplit, kBKs>::kStageBytes;
+  static constexpr size_t kRing =
+      (size_t)kStages * TileCfg<BN, kSplit, kBKs, kATmem>::kStageBytes;
   static constexpr bool kSeparate = kRing + 1280 + kEpiTBytes <= 232448;
   static constexpr size_t kOff = kSeparate ? kRing + 256 : kRing - kEpiTBytes;
   static constexpr size_t kRingFree = kSeparate ? kRing : kRing - kEpiTBytes;
@@ -145,8 +160,10 @@ __global__ void __launch_bounds__(kThreads, kEpi == kEpiDW ? 2 : 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const TcArgs args) {
   constexpr int kBK = stage_k(kSplit, kEpi);
-  using Cfg = TileCfg<BN, kSplit, kBK>;
-  using Epi = EpiT<BN, kSplit, kStages, kBK>;
+  constexpr bool kATmem = a_in_tmem(kSplit, kEpi, BN);
+  using Cfg = TileCfg<BN, kSplit, kBK, kATmem>;
+  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem>;
+  static_assert(!kATmem || Cfg::kAccCols + kStages * Cfg::kACols <= Cfg::kTmemCols, "TMEM");
   constexpr int kABytes = Cfg::kABytes;
   constexpr uint32_t kA32Bytes = Cfg::kA32Bytes;
   constexpr int kBox = kBK * 128;   // one 64-wide MN box of kBK rows (MN-major operands)
@@ -218,10 +235,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // for it (pdl_begin), except the producer's loads of the weights for the
   // first stages (forward and dX: A = W, last written two or more kernels
   // back, and the preceding kernel only starts once its own predecessor is
-  // complete).
+  // complete) and the converter warps, which touch only shared and tensor
+  // memory until the epilogue (they wait before it): the prefetched weight
+  // stages are converted while the preceding kernel still runs.
   constexpr bool kPrefetchA = kEpi != kEpiDW;
   const bool producer = warp == 0 && lane == 0;
-  if (!producer) pdl_begin();
+  const bool converter = kWConv && warp >= 2;
+  if (!producer && !converter) pdl_begin();
   if (warp == 0) {
     if (lane == 0) {
       // one box of 3D maps (kSplit = 1) or of 4D maps with the piece index
@@ -277,7 +297,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
         if (*abort_flag) break;
         uint8_t* sa0 = smem + s * Cfg::kStageBytes;
-        uint8_t* sb0 = sa0 + kSplit * kABytes;
+        uint8_t* sb0 = sa0 + Cfg::kAArea;
         if (kt >= npre) {
           tc::mbar_arrive_expect_tx(&full[s], kABytesAll + kBBytesAll);
           if (kWConv) load_a32(kt, s);
@@ -310,6 +330,73 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             tc::mbar_wait_bounded(&afull[j % kStages], (j / kStages) & 1, kWaitNs);
       }
     }
+  } else if (kWConv && kATmem && warp >= 2) {
+    if constexpr (kATmem) {
+      // Converters, A in tensor memory: warp w writes TMEM lanes 32 (w % 4) ..
+      // + 31, the rows (features; dX: inputs) of that quadrant.  Quadrants 2
+      // and 3 have two converter warps (2, 6 and 3, 7), each taking half of the
+      // k step; quadrants 0 and 1 have one (4, 5), taking all of it.  A thread
+      // loads its row's fp32 values (the forward's K-major tile lands with a
+      // 128-byte swizzle, so the warp's 16-byte loads do not conflict; dX's
+      // MN-major tile is read down a column), splits them into three pieces and
+      // stores each piece's bf16 pairs (the lower k in the lower half) into its
+      // lane's columns: piece p of the stage at columns p kBK / 2 .. + kBK / 2.
+      constexpr int kHalfK = kBK / 2;
+      const int qd = warp & 3;
+      const int kb = qd >= 2 ? (warp >= 6 ? kHalfK : 0) : 0;   // first k of this warp
+      const int ke = qd >= 2 ? kb + kHalfK : kBK;
+      const int row = 32 * qd + lane;
+      const uint32_t lane_addr = (uint32_t)(32 * qd) << 16;
+      for (int kt = 0; kt < KT; ++kt) {
+        const int s = kt % kStages;
+        if (!__all_sync(0xffffffffu, wait_or_abort(&afull[s], (kt / kStages) & 1, abort_flag))) {
+          if (lane == 0) *abort_flag = 1;
+          break;
+        }
+        const float* a32 = reinterpret_cast<const float*>(smem + s * Cfg::kStageBytes);
+        const uint32_t acol = tmem + lane_addr + Cfg::kAccCols + (uint32_t)s * Cfg::kACols;
+  #pragma unroll 1
+        for (int h0 = kb; h0 < ke; h0 += kHalfK) {
+          float x[kHalfK];
+          if (!kAMN) {
+  #pragma unroll
+            for (int c = 0; c < kHalfK / 4; ++c) {
+              const int cc = (h0 / 4 + c) ^ (row & 7);
+              const float4 v = *reinterpret_cast<const float4*>(a32 + row * kBK + 4 * cc);
+              x[4 * c] = v.x;
+              x[4 * c + 1] = v.y;
+              x[4 * c + 2] = v.z;
+              x[4 * c + 3] = v.w;
+            }
+          } else {
+  #pragma unroll
+            for (int k = 0; k < kHalfK; ++k) x[k] = a32[(h0 + k) * 128 + row];
+          }
+          uint32_t p0[kHalfK / 2], p1[kHalfK / 2], p2[kHalfK / 2];
+  #pragma unroll
+          for (int j = 0; j < kHalfK / 2; ++j) {
+            bf16 a0, a1, a2, b0, b1, b2;
+            split3(x[2 * j], a0, a1, a2);
+            split3(x[2 * j + 1], b0, b1, b2);
+            const __nv_bfloat162 v0 = __halves2bfloat162(a0, b0);
+            const __nv_bfloat162 v1 = __halves2bfloat162(a1, b1);
+            const __nv_bfloat162 v2 = __halves2bfloat162(a2, b2);
+            p0[j] = *reinterpret_cast<const uint32_t*>(&v0);
+            p1[j] = *reinterpret_cast<const uint32_t*>(&v1);
+            p2[j] = *reinterpret_cast<const uint32_t*>(&v2);
+          }
+          const uint32_t col = acol + (uint32_t)(h0 / 2);
+          tc::tmem_st_32x32b_x8(col, p0);
+          tc::tmem_st_32x32b_x8(col + kBK / 2, p1);
+          tc::tmem_st_32x32b_x8(col + kBK, p2);
+        }
+        tc::tmem_st_wait();
+        tc::tc_fence_before();   // the stores, before the MMA thread's wait on conv[s]
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&conv[s]);
+      }
+    }
+    pdl_begin();   // before the epilogue's global accesses
   } else if (kWConv && warp >= 2) {
     // Converters: the fp32 weight tile of each k step into its three bf16
     // pieces (x0 = bf16(x), x1 = bf16(x - x0), x2 = bf16(x - x0 - x1)), in
@@ -372,9 +459,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&conv[s]);
     }
+    pdl_begin();   // before the epilogue's global accesses
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, BN, kAMN, kBMN);
+      // A in TMEM is read row by row (K-major) whatever the weights' layout
+      constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, BN, kATmem ? false : kAMN, kBMN);
       for (int kt = 0; kt < KT; ++kt) {
         const int s = kt % kStages;
         if (!wait_or_abort(&full[s], (kt / kStages) & 1, abort_flag) ||
@@ -384,7 +473,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
         tc::tc_fence_after();
         const uint32_t sa0 = tc::smem_u32(smem + s * Cfg::kStageBytes);
-        const uint32_t sb0 = sa0 + kSplit * kABytes;
+        const uint32_t sb0 = sa0 + Cfg::kAArea;
+        const uint32_t ta0 = tmem + Cfg::kAccCols + (uint32_t)s * Cfg::kACols;   // A in TMEM
         constexpr int kPairs = kSplit == 1 ? 1 : 6;
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk) {
@@ -404,7 +494,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const uint32_t dcol = (kSplit == 3 && q > 0) ? (uint32_t)BN : 0u;
             const bool acc_on = kSplit == 1 ? (kt | kk | q) != 0
                                             : (q == 0 ? (kt | kk) != 0 : ((kt | kk) != 0 || q > 1));
-            tc::mma_bf16(tmem + dcol, ad, bd, kIdesc, acc_on ? 1u : 0u);
+            if (kATmem)
+              tc::mma_bf16_ts(tmem + dcol, ta0 + (uint32_t)(kPairA[q] * (kBK / 2) + kk * 8), bd,
+                              kIdesc, acc_on ? 1u : 0u);
+            else
+              tc::mma_bf16(tmem + dcol, ad, bd, kIdesc, acc_on ? 1u : 0u);
           }
         }
         tc::mma_commit(&empty[s]);
@@ -1002,14 +1096,14 @@ __global__ void split_pieces_kernel(const float* __restrict__ x, bf16* __restric
   }
 }
 
-template <int BN, int kSplit, int kStages, int kBK>
+template <int BN, int kSplit, int kStages, int kBK, bool kATmem>
 size_t smem_bytes() {
   // Shared memory requested per CTA also caps the CTAs per SM so that their
   // TMEM columns never exceed the 512 an SM has.
-  const size_t ring = (size_t)kStages * TileCfg<BN, kSplit, kBK>::kStageBytes + 1024 + 256 +
-                      (EpiT<BN, kSplit, kStages, kBK>::kSeparate ? kEpiTBytes : 0);
-  const size_t floor_for_tmem =
-      (size_t)(233472 / (512 / TileCfg<BN, kSplit, kBK>::kTmemCols + 1)) + 1024;
+  using Cfg = TileCfg<BN, kSplit, kBK, kATmem>;
+  const size_t ring = (size_t)kStages * Cfg::kStageBytes + 1024 + 256 +
+                      (EpiT<BN, kSplit, kStages, kBK, kATmem>::kSeparate ? kEpiTBytes : 0);
+  const size_t floor_for_tmem = (size_t)(233472 / (512 / Cfg::kTmemCols + 1)) + 1024;
   return std::max(ring, floor_for_tmem);
 }
 
@@ -1017,10 +1111,11 @@ template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
 Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, int slots,
                  cudaStream_t st, bool* launched = nullptr) {
   constexpr int kBK = stage_k(kSplit, kEpi);
-  using Epi = EpiT<BN, kSplit, kStages, kBK>;
-  static_assert(kStages * TileCfg<BN, kSplit, kBK>::kStageBytes + 1280 <= 232448, "smem");
+  constexpr bool kATmem = a_in_tmem(kSplit, kEpi, BN);
+  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem>;
+  static_assert(kStages * TileCfg<BN, kSplit, kBK, kATmem>::kStageBytes + 1280 <= 232448, "smem");
   auto kern = tc_gemm_kernel<BN, kAMN, kBMN, kEpi, kStages, kSplit>;
-  const size_t smem = smem_bytes<BN, kSplit, kStages, kBK>();
+  const size_t smem = smem_bytes<BN, kSplit, kStages, kBK, kATmem>();
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -1141,12 +1236,12 @@ Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uin
 
 Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                         uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
-                        uint32_t box_inner, uint32_t box_rows) {
+                        uint32_t box_inner, uint32_t box_rows, bool swizzle128) {
   cuuint64_t dims[3] = {inner, rows, batch};
   cuuint64_t strides[2] = {row_stride_elems * 4, batch_stride_elems * 4};
   cuuint32_t box[3] = {box_inner, box_rows, 1};
   return encode(map, 3, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4,
-                CU_TENSOR_MAP_SWIZZLE_NONE);
+                swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,

@@ -90,10 +90,11 @@ Status tc_init();
 Status make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                          uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
                          uint32_t box_inner, uint32_t box_rows);
-// 3D fp32 tensor map (inner, rows, batch), no swizzle, zero fill.
+// 3D fp32 tensor map (inner, rows, batch), zero fill; no swizzle, or the
+// 128-byte swizzle (box rows of 32 floats) when swizzle128.
 Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                         uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
-                        uint32_t box_inner, uint32_t box_rows);
+                        uint32_t box_inner, uint32_t box_rows, bool swizzle128 = false);
 // 4D bf16 tensor map (inner, rows, batch, piece) over three piece planes.
 Status make_tmap_bf16_4d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                          uint64_t batch, uint64_t row_stride_elems, uint64_t batch_stride_elems,
