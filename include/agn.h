@@ -105,7 +105,9 @@ typedef struct agn_options {
      instead of the persistent one, for comparison.  Bit 4 runs the forward
      and dX GEMMs without split K (one CTA per output tile).  Bit 5 runs the
      output layer (forward, softmax-CE, dX) as a kernel of its own instead of
-     in the epilogue of the last hidden layer's forward GEMM. */
+     in the epilogue of the last hidden layer's forward GEMM.  Bit 6 gathers
+     each local step's minibatch into a buffer of its own (one launch per
+     step) instead of reading it from the padded shards in place. */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);

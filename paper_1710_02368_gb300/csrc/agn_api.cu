@@ -258,6 +258,14 @@ struct agn_handle {
   // alternates between two buffers by local step (gparity)
   bool early_gather = false;
   int gparity = 0;
+  // padded shards: layer 1's tensor-core operand and the labels read in
+  // place, worker w's shard stored as S + m rows (row r = dataset row
+  // w S + r mod S), so a local step's minibatch is m consecutive rows and
+  // no gather runs; yb is then the padded labels [n][S + m]
+  bool direct_x = false;
+  void* Xpad = nullptr;           // bf16 mode: [n][S + m][d0]
+  bf16* Hs0_pad = nullptr;        // fp32 mode: pieces [3][n][S + m][d0]
+  long long* zero_t0 = nullptr;   // [n] zeros (the fill's step counters)
   void* Xb_alt = nullptr;         // bf16 mode: [n][m][d0]
   bf16* Hs0_alt = nullptr;        // fp32 mode: pieces [3][n][m][d0]
   // test hook of the bounded waits (agn_debug_waits)
@@ -405,9 +413,12 @@ void collect_profile(agn_handle* h) {
 // Layer l (1-based) runs on the tensor cores: bf16 mode, a hidden layer.
 bool tc_layer(const agn_handle* h, int l) { return h->use_tc && l < h->L; }
 
-agn::TcArgs tc_args(agn_handle* h, const int* sw) {
+agn::TcArgs tc_args(agn_handle* h, const int* sw, const long long* st0, int step) {
   agn::TcArgs t{};
   t.slot_worker = sw;
+  t.slot_t0 = st0;
+  t.step = step;
+  t.x_shard = h->direct_x ? h->S : 0;
   t.ksplit = 1;
   t.part = h->tc_part;
   t.counter = nullptr;            // set per forward / dX launch (next_counters)
@@ -476,6 +487,22 @@ Status build_tc_maps(agn_handle* h) {
     const void* dZ = h->dZ[l];
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_k, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, bn));
     AGN_TRY(agn::make_tmap_bf16_3d(&mp.dz_mn, dZ, fo, m, n, fo, (uint64_t)m * fo, 64, 64));
+  }
+  if (h->direct_x) {   // layer 1's operand maps over the padded shards
+    const uint64_t fi = h->dims[0], rows = (uint64_t)(h->S + m);
+    auto& mp = h->tmaps[0];
+    if (h->split) {
+      const uint64_t hp = (uint64_t)n * rows * fi;
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_k, h->Hs0_pad, fi, rows, n, fi, rows * fi, hp,
+                                     agn::kTcSplitBK, bn));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn, h->Hs0_pad, fi, rows, n, fi, rows * fi, hp, 64,
+                                     64));
+      AGN_TRY(agn::make_tmap_bf16_4d(&mp.h_mn32, h->Hs0_pad, fi, rows, n, fi, rows * fi, hp, 64,
+                                     32));
+    } else {
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_k, h->Xpad, fi, rows, n, fi, rows * fi, 64, bn));
+      AGN_TRY(agn::make_tmap_bf16_3d(&mp.h_mn, h->Xpad, fi, rows, n, fi, rows * fi, 64, 64));
+    }
   }
   if (h->early_gather) {   // layer 1's operand maps over the alternate buffer
     const uint64_t fi = h->dims[0];
@@ -571,7 +598,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     const bool alt = h->early_gather && h->gparity;
     const agn_handle::LayerMaps& l1 = alt ? h->l1_alt : h->tmaps.empty() ? h->l1_alt : h->tmaps[0];
     auto maps_of = [&](int l) -> const agn_handle::LayerMaps& { return l == 1 ? l1 : h->tmaps[l - 1]; };
-    {
+    if (!h->direct_x) {
       // fp32 mode with the early gather: the fp32 rows are not read by the
       // tensor-core kernels, only their pieces
       T* xb = h->early_gather ? (h->split ? nullptr : static_cast<T*>(alt ? h->Xb_alt : h->Xb))
@@ -604,6 +631,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         a.woff = h->woff[L - 1]; a.boff = h->boff[L - 1];
         a.K = fi; a.C = C; a.m = m;
         a.slot_worker = sw; a.yb = h->yb;
+        a.slot_t0 = st0; a.x_shard = h->direct_x ? h->S : 0;
         a.dZL = h->dZ[L]; a.ldz = h->ldz_out;
         a.dZL_pieces = (h->fuse_out_dw && h->split) ? h->dZp[L] : nullptr;
         a.dZL_plane = (int64_t)n * m * h->ldz_out;
@@ -650,7 +678,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
                            : 0.0),
                  launches);
         if (fuse) {
-          agn::TcArgs t = tc_args(h, sw);
+          agn::TcArgs t = tc_args(h, sw, st0, i);
           t.M = fo; t.N = m; t.K = fi;
           t.a_by_worker = 1;
           t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
@@ -673,6 +701,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.loss_parts = h->loss_parts; t.slot_commit = sc; t.lam = h->lam; t.step = i;
           t.nonfinite = h->flag;
           const auto& mp = maps_of(l);
+          t.x_b_direct = l == 1;
           t.ksplit = pick_ksplit(h, fo, fi, s);
           next_counters(h, &t);
           bool launched = false;
@@ -683,13 +712,14 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           head_done = true;
           dz_ready = t.dh_pieces != nullptr;
         } else if (tc_layer(h, l) && (h->tc_mask & 1)) {
-          agn::TcArgs t = tc_args(h, sw);
+          agn::TcArgs t = tc_args(h, sw, st0, i);
           t.M = fo; t.N = m; t.K = fi;
           t.a_by_worker = 1;
           t.out = h->H[l]; t.ldo = fo; t.out_bstride = (int64_t)m * fo;
           t.relu = 1; t.boff = h->boff[l - 1];
           t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
           const auto& mp = maps_of(l);
+          t.x_b_direct = l == 1;
           t.ksplit = pick_ksplit(h, fo, fi, s);
           next_counters(h, &t);
           AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split, agn::tc_bn(m)));
@@ -727,7 +757,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
                launches);
       if (tc_layer(h, l) && (h->tc_mask & 2)) {
         AGN_TRY(ensure_pieces(l));
-        agn::TcArgs t = tc_args(h, sw);
+        agn::TcArgs t = tc_args(h, sw, st0, i);
         t.M = fi; t.N = m; t.K = fo;
         t.a_by_worker = 1;
         t.out = h->dZ[l - 1]; t.ldo = fi; t.out_bstride = (int64_t)m * fi;
@@ -765,7 +795,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         AGN_TRY(ensure_pieces(l));
         if (h->tc_mask & 8) {   // the earlier one-tile-per-CTA kernel, layer by layer
           Launch k(h, AGN_K_BACKWARD_DW, flops, bytes, launches);
-          agn::TcArgs t = tc_args(h, sw);
+          agn::TcArgs t = tc_args(h, sw, st0, i);
           t.M = fi; t.N = fo; t.K = m;
           t.woff = h->woff[l - 1]; t.eta = eta;
           const auto& mp = h->tmaps[l - 1];
@@ -776,7 +806,8 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
         } else {
           const auto& mp = maps_of(l);
           tc_dw.push_back({h->split ? &mp.h_mn32 : &mp.h_mn, h->split ? &mp.dz_mn32 : &mp.dz_mn,
-                           &mp.theta, &mp.acc, fi, fo, h->woff[l - 1], h->boff[l - 1]});
+                           &mp.theta, &mp.acc, fi, fo, h->woff[l - 1], h->boff[l - 1],
+                           l == 1 ? 1 : 0});
           tc_flops += flops;
           tc_bytes += bytes;
         }
@@ -818,7 +849,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
     }
     if (!tc_dw.empty()) {
       Launch k(h, AGN_K_BACKWARD_DW, tc_flops, tc_bytes, launches);
-      agn::TcArgs t = tc_args(h, sw);
+      agn::TcArgs t = tc_args(h, sw, st0, i);
       t.K = m; t.eta = eta;
       AGN_TRY(agn::tc_backward_dw(tc_dw.data(), (int)tc_dw.size(), t, s, h->stream, h->split,
                                   h->num_sms));
@@ -1118,7 +1149,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 63) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 63]");
+  if (o.tc_mask < 0 || o.tc_mask > 127) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 127]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)
@@ -1277,11 +1308,22 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   // layer 1's operand is a tensor-core kernel (forward and dW)
   h->early_gather = h->use_tc && (h->tc_mask & 1) && (h->tc_mask & 4) && !(h->tc_mask & 8) &&
                     h->L >= 2 && d0 % 4 == 0;
+  // no gather at all when, besides, every reader of the labels is one of the
+  // output-layer kernels (the padded shards replace the alternate buffers)
+  h->direct_x = h->early_gather && h->use_head && !(h->tc_mask & 64);
+  if (h->direct_x) {
+    h->early_gather = false;
+    const size_t rows = (size_t)(n * (h->S + m));
+    if (h->split) AGN_TRY(dalloc_t(h, &h->Hs0_pad, 3 * rows * (size_t)d0));
+    else AGN_TRY(dalloc(h, &h->Xpad, rows * (size_t)d0 * es));
+    AGN_TRY(dalloc_t(h, &h->zero_t0, (size_t)n));
+    AGN_TRY_CUDA(cudaMemset(h->zero_t0, 0, (size_t)n * sizeof(long long)));
+  }
   if (h->early_gather) {
     if (h->split) AGN_TRY(dalloc_t(h, &h->Hs0_alt, (size_t)(3 * n * m * d0)));
     else AGN_TRY(dalloc(h, &h->Xb_alt, (size_t)(n * m * d0) * es));
   }
-  AGN_TRY(dalloc_t(h, &h->yb, (size_t)(n * m)));
+  AGN_TRY(dalloc_t(h, &h->yb, (size_t)(n * (h->direct_x ? h->S + m : m))));
   h->H.assign(h->L, nullptr);
   for (int l = 1; l < h->L; ++l) AGN_TRY(dalloc(h, &h->H[l], (size_t)(n * m * dims[l]) * es));
   AGN_TRY(dalloc_t(h, &h->Z, (size_t)(n * m * dims[h->L])));
@@ -1360,6 +1402,21 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   AGN_TRY_CUDA(cudaMemcpyAsync(h->pull_list, all.data(), n * sizeof(int), cudaMemcpyHostToDevice,
                                h->stream));
   AGN_TRY(agn::bounds_upload(h->stream));   // bounds-checked build: the handle's buffers
+  if (h->direct_x) {
+    // the padded shards: worker w's rows r = 0 .. S + m - 1 are the gather of
+    // one "step" of S + m rows from step counter 0 (row (0 + r) mod S)
+    const int rows = (int)(h->S + m);
+    const int64_t plane = n * (int64_t)rows * d0;
+    if (h->split)
+      AGN_TRY(agn::gather_batch<float>(static_cast<const float*>(h->X), h->y, nullptr, h->yb,
+                                       d0, rows, h->S, h->pull_list, h->zero_t0, 0, (int)n,
+                                       h->stream, h->Hs0_pad, plane, 0));
+    else   // (the tensor cores' fp32 mode is the split one: this is bf16)
+      AGN_TRY(agn::gather_batch<bf16>(static_cast<const bf16*>(h->X), h->y,
+                                      static_cast<bf16*>(h->Xpad), h->yb, d0, rows, h->S,
+                                      h->pull_list, h->zero_t0, 0, (int)n, h->stream, nullptr, 0,
+                                      0));
+  }
   AGN_TRY(agn::pull_replicas(h->theta_c, h->rep, h->rep_b, h->P_pad, h->P_pad, h->pull_list,
                              (int)n, h->stream, h->piece_plane,
                              h->elide ? h->acc : nullptr));   // every worker pulls version 0

@@ -98,6 +98,17 @@ inline Status bounds_collect(cudaStream_t) { return Status::Ok(); }
 constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
 
+// Padded shards (the tensor-core path's layer-1 operand and labels): worker
+// w's shard of S dataset rows is stored as S + m rows, row r holding dataset
+// row w S + (r mod S), so that the minibatch of local step `step` of slot z,
+// rows (t m + j) mod S for j < m (t = slot_t0[z] + step, Algorithm 1's
+// FetchNextMiniBatch), is the m consecutive rows starting at this row.
+__device__ __forceinline__ int64_t batch_row0(const long long* slot_t0, int slot, int step,
+                                              int m, int64_t S) {
+  const unsigned long long t = (unsigned long long)(AGN_LD(slot_t0 + slot) + step);
+  return (int64_t)((t * (unsigned long long)m) % (unsigned long long)S);
+}
+
 // x = q0 + q1 + q2 exactly, each a bf16 (round to nearest even): q0 keeps the
 // leading 8 significant bits of x, q1 the next 8, q2 the last 8.  The two
 // residuals are exact float subtractions (Sterbenz); x must not be so small

@@ -88,6 +88,10 @@ struct HeadArgs {
   const int* slot_commit;
   int lam, step;
   int* flag;
+  // padded labels (batch_row0): x_shard = S > 0 reads yb [n][S + m] at the
+  // slot's minibatch rows instead of yb [slots][m]
+  const long long* slot_t0;
+  int64_t x_shard;
 };
 template <typename T>
 Status head_forward_backward(const HeadArgs& a, int slots, cudaStream_t st);

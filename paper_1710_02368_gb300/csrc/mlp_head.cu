@@ -129,7 +129,10 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
       for (int r = 0; r < kHeadSplit; ++r) v += red[sj][r][c < C ? c : 0];
       zc[c] = c < C ? v + AGN_LD(bias + c) : -INFINITY;
     }
-    const int y = AGN_LD(a.yb + (int64_t)z * m + j);
+    const int y = a.x_shard > 0
+                      ? AGN_LD(a.yb + (int64_t)w * (a.x_shard + m) +
+                               batch_row0(a.slot_t0, z, a.step, m, a.x_shard) + j)
+                      : AGN_LD(a.yb + (int64_t)z * m + j);
     float mx = zc[0];
 #pragma unroll
     for (int c = 1; c < kMaxC; ++c) mx = fmaxf(mx, zc[c]);

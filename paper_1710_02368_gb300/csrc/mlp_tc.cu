@@ -203,7 +203,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int kt0 = sk * kt_per;
   const int KT = min(KT_all, kt0 + kt_per) - kt0;
   const int a_z = args.a_by_worker ? worker : slot;
-  const int b_z = args.b_by_worker ? worker : slot;
+  // layer 1's B straight from the padded shards: the worker's shard at the
+  // slot's minibatch row (tile rows past m belong to the next rows of the
+  // shard; their accumulator columns are never stored)
+  const bool b_direct = !kBMN && args.x_b_direct && args.x_shard > 0;
+  const int b_z = b_direct ? worker : args.b_by_worker ? worker : slot;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -279,10 +283,33 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       constexpr uint32_t kABytesAll = kWConv ? 0u : kSplit * kABytes;   // A bytes on full[s]
       constexpr uint32_t kBBytesAll = kSplit * Cfg::kBBytes;
       const int npre = kPrefetchA ? min(KT, kStages) : 0;
+      // (slot_t0 is written by the host before the launch)
+      const int b_row0 =
+          b_direct ? (int)batch_row0(args.slot_t0, slot, args.step, args.N, args.x_shard) : 0;
+      auto load_b = [&](int kt, int s) {
+        uint8_t* sb0 = smem + s * Cfg::kStageBytes + Cfg::kAArea;
+        const int kc = (kt0 + kt) * kBK;
+#pragma unroll
+        for (int p = 0; p < kSplit; ++p) {
+          uint8_t* sb = sb0 + p * Cfg::kBBytes;
+          if (!kBMN) {
+            load(sb, &tmB, kc, n_tile * BN + b_row0, b_z, p, &full[s]);
+          } else {
+#pragma unroll
+            for (int c = 0; c < BN / 64; ++c)
+              load(sb + c * kBox, &tmB, n_tile * BN + c * 64, kc, b_z, p, &full[s]);
+          }
+        }
+      };
       for (int kt = 0; kt < npre; ++kt) {
-        if (kWConv) {
-          load_a32(kt, kt);
-        } else {
+        if (kWConv) load_a32(kt, kt);
+        if (b_direct) {
+          // B from the padded shards, which no kernel writes: the whole stage
+          // is requested before the wait
+          tc::mbar_arrive_expect_tx(&full[kt], kABytesAll + kBBytesAll);
+          if (!kWConv) load_a(kt, kt);
+          load_b(kt, kt);
+        } else if (!kWConv) {
           tc::mbar_expect_tx(&full[kt], kABytesAll);
           load_a(kt, kt);
         }
@@ -296,32 +323,23 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           break;
         }
         if (*abort_flag) break;
-        uint8_t* sa0 = smem + s * Cfg::kStageBytes;
-        uint8_t* sb0 = sa0 + Cfg::kAArea;
         if (kt >= npre) {
           tc::mbar_arrive_expect_tx(&full[s], kABytesAll + kBBytesAll);
           if (kWConv) load_a32(kt, s);
           else load_a(kt, s);
+        } else if (b_direct) {
+          continue;   // requested whole before the wait
         } else {
           tc::mbar_arrive_expect_tx(&full[s], kBBytesAll);
         }
-#pragma unroll
-        for (int p = 0; p < kSplit; ++p) {
-          uint8_t* sb = sb0 + p * Cfg::kBBytes;
-          const int kc = (kt0 + kt) * kBK;
-          if (!kBMN) {
-            load(sb, &tmB, kc, n_tile * BN, b_z, p, &full[s]);
-          } else {
-#pragma unroll
-            for (int c = 0; c < BN / 64; ++c)
-              load(sb + c * kBox, &tmB, n_tile * BN + c * 64, kc, b_z, p, &full[s]);
-          }
-        }
+        load_b(kt, s);
       }
       if (*abort_flag) {
         // drain: wait (bounded) for the copies of the last stages we armed;
-        // prefetched stages not reached yet get their arrival first
-        for (int j = kt; j < npre; ++j) tc::mbar_arrive(&full[j]);
+        // prefetched stages not reached yet get their arrival first (with B
+        // from the padded shards they had it before the wait)
+        if (!b_direct)
+          for (int j = kt; j < npre; ++j) tc::mbar_arrive(&full[j]);
         for (int j = kt; j < npre; ++j) tc::mbar_wait_bounded(&full[j], 0, kWaitNs);
         for (int j = kt - 1; j >= 0 && j >= kt - kStages; --j)
           tc::mbar_wait_bounded(&full[j % kStages], (j / kStages) & 1, kWaitNs);
@@ -898,7 +916,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               float se = ex;
 #pragma unroll
               for (int off = 8; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
-              const int y = valid ? AGN_LD(args.yb + (int64_t)slot * args.N + j) : -1;
+              const int y = !valid ? -1
+                            : args.x_shard > 0
+                                ? AGN_LD(args.yb + (int64_t)worker * (args.x_shard + args.N) +
+                                         batch_row0(args.slot_t0, slot, args.step, args.N,
+                                                    args.x_shard) + j)
+                                : AGN_LD(args.yb + (int64_t)slot * args.N + j);
               const float zy = __shfl_sync(0xffffffffu, z, (lane & 16) + (y > 0 ? y : 0));
               float pr = ex * (1.0f / se);
               if (cl == y) pr -= 1.0f;

@@ -76,6 +76,14 @@ struct TcArgs {
   // tile counter (0 = none), so that the ranks waiting for it give up.
   uint64_t wait_ns;
   int withhold_rank;
+  // Padded shards (batch_row0): x_shard = S > 0 makes the layer-1 operand
+  // (the forward's B, dW's A of layer 1) rows of the padded-shard maps at the
+  // slot's minibatch row, batch coordinate the worker; and labels come from
+  // yb = the padded labels [n][S + m] at the same rows.  x_b_direct: this
+  // launch's B operand is layer 1's (forward of layer 1).
+  const long long* slot_t0;
+  int64_t x_shard;
+  int x_b_direct;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
@@ -126,6 +134,7 @@ struct DwLayerMaps {
   const CUtensorMap *h_mn, *dz_mn, *theta, *acc;
   int M, N;
   int64_t woff, boff;
+  int a_direct = 0;   // h_mn is a padded-shard map (layer 1; args.x_shard > 0)
 };
 // dW with the local step and accumulation of the weights and biases of all
 // `layers` in one persistent launch (mlp_tc_dw.cu, grid min(tiles, num_sms)).

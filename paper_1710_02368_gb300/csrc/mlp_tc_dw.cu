@@ -108,6 +108,7 @@ struct DwLayer {
   int M, N;          // inputs d_{l-1}, outputs d_l
   int mt, nt;        // input tiles (M / 128 + 1: the last holds the bias row), feature tiles
   int tile_begin;    // first tile of this layer in the launch
+  int a_direct;      // A = the padded shards' rows of the slot's minibatch (layer 1)
   int64_t woff, boff;
 };
 struct DwBatch {
@@ -229,6 +230,12 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         const TileIdx ti = decode(B, t);
         const CUtensorMap* tmA = &B.a[ti.layer];
         const CUtensorMap* tmB = &B.b[ti.layer];
+        // layer 1's A from the padded shards: the worker's shard at the slot's
+        // minibatch row (samples past m multiply dZ rows that are zero fill)
+        const bool a_direct = B.layer[ti.layer].a_direct && args.x_shard > 0;
+        const int a_row0 =
+            a_direct ? (int)batch_row0(args.slot_t0, ti.slot, args.step, args.K, args.x_shard) : 0;
+        const int a_z = a_direct ? AGN_LD(args.slot_worker + ti.slot) : ti.slot;
         if (throttle && itp > 0 && *chunk_tiles < itp) {
           const uint64_t t0 = tc::globaltimer_ns();
           while (*chunk_tiles < itp) {
@@ -255,16 +262,17 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
             uint8_t* sa = sa0 + p * kABytes;
             uint8_t* sb = sb0 + p * Cfg::kBBytes;
             if (kSplit == 1) {
-              tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot);
-              tc::tma_load_3d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot);
+              tc::tma_load_3d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK + a_row0, a_z);
+              tc::tma_load_3d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK + a_row0,
+                              a_z);
   #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
                 tc::tma_load_3d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
                                 ti.slot);
             } else {
-              tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK, ti.slot, p);
-              tc::tma_load_4d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK, ti.slot,
-                              p);
+              tc::tma_load_4d(sa, tmA, &full[s], ti.m_tile * 128, kt * kBK + a_row0, a_z, p);
+              tc::tma_load_4d(sa + kBox, tmA, &full[s], ti.m_tile * 128 + 64, kt * kBK + a_row0,
+                              a_z, p);
   #pragma unroll
               for (int c = 0; c < BN / 64; ++c)
                 tc::tma_load_4d(sb + c * kBox, tmB, &full[s], ti.n_tile * BN + c * 64, kt * kBK,
@@ -593,6 +601,7 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
       L.M = d.M;
       L.N = d.N;
       L.woff = d.woff;
+      L.a_direct = d.a_direct;
       L.boff = d.boff;
       L.mt = d.M / 128 + 1;          // rows 0 .. M, row M the bias
       L.nt = (d.N + bn - 1) / bn;
