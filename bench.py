@@ -172,12 +172,13 @@ def cpu_baseline(wl, seconds=15.0):
         ds(np.array([k * wl.shard]))
     t0 = time.perf_counter()
     O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:1], tau[:1], ds, wl.batch, wl.shard,
+              normalize=bool(wl.normalize),
               dtype=dtype)
     per_commit = time.perf_counter() - t0
     n_commits = max(1, min(wl.commits, int(seconds / max(per_commit, 1e-6))))
     t0 = time.perf_counter()
     O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:n_commits], tau[:n_commits], ds, wl.batch,
-              wl.shard, dtype=dtype)
+              wl.shard, normalize=bool(wl.normalize), dtype=dtype)
     dt = time.perf_counter() - t0
     return {"value": n_commits * wl.lam * wl.batch / dt, "unit": UNIT, "cores": os.cpu_count(),
             "kind": "oracle",
@@ -201,7 +202,8 @@ def run_reference(args, wl):
 
     def step():
         O.agn_run(mlp, th0, wl.n, wl.lam, wl.eta, w[:per_step], tau[:per_step], ds, wl.batch,
-                  wl.shard, dtype=dtype, staleness_scaled=args.commit_rule == "dynsgd",
+                  wl.shard, normalize=bool(wl.normalize), dtype=dtype,
+                  staleness_scaled=args.commit_rule == "dynsgd",
                   elide_accumulator=args.elide_accumulator, optimizer=args.optimizer)
     for _ in range(args.warmup):
         step()
@@ -439,11 +441,15 @@ def measure_workload(args, wl, agn, torch, dev, per_step, ws, clock_index=None):
     h.profile(1)
     barrier()
     p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if args.profile_region:
+        torch.cuda.profiler.start()
     p0.record(st)
     for i in range(args.warmup + args.steps, args.warmup + 2 * args.steps):
         step(i)
     p1.record(st)
     barrier()
+    if args.profile_region:
+        torch.cuda.profiler.stop()
     h.profile(0)
     prof_ms = p0.elapsed_time(p1)
     kst = h.kernel_stats()
@@ -607,6 +613,13 @@ def main():
                     help="comma-separated log2 P of the commit kernel runs (default: 20,24,26,28)")
     ap.add_argument("--commit-only", action="store_true",
                     help="time only the standalone commit+pull kernel")
+    ap.add_argument("--lam", type=int, default=0,
+                    help="local steps per commit (lambda) instead of the workload's own: the "
+                         "lambda sweep of the 64-worker workload (1, 5, 10, 20, 40)")
+    ap.add_argument("--profile-region", action="store_true",
+                    help="bracket the per-kernel timing region with cudaProfilerStart/Stop, so "
+                         "that ncu --profile-from-start off captures the launches the roofline "
+                         "figures come from")
     ap.add_argument("--no-sub-workloads", action="store_true",
                     help="time only the headline workload (not the two bf16 workloads)")
     args = ap.parse_args()
@@ -619,6 +632,11 @@ def main():
                                  n_samples=wl.shard * args.workers,
                                  tau_lo=min(wl.tau_lo, args.workers - 1),
                                  tau_hi=min(wl.tau_hi, args.workers - 1))
+    if args.lam:
+        import dataclasses
+        name = wl.name.replace(f"-lam{wl.lam}-", f"-lam{args.lam}-")
+        wl = dataclasses.replace(wl, name=name if name != wl.name else f"{wl.name}-lam{args.lam}",
+                                 lam=args.lam)
     if args.impl == "reference":
         return run_reference(args, wl)
     if args.commit_only:
