@@ -107,7 +107,9 @@ typedef struct agn_options {
      output layer (forward, softmax-CE, dX) as a kernel of its own instead of
      in the epilogue of the last hidden layer's forward GEMM.  Bit 6 gathers
      each local step's minibatch into a buffer of its own (one launch per
-     step) instead of reading it from the padded shards in place. */
+     step) instead of reading it from the padded shards in place.  Bit 7
+     runs the bf16 forward and dX GEMMs of full waves with one 128-row tile
+     per CTA instead of two that share each B stage. */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);

@@ -63,7 +63,9 @@ constexpr int kHeadScratch = (kHC * 128 + 8 * 16 * kHC + 32 * kHC) * 4 + 8 * 256
 // kBK k each (rows of 2 kBK bytes).  With A in tensor memory (kATmem) the
 // stage holds the fp32 weight tile the converters read, then the B pieces,
 // and A's pieces take kACols TMEM columns per stage after the accumulators.
-template <int BN, int kSplit, int kBKs = 64, bool kATmemT = false>
+// kMT = 2 (bf16 forward and dX of full waves): two 128-row A tiles per stage
+// share the B tile, each with its own accumulator.
+template <int BN, int kSplit, int kBKs = 64, bool kATmemT = false, int kMTT = 1>
 struct TileCfg {
   static constexpr int kBK = kBKs;
   static constexpr bool kATmem = kATmemT;
@@ -71,12 +73,12 @@ struct TileCfg {
   static constexpr int kABytes = 128 * kRowBytes;
   static constexpr int kBBytes = BN * kRowBytes;
   static constexpr uint32_t kA32Bytes = 128 * kBK * 4;   // an fp32 weight tile
-  static constexpr int kAArea = kATmem ? (int)kA32Bytes : kSplit * kABytes;
+  static constexpr int kAArea = kATmem ? (int)kA32Bytes : kSplit * kABytes * kMTT;
   static constexpr int kStageBytes = kAArea + kSplit * kBBytes;
   // split mode keeps two accumulators: columns [0, BN) take the leading
   // piece products a0 b0, columns [BN, 2 BN) the five smaller pairs, so the
   // rounding of the tensor core's running sums is relative to each part
-  static constexpr uint32_t kAccCols = (kSplit == 1 ? 1 : 2) * BN;
+  static constexpr uint32_t kAccCols = (kSplit == 1 ? 1 : 2) * BN * kMTT;
   static constexpr uint32_t kACols = kSplit * kBK / 2;   // A pieces of one stage in TMEM
   static constexpr uint32_t kTmemCols = kATmem ? 512 : kAccCols;   // power of two >= 32
 };
@@ -84,10 +86,10 @@ struct TileCfg {
 // The forward / dX epilogue's transpose tiles sit after the barriers when the
 // CTA's shared memory has room for them (then the whole stage ring can hold
 // split-K partial sums), else at the end of the ring.
-template <int BN, int kSplit, int kStages, int kBKs, bool kATmem>
+template <int BN, int kSplit, int kStages, int kBKs, bool kATmem, int kMT = 1>
 struct EpiT {
   static constexpr size_t kRing =
-      (size_t)kStages * TileCfg<BN, kSplit, kBKs, kATmem>::kStageBytes;
+      (size_t)kStages * TileCfg<BN, kSplit, kBKs, kATmem, kMT>::kStageBytes;
   static constexpr bool kSeparate = kRing + 1280 + kEpiTBytes <= 232448;
   static constexpr size_t kOff = kSeparate ? kRing + 256 : kRing - kEpiTBytes;
   static constexpr size_t kRingFree = kSeparate ? kRing : kRing - kEpiTBytes;
@@ -155,14 +157,19 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity,
 // kSplit = 3: fp32 operands as three exact bf16 pieces, 4D tensor maps
 // (inner, rows, batch, piece), fp32 activations in the epilogues and the
 // three pieces of the updated weights written by dW.
-template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
+// kMT = 2: a CTA computes two 128-row tiles (rows 256 x blockIdx.x ..) that
+// share each B stage (bf16 forward and dX without split K): half the B bytes
+// per output, half the CTAs of a full wave.
+template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit, int kMT = 1>
 __global__ void __launch_bounds__(kThreads, kEpi == kEpiDW ? 2 : 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const TcArgs args) {
   constexpr int kBK = stage_k(kSplit, kEpi);
   constexpr bool kATmem = a_in_tmem(kSplit, kEpi, BN);
-  using Cfg = TileCfg<BN, kSplit, kBK, kATmem>;
-  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem>;
+  static_assert(kMT == 1 || (kSplit == 1 && (kEpi == kEpiFwd || kEpi == kEpiDX)),
+                "two row tiles per CTA: bf16 forward and dX only");
+  using Cfg = TileCfg<BN, kSplit, kBK, kATmem, kMT>;
+  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem, kMT>;
   static_assert(!kATmem || Cfg::kAccCols + kStages * Cfg::kACols <= Cfg::kTmemCols, "TMEM");
   constexpr int kABytes = Cfg::kABytes;
   constexpr uint32_t kA32Bytes = Cfg::kA32Bytes;
@@ -193,7 +200,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __syncthreads();
   if (s_skip != 0) return;   // uniform across the CTA
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ks = kEpi == kEpiDW ? 1 : args.ksplit;   // CTAs sharing one output tile
+  const int ks = kEpi == kEpiDW || kMT > 1 ? 1 : args.ksplit;   // CTAs sharing one output tile
   const int m_tile = blockIdx.x, n_tile = blockIdx.y;
   const int slot = blockIdx.z / ks, sk = blockIdx.z % ks;
   const int worker = AGN_LD(args.slot_worker + slot);
@@ -232,7 +239,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
-  const uint32_t tmem = *tmem_holder;
+  const uint32_t tmem_base = *tmem_holder;
+  const uint32_t tmem = tmem_base;
 
   // Programmatic dependent launch: the setup above ran while the preceding
   // kernel finished.  Everything that reads or writes global memory waits
@@ -258,13 +266,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         uint8_t* sa0 = smem + s * Cfg::kStageBytes;
         const int kc = (kt0 + kt) * kBK;
 #pragma unroll
-        for (int p = 0; p < kSplit; ++p) {
-          uint8_t* sa = sa0 + p * kABytes;
-          if (!kAMN) {
-            load(sa, &tmA, kc, m_tile * 128, a_z, p, &full[s]);
-          } else {
-            load(sa, &tmA, m_tile * 128, kc, a_z, p, &full[s]);
-            load(sa + kBox, &tmA, m_tile * 128 + 64, kc, a_z, p, &full[s]);
+        for (int mh = 0; mh < kMT; ++mh) {
+          const int r0 = (m_tile * kMT + mh) * 128;
+#pragma unroll
+          for (int p = 0; p < kSplit; ++p) {
+            uint8_t* sa = sa0 + (mh * kSplit + p) * kABytes;
+            if (!kAMN) {
+              load(sa, &tmA, kc, r0, a_z, p, &full[s]);
+            } else {
+              load(sa, &tmA, r0, kc, a_z, p, &full[s]);
+              load(sa + kBox, &tmA, r0 + 64, kc, a_z, p, &full[s]);
+            }
           }
         }
       };
@@ -280,7 +292,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       };
       // prefetched stages count the A bytes now and arrive with the B bytes
       // below, so no phase can complete before its B boxes are requested
-      constexpr uint32_t kABytesAll = kWConv ? 0u : kSplit * kABytes;   // A bytes on full[s]
+      constexpr uint32_t kABytesAll = kWConv ? 0u : kSplit * kABytes * kMT;   // A bytes on full[s]
       constexpr uint32_t kBBytesAll = kSplit * Cfg::kBBytes;
       const int npre = kPrefetchA ? min(KT, kStages) : 0;
       // (slot_t0 is written by the host before the launch)
@@ -497,8 +509,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk) {
 #pragma unroll
-          for (int q = 0; q < kPairs; ++q) {
-            const uint32_t sa = sa0 + (kSplit == 1 ? 0 : kPairA[q]) * kABytes;
+          for (int mq = 0; mq < kMT * kPairs; ++mq) {
+            const int q = mq % kPairs, mh = mq / kPairs;   // (kMT > 1: kPairs = 1)
+            const uint32_t sa = sa0 + (mh * kSplit + (kSplit == 1 ? 0 : kPairA[q])) * kABytes;
             const uint32_t sb = sb0 + (kSplit == 1 ? 0 : kPairB[q]) * Cfg::kBBytes;
             // MN-major: 16 k rows of 128 bytes per k16 step, the two 64-wide
             // boxes kBox apart; K-major: 32 bytes along the row per k16 step,
@@ -509,7 +522,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const uint64_t bd = kBMN ? tc::smem_desc_sw128(sb + kk * 2048, kBox, 1024)
                                 : kBK == 64 ? tc::smem_desc_sw128(sb + kk * 32, 16, 1024)
                                             : tc::smem_desc_sw64(sb + kk * 32, 16, 512);
-            const uint32_t dcol = (kSplit == 3 && q > 0) ? (uint32_t)BN : 0u;
+            const uint32_t dcol = (kSplit == 3 && q > 0) ? (uint32_t)BN : (uint32_t)(mh * BN);
             const bool acc_on = kSplit == 1 ? (kt | kk | q) != 0
                                             : (q == 0 ? (kt | kk) != 0 : ((kt | kk) != 0 || q > 1));
             if (kATmem)
@@ -544,524 +557,530 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (!ok) {
     if (threadIdx.x == 0) atomicExch(args.err, 1);
   } else {
-    const int g = warp & 3, half = warp >> 2;
-    const int row = 128 * m_tile + 32 * g + lane;   // M index of this thread
-    const bool row_ok = row < args.M;
-    const uint32_t lane_base = (uint32_t)(32 * g) << 16;
-    float* theta = args.theta + (int64_t)worker * args.ld_param;
-    // Accumulated values of this thread's row for columns c0 .. c0 + 15: from
-    // TMEM (the sum of the two accumulators in the split mode), or, with
-    // split K, the partial sums of all ks CTAs of the tile in rank order.
-    const int64_t tile_id = ((int64_t)slot * gridDim.y + n_tile) * gridDim.x + m_tile;
-    const int trow = 32 * g + lane;
-    auto tmem_vals = [&](int c0, uint32_t (&r)[16]) {
-      tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)c0, r);
-      if (kSplit == 3) {
-        uint32_t r2[16];
-        tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(BN + c0), r2);
+    // kMT = 2: the CTA's two row tiles in turn, accumulators BN columns apart
+#pragma unroll 1
+    for (int mh = 0; mh < kMT; ++mh) {
+      const int m_tile = (int)blockIdx.x * kMT + mh;
+      const uint32_t tmem = tmem_base + (uint32_t)(mh * BN);
+      const int g = warp & 3, half = warp >> 2;
+      const int row = 128 * m_tile + 32 * g + lane;   // M index of this thread
+      const bool row_ok = row < args.M;
+      const uint32_t lane_base = (uint32_t)(32 * g) << 16;
+      float* theta = args.theta + (int64_t)worker * args.ld_param;
+      // Accumulated values of this thread's row for columns c0 .. c0 + 15: from
+      // TMEM (the sum of the two accumulators in the split mode), or, with
+      // split K, the partial sums of all ks CTAs of the tile in rank order.
+      const int64_t tile_id = ((int64_t)slot * gridDim.y + n_tile) * gridDim.x + m_tile;
+      const int trow = 32 * g + lane;
+      auto tmem_vals = [&](int c0, uint32_t (&r)[16]) {
+        tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)c0, r);
+        if (kSplit == 3) {
+          uint32_t r2[16];
+          tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(BN + c0), r2);
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
+        }
         tc::tmem_ld_wait();
+      };
+      // Split K (forward / dX): chunk j of the tile (columns 32 j .. 32 j + 31)
+      // is finished by rank j % ks.  Every rank stores its partial sums of the
+      // chunks it does not finish ([column][row], rows contiguous) and counts
+      // itself in on the tile's counter (an array the previous launch cleared).
+      // A rank that finishes chunks waits until all ks ranks are in (the CTAs
+      // of a launch with ks > 1 are resident together: at most one per SM, no
+      // more than the SMs), copies the other ranks' partial sums of its chunks
+      // into its stage ring and adds them in rank order, its own from TMEM.
+      // Warps 0-3 take columns 0-15 of every chunk, warps 4-7 columns 16-31.
+      constexpr int kNch = BN / 32;
+      constexpr uint32_t kChunkBytes = 128u * 32u * 4u;
+      const bool split_k = kEpi != kEpiDW && ks > 1;
+      const int own_rank = split_k ? sk : 0, kstride = split_k ? ks : 1;
+      const int n_own = (kNch - own_rank + kstride - 1) / kstride;   // chunks own_rank + o ks
+      const int co = 16 * half;                                       // this warp's columns of a chunk
+      const float* red_smem = reinterpret_cast<const float*>(smem);   // the free stage ring
+      // Forward and dX epilogues: the warp's 32 rows x 16 columns go through a
+      // warp-private shared-memory tile (column-major) so that each lane then
+      // handles four consecutive rows (features, contiguous in memory) of four
+      // columns: 16-byte bias / mask loads, 16-byte stores of the output and
+      // 8-byte stores of each bf16 piece.
+      float* tT = reinterpret_cast<float*>(smem + Epi::kOff) +
+                  warp * (32 * 32);
+      const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
+      const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
+      const bool row4_ok = row4 < args.M;                      // M % 4 == 0: all four or none
+      const TAct* mask = kEpi == kEpiDX
+                             ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
+                             : nullptr;
+      // the mask of the warp's first columns (and the bias) are loaded before
+      // the split-K exchange: they do not depend on it
+      float4 hm[4];
+      auto load_mask = [&](int c0) {
+        if (kEpi == kEpiDX && row4_ok) {   // all mask loads in flight before any store
 #pragma unroll
-        for (int i = 0; i < 16; ++i)
-          r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
-      }
-      tc::tmem_ld_wait();
-    };
-    // Split K (forward / dX): chunk j of the tile (columns 32 j .. 32 j + 31)
-    // is finished by rank j % ks.  Every rank stores its partial sums of the
-    // chunks it does not finish ([column][row], rows contiguous) and counts
-    // itself in on the tile's counter (an array the previous launch cleared).
-    // A rank that finishes chunks waits until all ks ranks are in (the CTAs
-    // of a launch with ks > 1 are resident together: at most one per SM, no
-    // more than the SMs), copies the other ranks' partial sums of its chunks
-    // into its stage ring and adds them in rank order, its own from TMEM.
-    // Warps 0-3 take columns 0-15 of every chunk, warps 4-7 columns 16-31.
-    constexpr int kNch = BN / 32;
-    constexpr uint32_t kChunkBytes = 128u * 32u * 4u;
-    const bool split_k = kEpi != kEpiDW && ks > 1;
-    const int own_rank = split_k ? sk : 0, kstride = split_k ? ks : 1;
-    const int n_own = (kNch - own_rank + kstride - 1) / kstride;   // chunks own_rank + o ks
-    const int co = 16 * half;                                       // this warp's columns of a chunk
-    const float* red_smem = reinterpret_cast<const float*>(smem);   // the free stage ring
-    // Forward and dX epilogues: the warp's 32 rows x 16 columns go through a
-    // warp-private shared-memory tile (column-major) so that each lane then
-    // handles four consecutive rows (features, contiguous in memory) of four
-    // columns: 16-byte bias / mask loads, 16-byte stores of the output and
-    // 8-byte stores of each bf16 piece.
-    float* tT = reinterpret_cast<float*>(smem + Epi::kOff) +
-                warp * (32 * 32);
-    const int r4 = (lane & 7) * 4, jl = lane >> 3;          // rows r4 .. r4 + 3, columns jl + 4 u
-    const int row4 = 128 * m_tile + 32 * g + r4;             // first row of this lane
-    const bool row4_ok = row4 < args.M;                      // M % 4 == 0: all four or none
-    const TAct* mask = kEpi == kEpiDX
-                           ? static_cast<const TAct*>(args.mask) + (int64_t)slot * args.mask_bstride
-                           : nullptr;
-    // the mask of the warp's first columns (and the bias) are loaded before
-    // the split-K exchange: they do not depend on it
-    float4 hm[4];
-    auto load_mask = [&](int c0) {
-      if (kEpi == kEpiDX && row4_ok) {   // all mask loads in flight before any store
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int j = n_tile * BN + c0 + jl + 4 * u;
-          hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
-                             : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
-    };
-    constexpr bool kFwd = kEpi == kEpiFwd || kEpi == kEpiFwdHead;
-    float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (kFwd && row4_ok && n_own > 0)
-      bias4 = AGN_LD(reinterpret_cast<const float4*>(theta + args.boff + row4));
-    if (n_own > 0) load_mask(32 * own_rank + co);
-    // fused output layer: this tile's 128 columns of W_L (kHC x 128, zero past
-    // C and M), loads in flight across the split-K exchange
-    constexpr int kW3Per = kHC * 128 / kThreads;
-    float w3v_reg[kEpi == kEpiFwdHead ? kW3Per : 1];
-    if (kEpi == kEpiFwdHead) {
-      const float* w3g = theta + args.head_woff;
-#pragma unroll
-      for (int k = 0; k < kW3Per; ++k) {
-        const int i = threadIdx.x + k * kThreads;
-        const int c = i >> 7, rr = 128 * m_tile + (i & 127);
-        w3v_reg[k] = (c < args.head_C && rr < args.M) ? AGN_LD(w3g + (int64_t)c * args.M + rr) : 0.f;
-      }
-    }
-    bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
-    if (split_k) {
-      float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
-#pragma unroll 1
-      for (int j = 0; j < kNch; ++j) {
-        if (j % ks == sk) continue;
-        uint32_t r[16];
-        tmem_vals(32 * j + co, r);
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-          AGN_STCG(mine + (int64_t)(32 * j + co + i) * 128 + trow, __uint_as_float(r[i]));
-      }
-      // the CTA's stores, ordered by the barrier, are released by one
-      // acquire-release arrival; the wait acquires the other ranks'
-      __shared__ int s_have;
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        int* ctr = args.counter + tile_id;
-        bool got = AGN_BOUNDS_OK(ctr, 4);
-        if (!got) AGN_BOUNDS_FAIL(ctr);   // bounds-checked build: no wait on a stray counter
-        if (got && sk + 1 != args.withhold_rank) tc::atomic_add_acq_rel_gpu(ctr, 1);
-        if (got && n_own > 0) {
-          got = tc::wait_count_low(ctr, ks, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
-          if (got) {
-            tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
-            tc::mbar_arrive_expect_tx(red, kChunkBytes * (uint32_t)(n_own * (ks - 1)));
-            for (int o = 0, d = 0; o < n_own; ++o) {
-              const int j = sk + o * ks;
-              for (int q = 0; q < ks; ++q) {
-                if (q == sk) continue;
-                const float* src = args.part + (tile_id * ks + q) * (int64_t)(128 * BN) +
-                                   (int64_t)j * (32 * 128);
-                if (AGN_BOUNDS_OK(src, kChunkBytes)) {
-                  tc::bulk_load(smem + (size_t)d * kChunkBytes, src, kChunkBytes, red);
-                } else {   // bounds-checked build: account for the bytes, skip the copy
-                  AGN_BOUNDS_FAIL(src);
-                  tc::mbar_complete_tx(red, kChunkBytes);
-                }
-                ++d;
-              }
-            }
-          }
-        }
-        s_have = got;
-      }
-      __syncthreads();
-      have = s_have != 0;
-      if (have && n_own > 0) have = __syncthreads_and(wait_or_abort(red, 0, abort_flag)) != 0;
-      if (threadIdx.x == 0 && !have) atomicExch(args.err, 1);   // gave up: report, skip the epilogue
-    }
-    // the accumulated values of this thread's row for columns c0 .. c0 + 15
-    // of chunk j = own_rank + o ks (c0 = 32 j + co)
-    auto vals = [&](int o, int c0, uint32_t (&r)[16]) {
-      tmem_vals(c0, r);
-      if (!split_k) return;
-      float v[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] = 0.f;
-      for (int q = 0, d = 0; q < ks; ++q) {
-        if (q == sk) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] += __uint_as_float(r[i]);
-        } else {
-          const float* pq = red_smem + (size_t)(o * (ks - 1) + d) * (32 * 128) + co * 128 + trow;
-#pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] += pq[i * 128];
-          ++d;
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(v[i]);
-    };
-    // fused output layer: W_L's rows for this tile's 128 features, the number
-    // of 32-sample chunks with samples, and the scratch
-    float* sW3 = reinterpret_cast<float*>(smem + Epi::kHeadOff);
-    float* sPart = sW3 + kHC * 128;
-    float* sG = sPart + 8 * 16 * kHC;
-    uint16_t* sMask = reinterpret_cast<uint16_t*>(sG + 32 * kHC);   // [owned chunk][thread]
-    const int nchk = (args.N + 31) / 32;
-    if (kEpi == kEpiFwdHead && have) {
-#pragma unroll
-      for (int k = 0; k < kW3Per; ++k) sW3[threadIdx.x + k * kThreads] = w3v_reg[k];
-      __syncthreads();
-    }
-    if (!have) {
-      // reported above
-    } else if (kEpi == kEpiFwd || kEpi == kEpiDX || kEpi == kEpiFwdHead) {
-      TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
-#pragma unroll 1
-      for (int o = 0; o < n_own; ++o) {
-        const int c0 = 32 * (own_rank + o * kstride) + co;
-        if (o > 0) load_mask(c0);
-        uint32_t r[16];
-        vals(o, c0, r);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
-        __syncwarp();
-        if (kEpi == kEpiFwdHead && (c0 - co) / 32 < nchk) {
-          // Pass 1 of the fused output layer, before this chunk's stores (so
-          // that the release below orders only the partials): this CTA's
-          // share of the chunk's logits, sum over its 128 features of
-          // H_{L-1}[j][f] W_L[c][f].  A lane sums its four features; the eight
-          // lanes of a column fold by a fixed shuffle tree; the four row
-          // quadrants of a column half are added in order below.  The ReLU
-          // mask of the lane's 4 x 4 values goes to shared memory for pass 2.
-          // This code runs once per chunk and launch, from a cold instruction
-          // cache: it loops over the lane's four columns (u) rather than
-          // unrolling them, which keeps it a quarter of the size.
-          const int C = args.head_C;
-          uint32_t mbits = 0;
-          // W_L rows past C are zero in shared memory: all kHC classes are
-          // summed unguarded, as independent chains
-          const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
-#pragma unroll 1
           for (int u = 0; u < 4; ++u) {
             const int j = n_tile * BN + c0 + jl + 4 * u;
-            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (row4_ok && j < args.N) {
-              a = *reinterpret_cast<const float4*>(tT + (jl + 4 * u) * 32 + r4);
-              a.x = fmaxf(a.x + bias4.x, 0.f);
-              a.y = fmaxf(a.y + bias4.y, 0.f);
-              a.z = fmaxf(a.z + bias4.z, 0.f);
-              a.w = fmaxf(a.w + bias4.w, 0.f);
-            }
-            const float hq[4] = {a.x, a.y, a.z, a.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e)   // the mask of the value as stored
-              mbits |= (static_cast<float>(static_cast<TAct>(hq[e])) > 0.f ? 1u : 0u)
-                       << (4 * u + e);
-            float zp[kHC];
-#pragma unroll
-            for (int c = 0; c < kHC; ++c) {
-              const float4 w = w3v[c * 32];
-              float t = hq[0] * w.x;
-              t = fmaf(hq[1], w.y, t);
-              t = fmaf(hq[2], w.z, t);
-              zp[c] = fmaf(hq[3], w.w, t);
-            }
-            // fold the eight lanes of the column (lane bits 0-2) by a fixed
-            // reduce-scatter: each round a lane keeps half of its classes and
-            // adds its partner's share of them; afterwards the lane holds the
-            // column's sums of classes kb and kb + 1, kb = 8 b2 + 4 b1 + 2 b0
-            static_assert(kHC == 16, "the reduce-scatter folds 16 classes");
-            const int b2 = (lane >> 2) & 1, b1 = (lane >> 1) & 1, b0 = lane & 1;
-            float k8[8], k4[4], k2[2];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const float keep = b2 ? zp[k + 8] : zp[k], send = b2 ? zp[k] : zp[k + 8];
-              k8[k] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-            }
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const float keep = b1 ? k8[k + 4] : k8[k], send = b1 ? k8[k] : k8[k + 4];
-              k4[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
-            }
-#pragma unroll
-            for (int k = 0; k < 2; ++k) {
-              const float keep = b0 ? k4[k + 2] : k4[k], send = b0 ? k4[k] : k4[k + 2];
-              k2[k] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
-            }
-            *reinterpret_cast<float2*>(sPart + (warp * 16 + jl + 4 * u) * kHC + 8 * b2 + 4 * b1 +
-                                       2 * b0) = make_float2(k2[0], k2[1]);
-          }
-          sMask[o * kThreads + threadIdx.x] = (uint16_t)mbits;
-          __syncthreads();
-          const int chunk = (c0 - co) / 32;
-          float* gp = args.head_part +
-                      (((int64_t)slot * nchk + chunk) * gridDim.x + m_tile) * (32 * kHC);
-          for (int i = threadIdx.x; i < 32 * kHC; i += kThreads) {
-            const int cc = i / kHC, c = i % kHC, hf = cc >> 4, jcl = cc & 15;
-            float sum = 0.f;
-            if (c < C)
-              for (int gq = 0; gq < 4; ++gq) sum += sPart[((gq + 4 * hf) * 16 + jcl) * kHC + c];
-            AGN_STCG(gp + i, sum);
-          }
-          __syncthreads();
-          // count in: the CTA's partials, ordered before by the barrier, are
-          // released by one acquire-release arrival
-          if (threadIdx.x == 0) {
-            int* hc = args.head_counter + slot * nchk + chunk;
-            if (AGN_BOUNDS_OK(hc, 4)) tc::atomic_add_acq_rel_gpu(hc, 1);
-            else AGN_BOUNDS_FAIL(hc);
-          }
-        }
-        if (row4_ok) {
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const int jc = jl + 4 * u;
-            const int j = n_tile * BN + c0 + jc;
-            if (j < args.N) {
-              const float4 a = *reinterpret_cast<const float4*>(tT + jc * 32 + r4);
-              float v[4] = {a.x, a.y, a.z, a.w};
-              if (kFwd) {
-                v[0] += bias4.x; v[1] += bias4.y; v[2] += bias4.z; v[3] += bias4.w;
-                if (args.relu) {
-#pragma unroll
-                  for (int e = 0; e < 4; ++e) v[e] = fmaxf(v[e], 0.f);
-                }
-              } else {
-                const float hv[4] = {hm[u].x, hm[u].y, hm[u].z, hm[u].w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) v[e] = hv[e] > 0.f ? v[e] : 0.f;
-              }
-              const int64_t o4 = (int64_t)j * args.ldo + row4;
-              store4(out + o4, v);
-              if (kSplit == 3 && args.out_pieces) {
-                uint2 q0, q1, q2;
-                split3_x4(v, q0, q1, q2);
-                bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o4;
-                AGN_ST(reinterpret_cast<uint2*>(pp), q0);
-                AGN_ST(reinterpret_cast<uint2*>(pp + args.out_plane), q1);
-                AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.out_plane), q2);
-              }
-            }
-          }
-        }
-        __syncwarp();
-      }
-      if (kEpi == kEpiFwdHead) {
-        // Pass 2: once every feature tile's partials of a chunk are in (all
-        // CTAs of this launch are resident), the chunk's logits are summed in
-        // tile order plus b_L; every half-warp takes softmax cross-entropy and
-        // dZ_L = (softmax - onehot(y)) / m of a sample (the first feature tile
-        // writes dZ_L and the chunk's loss); every CTA then writes dZ_{L-1} =
-        // (dZ_L W_L) [H_{L-1} > 0] for its own features (W_L before its
-        // update).
-        __shared__ int s_hok;
-        const int C = args.head_C;
-        const float* bl = theta + args.head_boff;
-        TAct* dh = static_cast<TAct*>(args.dh) + (int64_t)slot * args.out_bstride;
-        const int mtn = (int)gridDim.x;
-#pragma unroll 1
-        for (int o = 0; o < n_own; ++o) {
-          const int chunk = own_rank + o * kstride;
-          if (chunk >= nchk) continue;   // CTA-uniform
-          int* ctr = args.head_counter + slot * nchk + chunk;
-          if (threadIdx.x == 0)
-            s_hok = AGN_BOUNDS_OK(ctr, 4) &&
-                    tc::wait_count_low(ctr, mtn, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
-          __syncthreads();
-          if (!s_hok) {
-            if (threadIdx.x == 0) atomicExch(args.err, 1);
-            break;
-          }
-          // the feature tiles' partials in tile order: each thread sums two of
-          // the chunk's 32 x kHC logits, up to 2 x 16 loads in flight; thread
-          // t holds class t % kHC of samples t / kHC and 16 + t / kHC, so the
-          // 16 lanes of a half-warp hold one sample's logits
-          static_assert(32 * kHC == 2 * kThreads, "two logits per thread");
-          static_assert(kHC == 16, "one sample per half-warp");
-          const float* gp0 = args.head_part + ((int64_t)slot * nchk + chunk) * mtn * (32 * kHC);
-          float zz[2] = {0.f, 0.f};
-          for (int m0 = 0; m0 < mtn; m0 += 16) {
-            float p0[16], p1[16];
-#pragma unroll
-            for (int q = 0; q < 16; ++q) {
-              const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
-              p0[q] = m0 + q < mtn ? AGN_LDCG(pq) : 0.f;
-              p1[q] = m0 + q < mtn ? AGN_LDCG(pq + kThreads) : 0.f;
-            }
-#pragma unroll
-            for (int q = 0; q < 16; ++q) {
-              zz[0] += p0[q];
-              zz[1] += p1[q];
-            }
-          }
-          // softmax cross-entropy and dZ_L = (softmax - onehot(y)) / m of the
-          // thread's two (sample, class) entries: max and sum over the
-          // sample's classes by a fixed shuffle tree within the half-warp;
-          // the first feature tile writes dZ_L
-          float* sCE = sPart;   // [32] per-sample cross-entropy (pass 1 is done with sPart)
-          {
-            const int cl = threadIdx.x % kHC;
-            const bool cv = cl < C;
-            const float inv_m = 1.0f / (float)args.N;
-            const float bc = cv ? AGN_LD(bl + cl) : 0.f;
-#pragma unroll 1
-            for (int hh = 0; hh < 2; ++hh) {
-              const int sl = 16 * hh + (threadIdx.x >> 4);   // sample within the chunk
-              const int j = n_tile * BN + 32 * chunk + sl;
-              const bool valid = j < args.N;
-              const float z = cv ? (hh ? zz[1] : zz[0]) + bc : -INFINITY;
-              float mx = z;
-#pragma unroll
-              for (int off = 8; off > 0; off >>= 1)
-                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-              const float ex = cv ? expf(z - mx) : 0.f;
-              float se = ex;
-#pragma unroll
-              for (int off = 8; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
-              const int y = !valid ? -1
-                            : args.x_shard > 0
-                                ? AGN_LD(args.yb + (int64_t)worker * (args.x_shard + args.N) +
-                                         batch_row0(args.slot_t0, slot, args.step, args.N,
-                                                    args.x_shard) + j)
-                                : AGN_LD(args.yb + (int64_t)slot * args.N + j);
-              const float zy = __shfl_sync(0xffffffffu, z, (lane & 16) + (y > 0 ? y : 0));
-              float pr = ex * (1.0f / se);
-              if (cl == y) pr -= 1.0f;
-              const float gz = valid ? pr * inv_m : 0.f;
-              sG[sl * kHC + cl] = gz;
-              if (m_tile == 0 && valid && cv) {
-                const TAct gv = static_cast<TAct>(gz);
-                const int64_t zi = ((int64_t)slot * args.N + j) * args.ldz + cl;
-                AGN_ST(static_cast<TAct*>(args.dzl) + zi, gv);
-                if (args.dzl_pieces) {
-                  bf16 q0, q1, q2;
-                  split3(static_cast<float>(gv), q0, q1, q2);
-                  AGN_ST(args.dzl_pieces + zi, q0);
-                  AGN_ST(args.dzl_pieces + args.dzl_plane + zi, q1);
-                  AGN_ST(args.dzl_pieces + 2 * args.dzl_plane + zi, q2);
-                }
-              }
-              if (cl == 0) sCE[sl] = valid ? (logf(se) + mx) - zy : 0.f;
-            }
-          }
-          __syncthreads();
-          float ce = 0.f;
-          if (warp == 0) {   // the chunk's cross-entropy sum, fixed tree over its samples
-            ce = sCE[lane];
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) ce += __shfl_xor_sync(0xffffffffu, ce, off);
-          }
-          if (row4_ok) {
-            const uint32_t mbits = sMask[o * kThreads + threadIdx.x];
-            const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
-            // dZ_{L-1} of the lane's 4 features x 4 columns: 16 independent
-            // chains over the classes (dZ_L is zero past C)
-            float d[4][4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-              for (int e = 0; e < 4; ++e) d[u][e] = 0.f;
-#pragma unroll 2
-            for (int c = 0; c < kHC; ++c) {
-              const float4 w = w3v[c * 32];
-#pragma unroll
-              for (int u = 0; u < 4; ++u) {
-                const float gzc = sG[(co + jl + 4 * u) * kHC + c];
-                d[u][0] = fmaf(gzc, w.x, d[u][0]);
-                d[u][1] = fmaf(gzc, w.y, d[u][1]);
-                d[u][2] = fmaf(gzc, w.z, d[u][2]);
-                d[u][3] = fmaf(gzc, w.w, d[u][3]);
-              }
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const int j = n_tile * BN + 32 * chunk + co + jl + 4 * u;
-              if (j < args.N) {
-                float dv[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) dv[e] = (mbits >> (4 * u + e)) & 1u ? d[u][e] : 0.f;
-                const int64_t o4 = (int64_t)j * args.ldo + row4;
-                store4(dh + o4, dv);
-                if (kSplit == 3 && args.dh_pieces) {
-                  uint2 q0, q1, q2;
-                  split3_x4(dv, q0, q1, q2);
-                  bf16* pp = args.dh_pieces + (int64_t)slot * args.out_bstride + o4;
-                  AGN_ST(reinterpret_cast<uint2*>(pp), q0);
-                  AGN_ST(reinterpret_cast<uint2*>(pp + args.dh_plane), q1);
-                  AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.dh_plane), q2);
-                }
-              }
-            }
-          }
-          if (threadIdx.x == 0) {
-            // the chunk's loss contribution (sum of its samples' cross-entropy
-            // over m) in the chunk's slot; the run's loss kernel adds the slots
-            // in order
-            if (m_tile == 0) {
-              const float part = ce / (float)args.N;
-              AGN_ST(args.loss_parts +
-                         ((int64_t)AGN_LD(args.slot_commit + slot) * args.lam + args.step) * nchk +
-                         chunk,
-                     part);
-              if (!isfinite(part)) atomicExch(args.nonfinite, 1);
-            }
-          }
-        }
-      }
-    } else {   // kEpiDW
-      float* acc = args.acc + (int64_t)worker * args.ld_param;
-      bf16* tb = args.theta_b + (int64_t)worker * args.ld_param;
-      const float eta = args.eta;
-      // Chunks of 16 columns; the loads of chunk c + 1 are issued before the
-      // stores of chunk c, so every thread keeps 32 loads in flight while it
-      // writes (the epilogue is bound by DRAM latency x bandwidth).
-      constexpr int kCh = 16;
-      constexpr int kChunks = (BN / 2) / kCh;
-      const float* __restrict__ th_in = theta;
-      const float* __restrict__ ac_in = acc;
-      const int cbase = n_tile * BN + half * (BN / 2);     // first column of this half
-      const int64_t pbase = args.woff + (int64_t)cbase * args.M + row;
-      float thn[kCh], acn[kCh];
-      auto load_chunk = [&](int ch) {
-        const int nvalid = row_ok ? min(kCh, args.N - (cbase + ch * kCh)) : 0;
-#pragma unroll
-        for (int i = 0; i < kCh; ++i) {
-          if (i < nvalid) {
-            const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
-            thn[i] = AGN_LDCS(th_in + p);
-            acn[i] = AGN_LDCS(ac_in + p);
+            hm[u] = j < args.N ? load4(mask + (int64_t)j * args.ldo + row4)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
           }
         }
       };
-      load_chunk(0);
+      constexpr bool kFwd = kEpi == kEpiFwd || kEpi == kEpiFwdHead;
+      float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kFwd && row4_ok && n_own > 0)
+        bias4 = AGN_LD(reinterpret_cast<const float4*>(theta + args.boff + row4));
+      if (n_own > 0) load_mask(32 * own_rank + co);
+      // fused output layer: this tile's 128 columns of W_L (kHC x 128, zero past
+      // C and M), loads in flight across the split-K exchange
+      constexpr int kW3Per = kHC * 128 / kThreads;
+      float w3v_reg[kEpi == kEpiFwdHead ? kW3Per : 1];
+      if (kEpi == kEpiFwdHead) {
+        const float* w3g = theta + args.head_woff;
 #pragma unroll
-      for (int ch = 0; ch < kChunks; ++ch) {
-        float th[kCh], ac[kCh];
-#pragma unroll
-        for (int i = 0; i < kCh; ++i) {
-          th[i] = thn[i];
-          ac[i] = acn[i];
+        for (int k = 0; k < kW3Per; ++k) {
+          const int i = threadIdx.x + k * kThreads;
+          const int c = i >> 7, rr = 128 * m_tile + (i & 127);
+          w3v_reg[k] = (c < args.head_C && rr < args.M) ? AGN_LD(w3g + (int64_t)c * args.M + rr) : 0.f;
         }
-        uint32_t r[kCh];
-        const uint32_t col = (uint32_t)(half * (BN / 2) + ch * kCh);
-        tc::tmem_ld_32x32b_x16(tmem + lane_base + col, r);
-        uint32_t r2[kCh];
-        if (kSplit == 3) tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)BN + col, r2);
-        if (ch + 1 < kChunks) load_chunk(ch + 1);
-        tc::tmem_ld_wait();
-        if (kSplit == 3) {
+      }
+      bool have = true;   // the other ranks' partial sums of this CTA's chunks are in the ring
+      if (split_k) {
+        float* mine = args.part + (tile_id * ks + sk) * (int64_t)(128 * BN);
+#pragma unroll 1
+        for (int j = 0; j < kNch; ++j) {
+          if (j % ks == sk) continue;
+          uint32_t r[16];
+          tmem_vals(32 * j + co, r);
 #pragma unroll
-          for (int i = 0; i < kCh; ++i)
-            r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
+          for (int i = 0; i < 16; ++i)
+            AGN_STCG(mine + (int64_t)(32 * j + co + i) * 128 + trow, __uint_as_float(r[i]));
         }
-        const int nvalid = row_ok ? min(kCh, args.N - (cbase + ch * kCh)) : 0;
+        // the CTA's stores, ordered by the barrier, are released by one
+        // acquire-release arrival; the wait acquires the other ranks'
+        __shared__ int s_have;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+          int* ctr = args.counter + tile_id;
+          bool got = AGN_BOUNDS_OK(ctr, 4);
+          if (!got) AGN_BOUNDS_FAIL(ctr);   // bounds-checked build: no wait on a stray counter
+          if (got && sk + 1 != args.withhold_rank) tc::atomic_add_acq_rel_gpu(ctr, 1);
+          if (got && n_own > 0) {
+            got = tc::wait_count_low(ctr, ks, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
+            if (got) {
+              tc::fence_proxy_async_global();   // the ranks' stores, before the bulk reads
+              tc::mbar_arrive_expect_tx(red, kChunkBytes * (uint32_t)(n_own * (ks - 1)));
+              for (int o = 0, d = 0; o < n_own; ++o) {
+                const int j = sk + o * ks;
+                for (int q = 0; q < ks; ++q) {
+                  if (q == sk) continue;
+                  const float* src = args.part + (tile_id * ks + q) * (int64_t)(128 * BN) +
+                                     (int64_t)j * (32 * 128);
+                  if (AGN_BOUNDS_OK(src, kChunkBytes)) {
+                    tc::bulk_load(smem + (size_t)d * kChunkBytes, src, kChunkBytes, red);
+                  } else {   // bounds-checked build: account for the bytes, skip the copy
+                    AGN_BOUNDS_FAIL(src);
+                    tc::mbar_complete_tx(red, kChunkBytes);
+                  }
+                  ++d;
+                }
+              }
+            }
+          }
+          s_have = got;
+        }
+        __syncthreads();
+        have = s_have != 0;
+        if (have && n_own > 0) have = __syncthreads_and(wait_or_abort(red, 0, abort_flag)) != 0;
+        if (threadIdx.x == 0 && !have) atomicExch(args.err, 1);   // gave up: report, skip the epilogue
+      }
+      // the accumulated values of this thread's row for columns c0 .. c0 + 15
+      // of chunk j = own_rank + o ks (c0 = 32 j + co)
+      auto vals = [&](int o, int c0, uint32_t (&r)[16]) {
+        tmem_vals(c0, r);
+        if (!split_k) return;
+        float v[16];
 #pragma unroll
-        for (int i = 0; i < kCh; ++i) {
-          if (i < nvalid) {
-            const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
-            const float gr = __uint_as_float(r[i]);
-            const float t = fmaf(-eta, gr, th[i]);
-            AGN_ST(theta + p, t);
-            AGN_ST(acc + p, ac[i] + gr);
-            if (kSplit == 1) AGN_ST(tb + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        for (int q = 0, d = 0; q < ks; ++q) {
+          if (q == sk) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] += __uint_as_float(r[i]);
+          } else {
+            const float* pq = red_smem + (size_t)(o * (ks - 1) + d) * (32 * 128) + co * 128 + trow;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] += pq[i * 128];
+            ++d;
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(v[i]);
+      };
+      // fused output layer: W_L's rows for this tile's 128 features, the number
+      // of 32-sample chunks with samples, and the scratch
+      float* sW3 = reinterpret_cast<float*>(smem + Epi::kHeadOff);
+      float* sPart = sW3 + kHC * 128;
+      float* sG = sPart + 8 * 16 * kHC;
+      uint16_t* sMask = reinterpret_cast<uint16_t*>(sG + 32 * kHC);   // [owned chunk][thread]
+      const int nchk = (args.N + 31) / 32;
+      if (kEpi == kEpiFwdHead && have) {
+#pragma unroll
+        for (int k = 0; k < kW3Per; ++k) sW3[threadIdx.x + k * kThreads] = w3v_reg[k];
+        __syncthreads();
+      }
+      if (!have) {
+        // reported above
+      } else if (kEpi == kEpiFwd || kEpi == kEpiDX || kEpi == kEpiFwdHead) {
+        TAct* out = static_cast<TAct*>(args.out) + (int64_t)slot * args.out_bstride;
+#pragma unroll 1
+        for (int o = 0; o < n_own; ++o) {
+          const int c0 = 32 * (own_rank + o * kstride) + co;
+          if (o > 0) load_mask(c0);
+          uint32_t r[16];
+          vals(o, c0, r);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) tT[i * 32 + lane] = __uint_as_float(r[i]);
+          __syncwarp();
+          if (kEpi == kEpiFwdHead && (c0 - co) / 32 < nchk) {
+            // Pass 1 of the fused output layer, before this chunk's stores (so
+            // that the release below orders only the partials): this CTA's
+            // share of the chunk's logits, sum over its 128 features of
+            // H_{L-1}[j][f] W_L[c][f].  A lane sums its four features; the eight
+            // lanes of a column fold by a fixed shuffle tree; the four row
+            // quadrants of a column half are added in order below.  The ReLU
+            // mask of the lane's 4 x 4 values goes to shared memory for pass 2.
+            // This code runs once per chunk and launch, from a cold instruction
+            // cache: it loops over the lane's four columns (u) rather than
+            // unrolling them, which keeps it a quarter of the size.
+            const int C = args.head_C;
+            uint32_t mbits = 0;
+            // W_L rows past C are zero in shared memory: all kHC classes are
+            // summed unguarded, as independent chains
+            const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
+#pragma unroll 1
+            for (int u = 0; u < 4; ++u) {
+              const int j = n_tile * BN + c0 + jl + 4 * u;
+              float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+              if (row4_ok && j < args.N) {
+                a = *reinterpret_cast<const float4*>(tT + (jl + 4 * u) * 32 + r4);
+                a.x = fmaxf(a.x + bias4.x, 0.f);
+                a.y = fmaxf(a.y + bias4.y, 0.f);
+                a.z = fmaxf(a.z + bias4.z, 0.f);
+                a.w = fmaxf(a.w + bias4.w, 0.f);
+              }
+              const float hq[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e)   // the mask of the value as stored
+                mbits |= (static_cast<float>(static_cast<TAct>(hq[e])) > 0.f ? 1u : 0u)
+                         << (4 * u + e);
+              float zp[kHC];
+#pragma unroll
+              for (int c = 0; c < kHC; ++c) {
+                const float4 w = w3v[c * 32];
+                float t = hq[0] * w.x;
+                t = fmaf(hq[1], w.y, t);
+                t = fmaf(hq[2], w.z, t);
+                zp[c] = fmaf(hq[3], w.w, t);
+              }
+              // fold the eight lanes of the column (lane bits 0-2) by a fixed
+              // reduce-scatter: each round a lane keeps half of its classes and
+              // adds its partner's share of them; afterwards the lane holds the
+              // column's sums of classes kb and kb + 1, kb = 8 b2 + 4 b1 + 2 b0
+              static_assert(kHC == 16, "the reduce-scatter folds 16 classes");
+              const int b2 = (lane >> 2) & 1, b1 = (lane >> 1) & 1, b0 = lane & 1;
+              float k8[8], k4[4], k2[2];
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const float keep = b2 ? zp[k + 8] : zp[k], send = b2 ? zp[k] : zp[k + 8];
+                k8[k] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+              }
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const float keep = b1 ? k8[k + 4] : k8[k], send = b1 ? k8[k] : k8[k + 4];
+                k4[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+              }
+#pragma unroll
+              for (int k = 0; k < 2; ++k) {
+                const float keep = b0 ? k4[k + 2] : k4[k], send = b0 ? k4[k] : k4[k + 2];
+                k2[k] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+              }
+              *reinterpret_cast<float2*>(sPart + (warp * 16 + jl + 4 * u) * kHC + 8 * b2 + 4 * b1 +
+                                         2 * b0) = make_float2(k2[0], k2[1]);
+            }
+            sMask[o * kThreads + threadIdx.x] = (uint16_t)mbits;
+            __syncthreads();
+            const int chunk = (c0 - co) / 32;
+            float* gp = args.head_part +
+                        (((int64_t)slot * nchk + chunk) * gridDim.x + m_tile) * (32 * kHC);
+            for (int i = threadIdx.x; i < 32 * kHC; i += kThreads) {
+              const int cc = i / kHC, c = i % kHC, hf = cc >> 4, jcl = cc & 15;
+              float sum = 0.f;
+              if (c < C)
+                for (int gq = 0; gq < 4; ++gq) sum += sPart[((gq + 4 * hf) * 16 + jcl) * kHC + c];
+              AGN_STCG(gp + i, sum);
+            }
+            __syncthreads();
+            // count in: the CTA's partials, ordered before by the barrier, are
+            // released by one acquire-release arrival
+            if (threadIdx.x == 0) {
+              int* hc = args.head_counter + slot * nchk + chunk;
+              if (AGN_BOUNDS_OK(hc, 4)) tc::atomic_add_acq_rel_gpu(hc, 1);
+              else AGN_BOUNDS_FAIL(hc);
+            }
+          }
+          if (row4_ok) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int jc = jl + 4 * u;
+              const int j = n_tile * BN + c0 + jc;
+              if (j < args.N) {
+                const float4 a = *reinterpret_cast<const float4*>(tT + jc * 32 + r4);
+                float v[4] = {a.x, a.y, a.z, a.w};
+                if (kFwd) {
+                  v[0] += bias4.x; v[1] += bias4.y; v[2] += bias4.z; v[3] += bias4.w;
+                  if (args.relu) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) v[e] = fmaxf(v[e], 0.f);
+                  }
+                } else {
+                  const float hv[4] = {hm[u].x, hm[u].y, hm[u].z, hm[u].w};
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) v[e] = hv[e] > 0.f ? v[e] : 0.f;
+                }
+                const int64_t o4 = (int64_t)j * args.ldo + row4;
+                store4(out + o4, v);
+                if (kSplit == 3 && args.out_pieces) {
+                  uint2 q0, q1, q2;
+                  split3_x4(v, q0, q1, q2);
+                  bf16* pp = args.out_pieces + (int64_t)slot * args.out_bstride + o4;
+                  AGN_ST(reinterpret_cast<uint2*>(pp), q0);
+                  AGN_ST(reinterpret_cast<uint2*>(pp + args.out_plane), q1);
+                  AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.out_plane), q2);
+                }
+              }
+            }
+          }
+          __syncwarp();
+        }
+        if (kEpi == kEpiFwdHead) {
+          // Pass 2: once every feature tile's partials of a chunk are in (all
+          // CTAs of this launch are resident), the chunk's logits are summed in
+          // tile order plus b_L; every half-warp takes softmax cross-entropy and
+          // dZ_L = (softmax - onehot(y)) / m of a sample (the first feature tile
+          // writes dZ_L and the chunk's loss); every CTA then writes dZ_{L-1} =
+          // (dZ_L W_L) [H_{L-1} > 0] for its own features (W_L before its
+          // update).
+          __shared__ int s_hok;
+          const int C = args.head_C;
+          const float* bl = theta + args.head_boff;
+          TAct* dh = static_cast<TAct*>(args.dh) + (int64_t)slot * args.out_bstride;
+          const int mtn = (int)gridDim.x;
+#pragma unroll 1
+          for (int o = 0; o < n_own; ++o) {
+            const int chunk = own_rank + o * kstride;
+            if (chunk >= nchk) continue;   // CTA-uniform
+            int* ctr = args.head_counter + slot * nchk + chunk;
+            if (threadIdx.x == 0)
+              s_hok = AGN_BOUNDS_OK(ctr, 4) &&
+                      tc::wait_count_low(ctr, mtn, abort_flag, args.wait_ns ? args.wait_ns : kWaitNs);
+            __syncthreads();
+            if (!s_hok) {
+              if (threadIdx.x == 0) atomicExch(args.err, 1);
+              break;
+            }
+            // the feature tiles' partials in tile order: each thread sums two of
+            // the chunk's 32 x kHC logits, up to 2 x 16 loads in flight; thread
+            // t holds class t % kHC of samples t / kHC and 16 + t / kHC, so the
+            // 16 lanes of a half-warp hold one sample's logits
+            static_assert(32 * kHC == 2 * kThreads, "two logits per thread");
+            static_assert(kHC == 16, "one sample per half-warp");
+            const float* gp0 = args.head_part + ((int64_t)slot * nchk + chunk) * mtn * (32 * kHC);
+            float zz[2] = {0.f, 0.f};
+            for (int m0 = 0; m0 < mtn; m0 += 16) {
+              float p0[16], p1[16];
+#pragma unroll
+              for (int q = 0; q < 16; ++q) {
+                const float* pq = gp0 + (int64_t)(m0 + q) * (32 * kHC) + threadIdx.x;
+                p0[q] = m0 + q < mtn ? AGN_LDCG(pq) : 0.f;
+                p1[q] = m0 + q < mtn ? AGN_LDCG(pq + kThreads) : 0.f;
+              }
+#pragma unroll
+              for (int q = 0; q < 16; ++q) {
+                zz[0] += p0[q];
+                zz[1] += p1[q];
+              }
+            }
+            // softmax cross-entropy and dZ_L = (softmax - onehot(y)) / m of the
+            // thread's two (sample, class) entries: max and sum over the
+            // sample's classes by a fixed shuffle tree within the half-warp;
+            // the first feature tile writes dZ_L
+            float* sCE = sPart;   // [32] per-sample cross-entropy (pass 1 is done with sPart)
+            {
+              const int cl = threadIdx.x % kHC;
+              const bool cv = cl < C;
+              const float inv_m = 1.0f / (float)args.N;
+              const float bc = cv ? AGN_LD(bl + cl) : 0.f;
+#pragma unroll 1
+              for (int hh = 0; hh < 2; ++hh) {
+                const int sl = 16 * hh + (threadIdx.x >> 4);   // sample within the chunk
+                const int j = n_tile * BN + 32 * chunk + sl;
+                const bool valid = j < args.N;
+                const float z = cv ? (hh ? zz[1] : zz[0]) + bc : -INFINITY;
+                float mx = z;
+#pragma unroll
+                for (int off = 8; off > 0; off >>= 1)
+                  mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+                const float ex = cv ? expf(z - mx) : 0.f;
+                float se = ex;
+#pragma unroll
+                for (int off = 8; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
+                const int y = !valid ? -1
+                              : args.x_shard > 0
+                                  ? AGN_LD(args.yb + (int64_t)worker * (args.x_shard + args.N) +
+                                           batch_row0(args.slot_t0, slot, args.step, args.N,
+                                                      args.x_shard) + j)
+                                  : AGN_LD(args.yb + (int64_t)slot * args.N + j);
+                const float zy = __shfl_sync(0xffffffffu, z, (lane & 16) + (y > 0 ? y : 0));
+                float pr = ex * (1.0f / se);
+                if (cl == y) pr -= 1.0f;
+                const float gz = valid ? pr * inv_m : 0.f;
+                sG[sl * kHC + cl] = gz;
+                if (m_tile == 0 && valid && cv) {
+                  const TAct gv = static_cast<TAct>(gz);
+                  const int64_t zi = ((int64_t)slot * args.N + j) * args.ldz + cl;
+                  AGN_ST(static_cast<TAct*>(args.dzl) + zi, gv);
+                  if (args.dzl_pieces) {
+                    bf16 q0, q1, q2;
+                    split3(static_cast<float>(gv), q0, q1, q2);
+                    AGN_ST(args.dzl_pieces + zi, q0);
+                    AGN_ST(args.dzl_pieces + args.dzl_plane + zi, q1);
+                    AGN_ST(args.dzl_pieces + 2 * args.dzl_plane + zi, q2);
+                  }
+                }
+                if (cl == 0) sCE[sl] = valid ? (logf(se) + mx) - zy : 0.f;
+              }
+            }
+            __syncthreads();
+            float ce = 0.f;
+            if (warp == 0) {   // the chunk's cross-entropy sum, fixed tree over its samples
+              ce = sCE[lane];
+#pragma unroll
+              for (int off = 16; off > 0; off >>= 1) ce += __shfl_xor_sync(0xffffffffu, ce, off);
+            }
+            if (row4_ok) {
+              const uint32_t mbits = sMask[o * kThreads + threadIdx.x];
+              const float4* w3v = reinterpret_cast<const float4*>(sW3 + 32 * g + r4);
+              // dZ_{L-1} of the lane's 4 features x 4 columns: 16 independent
+              // chains over the classes (dZ_L is zero past C)
+              float d[4][4];
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) d[u][e] = 0.f;
+#pragma unroll 2
+              for (int c = 0; c < kHC; ++c) {
+                const float4 w = w3v[c * 32];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                  const float gzc = sG[(co + jl + 4 * u) * kHC + c];
+                  d[u][0] = fmaf(gzc, w.x, d[u][0]);
+                  d[u][1] = fmaf(gzc, w.y, d[u][1]);
+                  d[u][2] = fmaf(gzc, w.z, d[u][2]);
+                  d[u][3] = fmaf(gzc, w.w, d[u][3]);
+                }
+              }
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const int j = n_tile * BN + 32 * chunk + co + jl + 4 * u;
+                if (j < args.N) {
+                  float dv[4];
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) dv[e] = (mbits >> (4 * u + e)) & 1u ? d[u][e] : 0.f;
+                  const int64_t o4 = (int64_t)j * args.ldo + row4;
+                  store4(dh + o4, dv);
+                  if (kSplit == 3 && args.dh_pieces) {
+                    uint2 q0, q1, q2;
+                    split3_x4(dv, q0, q1, q2);
+                    bf16* pp = args.dh_pieces + (int64_t)slot * args.out_bstride + o4;
+                    AGN_ST(reinterpret_cast<uint2*>(pp), q0);
+                    AGN_ST(reinterpret_cast<uint2*>(pp + args.dh_plane), q1);
+                    AGN_ST(reinterpret_cast<uint2*>(pp + 2 * args.dh_plane), q2);
+                  }
+                }
+              }
+            }
+            if (threadIdx.x == 0) {
+              // the chunk's loss contribution (sum of its samples' cross-entropy
+              // over m) in the chunk's slot; the run's loss kernel adds the slots
+              // in order
+              if (m_tile == 0) {
+                const float part = ce / (float)args.N;
+                AGN_ST(args.loss_parts +
+                           ((int64_t)AGN_LD(args.slot_commit + slot) * args.lam + args.step) * nchk +
+                           chunk,
+                       part);
+                if (!isfinite(part)) atomicExch(args.nonfinite, 1);
+              }
+            }
+          }
+        }
+      } else {   // kEpiDW
+        float* acc = args.acc + (int64_t)worker * args.ld_param;
+        bf16* tb = args.theta_b + (int64_t)worker * args.ld_param;
+        const float eta = args.eta;
+        // Chunks of 16 columns; the loads of chunk c + 1 are issued before the
+        // stores of chunk c, so every thread keeps 32 loads in flight while it
+        // writes (the epilogue is bound by DRAM latency x bandwidth).
+        constexpr int kCh = 16;
+        constexpr int kChunks = (BN / 2) / kCh;
+        const float* __restrict__ th_in = theta;
+        const float* __restrict__ ac_in = acc;
+        const int cbase = n_tile * BN + half * (BN / 2);     // first column of this half
+        const int64_t pbase = args.woff + (int64_t)cbase * args.M + row;
+        float thn[kCh], acn[kCh];
+        auto load_chunk = [&](int ch) {
+          const int nvalid = row_ok ? min(kCh, args.N - (cbase + ch * kCh)) : 0;
+#pragma unroll
+          for (int i = 0; i < kCh; ++i) {
+            if (i < nvalid) {
+              const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
+              thn[i] = AGN_LDCS(th_in + p);
+              acn[i] = AGN_LDCS(ac_in + p);
+            }
+          }
+        };
+        load_chunk(0);
+#pragma unroll
+        for (int ch = 0; ch < kChunks; ++ch) {
+          float th[kCh], ac[kCh];
+#pragma unroll
+          for (int i = 0; i < kCh; ++i) {
+            th[i] = thn[i];
+            ac[i] = acn[i];
+          }
+          uint32_t r[kCh];
+          const uint32_t col = (uint32_t)(half * (BN / 2) + ch * kCh);
+          tc::tmem_ld_32x32b_x16(tmem + lane_base + col, r);
+          uint32_t r2[kCh];
+          if (kSplit == 3) tc::tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)BN + col, r2);
+          if (ch + 1 < kChunks) load_chunk(ch + 1);
+          tc::tmem_ld_wait();
+          if (kSplit == 3) {
+#pragma unroll
+            for (int i = 0; i < kCh; ++i)
+              r[i] = __float_as_uint(__fadd_rn(__uint_as_float(r[i]), __uint_as_float(r2[i])));
+          }
+          const int nvalid = row_ok ? min(kCh, args.N - (cbase + ch * kCh)) : 0;
+#pragma unroll
+          for (int i = 0; i < kCh; ++i) {
+            if (i < nvalid) {
+              const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
+              const float gr = __uint_as_float(r[i]);
+              const float t = fmaf(-eta, gr, th[i]);
+              AGN_ST(theta + p, t);
+              AGN_ST(acc + p, ac[i] + gr);
+              if (kSplit == 1) AGN_ST(tb + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces
+            }
           }
         }
       }
@@ -1119,26 +1138,27 @@ __global__ void split_pieces_kernel(const float* __restrict__ x, bf16* __restric
   }
 }
 
-template <int BN, int kSplit, int kStages, int kBK, bool kATmem>
+template <int BN, int kSplit, int kStages, int kBK, bool kATmem, int kMT = 1>
 size_t smem_bytes() {
   // Shared memory requested per CTA also caps the CTAs per SM so that their
   // TMEM columns never exceed the 512 an SM has.
-  using Cfg = TileCfg<BN, kSplit, kBK, kATmem>;
+  using Cfg = TileCfg<BN, kSplit, kBK, kATmem, kMT>;
   const size_t ring = (size_t)kStages * Cfg::kStageBytes + 1024 + 256 +
-                      (EpiT<BN, kSplit, kStages, kBK, kATmem>::kSeparate ? kEpiTBytes : 0);
+                      (EpiT<BN, kSplit, kStages, kBK, kATmem, kMT>::kSeparate ? kEpiTBytes : 0);
   const size_t floor_for_tmem = (size_t)(233472 / (512 / Cfg::kTmemCols + 1)) + 1024;
   return std::max(ring, floor_for_tmem);
 }
 
-template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit>
+template <int BN, bool kAMN, bool kBMN, int kEpi, int kStages, int kSplit, int kMT = 1>
 Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, int slots,
                  cudaStream_t st, bool* launched = nullptr) {
   constexpr int kBK = stage_k(kSplit, kEpi);
   constexpr bool kATmem = a_in_tmem(kSplit, kEpi, BN);
-  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem>;
-  static_assert(kStages * TileCfg<BN, kSplit, kBK, kATmem>::kStageBytes + 1280 <= 232448, "smem");
-  auto kern = tc_gemm_kernel<BN, kAMN, kBMN, kEpi, kStages, kSplit>;
-  const size_t smem = smem_bytes<BN, kSplit, kStages, kBK, kATmem>();
+  using Epi = EpiT<BN, kSplit, kStages, kBK, kATmem, kMT>;
+  static_assert(kStages * TileCfg<BN, kSplit, kBK, kATmem, kMT>::kStageBytes + 1280 <= 232448,
+                "smem");
+  auto kern = tc_gemm_kernel<BN, kAMN, kBMN, kEpi, kStages, kSplit, kMT>;
+  const size_t smem = smem_bytes<BN, kSplit, kStages, kBK, kATmem, kMT>();
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -1146,7 +1166,7 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
   });
   AGN_TRY_CUDA(attr_err);
   // split K: every rank with a non-empty range of k steps
-  int ks = kEpi == kEpiDW ? 1 : std::max(1, args.ksplit);
+  int ks = kEpi == kEpiDW || kMT > 1 ? 1 : std::max(1, args.ksplit);
   if (ks > 1) {
     // a rank that finishes chunks holds the other ranks' partial sums of
     // them (16 KB per chunk and rank) in its stage ring
@@ -1172,7 +1192,7 @@ Status launch_tc(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
   }
   if (ks > 1 && (!args.part || !args.counter))
     return Status::Err(AGN_E_INVALID, "split-K GEMM without workspace");
-  dim3 grid((unsigned)ceil_div(args.M, 128), (unsigned)ceil_div(args.N, BN),
+  dim3 grid((unsigned)ceil_div(args.M, 128 * kMT), (unsigned)ceil_div(args.N, BN),
             (unsigned)(slots * ks));
   TcArgs a2 = args;
   a2.ksplit = ks;
@@ -1267,12 +1287,36 @@ Status make_tmap_f32_3d(CUtensorMap* map, const void* base, uint64_t inner, uint
                 swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
+// Two 128-row tiles per CTA (kMT = 2) for the bf16 forward and dX when the
+// one-tile launch would need more than one round of CTAs on the SMs (full
+// waves): each B stage then feeds twice the MMAs, and the CTAs of a full
+// wave halve.  Not with split K, nor with column tiles under 128 (there the
+// weights, read once anyway, dominate the stages' bytes).
+bool use_row_pairs(const TcArgs& args, int slots, bool split, int bn) {
+  if (split || bn < 128 || args.ksplit > 1 || args.one_row_tile) return false;
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return false;
+    }
+    sms = n;
+  }
+  return ceil_div(args.M, 128) * ceil_div(args.N, bn) * (int64_t)slots > sms;
+}
+
 Status tc_forward(const CUtensorMap& w_k, const CUtensorMap& h_k, const TcArgs& args, int slots,
                   cudaStream_t st, bool split, int bn) {
   if (split) {
     if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 6, 3>(w_k, h_k, args, slots, st);
     if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 4, 3>(w_k, h_k, args, slots, st);
     return launch_tc<256, false, false, kEpiFwd, 3, 3>(w_k, h_k, args, slots, st);
+  }
+  if (use_row_pairs(args, slots, split, bn)) {
+    if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 4, 1, 2>(w_k, h_k, args, slots, st);
+    return launch_tc<256, false, false, kEpiFwd, 3, 1, 2>(w_k, h_k, args, slots, st);
   }
   if (bn == 64) return launch_tc<64, false, false, kEpiFwd, 6, 1>(w_k, h_k, args, slots, st);
   if (bn == 128) return launch_tc<128, false, false, kEpiFwd, 5, 1>(w_k, h_k, args, slots, st);
@@ -1307,6 +1351,10 @@ Status tc_backward_dx(const CUtensorMap& w_mn, const CUtensorMap& dz_k, const Tc
     if (bn == 64) return launch_tc<64, true, false, kEpiDX, 6, 3>(w_mn, dz_k, args, slots, st);
     if (bn == 128) return launch_tc<128, true, false, kEpiDX, 4, 3>(w_mn, dz_k, args, slots, st);
     return launch_tc<256, true, false, kEpiDX, 3, 3>(w_mn, dz_k, args, slots, st);
+  }
+  if (use_row_pairs(args, slots, split, bn)) {
+    if (bn == 128) return launch_tc<128, true, false, kEpiDX, 4, 1, 2>(w_mn, dz_k, args, slots, st);
+    return launch_tc<256, true, false, kEpiDX, 3, 1, 2>(w_mn, dz_k, args, slots, st);
   }
   if (bn == 64) return launch_tc<64, true, false, kEpiDX, 6, 1>(w_mn, dz_k, args, slots, st);
   if (bn == 128) return launch_tc<128, true, false, kEpiDX, 5, 1>(w_mn, dz_k, args, slots, st);

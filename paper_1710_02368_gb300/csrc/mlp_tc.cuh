@@ -84,6 +84,9 @@ struct TcArgs {
   const long long* slot_t0;
   int64_t x_shard;
   int x_b_direct;
+  // 1: one 128-row tile per CTA even where two would share the B stages
+  // (the bf16 forward and dX of full waves)
+  int one_row_tile;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N
