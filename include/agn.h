@@ -109,7 +109,10 @@ typedef struct agn_options {
      each local step's minibatch into a buffer of its own (one launch per
      step) instead of reading it from the padded shards in place.  Bit 7
      runs the bf16 forward and dX GEMMs of full waves with one 128-row tile
-     per CTA instead of two that share each B stage. */
+     per CTA instead of two that share each B stage.  Bit 8 makes the
+     persistent dW kernel read each accumulator chunk into shared memory and
+     store a_k + g even for waves whose accumulators fit well within the L2,
+     where it otherwise adds g to a_k in the L2 (red.add). */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);

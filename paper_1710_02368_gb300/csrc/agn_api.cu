@@ -432,6 +432,7 @@ agn::TcArgs tc_args(agn_handle* h, const int* sw, const long long* st0, int step
   t.wait_ns = h->dbg_wait_ns;
   t.withhold_rank = h->dbg_withhold;
   t.one_row_tile = (h->tc_mask & 128) ? 1 : 0;
+  t.acc_ring = (h->tc_mask & 256) ? 1 : 0;
   return t;
 }
 
@@ -1150,7 +1151,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 255) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 255]");
+  if (o.tc_mask < 0 || o.tc_mask > 511) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 511]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)

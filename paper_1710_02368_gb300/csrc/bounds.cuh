@@ -1,17 +1,17 @@
 // The bounds-checked build (compiled with -DAGN_BOUNDS_CHECK; build.py's
 // `check` variant, libagn_gb300_check.so).  compute-sanitizer cannot be used
 // on the GPUs this library is tested on, so this build stands in for its
-// memcheck on the hot path: every generic global load and store of the
-// kernels that AGN_ST / AGN_LD and their cache-hint forms wrap is first checked
-// against the table of device buffers the library knows (the handles'
-// allocations and the caller's buffers of a standalone commit call).  An
-// access outside every buffer is not performed: the kernel records its
-// address and counts it, a load returns zero, and the host turns the count
-// into AGN_E_BOUNDS after the call.  Tensor-map (TMA) copies are checked on
-// the host when the map is encoded (the whole span of the map must lie in
-// one buffer; the copy engine itself stays within the map), and bulk copies
-// on the device before they are issued.  In the normal build the macros are
-// the plain accesses.
+// memcheck on the hot path: every generic global load, store and L2 add of
+// the kernels that AGN_ST / AGN_LD, their cache-hint forms and AGN_RED4 /
+// AGN_RED wrap is first checked against the table of device buffers the
+// library knows (the handles' allocations and the caller's buffers of a
+// standalone commit call).  An access outside every buffer is not performed:
+// the kernel records its address and counts it, a load returns zero, and the
+// host turns the count into AGN_E_BOUNDS after the call.  Tensor-map (TMA)
+// copies are checked on the host when the map is encoded (the whole span of
+// the map must lie in one buffer; the copy engine itself stays within the
+// map), and bulk copies on the device before they are issued.  In the normal
+// build the macros are the plain accesses.
 #pragma once
 
 #include <cstdint>
@@ -86,6 +86,17 @@ __device__ __forceinline__ T ldcs_checked(const T* p) {
 #define AGN_STCS(p, v) ::agn::stcs_checked((p), (v))
 #define AGN_BOUNDS_OK(p, bytes) ::agn::bounds_ok((p), (bytes))
 #define AGN_BOUNDS_FAIL(p) ::agn::bounds_fail(p)
+// L2 adds (tc_ptx.cuh): four floats or one
+#define AGN_RED4(p, v)                                                        \
+  do {                                                                        \
+    if (::agn::bounds_ok((p), 16)) ::agn::tc::red_add_f32x4((p), (v));        \
+    else ::agn::bounds_fail(p);                                               \
+  } while (0)
+#define AGN_RED(p, v)                                                         \
+  do {                                                                        \
+    if (::agn::bounds_ok((p), 4)) ::agn::tc::red_add_f32((p), (v));           \
+    else ::agn::bounds_fail(p);                                               \
+  } while (0)
 
 // Host side of one translation unit's table: bounds_set_<unit> uploads the
 // table and clears the unit's record, bounds_get_<unit> reads the record
@@ -123,6 +134,8 @@ __device__ __forceinline__ T ldcs_checked(const T* p) {
 #define AGN_STCS(p, v) __stcs((p), (v))
 #define AGN_BOUNDS_OK(p, bytes) true
 #define AGN_BOUNDS_FAIL(p) ((void)0)
+#define AGN_RED4(p, v) ::agn::tc::red_add_f32x4((p), (v))
+#define AGN_RED(p, v) ::agn::tc::red_add_f32((p), (v))
 #define AGN_BOUNDS_UNIT(unit)
 
 #endif

@@ -87,6 +87,9 @@ struct TcArgs {
   // 1: one 128-row tile per CTA even where two would share the B stages
   // (the bf16 forward and dX of full waves)
   int one_row_tile;
+  // dW: 1 reads a_k's chunks through the parameter ring and stores a_k + g;
+  // 0 adds g to a_k in the L2 (red.add) and keeps the ring for theta_k
+  int acc_ring;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N

@@ -66,17 +66,21 @@ constexpr int kThrottleTiles = 8;              // tiles per CTA from which opera
 // kBK samples per stage: one TMA box is 64 MN-elements x kBK samples of bf16
 // (kBK rows of 128 bytes, 128-byte swizzle); A = two boxes (128 inputs),
 // B = BN / 64 boxes.
-// kMode: kDwUpdAcc = the local step and accumulation, theta_k and a_k per
-// chunk (3 slots in flight); kDwUpd = the local step without accumulator
-// (elided: commits from a pull snapshot), theta_k alone (6 slots); kDwGrad =
-// the raw gradient only, stored for a separate optimizer kernel (no chunks).
-enum { kDwUpdAcc = 0, kDwUpd = 1, kDwGrad = 2 };
+// kMode: kDwUpdRed = the local step and accumulation, theta_k per chunk
+// through the ring (6 slots in flight) and a_k += g as L2 adds (red.add,
+// nothing read back into the SM); kDwUpdAcc = the same with a_k's chunk read
+// through the ring beside theta_k's and stored back (3 slots); kDwUpd = the
+// local step without accumulator (elided: commits from a pull snapshot),
+// theta_k alone (6 slots); kDwGrad = the raw gradient only, stored for a
+// separate optimizer kernel (no chunks).
+enum { kDwUpdAcc = 0, kDwUpd = 1, kDwGrad = 2, kDwUpdRed = 3 };
 template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 struct DwCfg {
-  static constexpr bool kAcc = kMode == kDwUpdAcc;
-  static constexpr int kArrays = kMode == kDwUpdAcc ? 2 : 1;
+  static constexpr bool kAcc = kMode == kDwUpdAcc || kMode == kDwUpdRed;   // a_k += g
+  static constexpr bool kAccRing = kMode == kDwUpdAcc;                     // a_k via the ring
+  static constexpr int kArrays = kAccRing ? 2 : 1;
   static constexpr int kSlotBytes = kArrays * (kChunkBytes + kBiasHalf);
-  static constexpr int kRing = kAcc ? 3 : 6;
+  static constexpr int kRing = kAccRing ? 3 : 6;
   static constexpr int kBK = kBKs;
   static constexpr int kBox = kBK * 128;
   static constexpr int kABytes = 2 * kBox;
@@ -151,7 +155,7 @@ template <int BN, int kSplit, int kStages, int kBKs, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   using Cfg = DwCfg<BN, kSplit, kStages, kBKs, kMode>;
-  constexpr bool kAcc = Cfg::kAcc, kGrad = kMode == kDwGrad;
+  constexpr bool kAcc = Cfg::kAcc, kAccRing = Cfg::kAccRing, kGrad = kMode == kDwGrad;
   constexpr int kRing = Cfg::kRing, kSlotBytes = Cfg::kSlotBytes;
   constexpr int kBK = Cfg::kBK, kABytes = Cfg::kABytes, kBox = Cfg::kBox;
   extern __shared__ uint8_t smem_raw[];
@@ -302,7 +306,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
         constexpr int kA = Cfg::kArrays;
         tc::mbar_arrive_expect_tx(&cfull[r], kA * (kChunkBytes + (bias_tile ? kBiasHalf : 0)));
         tc::tma_load_3d(dst, &B.th[ti.layer], &cfull[r], ti.m_tile * 128, f0, worker);
-        if (kAcc)
+        if (kAccRing)
           tc::tma_load_3d(dst + kChunkBytes, &B.ac[ti.layer], &cfull[r], ti.m_tile * 128, f0,
                           worker);
         if (bias_tile) {   // b_l[f0 .. f0 + 31] and its accumulator (within the replica)
@@ -313,7 +317,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
             AGN_BOUNDS_FAIL(args.theta + pb);
             tc::mbar_complete_tx(&cfull[r], kBiasHalf);
           }
-          if (kAcc) {
+          if (kAccRing) {
             if (AGN_BOUNDS_OK(args.acc + pb, kBiasHalf)) {
               tc::bulk_load(dst + kA * kChunkBytes + kBiasHalf, args.acc + pb, kBiasHalf,
                             &cfull[r]);
@@ -511,11 +515,13 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
               tn[3] = fmaf(-eta, gv.w, tv.w);
               const int64_t p = L.woff + (int64_t)(fbase + i) * M + k0 + k4;
               AGN_ST(reinterpret_cast<float4*>(theta + p), make_float4(tn[0], tn[1], tn[2], tn[3]));
-              if (kAcc) {
+              if (kAccRing) {
                 const float4 av = *reinterpret_cast<const float4*>(
                     reinterpret_cast<const float*>(slot + kChunkBytes) + so);
                 AGN_ST(reinterpret_cast<float4*>(acc + p),
                        make_float4(av.x + gv.x, av.y + gv.y, av.z + gv.z, av.w + gv.w));
+              } else if (kAcc) {   // a_k += g in the L2 (one add per element and launch)
+                AGN_RED4(reinterpret_cast<float*>(acc + p), gv);
               }
               // the bf16 copy (bf16 mode); the fp32 mode's GEMMs split the
               // fp32 weights themselves
@@ -530,7 +536,8 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           const int64_t pb = L.boff + fbase + lane;
           const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
           AGN_ST(theta + pb, tn);
-          if (kAcc) AGN_ST(acc + pb, sTb[kCF + 16 * hf + lane] + gb);
+          if (kAccRing) AGN_ST(acc + pb, sTb[kCF + 16 * hf + lane] + gb);
+          else if (kAcc) AGN_RED(acc + pb, gb);
           if (kSplit == 1) AGN_ST(tb + pb, __float2bfloat16_rn(tn));
         }
         __syncwarp();
@@ -588,7 +595,7 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
   for (int l0 = 0; l0 < n_layers; l0 += kMaxDwLayers) {
     DwBatch batch;
     std::memset(&batch, 0, sizeof(batch));
-    int64_t tiles = 0;
+    int64_t tiles = 0, acc_bytes = 0;
     batch.n_layers = std::min(kMaxDwLayers, n_layers - l0);
     for (int i = 0; i < batch.n_layers; ++i) {
       const DwLayerMaps& d = layers[l0 + i];
@@ -605,6 +612,7 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
       L.boff = d.boff;
       L.mt = d.M / 128 + 1;          // rows 0 .. M, row M the bias
       L.nt = (d.N + bn - 1) / bn;
+      acc_bytes += ((int64_t)d.M + 1) * d.N * 4 * slots;
       L.tile_begin = (int)tiles;
       tiles += (int64_t)L.mt * L.nt * slots;
       if (tiles > INT32_MAX) return Status::Err(AGN_E_UNSUPPORTED, "dW tile count overflows");
@@ -612,17 +620,30 @@ Status tc_backward_dw(const DwLayerMaps* layers, int n_layers, const TcArgs& arg
     batch.total_tiles = (int)tiles;
     // split mode: 32 samples per stage, so that two stages fit beside the
     // parameter ring (the next tile's operands land while this one multiplies)
-    // grad_out: gradient only; else acc null: accumulator elided
-    const int mode = args.grad_out ? kDwGrad : args.acc ? kDwUpdAcc : kDwUpd;
+    // grad_out: gradient only; else acc null: accumulator elided; else a_k
+    // through L2 adds while the launch's accumulators fit well within the L2
+    // (small waves, where the chunk ring's latency bounds the kernel and
+    // half the ring's bytes per chunk buy twice the chunks in flight), or
+    // through the ring (large waves, which stream theta_k and a_k from DRAM
+    // at the copy bandwidth: there the L2's adds slowed the stream by 4 %;
+    // and always with args.acc_ring)
+    constexpr int64_t kRedAccBytes = 64ll << 20;
+    const bool ring = args.acc_ring || acc_bytes > kRedAccBytes;
+    const int mode = args.grad_out ? kDwGrad
+                     : !args.acc   ? kDwUpd
+                     : ring        ? kDwUpdAcc
+                                   : kDwUpdRed;
     Status r = Status::Ok();
     if (split) {
-      r = mode == kDwGrad ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwGrad>(batch, args, num_sms, st)
-          : mode == kDwUpd ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpd>(batch, args, num_sms, st)
-                           : launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpdAcc>(batch, args, num_sms, st);
+      r = mode == kDwGrad     ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwGrad>(batch, args, num_sms, st)
+          : mode == kDwUpd    ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpd>(batch, args, num_sms, st)
+          : mode == kDwUpdAcc ? launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpdAcc>(batch, args, num_sms, st)
+                              : launch_dw<kTcDwBNSplit, 3, 2, 32, kDwUpdRed>(batch, args, num_sms, st);
     } else {
-      r = mode == kDwGrad ? launch_dw<kTcDwBN, 1, 2, 64, kDwGrad>(batch, args, num_sms, st)
-          : mode == kDwUpd ? launch_dw<kTcDwBN, 1, 2, 64, kDwUpd>(batch, args, num_sms, st)
-                           : launch_dw<kTcDwBN, 1, 2, 64, kDwUpdAcc>(batch, args, num_sms, st);
+      r = mode == kDwGrad     ? launch_dw<kTcDwBN, 1, 2, 64, kDwGrad>(batch, args, num_sms, st)
+          : mode == kDwUpd    ? launch_dw<kTcDwBN, 1, 2, 64, kDwUpd>(batch, args, num_sms, st)
+          : mode == kDwUpdAcc ? launch_dw<kTcDwBN, 1, 2, 64, kDwUpdAcc>(batch, args, num_sms, st)
+                              : launch_dw<kTcDwBN, 1, 2, 64, kDwUpdRed>(batch, args, num_sms, st);
     }
     if (!r.ok()) return r;
   }

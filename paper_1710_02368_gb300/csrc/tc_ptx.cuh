@@ -112,6 +112,17 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
+// Fire-and-forget floating-point adds done by the L2 (no value returned):
+// *p += v, four consecutive floats (16-byte aligned) or one.
+__device__ __forceinline__ void red_add_f32x4(float* p, float4 v) {
+  asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};"
+               ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void red_add_f32(float* p, float v) {
+  asm volatile("red.relaxed.gpu.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+
 // atomicAdd with acquire-release semantics at GPU scope; returns the old value.
 __device__ __forceinline__ int atomic_add_acq_rel_gpu(int* p, int v) {
   int old;

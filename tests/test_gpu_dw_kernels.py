@@ -78,3 +78,20 @@ def test_persistent_dw_matches_tiled_dw(agn, dims, m, n, prec):
     tol = 1e-2 if prec == "bf16" else 1e-4
     assert np.linalg.norm(d1 - d2) <= tol * np.linalg.norm(d2)
     assert np.max(np.abs(l1 - l2)) <= tol * np.max(np.abs(l2))
+
+
+@pytest.mark.parametrize("dims,m,n", CASES)
+@pytest.mark.parametrize("prec", PRECS)
+def test_accumulator_l2_adds_match_ring(agn, dims, m, n, prec):
+    """a_k += g as L2 adds (red.add, the default for waves whose accumulators
+    fit well within the L2: all cases but the 8-worker 1024-2048-10 one,
+    whose 65 MB take the ring either way) against a_k's chunks read
+    through the parameter ring and stored back (tc_mask bit 8): one add of
+    the same two floats per element and local step either way, so after
+    several commits of three local steps theta~ and the losses agree bit for
+    bit."""
+    _, c1, l1 = _run(agn, dims, m, n, _prec(agn, prec), 7, lam=3, C=2 * n)
+    _, c2, l2 = _run(agn, dims, m, n, _prec(agn, prec), 7 | 256, lam=3, C=2 * n)
+    assert np.isfinite(c1).all()
+    assert np.array_equal(c1, c2), float(np.max(np.abs(c1 - c2)))
+    assert np.array_equal(l1, l2)
