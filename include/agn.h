@@ -112,7 +112,8 @@ typedef struct agn_options {
      per CTA instead of two that share each B stage.  Bit 8 makes the
      persistent dW kernel read each accumulator chunk into shared memory and
      store a_k + g even for waves whose accumulators fit well within the L2,
-     where it otherwise adds g to a_k in the L2 (red.add). */
+     where it otherwise adds g to a_k in the L2 (red.add).  Bit 9 makes the
+     forward of layer 1 request no weight stage before its dependency wait. */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);

@@ -704,6 +704,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.nonfinite = h->flag;
           const auto& mp = maps_of(l);
           t.x_b_direct = l == 1;
+          t.no_a_prefetch = l == 1 && (h->tc_mask & 512) ? 1 : 0;
           t.ksplit = pick_ksplit(h, fo, fi, s);
           next_counters(h, &t);
           bool launched = false;
@@ -722,6 +723,7 @@ Status run_wave_steps(agn_handle* h, const Wave& wv, int64_t* launches) {
           t.out_pieces = h_pieces; t.out_plane = (int64_t)n * m * fo;
           const auto& mp = maps_of(l);
           t.x_b_direct = l == 1;
+          t.no_a_prefetch = l == 1 && (h->tc_mask & 512) ? 1 : 0;
           t.ksplit = pick_ksplit(h, fo, fi, s);
           next_counters(h, &t);
           AGN_TRY(agn::tc_forward(mp.w_k, mp.h_k, t, s, h->stream, h->split, agn::tc_bn(m)));
@@ -1151,7 +1153,7 @@ Status create(agn_handle* h, const int32_t* dims, int32_t n_dims, int32_t n_work
   if (o.tau_lo < 0 || o.tau_hi < o.tau_lo) return Status::Err(AGN_E_INVALID, "bad tau range");
   if (o.gemm != AGN_GEMM_AUTO && o.gemm != AGN_GEMM_SIMT && o.gemm != AGN_GEMM_TCGEN05)
     return Status::Err(AGN_E_INVALID, "unknown gemm backend");
-  if (o.tc_mask < 0 || o.tc_mask > 511) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 511]");
+  if (o.tc_mask < 0 || o.tc_mask > 1023) return Status::Err(AGN_E_INVALID, "tc_mask must be in [0, 1023]");
   if (o.commit_rule != AGN_COMMIT_AGN && o.commit_rule != AGN_COMMIT_DYNSGD)
     return Status::Err(AGN_E_INVALID, "unknown commit_rule");
   if (o.n_eval < 0 || o.n_eval > (int64_t)1 << 31)

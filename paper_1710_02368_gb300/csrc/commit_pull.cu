@@ -317,7 +317,7 @@ __global__ void __launch_bounds__(kThreads)
 pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
             bf16* __restrict__ rep_bf16, int64_t P, int64_t ld, const int* __restrict__ workers,
             int64_t plane, float* __restrict__ snapshot) {
-  pdl_begin();
+  pdl_wait_only();   // the next forward may read the replicas before its own wait
   const int k = AGN_LD(workers + blockIdx.y);
   float* dst = replicas + (int64_t)k * ld;
   float* snap = snapshot ? snapshot + (int64_t)k * ld : nullptr;
@@ -339,6 +339,7 @@ pull_kernel(const float* __restrict__ theta_c, float* __restrict__ replicas,
       }
     }
   }
+  pdl_fence_exit();
 }
 
 __global__ void reduce_losses_kernel(const float* __restrict__ parts, int lambda, int q_per,

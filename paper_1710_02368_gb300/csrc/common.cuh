@@ -26,6 +26,18 @@ __device__ __forceinline__ void pdl_begin() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
+// The tensor-core forward and dX request their first weight stages before
+// their dependency wait.  That is safe for weights written two or more
+// kernels back (the preceding kernel let them launch only after its own
+// wait).  The kernels that write replicas the very next kernel may read so
+// (the dW local step, pulls, the Adam step) therefore wait without letting
+// the next kernel launch early (pdl_wait_only): it launches when all their
+// CTAs have exited, and every thread fences its writes before it exits
+// (pdl_fence_exit), so they are visible to those early reads.
+__device__ __forceinline__ void pdl_wait_only() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_fence_exit() { __threadfence(); }
 
 // Handles that time each kernel with CUDA events (agn_profile) turn the
 // overlap off while they do, so that an event pair brackets one kernel only.
@@ -97,6 +109,14 @@ inline Status bounds_collect(cudaStream_t) { return Status::Ok(); }
 
 constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
+
+// Algorithm 1's local step on one parameter, in its two steps: the update
+// g = -eta grad rounded to fp32, then theta + g rounded to fp32 (no fused
+// multiply-add; the L2-add form of the dW kernel performs the same two
+// roundings, so every path agrees bit for bit).
+__device__ __forceinline__ float local_step(float theta, float eta, float grad) {
+  return __fadd_rn(theta, __fmul_rn(-eta, grad));
+}
 
 // Padded shards (the tensor-core path's layer-1 operand and labels): worker
 // w's shard of S dataset rows is stored as S + m rows, row r holding dataset

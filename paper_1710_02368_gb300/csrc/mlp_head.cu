@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(32 * kDwGroups) head_dw_kernel(const HeadDwArg
   float* acc = a.acc ? a.acc + (int64_t)w * a.ld_param : nullptr;   // null: elided
   bf16* tb = a.theta_b ? a.theta_b + (int64_t)w * a.ld_param : nullptr;
   auto update = [&](int64_t p, float gr, float th, float ac) {
-    const float t = fmaf(-a.eta, gr, th);
+    const float t = local_step(th, a.eta, gr);
     AGN_ST(theta + p, t);
     if (acc) AGN_ST(acc + p, ac + gr);
     if (tb) {

@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
         if (n >= g.N) continue;
         const int64_t p = g.woff + m * g.N + n;
         const float gr = acc[i][j];
-        const float t = fmaf(-g.eta, gr, th[i][j]);
+        const float t = local_step(th[i][j], g.eta, gr);
         AGN_ST(theta + p, t);
         if (has_a) AGN_ST(a + p, av[i][j] + gr);
         if (tb) write_copy(tb, g.piece_plane, p, t);
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs g) {
     }
     if (do_bias && m0 + tid < g.M) {
       const int64_t p = g.boff + m0 + tid;
-      const float t = fmaf(-g.eta, bsum, AGN_LD(theta + p));
+      const float t = local_step(AGN_LD(theta + p), g.eta, bsum);
       AGN_ST(theta + p, t);
       if (has_a) AGN_ST(a + p, AGN_LD(a + p) + bsum);
       if (tb) write_copy(tb, g.piece_plane, p, t);

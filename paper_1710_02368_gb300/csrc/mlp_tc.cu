@@ -246,10 +246,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // kernel finished.  Everything that reads or writes global memory waits
   // for it (pdl_begin), except the producer's loads of the weights for the
   // first stages (forward and dX: A = W, last written two or more kernels
-  // back, and the preceding kernel only starts once its own predecessor is
-  // complete) and the converter warps, which touch only shared and tensor
-  // memory until the epilogue (they wait before it): the prefetched weight
-  // stages are converted while the preceding kernel still runs.
+  // back, where the preceding kernel only started once its own predecessor
+  // was complete, or by the preceding kernel itself when that is the dW, a
+  // pull or the Adam step, which let this one launch only after all their
+  // CTAs exited with their writes fenced) and the converter warps, which
+  // touch only shared and tensor memory until the epilogue (they wait before
+  // it): the prefetched weight stages are converted while the preceding
+  // kernel still runs.
   constexpr bool kPrefetchA = kEpi != kEpiDW;
   const bool producer = warp == 0 && lane == 0;
   const bool converter = kWConv && warp >= 2;
@@ -294,7 +297,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       // below, so no phase can complete before its B boxes are requested
       constexpr uint32_t kABytesAll = kWConv ? 0u : kSplit * kABytes * kMT;   // A bytes on full[s]
       constexpr uint32_t kBBytesAll = kSplit * Cfg::kBBytes;
-      const int npre = kPrefetchA ? min(KT, kStages) : 0;
+      const int npre = kPrefetchA && !args.no_a_prefetch ? min(KT, kStages) : 0;
       // (slot_t0 is written by the host before the launch)
       const int b_row0 =
           b_direct ? (int)batch_row0(args.slot_t0, slot, args.step, args.N, args.x_shard) : 0;
@@ -1076,7 +1079,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (i < nvalid) {
               const int64_t p = pbase + (int64_t)(ch * kCh + i) * args.M;
               const float gr = __uint_as_float(r[i]);
-              const float t = fmaf(-eta, gr, th[i]);
+              const float t = local_step(th[i], eta, gr);
               AGN_ST(theta + p, t);
               AGN_ST(acc + p, ac[i] + gr);
               if (kSplit == 1) AGN_ST(tb + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces
@@ -1118,7 +1121,7 @@ bias_update_kernel(const TD* __restrict__ dz, int m, int d, int64_t dz_bstride,
 #pragma unroll
   for (int q = 0; q < kBiasGroups; ++q) s += red[q][fx];
   const int64_t p = (int64_t)AGN_LD(slot_worker + z) * ld_param + boff + f;
-  const float t = fmaf(-eta, s, AGN_LD(theta + p));
+  const float t = local_step(AGN_LD(theta + p), eta, s);
   AGN_ST(theta + p, t);
   AGN_ST(acc + p, AGN_LD(acc + p) + s);
   if (kSplit == 1 && theta_b) AGN_ST(theta_b + p, __float2bfloat16_rn(t));   // fp32 mode: no pieces

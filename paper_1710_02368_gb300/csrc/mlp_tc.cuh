@@ -90,6 +90,8 @@ struct TcArgs {
   // dW: 1 reads a_k's chunks through the parameter ring and stores a_k + g;
   // 0 adds g to a_k in the L2 (red.add) and keeps the ring for theta_k
   int acc_ring;
+  // forward / dX: 1 requests no weight stage before the dependency wait
+  int no_a_prefetch;
 };
 
 // Column tile used for an N: the tensor map of the operand that spans N

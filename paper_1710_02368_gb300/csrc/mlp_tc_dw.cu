@@ -217,12 +217,14 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
   // kernel; global memory is touched only after it has completed, except the
   // producer's first parameter chunks (below)
 
-  if (!((warp == 0 || warp == kWarps - 1) && lane == 0)) pdl_begin();
+  // (the next forward may read theta_k before its own dependency wait: this
+  // kernel lets it launch only when all CTAs have exited, writes fenced)
+  if (!((warp == 0 || warp == kWarps - 1) && lane == 0)) pdl_wait_only();
   if (warp == 0 || warp == kWarps - 1) {
     if (warp == 0 && lane == 0) {
       // operand producer (warp 0): the GEMM operands of every tile into the
       // stage ring, as fast as the MMA frees stages
-      pdl_begin();
+      pdl_wait_only();
       uint32_t ml = 0;   // stage fills issued
       bool ok = true;
       // On a long stream of tiles (bound by DRAM) the operands of a tile are
@@ -342,7 +344,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
           ++ch;
         }
       }
-      pdl_begin();
+      pdl_wait_only();
       for (int t = blockIdx.x; !kGrad && ok && t < T; t += gridDim.x) {
         const TileIdx ti = decode(B, t);
         const DwLayer& L = B.layer[ti.layer];
@@ -509,10 +511,10 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
               const float4 tv = *reinterpret_cast<const float4*>(
                   reinterpret_cast<const float*>(slot) + so);
               float tn[4];
-              tn[0] = fmaf(-eta, gv.x, tv.x);
-              tn[1] = fmaf(-eta, gv.y, tv.y);
-              tn[2] = fmaf(-eta, gv.z, tv.z);
-              tn[3] = fmaf(-eta, gv.w, tv.w);
+              tn[0] = local_step(tv.x, eta, gv.x);
+              tn[1] = local_step(tv.y, eta, gv.y);
+              tn[2] = local_step(tv.z, eta, gv.z);
+              tn[3] = local_step(tv.w, eta, gv.w);
               const int64_t p = L.woff + (int64_t)(fbase + i) * M + k0 + k4;
               AGN_ST(reinterpret_cast<float4*>(theta + p), make_float4(tn[0], tn[1], tn[2], tn[3]));
               if (kAccRing) {
@@ -534,7 +536,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
               reinterpret_cast<const float*>(slot + Cfg::kArrays * kChunkBytes);
           const float gb = gS[lane * 32 + kb];
           const int64_t pb = L.boff + fbase + lane;
-          const float tn = fmaf(-eta, gb, sTb[16 * hf + lane]);
+          const float tn = local_step(sTb[16 * hf + lane], eta, gb);
           AGN_ST(theta + pb, tn);
           if (kAccRing) AGN_ST(acc + pb, sTb[kCF + 16 * hf + lane] + gb);
           else if (kAcc) AGN_RED(acc + pb, gb);
@@ -552,6 +554,7 @@ tc_dw_kernel(const __grid_constant__ DwBatch B, const TcArgs args) {
     if (!ok) *abort_flag = 1;
   }
   __syncwarp();
+  pdl_fence_exit();
   tc::tc_fence_before();
   __syncthreads();
   if (*abort_flag && threadIdx.x == 0) atomicExch(args.err, 1);

@@ -38,7 +38,7 @@ __device__ __forceinline__ void write_copy4(bf16* tb, int64_t plane, int64_t p, 
 }
 
 __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
-  pdl_begin();
+  pdl_wait_only();   // the next forward may read theta_k before its own wait
   const int z = blockIdx.y;
   const int w = AGN_LD(a.slot_worker + z);
   __shared__ float s_c1, s_c2;
@@ -79,6 +79,7 @@ __global__ void __launch_bounds__(kOptThreads) adam_kernel(const AdamArgs a) {
     }
     if (a.theta_b) write_copy4(a.theta_b, a.piece_plane, p, th);
   }
+  pdl_fence_exit();
 }
 
 }  // namespace
