@@ -11,11 +11,13 @@
 //              boxes, MN-major, 128-byte swizzle) into a ring of stages, as
 //              fast as the MMA frees them, so the next tile's GEMM runs while
 //              the current tile's epilogue drains.
-//   warp 10    parameter producer: each tile's theta_k and a_k rows, 32
-//              output features x 128 inputs per chunk, into a second ring.
-//              Each slot is refilled as soon as it frees, so DRAM reads of
-//              the next chunks (and of the next tile) are in flight while the
-//              current one is updated.
+//   warp 10    parameter producer: each tile's theta_k rows (and a_k's, for
+//              waves whose accumulators exceed 64 MB), 32 output features x
+//              128 inputs per chunk, into a second ring.  Each slot is
+//              refilled as soon as it frees, so DRAM reads of the next chunks
+//              (and of the next tile) are in flight while the current one is
+//              updated.  Smaller waves add g to a_k in the L2 (red.add) and
+//              keep twice the theta_k chunks in flight.
 //   warp 1     MMA issuer (one thread) and TMEM owner.  Two accumulators
 //              (double buffer): the GEMM of the next tile runs while the
 //              epilogue drains this one.
@@ -31,6 +33,9 @@
 // MMA warp, over the zero fill of the out-of-range row), so D[M][f] =
 // sum_j dZ_l[j][f] = g_b[f]; the epilogue updates b_l and its accumulator
 // from that row, with their 32 values per chunk copied in by the producer.
+//
+// The local step rounds as Algorithm 1 computes it: g = fp32(-eta grad), then
+// theta_k = fp32(theta_k + g) (local_step).
 //
 // The kernel is persistent (one CTA per SM: the rings take 210 KB of shared
 // memory and the accumulators all 512 TMEM columns); tiles (layer, slot,
