@@ -67,6 +67,38 @@ __device__ __forceinline__ void stage_wait() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
+// Eight consecutive elements (16-byte aligned) as floats: one 16-byte shared
+// load of bf16 (a bf16 is the upper half of the float it stands for), two of
+// floats.  st8 rounds eight floats to T and stores them (16 or 32 bytes).
+__device__ __forceinline__ void ld8(const bf16* p, float (&v)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    v[2 * i] = __uint_as_float(w[i] << 16);
+    v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
+}
+__device__ __forceinline__ void ld8(const float* p, float (&v)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ uint32_t bf16x2_bits(float lo, float hi) {
+  const __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&t);
+}
+__device__ __forceinline__ void st8(bf16* p, const float (&v)[8]) {
+  AGN_ST(reinterpret_cast<uint4*>(p),
+         make_uint4(bf16x2_bits(v[0], v[1]), bf16x2_bits(v[2], v[3]), bf16x2_bits(v[4], v[5]),
+                    bf16x2_bits(v[6], v[7])));
+}
+__device__ __forceinline__ void st8(float* p, const float (&v)[8]) {
+  AGN_ST(reinterpret_cast<float4*>(p), make_float4(v[0], v[1], v[2], v[3]));
+  AGN_ST(reinterpret_cast<float4*>(p + 4), make_float4(v[4], v[5], v[6], v[7]));
+}
+
 template <typename T, int kMaxC>
 __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   extern __shared__ __align__(16) uint8_t head_smem[];
@@ -97,15 +129,34 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
   const bool active = sj < nj;
   const T* h = Hs + (int64_t)sj * Kp;
   constexpr int kStride = 32 * kHeadSplit;
+  // K % 8 == 0: each lane takes eight consecutive inputs at a time (16-byte
+  // shared loads, 16- or 32-byte global stores); else one input at a time
+  const bool vec = K % 8 == 0;
   if (active) {
     float part[kMaxC];
 #pragma unroll
     for (int c = 0; c < kMaxC; ++c) part[c] = 0.f;
-    for (int k = 32 * q + lane; k < K; k += kStride) {
-      const float hv = cvt(h[k]);
+    if (vec) {
+      for (int k0 = 8 * (32 * q + lane); k0 < K; k0 += 8 * kStride) {
+        float hv[8];
+        ld8(h + k0, hv);
 #pragma unroll
-      for (int c = 0; c < kMaxC; ++c)
-        if (c < C) part[c] = fmaf(hv, cvt(Ws[(int64_t)c * Kp + k]), part[c]);
+        for (int c = 0; c < kMaxC; ++c) {
+          if (c < C) {
+            float wv[8];
+            ld8(Ws + (int64_t)c * Kp + k0, wv);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) part[c] = fmaf(hv[i], wv[i], part[c]);
+          }
+        }
+      }
+    } else {
+      for (int k = 32 * q + lane; k < K; k += kStride) {
+        const float hv = cvt(h[k]);
+#pragma unroll
+        for (int c = 0; c < kMaxC; ++c)
+          if (c < C) part[c] = fmaf(hv, cvt(Ws[(int64_t)c * Kp + k]), part[c]);
+      }
     }
 #pragma unroll
     for (int c = 0; c < kMaxC; ++c) {
@@ -172,7 +223,40 @@ __global__ void __launch_bounds__(kHeadThreads) head_kernel(const HeadArgs a) {
     // update); skipped when the output layer is the only layer (dH null)
     T* dh = a.dH ? static_cast<T*>(a.dH) + ((int64_t)z * m + j) * K : nullptr;
     bf16* dp = a.dH_pieces ? a.dH_pieces + ((int64_t)z * m + j) * K : nullptr;
-    for (int k = 32 * q + lane; dh && k < K; k += kStride) {
+    for (int k0 = 8 * (32 * q + lane); vec && dh && k0 < K; k0 += 8 * kStride) {
+      float v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = 0.f;
+#pragma unroll
+      for (int c = 0; c < kMaxC; ++c) {
+        if (c < C) {
+          float wv[8];
+          ld8(Ws + (int64_t)c * Kp + k0, wv);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[i] = fmaf(g[c], wv[i], v[i]);
+        }
+      }
+      float hv[8], o[8];
+      ld8(h + k0, hv);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = cvt(st_f<T>(hv[i] > 0.f ? v[i] : 0.f));
+      st8(dh + k0, o);
+      if (dp) {   // (fp32 mode: o holds the stored floats themselves)
+        float q0[8], q1[8], q2[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          bf16 b0, b1, b2;
+          split3(o[i], b0, b1, b2);
+          q0[i] = __bfloat162float(b0);
+          q1[i] = __bfloat162float(b1);
+          q2[i] = __bfloat162float(b2);
+        }
+        st8(dp + k0, q0);
+        st8(dp + a.dH_plane + k0, q1);
+        st8(dp + 2 * a.dH_plane + k0, q2);
+      }
+    }
+    for (int k = 32 * q + lane; !vec && dh && k < K; k += kStride) {
       float v0 = 0.f, v1 = 0.f;   // two chains: even and odd classes
 #pragma unroll
       for (int c = 0; c < kMaxC; c += 2) {
