@@ -157,3 +157,15 @@ def test_debug_waits_validates_its_arguments(agn):
     from paper_1710_02368_gb300 import _lib
     lib = _lib.load()
     assert lib.agn_debug_waits(None, 1000, 0) == agn.AGN_E_INVALID
+
+
+def test_create_rejects_unknown_tc_mask_bits(agn):
+    """tc_mask takes bits 0-9 (include/agn.h); anything outside is rejected
+    before any device access."""
+    for mask in (-1, 1024, 4096):
+        o = agn.agn_default_options()
+        o.tc_mask = mask
+        with pytest.raises(agn.AGNError) as e:
+            agn.agn_create((8, 4), 2, 1, 0.1, 1, o)
+        assert e.value.code == agn.AGN_E_INVALID
+        assert "tc_mask" in agn.agn_last_error()
