@@ -113,7 +113,8 @@ typedef struct agn_options {
      persistent dW kernel read each accumulator chunk into shared memory and
      store a_k + g even for waves whose accumulators fit well within the L2,
      where it otherwise adds g to a_k in the L2 (red.add).  Bit 9 makes the
-     forward of layer 1 request no weight stage before its dependency wait. */
+     forward of layer 1 request no weight stage before its dependency wait.
+     Any other bit: AGN_E_INVALID. */
   int32_t tc_mask;
   /* Commit rule (AGN_COMMIT_*): AGN_COMMIT_AGN (default) commits
      Delta = -eta a / lambda (Eq. 1; -eta a with normalize = 0);
